@@ -1,0 +1,173 @@
+/*
+ * lca.h - C ABI of the GB300 multi-byte-prediction (MBP) decode step of a byte-level
+ * hierarchical language model with a Latent-Causal-Attention (LCA) multi-byte head
+ * ("Dynamic Multi-Byte Prediction With Hierarchical Language Models").
+ *
+ * One decode step (Algorithm 1, one iteration of its loop) does, per sequence:
+ *   (1) draft n-1 bytes with the multi-byte head over the previous and current latent
+ *       group (Algorithm 1 lines 9-14; Section 3), or with independent MLP heads
+ *       (MLP-MBP, Section 4.1);
+ *   (2) embed the n candidates (next-byte byte c_1 plus the drafts) and run the encoder
+ *       module (Section 2.2 "Encoder Module") with its byte KV cache;
+ *   (3) split at space boundaries, mean-pool closed segments and run the LM module over
+ *       the new latents with its KV cache, only when a segment closes (Algorithm 1
+ *       lines 4-7; Eff-FxT rule, Section 4.1);
+ *   (4) run the next-byte decoder over all n candidates (Algorithm 1 line 8);
+ *   (5) accept: c_1 always, drafts left to right while their probability is >= tau
+ *       (Section 3.1 "Byte Acceptance"; LCA_THRESH), or while they equal the next-byte
+ *       argmax (speculative acceptance, Section 5.2 (ii); LCA_SPEC); then keep the
+ *       accepted prefix of every cache and drop the rest.
+ * The meaning of n used here: one next-byte byte plus n-1 drafts, so 1..n bytes are
+ * committed per step (the algorithm's "n-2 copies" and "h_2[-(n-1):]").
+ *
+ * Conventions
+ *   Status: every call returns LCA_OK (0) or a negative LCA_E_* code; lca_status_str
+ *     names it. After an error the context stays valid for lca_destroy and lca_prefill.
+ *   Ownership: the caller owns the weights, the workspace, the stream and all host
+ *     buffers; the library keeps the workspace and stream pointers until lca_destroy
+ *     and never frees them. Weights are copied (repacked) into the workspace by
+ *     lca_create and need not outlive it.
+ *   Memory: all device memory the library uses lies in the caller's workspace.
+ *   Sync: lca_prefill, lca_mbp_step, lca_generate and the debug calls return after the
+ *     stream has finished their work. lca_generate_async only enqueues.
+ *   Threads: no global state; one context is used by one host thread at a time.
+ */
+#ifndef LCA_H
+#define LCA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* status codes */
+#define LCA_OK 0
+#define LCA_E_ARG (-1)          /* bad pointer, size or enum value */
+#define LCA_E_CAPACITY (-2)     /* batch > max_batch, n outside 1..max_n, or bytes > max_bytes */
+#define LCA_E_WEIGHTS (-3)      /* a weight tensor is missing or has the wrong size or dtype */
+#define LCA_E_CUDA (-4)         /* a CUDA runtime call failed */
+#define LCA_E_DEVICE_STATE (-5) /* a kernel found an index out of range and skipped it */
+#define LCA_E_NUMERIC (-6)      /* non-finite logits were produced */
+#define LCA_E_TIMEOUT (-7)      /* a bounded device wait ran out */
+#define LCA_E_STATE (-8)        /* call order: e.g. a step before any prefill */
+
+/* storage types (weights, KV caches); activations are always fp32 */
+#define LCA_F32 0
+#define LCA_BF16 1
+
+/* multi-byte head kind */
+#define LCA_MB_LCA 0 /* transformer blocks with the LCA mask (Section 3) */
+#define LCA_MB_MLP 1 /* independent residual-SiLU MLP heads on the last next-byte state */
+
+/* acceptance rule */
+#define LCA_THRESH 0 /* draft kept while its drafter probability >= tau (Section 3.1) */
+#define LCA_SPEC 1   /* draft kept while it equals the next-byte argmax (Section 5.2) */
+
+typedef struct lca_ctx lca_ctx; /* opaque, owned by the library */
+
+/* Model shape and capacity. All fields are read; none is inferred. */
+typedef struct {
+  int32_t d_model, n_heads, head_dim, d_ff, vocab; /* vocab must be 256 */
+  int32_t n_enc, n_lm, n_nb, n_mb; /* blocks per module; MLP head: residual layers per head */
+  int32_t mb_kind;                 /* LCA_MB_LCA | LCA_MB_MLP */
+  int32_t n_mlp_heads;             /* MLP head only: heads (>= max_n - 1) */
+  int32_t boundary_byte;           /* byte that ends a segment (0x20) */
+  float rope_base, rms_eps, attn_scale; /* 1e5, 1e-6, 1/sqrt(head_dim) (Section 4.2) */
+  int32_t dtype;                   /* LCA_F32 | LCA_BF16 */
+  int32_t max_batch, max_bytes, max_n; /* max_bytes bounds prompt + generated + max_n */
+} lca_config;
+
+/* One named weight tensor: device pointer, element count, LCA_F32|LCA_BF16.
+ * Names (l = layer index, j = MLP head): "embed" [256,d]; "{enc,lm,nb,mb}.{l}.attn_norm"
+ * [d], ".wq" ".wk" ".wv" ".wo" [d,d], ".mlp_norm" [d], ".w1" ".w3" [d_ff,d], ".w2" [d,d_ff];
+ * "lm.bos" [d]; "nb.norm" [d]; "mb.norm" [d]; "mlp.{j}.{l}.w" [d,d]; "unembed" [256,d].
+ * Linear weights are [out, in] row-major. Norm gains and lm.bos are LCA_F32; every
+ * other tensor has the config dtype. */
+typedef struct {
+  const char* name;
+  const void* ptr;
+  int64_t numel;
+  int32_t dtype;
+} lca_tensor;
+
+/* Committed state of one sequence. */
+typedef struct {
+  int32_t t;                /* committed bytes */
+  int32_t K;                /* committed latents (closed segments) */
+  int32_t open_start;       /* first byte of the open segment */
+  int32_t prev_group_start; /* first byte of latent group K-1, or -1 when K == 0 */
+  int32_t group_start;      /* first byte of latent group K */
+  int32_t next_byte;        /* next-byte argmax at position t-1 (the next c_1) */
+  int32_t generated;        /* bytes generated by the last lca_generate */
+  int32_t pad;
+} lca_seq_state;
+
+/* Counters since lca_create (for throughput and algorithmic-byte accounting). */
+typedef struct {
+  int64_t steps;              /* decode steps run */
+  int64_t lm_steps;           /* steps in which the LM module ran (a candidate closed a segment) */
+  int64_t lm_rows;            /* latents the LM module processed (accepted or rolled back) */
+  int64_t mb_rows;            /* multi-byte window rows computed */
+  int64_t committed;          /* bytes committed */
+  int64_t kernels_per_step;   /* kernels one step graph of the last n launches, LM aside */
+  int64_t kernels_per_lm_run; /* kernels of the LM module when it runs */
+  int64_t workspace_bytes;
+} lca_stats;
+
+/* Bytes of device workspace a context with this config needs (out). */
+int lca_workspace_bytes(const lca_config* cfg, size_t* out);
+
+/* Create a context. workspace: device memory of >= lca_workspace_bytes, 256-byte aligned,
+ * caller-owned. stream: cudaStream_t the library enqueues on (caller-owned; 0 = legacy).
+ * Copies and repacks the n_weights tensors into the workspace. */
+int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, void* workspace,
+               size_t workspace_bytes, void* stream, lca_ctx** out);
+
+/* Start `batch` sequences from host prompts (prompts[b]: lens[b] >= 1 bytes). Runs the whole
+ * forward over the prompts (filling every cache) and the next-byte head at the last byte. */
+int lca_prefill(lca_ctx* ctx, int32_t batch, const uint8_t* const* prompts, const int32_t* lens);
+
+/* One MBP decode step (Algorithm 1, one loop iteration) for every sequence.
+ * out_bytes: host [batch * n], row b holds the committed bytes of sequence b;
+ * out_counts: host [batch], committed bytes 1..n. Either may be NULL. */
+int lca_mbp_step(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, uint8_t* out_bytes,
+                 int32_t* out_counts);
+
+/* lca_mbp_step without outputs: enqueue one step on the stream and return at once. The
+ * committed state is readable afterwards through lca_debug_state. */
+int lca_mbp_step_async(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode);
+
+/* Decode until every sequence has max_new more bytes (the last step is cut to the budget),
+ * as one device-side loop without host round trips. out: host [batch * max_new];
+ * out_len: host [batch] (= max_new); accepted_hist: host [n], steps by accepted drafts,
+ * summed over sequences. Any output pointer may be NULL. */
+int lca_generate(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t max_new,
+                 uint8_t* out, int32_t* out_len, int32_t* accepted_hist);
+
+/* lca_generate split in two: enqueue the loop on the stream and return at once; then wait
+ * and copy the results. Between the two the caller may record events on the stream. */
+int lca_generate_async(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t max_new);
+int lca_generate_fetch(lca_ctx* ctx, uint8_t* out, int32_t* out_len, int32_t* accepted_hist);
+
+/* Debug and test hooks. */
+int lca_debug_state(lca_ctx* ctx, int32_t b, lca_seq_state* out);
+int lca_debug_stats(lca_ctx* ctx, lca_stats* out);
+/* Logits of the last step: nb host [batch * n * 256] (next-byte rows of the n candidates),
+ * mb host [batch * (n-1) * 256] (drafter rows). Either may be NULL. */
+int lca_debug_logits(lca_ctx* ctx, float* nb, float* mb);
+/* Force the accepted-draft count of the NEXT step only: a host [batch], each in 0..n-1, or
+ * NULL to clear. */
+int lca_debug_force_accept(lca_ctx* ctx, const int32_t* a);
+/* Replace the n candidates (c_1, d_2..d_n) of the NEXT step only: cand host [batch * n], or
+ * NULL to clear. The drafter still runs and its logits stay readable. */
+int lca_debug_force_candidates(lca_ctx* ctx, const uint8_t* cand, int32_t n);
+
+int lca_destroy(lca_ctx* ctx);
+const char* lca_status_str(int status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LCA_H */

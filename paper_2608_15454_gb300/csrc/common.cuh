@@ -1,0 +1,240 @@
+// Shared device-side types of the MBP decode step: model shape, workspace layout,
+// per-sequence state and the launch wrappers each kernel file exports.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "lca.h"
+
+namespace lca {
+
+constexpr int kVocab = 256;
+constexpr int kMaxKSplit = 8;     // split-K ways of the skinny linear kernel
+constexpr int kMaxAttnSplit = 16; // key-range splits of decode attention
+constexpr int kAttnQT = 8;        // query rows per attention tile (decode)
+
+// device error word bits
+constexpr int kErrIndex = 1;   // an index was out of range; the access was skipped
+constexpr int kErrNumeric = 2; // non-finite logits
+
+// Linear epilogues.
+enum Epi : int {
+  EPI_STORE = 0,      // y = acc
+  EPI_RESID = 1,      // y = res + acc (res may alias y)
+  EPI_SWIGLU = 2,     // packed rows (2j, 2j+1) = (W1_j, W3_j): y_j = silu(acc_2j) * acc_2j+1
+  EPI_QKV = 3,        // packed rows [q | k | v]: RoPE on q and k, q -> y, k/v -> KV cache
+  EPI_RESID_SILU = 4, // y = res + silu(acc) (MLP-MBP head layer)
+};
+
+// Per-row descriptors of one stack run. Row r belongs to sequence b[r], sits at RoPE
+// position pos[r], writes its key/value to cache slot slot[r] and sees slots [0, kvlen[r]).
+struct Rows {
+  int* b;
+  int* pos;
+  int* slot;
+  int* kvlen;
+  int* seq_start; // [B] first row of each sequence (rows of a sequence are contiguous)
+  int* seq_count; // [B]
+  int* M;         // total rows (device scalar)
+};
+
+// One KV-cache layer: [B][H][S][hd] of the storage type.
+struct KV {
+  void* k;
+  void* v;
+  int S; // slots per (b, h)
+};
+
+struct EpiArgs {
+  int mode;
+  float* y;
+  int ldy;
+  const float* res;
+  int ldres;
+  // EPI_QKV
+  KV kv;
+  Rows rows;
+  const float2* rope; // [slots][hd/2] (cos, sin)
+  int H, hd, d;
+  int* err;
+};
+
+// Per-sequence committed state.
+struct SeqState {
+  int t;          // committed bytes
+  int K;          // committed latents
+  int open_start; // first byte of the open segment
+  int mb_start;   // first byte of the window the MB cache holds (-1: empty)
+  int mb_len;     // cached MB rows from mb_start
+  int next_c1;    // next-byte argmax at t-1
+  int generated;  // bytes generated in the current lca_generate
+  int budget;     // generation budget (lca_generate); INT_MAX for single steps
+  int done;       // budget reached
+  int active;     // sequence exists (b < batch of the last prefill)
+  int pad[6];
+};
+
+// Per-call parameters, copied to the device before each launch.
+struct Params {
+  int n;
+  float tau;
+  int accept;       // LCA_THRESH | LCA_SPEC
+  int gen;          // 1 inside lca_generate: budgets apply
+  int force_accept; // 1: this step uses forced_a
+  int force_cand;   // 1: this step uses forced_cand
+  int batch;
+  int iter;         // generate: steps run
+  int max_iter;     // generate: hard cap on steps
+  int pad[7];
+};
+
+// Counters of work done, for algorithmic-byte accounting.
+struct Stats {
+  unsigned long long steps;     // decode steps run
+  unsigned long long lm_steps;  // steps in which the LM module ran
+  unsigned long long lm_rows;   // LM rows (new latents, committed or not)
+  unsigned long long mb_rows;   // multi-byte window rows computed
+  unsigned long long committed; // bytes committed
+  unsigned long long pad[3];
+};
+
+// Kernels launched by this thread's wrappers (counted at capture time).
+extern thread_local long long g_launches;
+
+// Workspace layout (device pointers into the caller's workspace).
+struct Dev {
+  // shape
+  int d, H, hd, F, n_enc, n_lm, n_nb, n_mb, mb_kind, n_mlp_heads, dtype;
+  int B, S, L, NMAX, R; // batch cap, byte slots, latent slots, max n, row cap
+  int boundary;
+  float eps, scale;
+
+  // weights (storage type; norms and bos fp32)
+  void* embed;   // [256][d]
+  void* unembed; // [256][d]
+  const float* bos;
+  const float* nb_norm;
+  const float* mb_norm;
+  void* mlp_w; // [heads][n_mb][d][d]
+
+  // per-sequence state
+  SeqState* seq;
+  int* gstart;     // [B][L]  gstart[b][g] = first byte of latent group g
+  float* h_store;  // [B][S][d] encoder output of committed (and candidate) bytes
+  float* u_tab;    // [B][L][d] LM inputs u_0 = BOS, u_k = z_k
+  float* o_tab;    // [B][L][d] LM outputs
+  float* y_last;   // [B][d] next-byte hidden at t-1 (MLP head input)
+  int* kpos;       // [B][S] K(p) of committed positions (prefill scratch)
+
+  // rows
+  float* x_mb;
+  float* x_enc;
+  float* x_lm;
+  float* x_nb;
+  float* qbuf; // [R][d]
+  float* att;  // [R][d]
+  float* mid;  // [R][F]
+  float* xnorm; // [R][max(d,F)] normalised rows for the tiled GEMM
+  Rows r_mb, r_v, r_lm;
+
+  // heads
+  int* head_rows_mb; // [B*NMAX] row (into x_mb or x_mlp) of each draft, order b*(n-1)+j
+  int* head_rows_v;  // [B*NMAX]
+  int* M_head_mb;
+  int* M_head_v;
+  float* mb_logits; // [B*NMAX][256]
+  float* nb_logits; // [B*NMAX][256]
+  int* mb_arg;
+  float* mb_prob;
+  int* nb_arg;
+  float* nb_prob;
+
+  // candidates and outputs
+  int* cand;      // [B][NMAX]
+  int* kc;        // [B][NMAX] K(p) of candidate rows
+  uint8_t* out_step; // [B][NMAX]
+  int* out_cnt;      // [B]
+  uint8_t* out_gen;  // [B][S]
+  int* hist;         // [NMAX]
+  int* forced_a;     // [B]
+  int* forced_cand;  // [B][NMAX]
+  Params* params;
+  int* err;
+  Stats* stats;
+
+  // scratch
+  float* lin_part; // split-K partials
+  size_t lin_part_floats;
+  int* lin_cnt;    // split-K tile counters
+  int* head_cnt;   // head row-tile counters
+  float* attn_part; // attention split partials
+  int* attn_cnt;
+  float* inv_rms;  // [R]
+  float2* rope;    // [max(S,L)][hd/2]
+  int rope_slots;
+};
+
+struct Block {
+  const float* attn_norm;
+  const float* mlp_norm;
+  void* wqkv; // [3d][d]
+  void* wo;   // [d][d]
+  void* w13;  // [2F][d], rows interleaved (W1_j, W3_j)
+  void* w2;   // [d][F]
+  KV kv;
+};
+
+// ---------------------------------------------------------------- launch wrappers
+// Linear y = epi(norm?(x) . W^T) over the rows [0, *M) of x, groups along W (grouped GEMM).
+struct LinearArgs {
+  const float* x;
+  int ldx;
+  const void* W; // [groups][N][Kd]
+  int N, Kd;
+  int groups;    // row groups share nothing; group g uses W + g*N*Kd and rows g*Mg..
+  int Mg_stride; // rows per group (groups > 1)
+  const float* norm; // RMSNorm gain or nullptr
+  float eps;
+  const int* M;  // device row count (per group when groups > 1)
+  int M_cap;     // host upper bound of *M
+  EpiArgs epi;
+};
+void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s);
+
+size_t attention_scratch_floats(int B, int H, int hd);
+size_t attention_counters(int B, int H);
+void kernel_attrs_linear();
+void kernel_attrs_step();
+// Attention of query rows over a KV-cache layer (keys [0, kvlen[r]) of sequence b[r]).
+void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
+               int qtiles_grid, int splits, cudaStream_t s);
+
+// Step / prefill glue kernels (kernels_step.cu).
+void launch_mb_plan(const Dev& D, cudaStream_t s);
+void launch_mb_fill(const Dev& D, cudaStream_t s);
+void launch_mlp_plan(const Dev& D, cudaStream_t s);
+void launch_head(const Dev& D, const float* x, const int* rows, const int* M, int M_cap,
+                 const float* norm, float* logits, int* arg, float* prob, cudaStream_t s);
+void launch_verify_plan(const Dev& D, cudaStream_t s);
+void launch_segment(const Dev& D, cudaGraphConditionalHandle h, int use_handle, cudaStream_t s);
+void launch_lm_scatter(const Dev& D, cudaStream_t s);
+void launch_nb_input(const Dev& D, cudaStream_t s);
+void launch_commit(const Dev& D, cudaStream_t s);
+void launch_loop_ctl(const Dev& D, cudaGraphConditionalHandle h, cudaStream_t s);
+void launch_gen_init(const Dev& D, int max_new, cudaStream_t s);
+void launch_rope_table(const Dev& D, float base, cudaStream_t s);
+void launch_pack_rows(void* dst, const void* src, int rows, int cols, int dst_row0, int row_step,
+                      int elem_bytes, cudaStream_t s);
+
+// prefill
+void launch_prefill_embed(const Dev& D, const uint8_t* bytes, int M, cudaStream_t s);
+void launch_prefill_segment(const Dev& D, const uint8_t* bytes, const int* row0, const int* lens,
+                            int batch, const int* lm_row0, cudaStream_t s);
+void launch_prefill_pool(const Dev& D, const int* row0, const int* lens, const int* lm_row0,
+                         int batch, int max_lat, cudaStream_t s);
+void launch_prefill_nb_input(const Dev& D, int M, cudaStream_t s);
+void launch_prefill_finish(const Dev& D, const int* row0, const int* lens, const int* lm_row0,
+                           int batch, cudaStream_t s);
+
+} // namespace lca

@@ -1,0 +1,712 @@
+// Per-step glue of the MBP decode step and of prefill: window planning for the multi-byte
+// head, candidate embedding, space-rule segmentation with mean pooling, upsampling into the
+// next-byte decoder, the unembedding heads, and the acceptance scan with commit/rollback.
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+namespace lca {
+
+namespace {
+
+__device__ __forceinline__ float ld_w(const float* p, size_t i) { return p[i]; }
+__device__ __forceinline__ float ld_w(const __nv_bfloat16* p, size_t i) { return __bfloat162float(p[i]); }
+
+__device__ __forceinline__ void err_or(int* e, int bits) { atomicOr(e, bits); }
+
+// ---------------------------------------------------------------- multi-byte window plan
+// Algorithm 1 lines 9-12: the window of sequence b is the previous and the current latent
+// group, then n-2 copies of the last row. Inside the window the LCA mask is causal, and a
+// row depends only on the window start and the rows before it, so rows computed in earlier
+// steps stay valid while the window start is unchanged: their keys/values are kept in the
+// MB cache (slot = position - window start) and only new committed rows plus the copies are
+// computed. A changed window start (a committed boundary) rebuilds the cache.
+__global__ void k_mb_plan(Dev D) {
+  __shared__ int s_cnt[1024];
+  __shared__ int s_first[1024];
+  const Params P = *D.params;
+  const int n = P.n, batch = P.batch;
+  const int tid = threadIdx.x;
+  for (int b = tid; b < batch; b += blockDim.x) {
+    SeqState& st = D.seq[b];
+    const int t = st.t, g = st.K;
+    const int s = g >= 1 ? D.gstart[(size_t)b * D.L + g - 1] : 0;
+    if (st.mb_start != s) {
+      st.mb_start = s;
+      st.mb_len = 0;
+    }
+    int first = s + st.mb_len;
+    if (first > t - 1) first = t - 1;
+    s_first[b] = first;
+    s_cnt[b] = (t - first) + (n - 2);
+    st.mb_len = t - s;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int acc = 0;
+    for (int b = 0; b < batch; ++b) {
+      D.r_mb.seq_start[b] = acc;
+      D.r_mb.seq_count[b] = s_cnt[b];
+      acc += s_cnt[b];
+    }
+    for (int b = batch; b < D.B; ++b) {
+      D.r_mb.seq_start[b] = acc;
+      D.r_mb.seq_count[b] = 0;
+    }
+    if (acc > D.R) {
+      err_or(D.err, kErrIndex);
+      for (int b = 0; b < batch; ++b) D.r_mb.seq_count[b] = 0;
+      acc = 0;
+    }
+    *D.r_mb.M = acc;
+    *D.M_head_mb = batch * (n - 1);
+    D.stats->mb_rows += acc;
+  }
+  __syncthreads();
+  const int warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
+  for (int b = warp; b < batch; b += nw) {
+    const int st0 = D.r_mb.seq_start[b], cnt = D.r_mb.seq_count[b];
+    const int s = D.seq[b].mb_start, first = s_first[b];
+    for (int j = lane; j < cnt; j += 32) {
+      const int p = first + j;
+      const int r = st0 + j;
+      D.r_mb.b[r] = b;
+      D.r_mb.pos[r] = p;
+      D.r_mb.slot[r] = p - s;
+      D.r_mb.kvlen[r] = p - s + 1;
+    }
+    for (int j = lane; j < n - 1; j += 32)
+      D.head_rows_mb[b * (n - 1) + j] = cnt > 0 ? st0 + cnt - (n - 1) + j : 0;
+  }
+}
+
+// MB input rows: byte p of group k gets o_k + u_k (Algorithm 1 line 9, residual r_2 added
+// before upsampling); copies beyond t belong to the current group K.
+__global__ void k_mb_fill(Dev D) {
+  const int M = *D.r_mb.M;
+  const int d4 = D.d / 4;
+  for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < (size_t)M * d4;
+       idx += (size_t)gridDim.x * blockDim.x) {
+    const int r = (int)(idx / d4), c = (int)(idx - (size_t)r * d4) * 4;
+    const int b = D.r_mb.b[r], p = D.r_mb.pos[r];
+    const SeqState& st = D.seq[b];
+    const int g = st.K;
+    const int gs = D.gstart[(size_t)b * D.L + g];
+    const int k = (g >= 1 && p < gs) ? g - 1 : g;
+    const float4 o = *reinterpret_cast<const float4*>(D.o_tab + ((size_t)b * D.L + k) * D.d + c);
+    const float4 u = *reinterpret_cast<const float4*>(D.u_tab + ((size_t)b * D.L + k) * D.d + c);
+    *reinterpret_cast<float4*>(D.x_mb + (size_t)r * D.d + c) =
+        make_float4(o.x + u.x, o.y + u.y, o.z + u.z, o.w + u.w);
+  }
+}
+
+// MLP-MBP heads: row j*batch + b starts from the last next-byte hidden state of b.
+__global__ void k_mlp_plan(Dev D) {
+  const Params P = *D.params;
+  const int n = P.n, batch = P.batch;
+  const int rows = batch * (n - 1);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    *D.r_mb.M = batch;  // rows per head (grouped linear)
+    *D.M_head_mb = rows;
+  }
+  for (int q = blockIdx.x; q < rows; q += gridDim.x) {
+    const int j = q / batch, b = q - j * batch;
+    const int r = j * D.B + b;  // head j owns rows [j*B, j*B + batch)
+    for (int c = threadIdx.x; c < D.d; c += blockDim.x)
+      D.x_mb[(size_t)r * D.d + c] = D.y_last[(size_t)b * D.d + c];
+    if (threadIdx.x == 0) D.head_rows_mb[b * (n - 1) + j] = r;
+  }
+}
+
+// ---------------------------------------------------------------- unembedding heads
+// Final RMSNorm of the head, shared unembedding (Section 3), then per row the argmax (lowest
+// byte among equal maxima) and its softmax probability exp(l_max - logsumexp(l)).
+constexpr int kHR = 8;   // rows per CTA
+constexpr int kHV = 16;  // vocab entries per CTA
+
+template <typename TW>
+__global__ void __launch_bounds__(128)
+k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const int* Mp, int M_cap,
+       const float* __restrict__ norm, float* __restrict__ logits, int* __restrict__ arg,
+       float* __restrict__ prob, int* __restrict__ cnt) {
+  extern __shared__ float xs[];  // [kHR][d]
+  __shared__ float inv[kHR];
+  __shared__ int s_last;
+  int M = *Mp;
+  M = M < M_cap ? M : M_cap;
+  const int rt = blockIdx.x;
+  const int r0 = rt * kHR;
+  if (r0 >= M) return;
+  const int mr = min(kHR, M - r0);
+  const int d = D.d;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  for (int i = warp; i < mr; i += 4) {
+    const int src = rows ? rows[r0 + i] : r0 + i;
+    const float* xr = x + (size_t)src * d;
+    float ss = 0.f;
+    for (int k = lane; k < d; k += 32) ss += xr[k] * xr[k];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if (lane == 0) inv[i] = rsqrtf(ss / (float)d + D.eps);
+  }
+  __syncthreads();
+  for (int idx = tid; idx < kHR * d; idx += 128) {
+    const int i = idx / d, k = idx - i * d;
+    float v = 0.f;
+    if (i < mr) {
+      const int src = rows ? rows[r0 + i] : r0 + i;
+      v = x[(size_t)src * d + k] * inv[i] * norm[k];
+    }
+    xs[idx] = v;
+  }
+  __syncthreads();
+  const TW* Wu = reinterpret_cast<const TW*>(D.unembed);
+  // each warp: 4 vocab rows; each lane a strided slice of d
+  const int v0 = blockIdx.y * kHV + warp * 4;
+  for (int vv = 0; vv < 4; ++vv) {
+    const int v = v0 + vv;
+    float acc[kHR];
+#pragma unroll
+    for (int i = 0; i < kHR; ++i) acc[i] = 0.f;
+    for (int k = lane; k < d; k += 32) {
+      const float w = ld_w(Wu, (size_t)v * d + k);
+#pragma unroll
+      for (int i = 0; i < kHR; ++i) acc[i] = fmaf(w, xs[i * d + k], acc[i]);
+    }
+#pragma unroll
+    for (int i = 0; i < kHR; ++i) {
+      float s = acc[i];
+#pragma unroll
+      for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      if (lane == 0 && i < mr) logits[(size_t)(r0 + i) * kVocab + v] = s;
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = (atomicAdd(cnt + rt, 1) == (int)gridDim.y - 1);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  for (int i = warp; i < mr; i += 4) {
+    const float* lg = logits + (size_t)(r0 + i) * kVocab;
+    float best = -INFINITY;
+    int bi = kVocab;
+    bool bad = false;
+    for (int v = lane; v < kVocab; v += 32) {
+      const float l = __ldcg(lg + v);
+      if (!isfinite(l)) bad = true;
+      if (l > best || (l == best && v < bi)) {
+        best = l;
+        bi = v;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+      const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (ob > best || (ob == best && oi < bi)) {
+        best = ob;
+        bi = oi;
+      }
+    }
+    bad = __any_sync(0xffffffffu, bad);
+    float se = 0.f;
+    for (int v = lane; v < kVocab; v += 32) se += expf(__ldcg(lg + v) - best);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+    if (lane == 0) {
+      if (bad) {
+        err_or(D.err, kErrNumeric);
+        bi = 0;
+      }
+      arg[r0 + i] = bi;
+      prob[r0 + i] = bad ? 0.f : 1.f / se;
+    }
+  }
+  if (tid == 0) cnt[rt] = 0;
+}
+
+// ---------------------------------------------------------------- verify rows
+// Candidates c_1 (next-byte argmax) and d_2..d_n (drafts) at positions t..t+n-1; embed them.
+__global__ void k_verify_plan(Dev D) {
+  const Params P = *D.params;
+  const int n = P.n, batch = P.batch;
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x;
+  if (b >= batch) {
+    if (tid == 0) {
+      D.r_v.seq_start[b] = batch * n;
+      D.r_v.seq_count[b] = 0;
+    }
+    return;
+  }
+  const int t = D.seq[b].t;
+  if (b == 0 && tid == 0) *D.r_v.M = batch * n;
+  for (int i = tid; i < n; i += blockDim.x) {
+    int c;
+    if (P.force_cand) c = D.forced_cand[b * D.NMAX + i];
+    else c = i == 0 ? D.seq[b].next_c1 : D.mb_arg[b * (n - 1) + i - 1];
+    D.cand[b * D.NMAX + i] = c & 255;
+    const int r = b * n + i;
+    int p = t + i;
+    if (p >= D.S) {
+      err_or(D.err, kErrIndex);
+      p = D.S - 1;
+    }
+    D.r_v.b[r] = b;
+    D.r_v.pos[r] = p;
+    D.r_v.slot[r] = p;
+    D.r_v.kvlen[r] = p + 1;
+  }
+  if (tid == 0) {
+    D.r_v.seq_start[b] = b * n;
+    D.r_v.seq_count[b] = n;
+  }
+  __syncthreads();
+  for (int idx = tid; idx < n * D.d; idx += blockDim.x) {
+    const int i = idx / D.d, k = idx - i * D.d;
+    const int c = D.cand[b * D.NMAX + i];
+    const float e = D.dtype == LCA_BF16
+                        ? ld_w(reinterpret_cast<const __nv_bfloat16*>(D.embed), (size_t)c * D.d + k)
+                        : ld_w(reinterpret_cast<const float*>(D.embed), (size_t)c * D.d + k);
+    D.x_enc[(size_t)(b * n + i) * D.d + k] = e;
+  }
+}
+
+// ---------------------------------------------------------------- segments and latents
+// Space rule (b_p = [x_p == 0x20], the boundary byte ends its segment). Every boundary among
+// the candidates closes a segment: z = mean of the encoder output over the segment (committed
+// bytes from h_store, candidate rows from x_enc), which becomes the LM input of latent K+j.
+// K(p) of candidate row i counts boundaries at positions <= p. New latents of all sequences
+// are compacted into LM rows; the LM module runs (graph conditional) only if there are any.
+__global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handle) {
+  const Params P = *D.params;
+  const int n = P.n, batch = P.batch;
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x;
+  __shared__ int s_sp[64];
+  __shared__ int s_nsp, s_off;
+  if (b >= batch) {
+    if (tid == 0) {
+      D.r_lm.seq_start[b] = 0;
+      D.r_lm.seq_count[b] = 0;
+    }
+    return;
+  }
+  if (tid == 0) {
+    int off = 0, total = 0;
+    for (int bb = 0; bb < batch; ++bb) {
+      int c = 0;
+      for (int i = 0; i < n; ++i) c += D.cand[bb * D.NMAX + i] == D.boundary;
+      if (bb < b) off += c;
+      total += c;
+    }
+    s_off = off;
+    int m = 0;
+    for (int i = 0; i < n; ++i)
+      if (D.cand[b * D.NMAX + i] == D.boundary) s_sp[m++] = i;
+    s_nsp = m;
+    if (b == 0) {
+      *D.r_lm.M = total;
+      if (use_handle) cudaGraphSetConditional(hcond, total > 0 ? 1u : 0u);
+      D.stats->steps += 1;
+      D.stats->lm_steps += total > 0;
+      D.stats->lm_rows += total;
+    }
+  }
+  __syncthreads();
+  const SeqState st = D.seq[b];
+  const int t = st.t, K = st.K;
+  const int m = s_nsp, off = s_off;
+  if (tid < n) {
+    int k = K;
+    for (int i = 0; i <= tid; ++i) k += D.cand[b * D.NMAX + i] == D.boundary;
+    D.kc[b * D.NMAX + tid] = k;
+  }
+  if (tid == 0) {
+    D.r_lm.seq_start[b] = off;
+    D.r_lm.seq_count[b] = m;
+  }
+  for (int j = 0; j < m; ++j) {
+    const int i = s_sp[j];
+    const int k = K + 1 + j;
+    const int seg0 = j == 0 ? st.open_start : t + s_sp[j - 1] + 1;
+    const int seg1 = t + i;  // inclusive
+    const int row = off + j;
+    if (k >= D.L) {
+      if (tid == 0) err_or(D.err, kErrIndex);
+      continue;
+    }
+    const float inv_cnt = 1.f / (float)(seg1 - seg0 + 1);
+    for (int c = tid; c < D.d; c += blockDim.x) {
+      float s = 0.f;
+      for (int p = seg0; p <= seg1; ++p)
+        s += p < t ? D.h_store[((size_t)b * D.S + p) * D.d + c]
+                   : D.x_enc[(size_t)(b * n + p - t) * D.d + c];
+      const float z = s * inv_cnt;
+      D.x_lm[(size_t)row * D.d + c] = z;
+      D.u_tab[((size_t)b * D.L + k) * D.d + c] = z;
+    }
+    if (tid == 0) {
+      D.gstart[(size_t)b * D.L + k] = seg1;
+      D.r_lm.b[row] = b;
+      D.r_lm.pos[row] = k;
+      D.r_lm.slot[row] = k;
+      D.r_lm.kvlen[row] = k + 1;
+    }
+  }
+}
+
+// o_k of the latents the LM module just produced.
+__global__ void k_lm_scatter(Dev D) {
+  const int M = *D.r_lm.M;
+  for (int r = blockIdx.x; r < M; r += gridDim.x) {
+    const int b = D.r_lm.b[r], k = D.r_lm.pos[r];
+    for (int c = threadIdx.x; c < D.d; c += blockDim.x)
+      D.o_tab[((size_t)b * D.L + k) * D.d + c] = D.x_lm[(size_t)r * D.d + c];
+  }
+}
+
+// Next-byte decoder input: upsampled LM output plus the encoder residual r_1 (Algorithm 1
+// line 8): o_{K(p)} + h_e[p].
+__global__ void k_nb_input(Dev D) {
+  const Params P = *D.params;
+  const int n = P.n, batch = P.batch;
+  const int rows = batch * n;
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+    const int b = r / n, i = r - b * n;
+    const int k = D.kc[b * D.NMAX + i];
+    const float* o = D.o_tab + ((size_t)b * D.L + k) * D.d;
+    for (int c = threadIdx.x; c < D.d; c += blockDim.x)
+      D.x_nb[(size_t)r * D.d + c] = o[c] + D.x_enc[(size_t)r * D.d + c];
+  }
+}
+
+// ---------------------------------------------------------------- accept and commit
+// Section 3.1 "Byte Acceptance": c_1 is always kept; drafts are kept left to right while the
+// drafter's probability is >= tau (THRESH) or while they equal the next-byte argmax at the
+// position before them (SPEC); the first failure drops the rest. The accepted prefix of every
+// cache is kept by advancing t and K; everything beyond is dropped (overwritten later).
+__global__ void k_commit(Dev D) {
+  const Params P = *D.params;
+  const int n = P.n, batch = P.batch;
+  const int b = blockIdx.x;
+  if (b >= batch) return;
+  const int tid = threadIdx.x;
+  __shared__ int s_e, s_a, s_t, s_skip;
+  SeqState& st = D.seq[b];
+  if (tid == 0) {
+    s_skip = 0;
+    s_t = st.t;
+    if (P.gen && st.done) {
+      D.out_cnt[b] = 0;
+      s_skip = 1;
+    } else {
+      const int* cand = D.cand + b * D.NMAX;
+      int a = 0;
+      if (P.force_accept) {
+        a = D.forced_a[b];
+        a = a < 0 ? 0 : (a > n - 1 ? n - 1 : a);
+      } else {
+        for (int j = 0; j < n - 1; ++j) {
+          const bool ok = P.accept == LCA_SPEC ? cand[j + 1] == D.nb_arg[b * n + j]
+                                               : D.mb_prob[b * (n - 1) + j] >= P.tau;
+          if (!ok) break;
+          ++a;
+        }
+      }
+      int e = 1 + a;
+      if (P.gen) {
+        const int rem = st.budget - st.generated;
+        e = e < rem ? e : rem;
+      }
+      s_e = e;
+      s_a = a;
+    }
+  }
+  __syncthreads();
+  if (s_skip) return;
+  const int e = s_e, t = s_t;
+  // encoder outputs of the committed candidates join the pooled history
+  for (int idx = tid; idx < e * D.d; idx += blockDim.x) {
+    const int i = idx / D.d, c = idx - i * D.d;
+    D.h_store[((size_t)b * D.S + t + i) * D.d + c] = D.x_enc[(size_t)(b * n + i) * D.d + c];
+  }
+  for (int c = tid; c < D.d; c += blockDim.x)
+    D.y_last[(size_t)b * D.d + c] = D.x_nb[(size_t)(b * n + e - 1) * D.d + c];
+  if (tid == 0) {
+    const int* cand = D.cand + b * D.NMAX;
+    int last_sp = -1;
+    const int gen0 = st.generated;
+    for (int i = 0; i < n; ++i) {
+      const int c = cand[i];
+      D.out_step[b * D.NMAX + i] = (uint8_t)(i < e ? c : 0);
+      if (i < e) {
+        if (c == D.boundary) last_sp = i;
+        if (P.gen && gen0 + i < D.S) D.out_gen[(size_t)b * D.S + gen0 + i] = (uint8_t)c;
+      }
+    }
+    D.out_cnt[b] = e;
+    st.t = t + e;
+    st.K = D.kc[b * D.NMAX + e - 1];
+    if (last_sp >= 0) st.open_start = t + last_sp + 1;
+    st.next_c1 = D.nb_arg[b * n + e - 1];
+    st.generated = gen0 + e;
+    if (P.gen && st.generated >= st.budget) st.done = 1;
+    atomicAdd(D.hist + s_a, 1);
+    atomicAdd(&D.stats->committed, (unsigned long long)e);
+  }
+}
+
+// Generate loop control: keep looping while a sequence is short of its budget (and never more
+// than max_iter steps, each of which commits at least one byte per unfinished sequence).
+__global__ void k_loop_ctl(Dev D, cudaGraphConditionalHandle h) {
+  if (threadIdx.x != 0) return;
+  Params* P = D.params;
+  const int it = P->iter + 1;
+  P->iter = it;
+  int any = 0;
+  for (int b = 0; b < P->batch; ++b) any |= (D.seq[b].active && !D.seq[b].done);
+  cudaGraphSetConditional(h, (any && it < P->max_iter) ? 1u : 0u);
+}
+
+__global__ void k_gen_init(Dev D, int max_new) {
+  const int b = threadIdx.x;
+  if (b < D.B) {
+    SeqState& st = D.seq[b];
+    st.generated = 0;
+    st.budget = max_new;
+    st.done = st.active ? 0 : 1;
+  }
+  if (b < D.NMAX) D.hist[b] = 0;
+  if (b == 0) D.params->iter = 0;
+}
+
+// cos/sin of RoPE angles pos * base^(-2i/hd), computed in double.
+__global__ void k_rope_table(float2* tab, int slots, int hd, double base) {
+  const int half = hd / 2;
+  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < slots * half;
+       idx += gridDim.x * blockDim.x) {
+    const int p = idx / half, i = idx - p * half;
+    const double ang = (double)p * pow(base, -2.0 * i / hd);
+    tab[idx] = make_float2((float)cos(ang), (float)sin(ang));
+  }
+}
+
+// ---------------------------------------------------------------- prefill
+__global__ void k_prefill_embed(Dev D, const uint8_t* __restrict__ bytes, int M) {
+  for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < (size_t)M * D.d;
+       idx += (size_t)gridDim.x * blockDim.x) {
+    const int r = (int)(idx / D.d), k = (int)(idx - (size_t)r * D.d);
+    const int c = bytes[r];
+    D.x_enc[idx] = D.dtype == LCA_BF16
+                       ? ld_w(reinterpret_cast<const __nv_bfloat16*>(D.embed), (size_t)c * D.d + k)
+                       : ld_w(reinterpret_cast<const float*>(D.embed), (size_t)c * D.d + k);
+  }
+}
+
+// One CTA per sequence: K(p) for every prompt byte and the group starts.
+__global__ void k_prefill_segment(Dev D, const uint8_t* __restrict__ bytes, const int* row0,
+                                  const int* lens) {
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x;
+  __shared__ int s_scan[1024];
+  __shared__ int s_carry;
+  const int len = lens[b];
+  const uint8_t* x = bytes + row0[b];
+  if (tid == 0) {
+    s_carry = 0;
+    D.gstart[(size_t)b * D.L] = 0;
+  }
+  __syncthreads();
+  for (int base = 0; base < len; base += blockDim.x) {
+    const int p = base + tid;
+    const int isb = (p < len && x[p] == D.boundary) ? 1 : 0;
+    s_scan[tid] = isb;
+    __syncthreads();
+    for (int o = 1; o < (int)blockDim.x; o <<= 1) {
+      const int v = tid >= o ? s_scan[tid - o] : 0;
+      __syncthreads();
+      s_scan[tid] += v;
+      __syncthreads();
+    }
+    const int k = s_carry + s_scan[tid];
+    if (p < len) {
+      D.kpos[(size_t)b * D.S + p] = k;
+      if (isb) {
+        if (k < D.L) D.gstart[(size_t)b * D.L + k] = p;
+        else err_or(D.err, kErrIndex);
+      }
+    }
+    __syncthreads();
+    if (tid == blockDim.x - 1) s_carry = k;
+    __syncthreads();
+  }
+  if (tid == 0) {
+    const int K = s_carry;
+    D.seq[b].K = K;
+    D.seq[b].open_start = K > 0 ? D.gstart[(size_t)b * D.L + K] + 1 : 0;
+  }
+}
+
+// CTA (b, k): latent k of sequence b: BOS for k = 0, else the mean of segment k.
+__global__ void k_prefill_pool(Dev D, const int* row0, const int* lm_row0) {
+  const int b = blockIdx.x;
+  const int k = blockIdx.y;
+  const int K = D.seq[b].K;
+  if (k > K) return;
+  const int row = lm_row0[b] + k;
+  if (k == 0) {
+    for (int c = threadIdx.x; c < D.d; c += blockDim.x) {
+      D.x_lm[(size_t)row * D.d + c] = D.bos[c];
+      D.u_tab[((size_t)b * D.L) * D.d + c] = D.bos[c];
+    }
+    return;
+  }
+  const int seg1 = D.gstart[(size_t)b * D.L + k];
+  const int seg0 = k == 1 ? 0 : D.gstart[(size_t)b * D.L + k - 1] + 1;
+  const float inv_cnt = 1.f / (float)(seg1 - seg0 + 1);
+  for (int c = threadIdx.x; c < D.d; c += blockDim.x) {
+    float s = 0.f;
+    for (int p = seg0; p <= seg1; ++p) s += D.x_enc[(size_t)(row0[b] + p) * D.d + c];
+    const float z = s * inv_cnt;
+    D.x_lm[(size_t)row * D.d + c] = z;
+    D.u_tab[((size_t)b * D.L + k) * D.d + c] = z;
+  }
+}
+
+__global__ void k_prefill_nb_input(Dev D, int M) {
+  for (int r = blockIdx.x; r < M; r += gridDim.x) {
+    const int b = D.r_v.b[r], p = D.r_v.pos[r];
+    const int k = D.kpos[(size_t)b * D.S + p];
+    const float* o = D.o_tab + ((size_t)b * D.L + k) * D.d;
+    for (int c = threadIdx.x; c < D.d; c += blockDim.x) {
+      const float h = D.x_enc[(size_t)r * D.d + c];
+      D.h_store[((size_t)b * D.S + p) * D.d + c] = h;
+      D.x_nb[(size_t)r * D.d + c] = o[c] + h;
+    }
+  }
+}
+
+__global__ void k_prefill_finish(Dev D, const int* row0, const int* lens) {
+  const int b = blockIdx.x;
+  const int last = row0[b] + lens[b] - 1;
+  for (int c = threadIdx.x; c < D.d; c += blockDim.x)
+    D.y_last[(size_t)b * D.d + c] = D.x_nb[(size_t)last * D.d + c];
+  if (threadIdx.x == 0) {
+    SeqState& st = D.seq[b];
+    st.t = lens[b];
+    st.mb_start = -1;
+    st.mb_len = 0;
+    st.next_c1 = D.nb_arg[b];
+    st.generated = 0;
+    st.budget = 0x3fffffff;
+    st.done = 0;
+    st.active = 1;
+  }
+}
+
+// Repack rows: dst[(dst_row0 + i*row_step)] = src[i] for i < rows (row = cols elements).
+__global__ void k_pack_rows(uint8_t* dst, const uint8_t* src, int rows, size_t row_bytes,
+                            int dst_row0, int row_step) {
+  for (int i = blockIdx.x; i < rows; i += gridDim.x) {
+    const uint8_t* s = src + (size_t)i * row_bytes;
+    uint8_t* d = dst + (size_t)(dst_row0 + (size_t)i * row_step) * row_bytes;
+    for (size_t c = threadIdx.x * 16; c < row_bytes; c += blockDim.x * 16)
+      *reinterpret_cast<uint4*>(d + c) = *reinterpret_cast<const uint4*>(s + c);
+  }
+}
+
+} // namespace
+
+// ---------------------------------------------------------------- launch wrappers
+void kernel_attrs_step() {
+  cudaFuncSetAttribute(k_head<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  cudaFuncSetAttribute(k_head<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+}
+
+thread_local long long g_launches = 0;
+
+void launch_mb_plan(const Dev& D, cudaStream_t s) {
+  ++g_launches;
+  k_mb_plan<<<1, 1024, 0, s>>>(D);
+}
+void launch_mb_fill(const Dev& D, cudaStream_t s) {
+  ++g_launches;
+  k_mb_fill<<<152 * 2, 256, 0, s>>>(D);
+}
+void launch_mlp_plan(const Dev& D, cudaStream_t s) {
+  ++g_launches;
+  k_mlp_plan<<<256, 256, 0, s>>>(D);
+}
+
+void launch_head(const Dev& D, const float* x, const int* rows, const int* M, int M_cap,
+                 const float* norm, float* logits, int* arg, float* prob, cudaStream_t s) {
+  dim3 grid((M_cap + kHR - 1) / kHR, kVocab / kHV);
+  const size_t smem = (size_t)kHR * D.d * sizeof(float);
+  ++g_launches;
+  // the split-K counters double as head row-tile counters (different launches, same stream)
+  if (D.dtype == LCA_BF16)
+    k_head<__nv_bfloat16><<<grid, 128, smem, s>>>(D, x, rows, M, M_cap, norm, logits, arg, prob, D.head_cnt);
+  else
+    k_head<float><<<grid, 128, smem, s>>>(D, x, rows, M, M_cap, norm, logits, arg, prob, D.head_cnt);
+}
+
+void launch_verify_plan(const Dev& D, cudaStream_t s) {
+  ++g_launches;
+  k_verify_plan<<<D.B, 256, 0, s>>>(D);
+}
+void launch_segment(const Dev& D, cudaGraphConditionalHandle h, int use_handle, cudaStream_t s) {
+  ++g_launches;
+  k_segment<<<D.B, 256, 0, s>>>(D, h, use_handle);
+}
+void launch_lm_scatter(const Dev& D, cudaStream_t s) {
+  ++g_launches;
+  k_lm_scatter<<<256, 256, 0, s>>>(D);
+}
+void launch_nb_input(const Dev& D, cudaStream_t s) {
+  ++g_launches;
+  k_nb_input<<<256, 256, 0, s>>>(D);
+}
+void launch_commit(const Dev& D, cudaStream_t s) {
+  ++g_launches;
+  k_commit<<<D.B, 256, 0, s>>>(D);
+}
+void launch_loop_ctl(const Dev& D, cudaGraphConditionalHandle h, cudaStream_t s) {
+  ++g_launches;
+  k_loop_ctl<<<1, 32, 0, s>>>(D, h);
+}
+void launch_gen_init(const Dev& D, int max_new, cudaStream_t s) {
+  k_gen_init<<<1, 1024, 0, s>>>(D, max_new);
+}
+void launch_rope_table(const Dev& D, float base, cudaStream_t s) {
+  k_rope_table<<<256, 256, 0, s>>>(D.rope, D.rope_slots, D.hd, (double)base);
+}
+void launch_pack_rows(void* dst, const void* src, int rows, int cols, int dst_row0, int row_step,
+                      int elem_bytes, cudaStream_t s) {
+  k_pack_rows<<<256, 128, 0, s>>>((uint8_t*)dst, (const uint8_t*)src, rows,
+                                  (size_t)cols * elem_bytes, dst_row0, row_step);
+}
+void launch_prefill_embed(const Dev& D, const uint8_t* bytes, int M, cudaStream_t s) {
+  k_prefill_embed<<<1024, 256, 0, s>>>(D, bytes, M);
+}
+void launch_prefill_segment(const Dev& D, const uint8_t* bytes, const int* row0, const int* lens,
+                            int batch, const int* lm_row0, cudaStream_t s) {
+  (void)lm_row0;
+  k_prefill_segment<<<batch, 1024, 0, s>>>(D, bytes, row0, lens);
+}
+void launch_prefill_pool(const Dev& D, const int* row0, const int* lens, const int* lm_row0,
+                         int batch, int max_lat, cudaStream_t s) {
+  (void)lens;
+  k_prefill_pool<<<dim3(batch, max_lat + 1), 256, 0, s>>>(D, row0, lm_row0);
+}
+void launch_prefill_nb_input(const Dev& D, int M, cudaStream_t s) {
+  k_prefill_nb_input<<<1024, 256, 0, s>>>(D, M);
+}
+void launch_prefill_finish(const Dev& D, const int* row0, const int* lens, const int* lm_row0,
+                           int batch, cudaStream_t s) {
+  (void)lm_row0;
+  k_prefill_finish<<<batch, 256, 0, s>>>(D, row0, lens);
+}
+
+} // namespace lca

@@ -1,0 +1,961 @@
+// Host runtime behind include/lca.h: workspace layout, weight repacking, prefill, and the
+// decode step as a CUDA graph. One step is one graph replay with no host round trip; the
+// LM module sits in an IF conditional node that the segmentation kernel switches on only
+// when a segment closes (Algorithm 1 lines 4-7). lca_generate wraps the step in a WHILE
+// conditional node whose control kernel stops once every sequence has its bytes.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+
+using namespace lca;
+
+namespace {
+
+constexpr int kParamSlots = 8;
+constexpr int kMaxN = 16;
+
+struct Carver {
+  char* base;
+  size_t off = 0;
+  template <typename T>
+  T* take(size_t count) {
+    off = (off + 255) & ~size_t(255);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+struct Layout {
+  Dev D{};
+  std::vector<Block> enc, lm, nb, mb;
+  size_t bytes = 0;
+};
+
+size_t tw_bytes(int dtype) { return dtype == LCA_BF16 ? 2 : 4; }
+
+// Carve the whole workspace; base == nullptr only measures it.
+void carve(const lca_config& c, char* base, Layout& L) {
+  Carver cv{base};
+  Dev& D = L.D;
+  D.d = c.d_model;
+  D.H = c.n_heads;
+  D.hd = c.head_dim;
+  D.F = c.d_ff;
+  D.n_enc = c.n_enc;
+  D.n_lm = c.n_lm;
+  D.n_nb = c.n_nb;
+  D.n_mb = c.n_mb;
+  D.mb_kind = c.mb_kind;
+  D.n_mlp_heads = c.n_mlp_heads;
+  D.dtype = c.dtype;
+  D.B = c.max_batch;
+  D.S = c.max_bytes;
+  D.L = c.max_bytes + 1;
+  D.NMAX = c.max_n;
+  D.R = c.max_batch * (c.max_bytes + c.max_n);
+  D.boundary = c.boundary_byte;
+  D.eps = c.rms_eps;
+  D.scale = c.attn_scale;
+  const size_t d = D.d, F = D.F, tb = tw_bytes(c.dtype);
+  const size_t B = D.B, S = D.S, Lt = D.L, R = D.R, NM = D.NMAX;
+
+  D.embed = cv.take<char>(256 * d * tb);
+  D.unembed = cv.take<char>(256 * d * tb);
+  D.bos = cv.take<float>(d);
+  D.nb_norm = cv.take<float>(d);
+  D.mb_norm = cv.take<float>(d);
+  auto blocks = [&](std::vector<Block>& v, int n, size_t slots) {
+    v.resize(n);
+    for (auto& b : v) {
+      b.attn_norm = cv.take<float>(d);
+      b.mlp_norm = cv.take<float>(d);
+      b.wqkv = cv.take<char>(3 * d * d * tb);
+      b.wo = cv.take<char>(d * d * tb);
+      b.w13 = cv.take<char>(2 * F * d * tb);
+      b.w2 = cv.take<char>(d * F * tb);
+      b.kv.S = (int)slots;
+      b.kv.k = cv.take<char>(B * D.H * slots * D.hd * tb);
+      b.kv.v = cv.take<char>(B * D.H * slots * D.hd * tb);
+    }
+  };
+  blocks(L.enc, c.n_enc, S);
+  blocks(L.lm, c.n_lm, Lt);
+  blocks(L.nb, c.n_nb, S);
+  if (c.mb_kind == LCA_MB_LCA) {
+    blocks(L.mb, c.n_mb, S);
+    D.mlp_w = nullptr;
+  } else {
+    L.mb.clear();
+    D.mlp_w = cv.take<char>((size_t)c.n_mb * c.n_mlp_heads * d * d * tb);
+  }
+
+  D.seq = cv.take<SeqState>(B);
+  D.gstart = cv.take<int>(B * Lt);
+  D.h_store = cv.take<float>(B * S * d);
+  D.u_tab = cv.take<float>(B * Lt * d);
+  D.o_tab = cv.take<float>(B * Lt * d);
+  D.y_last = cv.take<float>(B * d);
+  D.kpos = cv.take<int>(B * S);
+
+  D.x_mb = cv.take<float>(R * d);
+  D.x_enc = cv.take<float>(R * d);
+  D.x_lm = cv.take<float>(R * d);
+  D.x_nb = cv.take<float>(R * d);
+  D.qbuf = cv.take<float>(R * d);
+  D.att = cv.take<float>(R * d);
+  D.mid = cv.take<float>(R * F);
+  D.xnorm = nullptr;
+  auto rows = [&](Rows& r) {
+    r.b = cv.take<int>(R);
+    r.pos = cv.take<int>(R);
+    r.slot = cv.take<int>(R);
+    r.kvlen = cv.take<int>(R);
+    r.seq_start = cv.take<int>(B);
+    r.seq_count = cv.take<int>(B);
+    r.M = cv.take<int>(1);
+  };
+  rows(D.r_mb);
+  rows(D.r_v);
+  rows(D.r_lm);
+
+  const size_t HR = std::max<size_t>(B * NM, B);
+  D.head_rows_mb = cv.take<int>(HR);
+  D.head_rows_v = cv.take<int>(HR);
+  D.M_head_mb = cv.take<int>(1);
+  D.M_head_v = cv.take<int>(1);
+  D.mb_logits = cv.take<float>(HR * 256);
+  D.nb_logits = cv.take<float>(HR * 256);
+  D.mb_arg = cv.take<int>(HR);
+  D.mb_prob = cv.take<float>(HR);
+  D.nb_arg = cv.take<int>(HR);
+  D.nb_prob = cv.take<float>(HR);
+
+  D.cand = cv.take<int>(B * NM);
+  D.kc = cv.take<int>(B * NM);
+  D.out_step = cv.take<uint8_t>(B * NM);
+  D.out_cnt = cv.take<int>(B);
+  D.out_gen = cv.take<uint8_t>(B * S);
+  D.hist = cv.take<int>(NM);
+  D.forced_a = cv.take<int>(B);
+  D.forced_cand = cv.take<int>(B * NM);
+  D.params = cv.take<Params>(kParamSlots);
+  D.err = cv.take<int>(1);
+  D.stats = cv.take<Stats>(1);
+
+  const size_t gemv_rows = B <= 4 ? R : 64;
+  D.lin_part_floats = (size_t)kMaxKSplit * gemv_rows * d;
+  D.lin_part = cv.take<float>(D.lin_part_floats);
+  D.lin_cnt = cv.take<int>(8192);
+  D.head_cnt = cv.take<int>(std::max<size_t>(R / 8 + 1, 1024));
+  D.attn_part = cv.take<float>(attention_scratch_floats(D.B, D.H, D.hd));
+  D.attn_cnt = cv.take<int>(attention_counters(D.B, D.H));
+  D.inv_rms = cv.take<float>(R);
+  D.rope_slots = (int)std::max(S, Lt);
+  D.rope = cv.take<float2>((size_t)D.rope_slots * (D.hd / 2));
+  L.bytes = cv.off + 256;
+}
+
+// Prefill staging lives after the layout: bytes and per-sequence offsets.
+struct Staging {
+  uint8_t* bytes;
+  int* row0;
+  int* lens;
+  int* lm_row0;
+};
+
+}  // namespace
+
+struct lca_ctx {
+  lca_config cfg{};
+  Layout L;
+  Staging stg{};
+  char* ws = nullptr;
+  size_t ws_bytes = 0;
+  cudaStream_t stream = nullptr;
+  cudaStream_t cap = nullptr, cap2 = nullptr;
+  Params* h_params = nullptr;  // pinned ring
+  int param_slot = 0;
+  Params host_params{};
+  int batch = 0;
+  bool prefilled = false;
+  std::vector<long long> t_host;
+  std::map<int, cudaGraphExec_t> step_exec, gen_exec;
+  std::vector<cudaGraph_t> graphs;
+  int last_n = 0;
+  int pending_force_accept = 0;
+  int pending_force_cand = 0;
+  int pending_force_cand_n = 0;
+  int gen_max_new = 0;
+  int gen_n = 0;
+  bool t_unsynced = false;
+  // kernels per step graph part, by n: [pre-LM + post-LM, LM body]
+  std::map<int, std::pair<long long, long long>> launches;
+};
+
+namespace {
+
+int check(cudaError_t e, const char* what) {
+  if (e != cudaSuccess) {
+    fprintf(stderr, "lca: %s: %s\n", what, cudaGetErrorString(e));
+    return LCA_E_CUDA;
+  }
+  return LCA_OK;
+}
+#define CK(x)                                   \
+  do {                                          \
+    int _s = check((x), #x);                    \
+    if (_s != LCA_OK) return _s;                \
+  } while (0)
+
+int validate(const lca_config* c) {
+  if (!c) return LCA_E_ARG;
+  if (c->vocab != 256 || c->d_model <= 0 || c->n_heads <= 0 || c->head_dim <= 0) return LCA_E_ARG;
+  if (c->n_heads * c->head_dim != c->d_model) return LCA_E_ARG;
+  if (c->head_dim != 32 && c->head_dim != 64) return LCA_E_ARG;
+  if (c->d_model % 16 || c->d_ff % 16) return LCA_E_ARG;
+  if (c->dtype != LCA_F32 && c->dtype != LCA_BF16) return LCA_E_ARG;
+  if (c->mb_kind != LCA_MB_LCA && c->mb_kind != LCA_MB_MLP) return LCA_E_ARG;
+  if (c->max_batch < 1 || c->max_batch > 1024 || c->max_bytes < 2 || c->max_n < 1 || c->max_n > kMaxN)
+    return LCA_E_ARG;
+  if (c->mb_kind == LCA_MB_MLP && c->n_mlp_heads < c->max_n - 1) return LCA_E_ARG;
+  if (c->n_enc < 0 || c->n_lm < 0 || c->n_nb < 0 || c->n_mb < 0) return LCA_E_ARG;
+  if (c->boundary_byte < 0 || c->boundary_byte > 255) return LCA_E_ARG;
+  return LCA_OK;
+}
+
+Params* next_params(lca_ctx* c) {
+  c->param_slot = (c->param_slot + 1) % kParamSlots;
+  Params* hp = c->h_params + c->param_slot;
+  *hp = c->host_params;
+  return hp;
+}
+
+int upload_params(lca_ctx* c) {
+  Params* hp = next_params(c);
+  CK(cudaMemcpyAsync(c->L.D.params, hp, sizeof(Params), cudaMemcpyHostToDevice, c->stream));
+  return LCA_OK;
+}
+
+bool tiled_for(int rows) { return rows > 64; }
+
+int attn_splits(const Dev& D, int batch_cap, int qtiles) {
+  int s = (2 * 152) / std::max(1, batch_cap * D.H * qtiles);
+  return std::max(1, std::min(s, kMaxAttnSplit));
+}
+
+// Run the pre-norm blocks of one module over rows [0, *rows.M) of x (in place).
+void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& rows, int M_cap,
+               int M_typ, int qt_grid, int splits, cudaStream_t s) {
+  Dev& D = c->L.D;
+  const bool tiled = tiled_for(M_typ);
+  for (auto& bk : blocks) {
+    LinearArgs a{};
+    a.groups = 1;
+    a.Mg_stride = 0;
+    a.eps = D.eps;
+    a.M = rows.M;
+    a.M_cap = M_cap;
+    // RMSNorm -> Q,K,V -> RoPE -> K,V appended to the cache
+    a.x = x;
+    a.ldx = D.d;
+    a.W = bk.wqkv;
+    a.N = 3 * D.d;
+    a.Kd = D.d;
+    a.norm = bk.attn_norm;
+    a.epi = EpiArgs{};
+    a.epi.mode = EPI_QKV;
+    a.epi.y = D.qbuf;
+    a.epi.ldy = D.d;
+    a.epi.kv = bk.kv;
+    a.epi.rows = rows;
+    a.epi.rope = D.rope;
+    a.epi.H = D.H;
+    a.epi.hd = D.hd;
+    a.epi.d = D.d;
+    a.epi.err = D.err;
+    linear(D, a, tiled, s);
+    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s);
+    // x += Wo . attn
+    a.x = D.att;
+    a.W = bk.wo;
+    a.N = D.d;
+    a.norm = nullptr;
+    a.epi.mode = EPI_RESID;
+    a.epi.y = x;
+    a.epi.res = x;
+    a.epi.ldy = a.epi.ldres = D.d;
+    linear(D, a, tiled, s);
+    // mid = silu(W1 . n(x)) * (W3 . n(x))
+    a.x = x;
+    a.W = bk.w13;
+    a.N = 2 * D.F;
+    a.norm = bk.mlp_norm;
+    a.epi.mode = EPI_SWIGLU;
+    a.epi.y = D.mid;
+    a.epi.ldy = D.F;
+    linear(D, a, tiled, s);
+    // x += W2 . mid
+    a.x = D.mid;
+    a.ldx = D.F;
+    a.W = bk.w2;
+    a.N = D.d;
+    a.Kd = D.F;
+    a.norm = nullptr;
+    a.epi.mode = EPI_RESID;
+    a.epi.y = x;
+    a.epi.res = x;
+    a.epi.ldy = a.epi.ldres = D.d;
+    linear(D, a, tiled, s);
+  }
+}
+
+// MLP-MBP drafter layers: v <- v + silu(W_{j,l} v) for every head j (grouped over heads).
+void run_mlp_heads(lca_ctx* c, int n, cudaStream_t s) {
+  Dev& D = c->L.D;
+  const size_t tb = tw_bytes(D.dtype);
+  for (int l = 0; l < D.n_mb; ++l) {
+    LinearArgs a{};
+    a.x = D.x_mb;
+    a.ldx = D.d;
+    a.W = reinterpret_cast<char*>(D.mlp_w) + (size_t)l * D.n_mlp_heads * D.d * D.d * tb;
+    a.N = D.d;
+    a.Kd = D.d;
+    a.groups = n - 1;
+    a.Mg_stride = D.B;
+    a.norm = nullptr;
+    a.eps = D.eps;
+    a.M = D.r_mb.M;
+    a.M_cap = D.B;
+    a.epi.mode = EPI_RESID_SILU;
+    a.epi.y = D.x_mb;
+    a.epi.res = D.x_mb;
+    a.epi.ldy = a.epi.ldres = D.d;
+    a.epi.err = D.err;
+    linear(D, a, tiled_for(D.B), s);
+  }
+}
+
+// Capture one decode step into graph g (which may be the body of a WHILE node).
+int capture_step(lca_ctx* c, cudaGraph_t g, int n, bool loop, cudaGraphConditionalHandle hwhile) {
+  Dev& D = c->L.D;
+  cudaStream_t s = c->cap;
+  CK(cudaStreamBeginCaptureToGraph(s, g, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+  const long long l0 = g_launches;
+  long long lm_launches = 0;
+  const int B = D.B;
+  // (3) draft
+  if (n >= 2) {
+    if (D.mb_kind == LCA_MB_LCA) {
+      launch_mb_plan(D, s);
+      launch_mb_fill(D, s);
+      const int typ = B * (2 * n);
+      run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2), s);  // window rows
+    } else {
+      launch_mlp_plan(D, s);
+      run_mlp_heads(c, n, s);
+    }
+    launch_head(D, D.x_mb, D.head_rows_mb, D.M_head_mb, B * (n - 1), D.mb_norm, D.mb_logits,
+                D.mb_arg, D.mb_prob, s);
+  }
+  // (1) embed + encoder over the n candidates
+  launch_verify_plan(D, s);
+  const int vs = attn_splits(D, B, 1);
+  run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, vs, s);
+  // segments closed by candidate boundaries -> LM rows; conditional on any
+  cudaStreamCaptureStatus st;
+  cudaGraph_t cg;
+  const cudaGraphNode_t* deps = nullptr;
+  const cudaGraphEdgeData* edata = nullptr;
+  size_t ndeps = 0;
+  CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &cg, nullptr, nullptr, nullptr));
+  cudaGraphConditionalHandle hlm;
+  CK(cudaGraphConditionalHandleCreate(&hlm, cg, 0, cudaGraphCondAssignDefault));
+  launch_segment(D, hlm, 1, s);
+  CK(cudaStreamGetCaptureInfo(s, &st, nullptr, &cg, &deps, &edata, &ndeps));
+  cudaGraphNodeParams cp{};
+  cp.type = cudaGraphNodeTypeConditional;
+  cp.conditional.handle = hlm;
+  cp.conditional.type = cudaGraphCondTypeIf;
+  cp.conditional.size = 1;
+  cudaGraphNode_t cnode;
+  CK(cudaGraphAddNode(&cnode, cg, deps, edata, ndeps, &cp));
+  cudaGraph_t body = cp.conditional.phGraph_out[0];
+  {
+    cudaStream_t s2 = c->cap2;
+    CK(cudaStreamBeginCaptureToGraph(s2, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+    // about one new latent per sequence every few bytes
+    const long long b0 = g_launches;
+    run_stack(c, c->L.lm, D.x_lm, D.r_lm, B * n, B, 1, vs, s2);
+    launch_lm_scatter(D, s2);
+    lm_launches = g_launches - b0;
+    cudaGraph_t tmp;
+    CK(cudaStreamEndCapture(s2, &tmp));
+  }
+  CK(cudaStreamUpdateCaptureDependencies(s, &cnode, nullptr, 1, cudaStreamSetCaptureDependencies));
+  // (4) upsample + next-byte decoder over the n candidates, head
+  launch_nb_input(D, s);
+  run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, vs, s);
+  launch_head(D, D.x_nb, nullptr, D.r_v.M, B * n, D.nb_norm, D.nb_logits, D.nb_arg, D.nb_prob, s);
+  // (5) accept + commit
+  launch_commit(D, s);
+  if (loop) launch_loop_ctl(D, hwhile, s);
+  cudaGraph_t out;
+  CK(cudaStreamEndCapture(s, &out));
+  if (!loop) c->launches[n] = {g_launches - l0 - lm_launches, lm_launches};
+  return LCA_OK;
+}
+
+int get_step_exec(lca_ctx* c, int n, cudaGraphExec_t* ex) {
+  auto it = c->step_exec.find(n);
+  if (it != c->step_exec.end()) {
+    *ex = it->second;
+    return LCA_OK;
+  }
+  cudaGraph_t g;
+  CK(cudaGraphCreate(&g, 0));
+  int st = capture_step(c, g, n, false, 0);
+  if (st != LCA_OK) return st;
+  cudaGraphExec_t e;
+  CK(cudaGraphInstantiate(&e, g, 0));
+  c->graphs.push_back(g);
+  c->step_exec[n] = e;
+  *ex = e;
+  return LCA_OK;
+}
+
+int get_gen_exec(lca_ctx* c, int n, cudaGraphExec_t* ex) {
+  auto it = c->gen_exec.find(n);
+  if (it != c->gen_exec.end()) {
+    *ex = it->second;
+    return LCA_OK;
+  }
+  cudaGraph_t g;
+  CK(cudaGraphCreate(&g, 0));
+  cudaGraphConditionalHandle hw;
+  CK(cudaGraphConditionalHandleCreate(&hw, g, 1, cudaGraphCondAssignDefault));
+  cudaGraphNodeParams cp{};
+  cp.type = cudaGraphNodeTypeConditional;
+  cp.conditional.handle = hw;
+  cp.conditional.type = cudaGraphCondTypeWhile;
+  cp.conditional.size = 1;
+  cudaGraphNode_t node;
+  CK(cudaGraphAddNode(&node, g, nullptr, nullptr, 0, &cp));
+  int st = capture_step(c, cp.conditional.phGraph_out[0], n, true, hw);
+  if (st != LCA_OK) return st;
+  cudaGraphExec_t e;
+  CK(cudaGraphInstantiate(&e, g, 0));
+  c->graphs.push_back(g);
+  c->gen_exec[n] = e;
+  *ex = e;
+  return LCA_OK;
+}
+
+int read_err(lca_ctx* c) {
+  int e = 0;
+  CK(cudaMemcpyAsync(&e, c->L.D.err, sizeof(int), cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  if (e) {
+    CK(cudaMemsetAsync(c->L.D.err, 0, sizeof(int), c->stream));
+    CK(cudaStreamSynchronize(c->stream));
+  }
+  if (e & kErrNumeric) return LCA_E_NUMERIC;
+  if (e & kErrIndex) return LCA_E_DEVICE_STATE;
+  return LCA_OK;
+}
+
+struct WeightSpec {
+  const void* ptr = nullptr;
+  int64_t numel = 0;
+  int dtype = 0;
+};
+
+int find_w(const std::map<std::string, WeightSpec>& m, const std::string& name, int64_t numel,
+           int dtype, const void** out) {
+  auto it = m.find(name);
+  if (it == m.end() || !it->second.ptr) {
+    fprintf(stderr, "lca: missing weight %s\n", name.c_str());
+    return LCA_E_WEIGHTS;
+  }
+  if (it->second.numel != numel || it->second.dtype != dtype) {
+    fprintf(stderr, "lca: weight %s has numel %lld dtype %d, expected %lld dtype %d\n", name.c_str(),
+            (long long)it->second.numel, it->second.dtype, (long long)numel, dtype);
+    return LCA_E_WEIGHTS;
+  }
+  *out = it->second.ptr;
+  return LCA_OK;
+}
+
+int load_weights(lca_ctx* c, const lca_tensor* w, int nw) {
+  std::map<std::string, WeightSpec> m;
+  for (int i = 0; i < nw; ++i) {
+    if (!w[i].name) return LCA_E_ARG;
+    m[w[i].name] = WeightSpec{w[i].ptr, w[i].numel, w[i].dtype};
+  }
+  Dev& D = c->L.D;
+  const int dt = c->cfg.dtype;
+  const size_t tb = tw_bytes(dt);
+  const int64_t d = D.d, F = D.F;
+  cudaStream_t s = c->stream;
+  const void* p;
+  auto copy = [&](void* dst, const std::string& name, int64_t numel, int dtype) -> int {
+    int st = find_w(m, name, numel, dtype, &p);
+    if (st != LCA_OK) return st;
+    CK(cudaMemcpyAsync(dst, p, numel * (dtype == LCA_BF16 ? 2 : 4), cudaMemcpyDeviceToDevice, s));
+    return LCA_OK;
+  };
+#define TRY(x)                       \
+  do {                               \
+    int _s = (x);                    \
+    if (_s != LCA_OK) return _s;     \
+  } while (0)
+  TRY(copy(D.embed, "embed", 256 * d, dt));
+  TRY(copy(D.unembed, "unembed", 256 * d, dt));
+  TRY(copy((void*)D.bos, "lm.bos", d, LCA_F32));
+  TRY(copy((void*)D.nb_norm, "nb.norm", d, LCA_F32));
+  TRY(copy((void*)D.mb_norm, "mb.norm", d, LCA_F32));
+  auto stack = [&](std::vector<Block>& v, const char* pre) -> int {
+    for (size_t l = 0; l < v.size(); ++l) {
+      const std::string b = std::string(pre) + "." + std::to_string(l) + ".";
+      Block& bk = v[l];
+      TRY(copy((void*)bk.attn_norm, b + "attn_norm", d, LCA_F32));
+      TRY(copy((void*)bk.mlp_norm, b + "mlp_norm", d, LCA_F32));
+      TRY(copy((char*)bk.wqkv, b + "wq", d * d, dt));
+      TRY(copy((char*)bk.wqkv + d * d * tb, b + "wk", d * d, dt));
+      TRY(copy((char*)bk.wqkv + 2 * d * d * tb, b + "wv", d * d, dt));
+      TRY(copy(bk.wo, b + "wo", d * d, dt));
+      TRY(copy(bk.w2, b + "w2", d * F, dt));
+      // interleave W1 and W3 rows: packed row 2j = W1_j, 2j+1 = W3_j
+      TRY(find_w(m, b + "w1", F * d, dt, &p));
+      launch_pack_rows(bk.w13, p, (int)F, (int)d, 0, 2, (int)tb, s);
+      TRY(find_w(m, b + "w3", F * d, dt, &p));
+      launch_pack_rows(bk.w13, p, (int)F, (int)d, 1, 2, (int)tb, s);
+    }
+    return LCA_OK;
+  };
+  TRY(stack(c->L.enc, "enc"));
+  TRY(stack(c->L.lm, "lm"));
+  TRY(stack(c->L.nb, "nb"));
+  if (D.mb_kind == LCA_MB_LCA) {
+    TRY(stack(c->L.mb, "mb"));
+  } else {
+    for (int l = 0; l < D.n_mb; ++l)
+      for (int j = 0; j < D.n_mlp_heads; ++j)
+        TRY(copy((char*)D.mlp_w + ((size_t)l * D.n_mlp_heads + j) * d * d * tb,
+                 "mlp." + std::to_string(j) + "." + std::to_string(l) + ".w", d * d, dt));
+  }
+#undef TRY
+  CK(cudaGetLastError());
+  return LCA_OK;
+}
+
+}  // namespace
+
+// ============================================================================ C ABI
+extern "C" {
+
+const char* lca_status_str(int s) {
+  switch (s) {
+    case LCA_OK: return "ok";
+    case LCA_E_ARG: return "bad argument";
+    case LCA_E_CAPACITY: return "capacity exceeded";
+    case LCA_E_WEIGHTS: return "missing or malformed weights";
+    case LCA_E_CUDA: return "CUDA error";
+    case LCA_E_DEVICE_STATE: return "device index out of range";
+    case LCA_E_NUMERIC: return "non-finite logits";
+    case LCA_E_TIMEOUT: return "device wait timed out";
+    case LCA_E_STATE: return "call out of order";
+    default: return "unknown status";
+  }
+}
+
+static size_t staging_bytes(const lca_config* c) {
+  return ((size_t)c->max_batch * c->max_bytes + 255) / 256 * 256 + 4 * 256 +
+         3 * (((size_t)c->max_batch * sizeof(int) + 255) / 256 * 256);
+}
+
+int lca_workspace_bytes(const lca_config* cfg, size_t* out) {
+  int st = validate(cfg);
+  if (st != LCA_OK) return st;
+  if (!out) return LCA_E_ARG;
+  Layout L;
+  carve(*cfg, nullptr, L);
+  *out = L.bytes + staging_bytes(cfg);
+  return LCA_OK;
+}
+
+int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, void* workspace,
+               size_t workspace_bytes, void* stream, lca_ctx** out) {
+  int st = validate(cfg);
+  if (st != LCA_OK) return st;
+  if (!out || !workspace || !weights || n_weights <= 0) return LCA_E_ARG;
+  if (reinterpret_cast<uintptr_t>(workspace) % 256) return LCA_E_ARG;
+  size_t need = 0;
+  lca_workspace_bytes(cfg, &need);
+  if (workspace_bytes < need) return LCA_E_CAPACITY;
+  lca_ctx* c = new lca_ctx();
+  c->cfg = *cfg;
+  c->ws = reinterpret_cast<char*>(workspace);
+  c->ws_bytes = workspace_bytes;
+  c->stream = reinterpret_cast<cudaStream_t>(stream);
+  carve(*cfg, c->ws, c->L);
+  {
+    char* sb = c->ws + c->L.bytes;
+    sb = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(sb) + 255) & ~uintptr_t(255));
+    c->stg.bytes = reinterpret_cast<uint8_t*>(sb);
+    sb += ((size_t)cfg->max_batch * cfg->max_bytes + 255) / 256 * 256 + 256;
+    const size_t ib = ((size_t)cfg->max_batch * sizeof(int) + 255) / 256 * 256;
+    c->stg.row0 = reinterpret_cast<int*>(sb);
+    c->stg.lens = reinterpret_cast<int*>(sb + ib);
+    c->stg.lm_row0 = reinterpret_cast<int*>(sb + 2 * ib);
+  }
+  auto fail = [&](int s) {
+    lca_destroy(c);
+    return s;
+  };
+  if (check(cudaStreamCreateWithFlags(&c->cap, cudaStreamNonBlocking), "stream") ||
+      check(cudaStreamCreateWithFlags(&c->cap2, cudaStreamNonBlocking), "stream") ||
+      check(cudaMallocHost(&c->h_params, sizeof(Params) * kParamSlots), "host params"))
+    return fail(LCA_E_CUDA);
+  kernel_attrs_linear();
+  kernel_attrs_step();
+  Dev& D = c->L.D;
+  // state and counters start at zero
+  if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);
+  st = load_weights(c, weights, n_weights);
+  if (st != LCA_OK) return fail(st);
+  launch_rope_table(D, cfg->rope_base, c->stream);
+  if (check(cudaGetLastError(), "rope") || check(cudaStreamSynchronize(c->stream), "create sync"))
+    return fail(LCA_E_CUDA);
+  c->host_params = Params{};
+  *out = c;
+  return LCA_OK;
+}
+
+int lca_destroy(lca_ctx* c) {
+  if (!c) return LCA_E_ARG;
+  if (c->stream) cudaStreamSynchronize(c->stream);
+  for (auto& kv : c->step_exec) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : c->gen_exec) cudaGraphExecDestroy(kv.second);
+  for (auto g : c->graphs) cudaGraphDestroy(g);
+  if (c->cap) cudaStreamDestroy(c->cap);
+  if (c->cap2) cudaStreamDestroy(c->cap2);
+  if (c->h_params) cudaFreeHost(c->h_params);
+  delete c;
+  return LCA_OK;
+}
+
+int lca_prefill(lca_ctx* c, int32_t batch, const uint8_t* const* prompts, const int32_t* lens) {
+  if (!c || !prompts || !lens) return LCA_E_ARG;
+  if (batch < 1 || batch > c->cfg.max_batch) return LCA_E_CAPACITY;
+  Dev& D = c->L.D;
+  cudaStream_t s = c->stream;
+  std::vector<int> row0(batch), lm_row0(batch), K(batch);
+  int M = 0, Mlm = 0, maxK = 0, maxlen = 0;
+  for (int b = 0; b < batch; ++b) {
+    if (!prompts[b] || lens[b] < 1) return LCA_E_ARG;
+    if (lens[b] + c->cfg.max_n > c->cfg.max_bytes) return LCA_E_CAPACITY;
+    row0[b] = M;
+    M += lens[b];
+    maxlen = std::max(maxlen, lens[b]);
+    int k = 0;
+    for (int p = 0; p < lens[b]; ++p) k += prompts[b][p] == c->cfg.boundary_byte;
+    K[b] = k;
+    maxK = std::max(maxK, k);
+    lm_row0[b] = Mlm;
+    Mlm += k + 1;
+  }
+  // host-built row descriptors (prompt structure is host data)
+  std::vector<int> rb(M), rp(M), rs(M), rk(M), ss(D.B, M), sc(D.B, 0);
+  std::vector<int> lb(Mlm), lp(Mlm), ls(D.B, Mlm), lc(D.B, 0);
+  std::vector<uint8_t> bytes(M);
+  for (int b = 0; b < batch; ++b) {
+    ss[b] = row0[b];
+    sc[b] = lens[b];
+    for (int p = 0; p < lens[b]; ++p) {
+      const int r = row0[b] + p;
+      rb[r] = b;
+      rp[r] = p;
+      bytes[r] = prompts[b][p];
+    }
+    ls[b] = lm_row0[b];
+    lc[b] = K[b] + 1;
+    for (int k = 0; k <= K[b]; ++k) {
+      lb[lm_row0[b] + k] = b;
+      lp[lm_row0[b] + k] = k;
+    }
+  }
+  std::vector<int> kv1(M), lkv1(Mlm);
+  for (int r = 0; r < M; ++r) kv1[r] = rp[r] + 1;
+  for (int r = 0; r < Mlm; ++r) lkv1[r] = lp[r] + 1;
+  std::vector<int> last(batch);
+  for (int b = 0; b < batch; ++b) last[b] = row0[b] + lens[b] - 1;
+  auto up = [&](void* dst, const void* src, size_t n) {
+    return check(cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s), "prefill upload");
+  };
+  if (up(c->stg.bytes, bytes.data(), M) || up(c->stg.row0, row0.data(), batch * 4) ||
+      up(c->stg.lens, lens, batch * 4) || up(c->stg.lm_row0, lm_row0.data(), batch * 4) ||
+      up(D.r_v.b, rb.data(), M * 4) || up(D.r_v.pos, rp.data(), M * 4) ||
+      up(D.r_v.slot, rp.data(), M * 4) || up(D.r_v.kvlen, kv1.data(), M * 4) ||
+      up(D.r_v.seq_start, ss.data(), D.B * 4) || up(D.r_v.seq_count, sc.data(), D.B * 4) ||
+      up(D.r_v.M, &M, 4) || up(D.r_lm.b, lb.data(), Mlm * 4) || up(D.r_lm.pos, lp.data(), Mlm * 4) ||
+      up(D.r_lm.slot, lp.data(), Mlm * 4) || up(D.r_lm.kvlen, lkv1.data(), Mlm * 4) ||
+      up(D.r_lm.seq_start, ls.data(), D.B * 4) || up(D.r_lm.seq_count, lc.data(), D.B * 4) ||
+      up(D.r_lm.M, &Mlm, 4) || up(D.head_rows_v, last.data(), batch * 4) || up(D.M_head_v, &batch, 4))
+    return LCA_E_CUDA;
+  // inactive sequences
+  {
+    std::vector<SeqState> zs(D.B);
+    for (auto& z : zs) memset(&z, 0, sizeof(z));
+    if (up(D.seq, zs.data(), sizeof(SeqState) * D.B)) return LCA_E_CUDA;
+  }
+  const int qt = std::min(64, (maxlen + kAttnQT - 1) / kAttnQT);
+  launch_prefill_embed(D, c->stg.bytes, M, s);
+  run_stack(c, c->L.enc, D.x_enc, D.r_v, M, M, qt, 1, s);
+  launch_prefill_segment(D, c->stg.bytes, c->stg.row0, c->stg.lens, batch, c->stg.lm_row0, s);
+  launch_prefill_pool(D, c->stg.row0, c->stg.lens, c->stg.lm_row0, batch, maxK, s);
+  const int lqt = std::min(64, (maxK + 1 + kAttnQT - 1) / kAttnQT);
+  run_stack(c, c->L.lm, D.x_lm, D.r_lm, Mlm, Mlm, lqt, 1, s);
+  launch_lm_scatter(D, s);
+  launch_prefill_nb_input(D, M, s);
+  run_stack(c, c->L.nb, D.x_nb, D.r_v, M, M, qt, 1, s);
+  launch_head(D, D.x_nb, D.head_rows_v, D.M_head_v, batch, D.nb_norm, D.nb_logits, D.nb_arg,
+              D.nb_prob, s);
+  launch_prefill_finish(D, c->stg.row0, c->stg.lens, c->stg.lm_row0, batch, s);
+  CK(cudaGetLastError());
+  c->batch = batch;
+  c->prefilled = true;
+  c->t_host.assign(batch, 0);
+  for (int b = 0; b < batch; ++b) c->t_host[b] = lens[b];
+  c->host_params.batch = batch;
+  c->pending_force_accept = c->pending_force_cand = 0;
+  int e = read_err(c);
+  return e;
+}
+
+static int step_prep(lca_ctx* c, int n, float tau, int mode) {
+  if (!c) return LCA_E_ARG;
+  if (!c->prefilled) return LCA_E_STATE;
+  if (n < 1 || n > c->cfg.max_n) return LCA_E_CAPACITY;
+  if (mode != LCA_THRESH && mode != LCA_SPEC) return LCA_E_ARG;
+  if (tau != tau) return LCA_E_ARG;
+  Params& P = c->host_params;
+  P.n = n;
+  P.tau = tau;
+  P.accept = mode;
+  P.batch = c->batch;
+  return LCA_OK;
+}
+
+int lca_mbp_step(lca_ctx* c, int32_t n, float tau, int32_t mode, uint8_t* out_bytes,
+                 int32_t* out_counts) {
+  int st = step_prep(c, n, tau, mode);
+  if (st != LCA_OK) return st;
+  for (int b = 0; b < c->batch; ++b)
+    if (c->t_host[b] + n > c->cfg.max_bytes) return LCA_E_CAPACITY;
+  if (c->pending_force_cand && c->pending_force_cand_n != n) return LCA_E_ARG;
+  cudaGraphExec_t ex;
+  st = get_step_exec(c, n, &ex);
+  if (st != LCA_OK) return st;
+  Params& P = c->host_params;
+  P.gen = 0;
+  P.force_accept = c->pending_force_accept;
+  P.force_cand = c->pending_force_cand;
+  st = upload_params(c);
+  if (st != LCA_OK) return st;
+  c->pending_force_accept = c->pending_force_cand = 0;
+  CK(cudaGraphLaunch(ex, c->stream));
+  std::vector<int> cnt(c->batch);
+  CK(cudaMemcpyAsync(cnt.data(), c->L.D.out_cnt, c->batch * sizeof(int), cudaMemcpyDeviceToHost,
+                     c->stream));
+  if (out_bytes)
+    CK(cudaMemcpy2DAsync(out_bytes, n, c->L.D.out_step, c->L.D.NMAX, n, c->batch,
+                         cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  c->last_n = n;
+  for (int b = 0; b < c->batch; ++b) c->t_host[b] += cnt[b];
+  if (out_counts) memcpy(out_counts, cnt.data(), c->batch * sizeof(int));
+  return read_err(c);
+}
+
+int lca_mbp_step_async(lca_ctx* c, int32_t n, float tau, int32_t mode) {
+  int st = step_prep(c, n, tau, mode);
+  if (st != LCA_OK) return st;
+  for (int b = 0; b < c->batch; ++b)
+    if (c->t_host[b] + n > c->cfg.max_bytes) return LCA_E_CAPACITY;
+  if (c->pending_force_cand && c->pending_force_cand_n != n) return LCA_E_ARG;
+  cudaGraphExec_t ex;
+  st = get_step_exec(c, n, &ex);
+  if (st != LCA_OK) return st;
+  Params& P = c->host_params;
+  P.gen = 0;
+  P.force_accept = c->pending_force_accept;
+  P.force_cand = c->pending_force_cand;
+  st = upload_params(c);
+  if (st != LCA_OK) return st;
+  c->pending_force_accept = c->pending_force_cand = 0;
+  CK(cudaGraphLaunch(ex, c->stream));
+  c->last_n = n;
+  for (int b = 0; b < c->batch; ++b) c->t_host[b] += n;  // upper bound until synced
+  c->t_unsynced = true;
+  return LCA_OK;
+}
+
+int lca_generate_async(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t max_new) {
+  int st = step_prep(c, n, tau, mode);
+  if (st != LCA_OK) return st;
+  if (max_new < 1) return LCA_E_ARG;
+  for (int b = 0; b < c->batch; ++b)
+    if (c->t_host[b] + max_new + n > c->cfg.max_bytes) return LCA_E_CAPACITY;
+  cudaGraphExec_t ex;
+  st = get_gen_exec(c, n, &ex);
+  if (st != LCA_OK) return st;
+  Params& P = c->host_params;
+  P.gen = 1;
+  P.force_accept = 0;
+  P.force_cand = 0;
+  P.iter = 0;
+  P.max_iter = max_new;
+  st = upload_params(c);
+  if (st != LCA_OK) return st;
+  launch_gen_init(c->L.D, max_new, c->stream);
+  CK(cudaGetLastError());
+  CK(cudaGraphLaunch(ex, c->stream));
+  c->gen_max_new = max_new;
+  c->gen_n = n;
+  c->last_n = n;
+  for (int b = 0; b < c->batch; ++b) c->t_host[b] += max_new;
+  return LCA_OK;
+}
+
+int lca_generate_fetch(lca_ctx* c, uint8_t* out, int32_t* out_len, int32_t* hist) {
+  if (!c) return LCA_E_ARG;
+  if (!c->gen_max_new) return LCA_E_STATE;
+  Dev& D = c->L.D;
+  const int mx = c->gen_max_new;
+  if (out)
+    CK(cudaMemcpy2DAsync(out, mx, D.out_gen, D.S, mx, c->batch, cudaMemcpyDeviceToHost, c->stream));
+  std::vector<SeqState> ss(c->batch);
+  CK(cudaMemcpyAsync(ss.data(), D.seq, sizeof(SeqState) * c->batch, cudaMemcpyDeviceToHost, c->stream));
+  std::vector<int> h(D.NMAX);
+  CK(cudaMemcpyAsync(h.data(), D.hist, sizeof(int) * D.NMAX, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  int st = LCA_OK;
+  for (int b = 0; b < c->batch; ++b) {
+    if (out_len) out_len[b] = ss[b].generated;
+    if (ss[b].generated != mx) st = LCA_E_DEVICE_STATE;
+  }
+  if (hist) memcpy(hist, h.data(), sizeof(int) * c->gen_n);
+  int e = read_err(c);
+  return e != LCA_OK ? e : st;
+}
+
+int lca_generate(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t max_new, uint8_t* out,
+                 int32_t* out_len, int32_t* hist) {
+  int st = lca_generate_async(c, n, tau, mode, max_new);
+  if (st != LCA_OK) return st;
+  return lca_generate_fetch(c, out, out_len, hist);
+}
+
+int lca_debug_state(lca_ctx* c, int32_t b, lca_seq_state* out) {
+  if (!c || !out) return LCA_E_ARG;
+  if (!c->prefilled) return LCA_E_STATE;
+  if (b < 0 || b >= c->batch) return LCA_E_ARG;
+  Dev& D = c->L.D;
+  SeqState s;
+  CK(cudaMemcpyAsync(&s, D.seq + b, sizeof(s), cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  if (c->t_unsynced) {
+    std::vector<SeqState> all(c->batch);
+    CK(cudaMemcpy(all.data(), D.seq, sizeof(SeqState) * c->batch, cudaMemcpyDeviceToHost));
+    for (int i = 0; i < c->batch; ++i) c->t_host[i] = all[i].t;
+    c->t_unsynced = false;
+  }
+  int g[2] = {-1, 0};
+  if (s.K >= 1)
+    CK(cudaMemcpyAsync(&g[0], D.gstart + (size_t)b * D.L + s.K - 1, 4, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaMemcpyAsync(&g[1], D.gstart + (size_t)b * D.L + s.K, 4, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  out->t = s.t;
+  out->K = s.K;
+  out->open_start = s.open_start;
+  out->prev_group_start = g[0];
+  out->group_start = g[1];
+  out->next_byte = s.next_c1;
+  out->generated = s.generated;
+  out->pad = 0;
+  return LCA_OK;
+}
+
+int lca_debug_logits(lca_ctx* c, float* nb, float* mb) {
+  if (!c) return LCA_E_ARG;
+  if (!c->last_n) return LCA_E_STATE;
+  const int n = c->last_n;
+  Dev& D = c->L.D;
+  if (nb)
+    CK(cudaMemcpyAsync(nb, D.nb_logits, sizeof(float) * 256 * c->batch * n, cudaMemcpyDeviceToHost,
+                       c->stream));
+  if (mb && n >= 2)
+    CK(cudaMemcpyAsync(mb, D.mb_logits, sizeof(float) * 256 * c->batch * (n - 1),
+                       cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  return LCA_OK;
+}
+
+int lca_debug_stats(lca_ctx* c, lca_stats* out) {
+  if (!c || !out) return LCA_E_ARG;
+  Stats s;
+  CK(cudaMemcpyAsync(&s, c->L.D.stats, sizeof(s), cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  out->steps = (int64_t)s.steps;
+  out->lm_steps = (int64_t)s.lm_steps;
+  out->lm_rows = (int64_t)s.lm_rows;
+  out->mb_rows = (int64_t)s.mb_rows;
+  out->committed = (int64_t)s.committed;
+  auto it = c->launches.find(c->last_n);
+  out->kernels_per_step = it == c->launches.end() ? 0 : it->second.first;
+  out->kernels_per_lm_run = it == c->launches.end() ? 0 : it->second.second;
+  out->workspace_bytes = (int64_t)c->ws_bytes;
+  return LCA_OK;
+}
+
+int lca_debug_force_accept(lca_ctx* c, const int32_t* a) {
+  if (!c) return LCA_E_ARG;
+  if (!c->prefilled) return LCA_E_STATE;
+  if (!a) {
+    c->pending_force_accept = 0;
+    return LCA_OK;
+  }
+  CK(cudaMemcpyAsync(c->L.D.forced_a, a, sizeof(int) * c->batch, cudaMemcpyHostToDevice, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  c->pending_force_accept = 1;
+  return LCA_OK;
+}
+
+int lca_debug_force_candidates(lca_ctx* c, const uint8_t* cand, int32_t n) {
+  if (!c) return LCA_E_ARG;
+  if (!c->prefilled) return LCA_E_STATE;
+  if (!cand) {
+    c->pending_force_cand = 0;
+    return LCA_OK;
+  }
+  if (n < 1 || n > c->cfg.max_n) return LCA_E_CAPACITY;
+  Dev& D = c->L.D;
+  std::vector<int> v((size_t)D.B * D.NMAX, 0);
+  for (int b = 0; b < c->batch; ++b)
+    for (int i = 0; i < n; ++i) v[(size_t)b * D.NMAX + i] = cand[(size_t)b * n + i];
+  CK(cudaMemcpyAsync(D.forced_cand, v.data(), sizeof(int) * v.size(), cudaMemcpyHostToDevice, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  c->pending_force_cand = 1;
+  c->pending_force_cand_n = n;
+  return LCA_OK;
+}
+
+}  // extern "C"

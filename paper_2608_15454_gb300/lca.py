@@ -1,0 +1,242 @@
+"""Thin ctypes binding of ``include/lca.h``: argument marshalling only.
+
+Every step of the decode path runs in the CUDA library ``liblca.so``; torch provides the
+device memory (workspace, weights) and the stream. There is no CPU fallback: if the
+library is missing, loading raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "liblca.so")
+
+LCA_OK = 0
+LCA_F32, LCA_BF16 = 0, 1
+LCA_MB_LCA, LCA_MB_MLP = 0, 1
+LCA_THRESH, LCA_SPEC = 0, 1
+
+STATUS = {0: "LCA_OK", -1: "LCA_E_ARG", -2: "LCA_E_CAPACITY", -3: "LCA_E_WEIGHTS", -4: "LCA_E_CUDA",
+          -5: "LCA_E_DEVICE_STATE", -6: "LCA_E_NUMERIC", -7: "LCA_E_TIMEOUT", -8: "LCA_E_STATE"}
+
+EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "lca_mbp_step_async",
+           "lca_generate",
+           "lca_generate_async", "lca_generate_fetch", "lca_debug_state", "lca_debug_stats",
+           "lca_debug_logits",
+           "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str")
+
+
+class LcaConfig(ctypes.Structure):
+    _fields_ = [("d_model", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("d_ff", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("n_enc", ctypes.c_int32), ("n_lm", ctypes.c_int32), ("n_nb", ctypes.c_int32),
+                ("n_mb", ctypes.c_int32), ("mb_kind", ctypes.c_int32), ("n_mlp_heads", ctypes.c_int32),
+                ("boundary_byte", ctypes.c_int32), ("rope_base", ctypes.c_float),
+                ("rms_eps", ctypes.c_float), ("attn_scale", ctypes.c_float), ("dtype", ctypes.c_int32),
+                ("max_batch", ctypes.c_int32), ("max_bytes", ctypes.c_int32), ("max_n", ctypes.c_int32)]
+
+
+class LcaTensor(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char_p), ("ptr", ctypes.c_void_p), ("numel", ctypes.c_int64),
+                ("dtype", ctypes.c_int32)]
+
+
+class LcaSeqState(ctypes.Structure):
+    _fields_ = [("t", ctypes.c_int32), ("K", ctypes.c_int32), ("open_start", ctypes.c_int32),
+                ("prev_group_start", ctypes.c_int32), ("group_start", ctypes.c_int32),
+                ("next_byte", ctypes.c_int32), ("generated", ctypes.c_int32), ("pad", ctypes.c_int32)]
+
+
+class LcaStats(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int64) for f in ("steps", "lm_steps", "lm_rows", "mb_rows", "committed",
+                                              "kernels_per_step", "kernels_per_lm_run",
+                                              "workspace_bytes")]
+
+
+class LcaError(RuntimeError):
+    def __init__(self, status, what):
+        super().__init__(f"{what}: {STATUS.get(status, status)}")
+        self.status = status
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load liblca.so (raises OSError when it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise OSError(f"CUDA library not built: {path} (run paper_2608_15454_gb300/build.py)")
+    lib = ctypes.CDLL(path)
+    P, I32, F32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_float
+    sig = {
+        "lca_workspace_bytes": [ctypes.POINTER(LcaConfig), ctypes.POINTER(ctypes.c_size_t)],
+        "lca_create": [ctypes.POINTER(LcaConfig), ctypes.POINTER(LcaTensor), ctypes.c_int, P,
+                       ctypes.c_size_t, P, ctypes.POINTER(P)],
+        "lca_prefill": [P, I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(I32)],
+        "lca_mbp_step": [P, I32, F32, I32, P, P],
+        "lca_mbp_step_async": [P, I32, F32, I32],
+        "lca_generate": [P, I32, F32, I32, I32, P, P, P],
+        "lca_generate_async": [P, I32, F32, I32, I32],
+        "lca_generate_fetch": [P, P, P, P],
+        "lca_debug_state": [P, I32, ctypes.POINTER(LcaSeqState)],
+        "lca_debug_stats": [P, ctypes.POINTER(LcaStats)],
+        "lca_debug_logits": [P, P, P],
+        "lca_debug_force_accept": [P, P],
+        "lca_debug_force_candidates": [P, P, I32],
+        "lca_destroy": [P],
+        "lca_status_str": [ctypes.c_int],
+    }
+    for name, args in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = ctypes.c_char_p if name == "lca_status_str" else ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def make_config(model, max_batch: int, max_bytes: int, max_n: int) -> LcaConfig:
+    """lca_config from a synth.ModelConfig."""
+    return LcaConfig(model.d_model, model.n_heads, model.head_dim, model.d_ff, model.vocab,
+                     model.n_enc, model.n_lm, model.n_nb, model.n_mb,
+                     LCA_MB_MLP if model.mb_kind == "mlp" else LCA_MB_LCA, model.n_mlp_heads,
+                     model.boundary_byte, model.rope_base, model.rms_eps, model.attn_scale,
+                     LCA_BF16 if model.dtype == "bf16" else LCA_F32, max_batch, max_bytes, max_n)
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+class Context:
+    """One lca_ctx: weights and workspace on a CUDA device, prompts and outputs on the host."""
+
+    def __init__(self, model, weights: dict, max_batch: int, max_bytes: int, max_n: int,
+                 device: str = "cuda", stream=None):
+        import torch
+        self.torch = torch
+        self.lib = load_library()
+        self.model = model
+        self.device = torch.device(device)
+        self.max_n = max_n
+        self.cfg = make_config(model, max_batch, max_bytes, max_n)
+        wdt = torch.bfloat16 if model.dtype == "bf16" else torch.float32
+        self._weights = {}
+        tensors = []
+        for name, a in weights.items():
+            is_f32 = name.endswith("norm") or name == "lm.bos"
+            t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(self.device)
+            t = t if is_f32 else t.to(wdt)
+            t = t.contiguous()
+            self._weights[name] = t
+            tensors.append(LcaTensor(name.encode(), t.data_ptr(), t.numel(),
+                                     LCA_F32 if (is_f32 or wdt == torch.float32) else LCA_BF16))
+        arr = (LcaTensor * len(tensors))(*tensors)
+        nbytes = ctypes.c_size_t(0)
+        self._check(self.lib.lca_workspace_bytes(ctypes.byref(self.cfg), ctypes.byref(nbytes)),
+                    "lca_workspace_bytes")
+        self.workspace_bytes = nbytes.value
+        self._ws = torch.empty(self.workspace_bytes + 256, dtype=torch.uint8, device=self.device)
+        base = (self._ws.data_ptr() + 255) // 256 * 256
+        self.stream = stream if stream is not None else torch.cuda.current_stream(self.device)
+        h = ctypes.c_void_p()
+        self._check(self.lib.lca_create(ctypes.byref(self.cfg), arr, len(tensors), base,
+                                        self.workspace_bytes, self.stream.cuda_stream, ctypes.byref(h)),
+                    "lca_create")
+        self.h = h
+        self.batch = 0
+        del self._weights  # repacked into the workspace
+
+    def _check(self, st, what):
+        if st != LCA_OK:
+            raise LcaError(st, what)
+
+    def close(self):
+        if getattr(self, "h", None):
+            self.lib.lca_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # ------------------------------------------------------------------ calls
+    def prefill(self, prompts):
+        n = len(prompts)
+        bufs = [ctypes.c_char_p(bytes(p)) for p in prompts]
+        arr = (ctypes.c_char_p * n)(*bufs)
+        lens = (ctypes.c_int32 * n)(*[len(p) for p in prompts])
+        self._check(self.lib.lca_prefill(self.h, n, arr, lens), "lca_prefill")
+        self.batch = n
+
+    def step(self, n, tau, mode=LCA_THRESH):
+        out = np.zeros((self.batch, n), dtype=np.uint8)
+        cnt = np.zeros(self.batch, dtype=np.int32)
+        self._check(self.lib.lca_mbp_step(self.h, n, tau, mode, _ptr(out), _ptr(cnt)), "lca_mbp_step")
+        return [bytes(out[b, :cnt[b]]) for b in range(self.batch)], cnt
+
+    def step_async(self, n, tau, mode=LCA_THRESH):
+        self._check(self.lib.lca_mbp_step_async(self.h, n, tau, mode), "lca_mbp_step_async")
+
+    def generate(self, n, tau, mode, max_new):
+        out = np.zeros((self.batch, max_new), dtype=np.uint8)
+        ln = np.zeros(self.batch, dtype=np.int32)
+        hist = np.zeros(n, dtype=np.int32)
+        self._check(self.lib.lca_generate(self.h, n, tau, mode, max_new, _ptr(out), _ptr(ln), _ptr(hist)),
+                    "lca_generate")
+        return [bytes(out[b, :ln[b]]) for b in range(self.batch)], hist
+
+    def generate_async(self, n, tau, mode, max_new):
+        self._check(self.lib.lca_generate_async(self.h, n, tau, mode, max_new), "lca_generate_async")
+        self._gen = (n, max_new)
+
+    def generate_fetch(self):
+        n, max_new = self._gen
+        out = np.zeros((self.batch, max_new), dtype=np.uint8)
+        ln = np.zeros(self.batch, dtype=np.int32)
+        hist = np.zeros(n, dtype=np.int32)
+        self._check(self.lib.lca_generate_fetch(self.h, _ptr(out), _ptr(ln), _ptr(hist)),
+                    "lca_generate_fetch")
+        return [bytes(out[b, :ln[b]]) for b in range(self.batch)], hist
+
+    def state(self, b):
+        s = LcaSeqState()
+        self._check(self.lib.lca_debug_state(self.h, b, ctypes.byref(s)), "lca_debug_state")
+        return {f: getattr(s, f) for f, _ in LcaSeqState._fields_ if f != "pad"}
+
+    def stats(self):
+        s = LcaStats()
+        self._check(self.lib.lca_debug_stats(self.h, ctypes.byref(s)), "lca_debug_stats")
+        return {f: getattr(s, f) for f, _ in LcaStats._fields_}
+
+    def logits(self, n):
+        nb = np.zeros((self.batch, n, 256), dtype=np.float32)
+        mb = np.zeros((self.batch, max(n - 1, 0), 256), dtype=np.float32)
+        self._check(self.lib.lca_debug_logits(self.h, _ptr(nb), _ptr(mb) if n > 1 else None),
+                    "lca_debug_logits")
+        return nb, mb
+
+    def force_accept(self, a):
+        if a is None:
+            self._check(self.lib.lca_debug_force_accept(self.h, None), "force_accept")
+            return
+        arr = np.ascontiguousarray(a, dtype=np.int32)
+        self._check(self.lib.lca_debug_force_accept(self.h, _ptr(arr)), "force_accept")
+
+    def force_candidates(self, cand, n):
+        if cand is None:
+            self._check(self.lib.lca_debug_force_candidates(self.h, None, 0), "force_candidates")
+            return
+        arr = np.frombuffer(b"".join(bytes(c) for c in cand), dtype=np.uint8).copy()
+        self._check(self.lib.lca_debug_force_candidates(self.h, _ptr(arr), n), "force_candidates")
+
+
+def status_str(st: int) -> str:
+    return load_library().lca_status_str(st).decode()
