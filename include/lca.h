@@ -154,6 +154,22 @@ int lca_generate_fetch(lca_ctx* ctx, uint8_t* out, int32_t* out_len, int32_t* ac
 /* Debug and test hooks. */
 int lca_debug_state(lca_ctx* ctx, int32_t b, lca_seq_state* out);
 int lca_debug_stats(lca_ctx* ctx, lca_stats* out);
+
+/* Run later steps as direct kernel launches instead of one graph (on != 0), so that
+ * per-kernel profilers can see them; the LM decision is then read back on the host.
+ * Results are identical. */
+int lca_debug_set_eager(lca_ctx* ctx, int32_t on);
+
+/* Per-kind timing of `steps` eager steps: CUDA events around every launch on the context
+ * stream. Kinds: 0 linear layers, 1 attention, 2 unembedding heads, 3 glue. bytes: the
+ * weight bytes each launch must read (linear layers and heads), summed. */
+typedef struct {
+  int64_t launches[4];
+  double ms[4];
+  double bytes[4];
+} lca_profile;
+int lca_debug_profile(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t steps,
+                      lca_profile* out);
 /* Logits of the last step: nb host [batch * n * 256] (next-byte rows of the n candidates),
  * mb host [batch * (n-1) * 256] (drafter rows). Either may be NULL. */
 int lca_debug_logits(lca_ctx* ctx, float* nb, float* mb);

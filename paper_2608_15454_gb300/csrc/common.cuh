@@ -102,6 +102,25 @@ struct Stats {
 // Kernels launched by this thread's wrappers (counted at capture time).
 extern thread_local long long g_launches;
 
+// Optional per-launch timing hook (eager steps only): the wrappers bracket each launch with
+// begin/end so the runtime can record CUDA events on the launching stream.
+enum ProfKind { PK_LINEAR = 0, PK_ATTN = 1, PK_HEAD = 2, PK_GLUE = 3, PK_COUNT = 4 };
+struct ProfHook {
+  virtual void begin(int kind, double bytes, cudaStream_t s) = 0;
+  virtual void end(cudaStream_t s) = 0;
+};
+extern thread_local ProfHook* g_prof;
+struct ProfScope {
+  cudaStream_t s;
+  bool on;
+  ProfScope(int kind, double bytes, cudaStream_t s_) : s(s_), on(g_prof != nullptr) {
+    if (on) g_prof->begin(kind, bytes, s);
+  }
+  ~ProfScope() {
+    if (on) g_prof->end(s);
+  }
+};
+
 // Workspace layout (device pointers into the caller's workspace).
 struct Dev {
   // shape

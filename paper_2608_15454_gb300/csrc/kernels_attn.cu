@@ -205,6 +205,7 @@ size_t attention_counters(int B, int H) { return (size_t)B * kQTMax * H; }
 
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s) {
+  ProfScope ps(PK_ATTN, 0.0, s);
   if (splits > kMaxAttnSplit) splits = kMaxAttnSplit;
   if (splits < 1) splits = 1;
   if (D.dtype == LCA_BF16) {

@@ -388,6 +388,7 @@ void kernel_attrs_linear() {
 
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s) {
   const bool norm = a.norm != nullptr;
+  ProfScope ps(PK_LINEAR, (double)a.N * a.Kd * a.groups * (D.dtype == LCA_BF16 ? 2 : 4), s);
   if (D.dtype == LCA_BF16) {
     if (tiled) norm ? launch_gemm<__nv_bfloat16, true>(D, a, s) : launch_gemm<__nv_bfloat16, false>(D, a, s);
     else norm ? launch_gemv<__nv_bfloat16, true>(D, a, s) : launch_gemv<__nv_bfloat16, false>(D, a, s);

@@ -626,17 +626,21 @@ void kernel_attrs_step() {
 }
 
 thread_local long long g_launches = 0;
+thread_local ProfHook* g_prof = nullptr;
 
 void launch_mb_plan(const Dev& D, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_mb_plan<<<1, 1024, 0, s>>>(D);
 }
 void launch_mb_fill(const Dev& D, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_mb_fill<<<152 * 2, 256, 0, s>>>(D);
 }
 void launch_mlp_plan(const Dev& D, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_mlp_plan<<<256, 256, 0, s>>>(D);
 }
 
@@ -645,6 +649,7 @@ void launch_head(const Dev& D, const float* x, const int* rows, const int* M, in
   dim3 grid((M_cap + kHR - 1) / kHR, kVocab / kHV);
   const size_t smem = (size_t)kHR * D.d * sizeof(float);
   ++g_launches;
+  ProfScope ps(PK_HEAD, 256.0 * D.d * (D.dtype == LCA_BF16 ? 2 : 4), s);
   // the split-K counters double as head row-tile counters (different launches, same stream)
   if (D.dtype == LCA_BF16)
     k_head<__nv_bfloat16><<<grid, 128, smem, s>>>(D, x, rows, M, M_cap, norm, logits, arg, prob, D.head_cnt);
@@ -654,26 +659,32 @@ void launch_head(const Dev& D, const float* x, const int* rows, const int* M, in
 
 void launch_verify_plan(const Dev& D, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_verify_plan<<<D.B, 256, 0, s>>>(D);
 }
 void launch_segment(const Dev& D, cudaGraphConditionalHandle h, int use_handle, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_segment<<<D.B, 256, 0, s>>>(D, h, use_handle);
 }
 void launch_lm_scatter(const Dev& D, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_lm_scatter<<<256, 256, 0, s>>>(D);
 }
 void launch_nb_input(const Dev& D, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_nb_input<<<256, 256, 0, s>>>(D);
 }
 void launch_commit(const Dev& D, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_commit<<<D.B, 256, 0, s>>>(D);
 }
 void launch_loop_ctl(const Dev& D, cudaGraphConditionalHandle h, cudaStream_t s) {
   ++g_launches;
+  ProfScope ps(PK_GLUE, 0.0, s);
   k_loop_ctl<<<1, 32, 0, s>>>(D, h);
 }
 void launch_gen_init(const Dev& D, int max_new, cudaStream_t s) {

@@ -196,6 +196,7 @@ struct lca_ctx {
   int gen_max_new = 0;
   int gen_n = 0;
   bool t_unsynced = false;
+  bool eager = false;
   // kernels per step graph part, by n: [pre-LM + post-LM, LM body]
   std::map<int, std::pair<long long, long long>> launches;
 };
@@ -343,21 +344,17 @@ void run_mlp_heads(lca_ctx* c, int n, cudaStream_t s) {
   }
 }
 
-// Capture one decode step into graph g (which may be the body of a WHILE node).
-int capture_step(lca_ctx* c, cudaGraph_t g, int n, bool loop, cudaGraphConditionalHandle hwhile) {
+// The three parts of one decode step, shared by graph capture and eager execution.
+void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
   Dev& D = c->L.D;
-  cudaStream_t s = c->cap;
-  CK(cudaStreamBeginCaptureToGraph(s, g, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
-  const long long l0 = g_launches;
-  long long lm_launches = 0;
   const int B = D.B;
   // (3) draft
   if (n >= 2) {
     if (D.mb_kind == LCA_MB_LCA) {
       launch_mb_plan(D, s);
       launch_mb_fill(D, s);
-      const int typ = B * (2 * n);
-      run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2), s);  // window rows
+      const int typ = B * (2 * n);  // typical window rows: the new committed bytes + copies
+      run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2), s);
     } else {
       launch_mlp_plan(D, s);
       run_mlp_heads(c, n, s);
@@ -367,9 +364,36 @@ int capture_step(lca_ctx* c, cudaGraph_t g, int n, bool loop, cudaGraphCondition
   }
   // (1) embed + encoder over the n candidates
   launch_verify_plan(D, s);
-  const int vs = attn_splits(D, B, 1);
-  run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, vs, s);
-  // segments closed by candidate boundaries -> LM rows; conditional on any
+  run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s);
+}
+
+void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
+  Dev& D = c->L.D;
+  // about one new latent per sequence every few bytes
+  run_stack(c, c->L.lm, D.x_lm, D.r_lm, D.B * n, D.B, 1, attn_splits(D, D.B, 1), s);
+  launch_lm_scatter(D, s);
+}
+
+void enqueue_verify_commit(lca_ctx* c, int n, cudaStream_t s) {
+  Dev& D = c->L.D;
+  const int B = D.B;
+  // (4) upsample + next-byte decoder over the n candidates, head
+  launch_nb_input(D, s);
+  run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s);
+  launch_head(D, D.x_nb, nullptr, D.r_v.M, B * n, D.nb_norm, D.nb_logits, D.nb_arg, D.nb_prob, s);
+  // (5) accept + commit
+  launch_commit(D, s);
+}
+
+// Capture one decode step into graph g (which may be the body of a WHILE node).
+int capture_step(lca_ctx* c, cudaGraph_t g, int n, bool loop, cudaGraphConditionalHandle hwhile) {
+  Dev& D = c->L.D;
+  cudaStream_t s = c->cap;
+  CK(cudaStreamBeginCaptureToGraph(s, g, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+  const long long l0 = g_launches;
+  long long lm_launches = 0;
+  enqueue_draft_encode(c, n, s);
+  // segments closed by candidate boundaries -> LM rows; the LM runs only if there are any
   cudaStreamCaptureStatus st;
   cudaGraph_t cg;
   const cudaGraphNode_t* deps = nullptr;
@@ -391,27 +415,81 @@ int capture_step(lca_ctx* c, cudaGraph_t g, int n, bool loop, cudaGraphCondition
   {
     cudaStream_t s2 = c->cap2;
     CK(cudaStreamBeginCaptureToGraph(s2, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
-    // about one new latent per sequence every few bytes
     const long long b0 = g_launches;
-    run_stack(c, c->L.lm, D.x_lm, D.r_lm, B * n, B, 1, vs, s2);
-    launch_lm_scatter(D, s2);
+    enqueue_lm(c, n, s2);
     lm_launches = g_launches - b0;
     cudaGraph_t tmp;
     CK(cudaStreamEndCapture(s2, &tmp));
   }
   CK(cudaStreamUpdateCaptureDependencies(s, &cnode, nullptr, 1, cudaStreamSetCaptureDependencies));
-  // (4) upsample + next-byte decoder over the n candidates, head
-  launch_nb_input(D, s);
-  run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, vs, s);
-  launch_head(D, D.x_nb, nullptr, D.r_v.M, B * n, D.nb_norm, D.nb_logits, D.nb_arg, D.nb_prob, s);
-  // (5) accept + commit
-  launch_commit(D, s);
+  enqueue_verify_commit(c, n, s);
   if (loop) launch_loop_ctl(D, hwhile, s);
   cudaGraph_t out;
   CK(cudaStreamEndCapture(s, &out));
   if (!loop) c->launches[n] = {g_launches - l0 - lm_launches, lm_launches};
   return LCA_OK;
 }
+
+// The same step as direct launches on the context stream; the LM decision is read back on
+// the host. Used for per-kernel profiling (profilers cannot see kernels inside graphs with
+// conditional nodes); results are identical to the graph.
+int run_step_eager(lca_ctx* c, int n) {
+  Dev& D = c->L.D;
+  cudaStream_t s = c->stream;
+  enqueue_draft_encode(c, n, s);
+  launch_segment(D, 0, 0, s);
+  int mlm = 0;
+  CK(cudaMemcpyAsync(&mlm, D.r_lm.M, sizeof(int), cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  if (mlm > 0) enqueue_lm(c, n, s);
+  enqueue_verify_commit(c, n, s);
+  CK(cudaGetLastError());
+  return LCA_OK;
+}
+
+// Records CUDA events around each launch of an eager step and sums them per kind.
+struct Profiler : ProfHook {
+  struct Rec {
+    int kind;
+    double bytes;
+    cudaEvent_t a, b;
+  };
+  std::vector<Rec> pool;
+  size_t used = 0;
+  double ms[PK_COUNT] = {0, 0, 0, 0};
+  double bytes[PK_COUNT] = {0, 0, 0, 0};
+  long long launches[PK_COUNT] = {0, 0, 0, 0};
+  void begin(int kind, double by, cudaStream_t s) override {
+    if (used == pool.size()) {
+      Rec r{};
+      cudaEventCreate(&r.a);
+      cudaEventCreate(&r.b);
+      pool.push_back(r);
+    }
+    Rec& r = pool[used];
+    r.kind = kind;
+    r.bytes = by;
+    cudaEventRecord(r.a, s);
+  }
+  void end(cudaStream_t s) override { cudaEventRecord(pool[used++].b, s); }
+  void collect() {
+    for (size_t i = 0; i < used; ++i) {
+      float t = 0.f;
+      cudaEventSynchronize(pool[i].b);
+      cudaEventElapsedTime(&t, pool[i].a, pool[i].b);
+      ms[pool[i].kind] += t;
+      bytes[pool[i].kind] += pool[i].bytes;
+      launches[pool[i].kind] += 1;
+    }
+    used = 0;
+  }
+  ~Profiler() {
+    for (auto& r : pool) {
+      cudaEventDestroy(r.a);
+      cudaEventDestroy(r.b);
+    }
+  }
+};
 
 int get_step_exec(lca_ctx* c, int n, cudaGraphExec_t* ex) {
   auto it = c->step_exec.find(n);
@@ -771,7 +849,12 @@ int lca_mbp_step(lca_ctx* c, int32_t n, float tau, int32_t mode, uint8_t* out_by
   st = upload_params(c);
   if (st != LCA_OK) return st;
   c->pending_force_accept = c->pending_force_cand = 0;
-  CK(cudaGraphLaunch(ex, c->stream));
+  if (c->eager) {
+    st = run_step_eager(c, n);
+    if (st != LCA_OK) return st;
+  } else {
+    CK(cudaGraphLaunch(ex, c->stream));
+  }
   std::vector<int> cnt(c->batch);
   CK(cudaMemcpyAsync(cnt.data(), c->L.D.out_cnt, c->batch * sizeof(int), cudaMemcpyDeviceToHost,
                      c->stream));
@@ -801,7 +884,12 @@ int lca_mbp_step_async(lca_ctx* c, int32_t n, float tau, int32_t mode) {
   st = upload_params(c);
   if (st != LCA_OK) return st;
   c->pending_force_accept = c->pending_force_cand = 0;
-  CK(cudaGraphLaunch(ex, c->stream));
+  if (c->eager) {
+    st = run_step_eager(c, n);
+    if (st != LCA_OK) return st;
+  } else {
+    CK(cudaGraphLaunch(ex, c->stream));
+  }
   c->last_n = n;
   for (int b = 0; b < c->batch; ++b) c->t_host[b] += n;  // upper bound until synced
   c->t_unsynced = true;
@@ -924,6 +1012,47 @@ int lca_debug_stats(lca_ctx* c, lca_stats* out) {
   out->kernels_per_lm_run = it == c->launches.end() ? 0 : it->second.second;
   out->workspace_bytes = (int64_t)c->ws_bytes;
   return LCA_OK;
+}
+
+int lca_debug_set_eager(lca_ctx* c, int32_t on) {
+  if (!c) return LCA_E_ARG;
+  c->eager = on != 0;
+  return LCA_OK;
+}
+
+int lca_debug_profile(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t steps,
+                      lca_profile* out) {
+  if (!out || steps < 1) return LCA_E_ARG;
+  int st = step_prep(c, n, tau, mode);
+  if (st != LCA_OK) return st;
+  for (int b = 0; b < c->batch; ++b)
+    if (c->t_host[b] + (long long)steps * n > c->cfg.max_bytes) return LCA_E_CAPACITY;
+  Params& P = c->host_params;
+  P.gen = 0;
+  P.force_accept = 0;
+  P.force_cand = 0;
+  Profiler prof;
+  for (int i = 0; i < steps; ++i) {
+    st = upload_params(c);
+    if (st != LCA_OK) return st;
+    g_prof = &prof;
+    st = run_step_eager(c, n);
+    g_prof = nullptr;
+    if (st != LCA_OK) return st;
+    prof.collect();
+  }
+  c->last_n = n;
+  std::vector<SeqState> all(c->batch);
+  CK(cudaMemcpyAsync(all.data(), c->L.D.seq, sizeof(SeqState) * c->batch, cudaMemcpyDeviceToHost,
+                     c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  for (int i = 0; i < c->batch; ++i) c->t_host[i] = all[i].t;
+  for (int k = 0; k < PK_COUNT && k < 4; ++k) {
+    out->launches[k] = prof.launches[k];
+    out->ms[k] = prof.ms[k];
+    out->bytes[k] = prof.bytes[k];
+  }
+  return read_err(c);
 }
 
 int lca_debug_force_accept(lca_ctx* c, const int32_t* a) {

@@ -25,6 +25,7 @@ STATUS = {0: "LCA_OK", -1: "LCA_E_ARG", -2: "LCA_E_CAPACITY", -3: "LCA_E_WEIGHTS
 EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "lca_mbp_step_async",
            "lca_generate",
            "lca_generate_async", "lca_generate_fetch", "lca_debug_state", "lca_debug_stats",
+           "lca_debug_set_eager", "lca_debug_profile",
            "lca_debug_logits",
            "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str")
 
@@ -54,6 +55,13 @@ class LcaStats(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int64) for f in ("steps", "lm_steps", "lm_rows", "mb_rows", "committed",
                                               "kernels_per_step", "kernels_per_lm_run",
                                               "workspace_bytes")]
+
+
+class LcaProfile(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_int64 * 4), ("ms", ctypes.c_double * 4), ("bytes", ctypes.c_double * 4)]
+
+
+PROFILE_KINDS = ("linear", "attention", "head", "glue")
 
 
 class LcaError(RuntimeError):
@@ -87,6 +95,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_debug_state": [P, I32, ctypes.POINTER(LcaSeqState)],
         "lca_debug_stats": [P, ctypes.POINTER(LcaStats)],
         "lca_debug_logits": [P, P, P],
+        "lca_debug_set_eager": [P, I32],
+        "lca_debug_profile": [P, I32, F32, I32, I32, ctypes.POINTER(LcaProfile)],
         "lca_debug_force_accept": [P, P],
         "lca_debug_force_candidates": [P, P, I32],
         "lca_destroy": [P],
@@ -215,6 +225,16 @@ class Context:
         s = LcaStats()
         self._check(self.lib.lca_debug_stats(self.h, ctypes.byref(s)), "lca_debug_stats")
         return {f: getattr(s, f) for f, _ in LcaStats._fields_}
+
+    def set_eager(self, on: bool):
+        self._check(self.lib.lca_debug_set_eager(self.h, 1 if on else 0), "lca_debug_set_eager")
+
+    def profile(self, n, tau, mode, steps):
+        p = LcaProfile()
+        self._check(self.lib.lca_debug_profile(self.h, n, tau, mode, steps, ctypes.byref(p)),
+                    "lca_debug_profile")
+        return {k: {"launches": p.launches[i], "ms": p.ms[i], "bytes": p.bytes[i]}
+                for i, k in enumerate(PROFILE_KINDS)}
 
     def logits(self, n):
         nb = np.zeros((self.batch, n, 256), dtype=np.float32)
