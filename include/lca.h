@@ -180,6 +180,26 @@ int lca_debug_force_accept(lca_ctx* ctx, const int32_t* a);
  * NULL to clear. The drafter still runs and its logits stay readable. */
 int lca_debug_force_candidates(lca_ctx* ctx, const uint8_t* cand, int32_t n);
 
+/* Decode attention as a standalone call: the attention every module of the decode step
+ * runs (causal softmax attention, Section 2.2; inside the multi-byte window of Algorithm 1
+ * line 12 the LCA mask reduces to the same causal form). Query row r of sequence b sees the
+ * cache slots [0, kv_len[r]) of its sequence; softmax scale `scale`; fp32 arithmetic.
+ *   q, out:   device fp32 [batch * n_rows][heads * head_dim] (RoPE already applied to q).
+ *   k_cache, v_cache: device [batch][heads][slots][head_dim] of `dtype` (LCA_F32|LCA_BF16).
+ *   kv_len:   device int32 [batch * n_rows], each 1..slots (larger values are clamped).
+ *   splits:   1..16; the key range of each (sequence, head) is split over `splits` CTAs whose
+ *             partial results are combined in a fixed order (deterministic).
+ *   scratch:  device memory of >= lca_decode_attention_scratch_bytes(...), 256-byte aligned,
+ *             caller-owned; overwritten by the call.
+ * head_dim must be 32 or 64. Asynchronous on `stream` (a cudaStream_t). Returns LCA_E_ARG for
+ * bad arguments and LCA_E_CAPACITY for too small a scratch. */
+int lca_decode_attention_scratch_bytes(int32_t batch, int32_t heads, int32_t head_dim,
+                                       int32_t splits, size_t* out);
+int lca_decode_attention(const float* q, float* out, const void* k_cache, const void* v_cache,
+                         int32_t dtype, int32_t batch, int32_t heads, int32_t head_dim,
+                         int32_t slots, int32_t n_rows, const int32_t* kv_len, float scale,
+                         int32_t splits, void* scratch, size_t scratch_bytes, void* stream);
+
 int lca_destroy(lca_ctx* ctx);
 const char* lca_status_str(int status);
 

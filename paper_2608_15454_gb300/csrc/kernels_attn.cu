@@ -188,12 +188,88 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
 }
 
 template <typename TC, int HD>
-void launch(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
-            int qtiles_grid, int splits, cudaStream_t s) {
-  dim3 grid(B, qtiles_grid, D.H * splits);
+void launch(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
+            int qtiles_grid, int splits, float* part, int* cnt, int* err, cudaStream_t s) {
+  dim3 grid(B, qtiles_grid, H * splits);
   ++g_launches;
-  k_attn<TC, HD><<<grid, kThreads, 0, s>>>(q, out, kv, rows, D.H, D.scale, splits, D.attn_part,
-                                           D.attn_cnt, D.err);
+  k_attn<TC, HD><<<grid, kThreads, 0, s>>>(q, out, kv, rows, H, scale, splits, part, cnt, err);
+}
+
+void launch_any(int dtype, int hd, const float* q, float* out, const KV& kv, const Rows& rows, int B,
+                int H, float scale, int qtiles_grid, int splits, float* part, int* cnt, int* err,
+                cudaStream_t s) {
+  if (dtype == LCA_BF16) {
+    if (hd == 64) launch<__nv_bfloat16, 64>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, part, cnt, err, s);
+    else launch<__nv_bfloat16, 32>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, part, cnt, err, s);
+  } else {
+    if (hd == 64) launch<float, 64>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, part, cnt, err, s);
+    else launch<float, 32>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, part, cnt, err, s);
+  }
+}
+
+// Rows of the standalone op: sequence b owns rows [b*n_rows, (b+1)*n_rows).
+__global__ void k_regular_rows(int* seq_start, int* seq_count, int batch, int n_rows) {
+  for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < batch; b += gridDim.x * blockDim.x) {
+    seq_start[b] = b * n_rows;
+    seq_count[b] = n_rows;
+  }
+}
+
+// Scratch of the standalone op: [error word][tile counters][seq_start][seq_count][partials].
+struct OpScratch {
+  int* err;
+  int* cnt;
+  int* seq_start;
+  int* seq_count;
+  float* part;
+  size_t header_bytes; // bytes that must be zero before a call (error word + counters)
+  size_t bytes;
+};
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+OpScratch op_scratch_layout(char* base, int batch, int heads, int head_dim, int splits) {
+  OpScratch o{};
+  size_t off = 0;
+  o.err = reinterpret_cast<int*>(base + off);
+  off += 256;
+  o.cnt = reinterpret_cast<int*>(base + off);
+  off += align256((size_t)batch * kQTMax * heads * sizeof(int));
+  o.header_bytes = off;
+  o.seq_start = reinterpret_cast<int*>(base + off);
+  off += align256((size_t)batch * sizeof(int));
+  o.seq_count = reinterpret_cast<int*>(base + off);
+  off += align256((size_t)batch * sizeof(int));
+  o.part = reinterpret_cast<float*>(base + off);
+  off += align256((size_t)batch * kQTMax * heads * splits * kAttnQT * (head_dim + 2) * sizeof(float));
+  o.bytes = off;
+  return o;
+}
+
+int op_check(const float* q, float* out, const void* k, const void* v, int dtype, int batch, int heads,
+             int head_dim, int slots, int n_rows, const int* kv_len, int splits) {
+  if (!q || !out || !k || !v || !kv_len) return LCA_E_ARG;
+  if (dtype != LCA_F32 && dtype != LCA_BF16) return LCA_E_ARG;
+  if (head_dim != 32 && head_dim != 64) return LCA_E_ARG;
+  if (batch < 1 || heads < 1 || slots < 1 || n_rows < 1) return LCA_E_ARG;
+  if (splits < 1 || splits > kMaxAttnSplit) return LCA_E_ARG;
+  return LCA_OK;
+}
+
+int op_run(const float* q, float* out, const void* k, const void* v, int dtype, int batch, int heads,
+           int head_dim, int slots, int n_rows, const int* kv_len, float scale, int splits,
+           const OpScratch& o, cudaStream_t s) {
+  if (cudaMemsetAsync(o.err, 0, o.header_bytes, s) != cudaSuccess) return LCA_E_CUDA;
+  k_regular_rows<<<(batch + 255) / 256, 256, 0, s>>>(o.seq_start, o.seq_count, batch, n_rows);
+  Rows rows{};
+  rows.kvlen = const_cast<int*>(kv_len);
+  rows.seq_start = o.seq_start;
+  rows.seq_count = o.seq_count;
+  KV kv{const_cast<void*>(k), const_cast<void*>(v), slots};
+  const int qt = (n_rows + kAttnQT - 1) / kAttnQT;
+  launch_any(dtype, head_dim, q, out, kv, rows, batch, heads, scale, qt < 64 ? qt : 64, splits,
+             o.part, o.cnt, o.err, s);
+  return cudaGetLastError() == cudaSuccess ? LCA_OK : LCA_E_CUDA;
 }
 
 } // namespace
@@ -208,13 +284,40 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
   ProfScope ps(PK_ATTN, 0.0, s);
   if (splits > kMaxAttnSplit) splits = kMaxAttnSplit;
   if (splits < 1) splits = 1;
-  if (D.dtype == LCA_BF16) {
-    if (D.hd == 64) launch<__nv_bfloat16, 64>(D, q, out, kv, rows, B, qtiles_grid, splits, s);
-    else launch<__nv_bfloat16, 32>(D, q, out, kv, rows, B, qtiles_grid, splits, s);
-  } else {
-    if (D.hd == 64) launch<float, 64>(D, q, out, kv, rows, B, qtiles_grid, splits, s);
-    else launch<float, 32>(D, q, out, kv, rows, B, qtiles_grid, splits, s);
-  }
+  launch_any(D.dtype, D.hd, q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.attn_part,
+             D.attn_cnt, D.err, s);
 }
+
+} // namespace lca
+
+using namespace lca;
+
+extern "C" {
+
+int lca_decode_attention_scratch_bytes(int32_t batch, int32_t heads, int32_t head_dim,
+                                       int32_t splits, size_t* out) {
+  if (!out || batch < 1 || heads < 1 || (head_dim != 32 && head_dim != 64) || splits < 1 ||
+      splits > kMaxAttnSplit)
+    return LCA_E_ARG;
+  *out = op_scratch_layout(nullptr, batch, heads, head_dim, splits).bytes;
+  return LCA_OK;
+}
+
+int lca_decode_attention(const float* q, float* out, const void* k_cache, const void* v_cache,
+                         int32_t dtype, int32_t batch, int32_t heads, int32_t head_dim,
+                         int32_t slots, int32_t n_rows, const int32_t* kv_len, float scale,
+                         int32_t splits, void* scratch, size_t scratch_bytes, void* stream) {
+  int st = op_check(q, out, k_cache, v_cache, dtype, batch, heads, head_dim, slots, n_rows, kv_len, splits);
+  if (st != LCA_OK) return st;
+  if (!scratch || reinterpret_cast<uintptr_t>(scratch) % 256) return LCA_E_ARG;
+  const OpScratch o = op_scratch_layout(reinterpret_cast<char*>(scratch), batch, heads, head_dim, splits);
+  if (scratch_bytes < o.bytes) return LCA_E_CAPACITY;
+  return op_run(q, out, k_cache, v_cache, dtype, batch, heads, head_dim, slots, n_rows, kv_len, scale,
+                splits, o, reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"
+
+namespace lca {
 
 } // namespace lca

@@ -27,7 +27,8 @@ EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "
            "lca_generate_async", "lca_generate_fetch", "lca_debug_state", "lca_debug_stats",
            "lca_debug_set_eager", "lca_debug_profile",
            "lca_debug_logits",
-           "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str")
+           "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str",
+           "lca_decode_attention_scratch_bytes", "lca_decode_attention")
 
 
 class LcaConfig(ctypes.Structure):
@@ -101,6 +102,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_debug_force_candidates": [P, P, I32],
         "lca_destroy": [P],
         "lca_status_str": [ctypes.c_int],
+        "lca_decode_attention_scratch_bytes": [I32, I32, I32, I32, ctypes.POINTER(ctypes.c_size_t)],
+        "lca_decode_attention": [P, P, P, P, I32, I32, I32, I32, I32, I32, P, F32, I32, P,
+                                 ctypes.c_size_t, P],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
@@ -256,6 +260,29 @@ class Context:
             return
         arr = np.frombuffer(b"".join(bytes(c) for c in cand), dtype=np.uint8).copy()
         self._check(self.lib.lca_debug_force_candidates(self.h, _ptr(arr), n), "force_candidates")
+
+
+def decode_attention(q, out, k_cache, v_cache, kv_len, scale, splits, scratch=None, stream=None):
+    """Standalone decode attention on torch CUDA tensors (see include/lca.h).
+    q/out: fp32 [batch*n_rows, heads*head_dim]; caches [batch, heads, slots, head_dim];
+    kv_len: int32 [batch*n_rows]. Returns the status code."""
+    import torch
+    lib = load_library()
+    batch, heads, slots, hd = k_cache.shape
+    n_rows = q.shape[0] // batch
+    dt = LCA_BF16 if k_cache.dtype == torch.bfloat16 else LCA_F32
+    st = stream if stream is not None else torch.cuda.current_stream(q.device)
+    args = [q.data_ptr(), out.data_ptr(), k_cache.data_ptr(), v_cache.data_ptr(), dt, batch, heads, hd,
+            slots, n_rows, kv_len.data_ptr(), scale, splits]
+    return lib.lca_decode_attention(*args, scratch.data_ptr(), scratch.numel(), st.cuda_stream)
+
+
+def decode_attention_scratch_bytes(batch, heads, head_dim, splits):
+    n = ctypes.c_size_t()
+    st = load_library().lca_decode_attention_scratch_bytes(batch, heads, head_dim, splits, ctypes.byref(n))
+    if st != LCA_OK:
+        raise LcaError(st, "lca_decode_attention_scratch_bytes")
+    return n.value
 
 
 def status_str(st: int) -> str:

@@ -15,7 +15,7 @@ def declared_functions():
             continue
         text = open(os.path.join(ROOT, "include", f)).read()
         text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-        names += re.findall(r"^\s*(?:int|const char\s*\*)\s+(lca_\w+)\s*\(", text, flags=re.M)
+        names += re.findall(r"^\s*(?:int|size_t|const char\s*\*)\s+(lca_\w+)\s*\(", text, flags=re.M)
     return names
 
 

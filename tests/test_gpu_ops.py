@@ -1,0 +1,69 @@
+"""The decode-attention kernel as a standalone call against a plain PyTorch fp32 reference."""
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def lca():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2608_15454_gb300 import build, lca as mod
+    build.build()
+    mod.load_library()
+    return mod
+
+
+def reference(q, k, v, kv_len, scale, n_rows):
+    """fp32 softmax attention: row r of sequence b over cache slots [0, kv_len[r])."""
+    import torch
+    B, H, S, hd = k.shape
+    out = torch.zeros_like(q)
+    kf, vf = k.float(), v.float()
+    for r in range(q.shape[0]):
+        b, L = r // n_rows, int(kv_len[r])
+        qr = q[r].view(H, hd)
+        s = torch.einsum("hd,hsd->hs", qr, kf[b, :, :L]) * scale
+        p = torch.softmax(s, dim=-1)
+        out[r] = torch.einsum("hs,hsd->hd", p, vf[b, :, :L]).reshape(-1)
+    return out
+
+
+def make_case(dtype, B, H, hd, S, n_rows, seed):
+    import torch
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    q = torch.randn(B * n_rows, H * hd, device="cuda", generator=g)
+    k = torch.randn(B, H, S, hd, device="cuda", generator=g).to(dtype)
+    v = torch.randn(B, H, S, hd, device="cuda", generator=g).to(dtype)
+    lens = torch.randint(1, S + 1, (B * n_rows,), device="cuda", generator=g, dtype=torch.int32)
+    lens[0] = S            # full cache
+    lens[-1] = 1           # one key
+    return q, k, v, lens
+
+
+@pytest.mark.parametrize("dtype_name,hd,splits,n_rows", [("float32", 32, 1, 3), ("bfloat16", 64, 8, 7),
+                                                         ("bfloat16", 64, 16, 20), ("float32", 64, 3, 1)])
+def test_decode_attention_matches_fp32_reference(lca, dtype_name, hd, splits, n_rows):
+    import torch
+    dtype = getattr(torch, dtype_name)
+    B, H, S = 3, 4, 301
+    q, k, v, lens = make_case(dtype, B, H, hd, S, n_rows, seed=hd + splits)
+    out = torch.empty_like(q)
+    nbytes = lca.decode_attention_scratch_bytes(B, H, hd, splits)
+    scratch = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    scale = 1.0 / hd ** 0.5
+    assert lca.decode_attention(q, out, k, v, lens, scale, splits, scratch) == 0
+    torch.cuda.synchronize()
+    want = reference(q, k, v, lens, scale, n_rows)
+    np.testing.assert_allclose(out.cpu().numpy(), want.cpu().numpy(), atol=1e-4, rtol=0)
+
+
+def test_decode_attention_rejects_bad_arguments(lca):
+    import torch
+    q, k, v, lens = make_case(torch.float32, 1, 2, 32, 16, 2, seed=0)
+    out = torch.empty_like(q)
+    small = torch.empty(256, dtype=torch.uint8, device="cuda")
+    assert lca.decode_attention(q, out, k, v, lens, 0.1, 4, small) == -2
+    assert lca.decode_attention(q, out, k, v, lens, 0.1, 99, small) == -1
