@@ -200,6 +200,26 @@ int lca_decode_attention(const float* q, float* out, const void* k_cache, const 
                          int32_t slots, int32_t n_rows, const int32_t* kv_len, float scale,
                          int32_t splits, void* scratch, size_t scratch_bytes, void* stream);
 
+/* lca_decode_attention for callers that cannot allocate device memory: plugin or custom-op
+ * hosts that hand a kernel only its input and output buffers, and code paths where an
+ * allocation call is not allowed because it may synchronize the device or break a fixed
+ * memory budget. (The paper has no counterpart; this is a library convenience.)
+ * Same arguments and results as lca_decode_attention without the scratch pair. The scratch is
+ * a fixed device array inside the library, lca_decode_attention_noalloc_capacity() bytes
+ * (8 MiB), which every GPU that loads the library holds until the process exits. Sizes whose
+ * scratch (lca_decode_attention_scratch_bytes) exceeds it return LCA_E_CAPACITY. The call
+ * allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
+ * The first call on a device looks up the array's device address (once per device, with that
+ * device current); make that first call before any stream capture. All calls share the one
+ * array and it keeps the last call's contents; each call clears the parts that must start at
+ * zero. Calls that may overlap on the GPU (other streams, other host threads) race on it:
+ * order them on one stream. */
+int lca_decode_attention_noalloc(const float* q, float* out, const void* k_cache, const void* v_cache,
+                                 int32_t dtype, int32_t batch, int32_t heads, int32_t head_dim,
+                                 int32_t slots, int32_t n_rows, const int32_t* kv_len, float scale,
+                                 int32_t splits, void* stream);
+size_t lca_decode_attention_noalloc_capacity(void);
+
 int lca_destroy(lca_ctx* ctx);
 const char* lca_status_str(int status);
 

@@ -6,6 +6,8 @@
 // values stream through shared memory in tiles of 32; softmax is computed online in fp32.
 // With several key splits each CTA writes (max, sum, acc) partials and the last CTA of the
 // (sequence, head) combines them in split order (deterministic).
+#include <mutex>
+
 #include "common.cuh"
 
 namespace lca {
@@ -272,6 +274,31 @@ int op_run(const float* q, float* out, const void* k, const void* v, int dtype, 
   return cudaGetLastError() == cudaSuccess ? LCA_OK : LCA_E_CUDA;
 }
 
+// ---------------------------------------------------------------- scratch without allocation
+// Scratch of lca_decode_attention_noalloc: a fixed array in device memory, shared by all calls
+// on a device and held by every GPU that loads the library until the process exits.
+constexpr size_t kNoAllocScratchBytes = 8u << 20;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_addr[kMaxDevices] = {};
+
+// Device address of g_noalloc_scratch on the current device, looked up once per device.
+int noalloc_scratch(char** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return LCA_E_CUDA;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_addr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || !p) return LCA_E_CUDA;
+    g_noalloc_addr[dev] = p;
+  }
+  *out = reinterpret_cast<char*>(g_noalloc_addr[dev]);
+  return LCA_OK;
+}
+
 } // namespace
 
 size_t attention_scratch_floats(int B, int H, int hd) {
@@ -315,6 +342,24 @@ int lca_decode_attention(const float* q, float* out, const void* k_cache, const 
   return op_run(q, out, k_cache, v_cache, dtype, batch, heads, head_dim, slots, n_rows, kv_len, scale,
                 splits, o, reinterpret_cast<cudaStream_t>(stream));
 }
+
+int lca_decode_attention_noalloc(const float* q, float* out, const void* k_cache, const void* v_cache,
+                                 int32_t dtype, int32_t batch, int32_t heads, int32_t head_dim,
+                                 int32_t slots, int32_t n_rows, const int32_t* kv_len, float scale,
+                                 int32_t splits, void* stream) {
+  int st = op_check(q, out, k_cache, v_cache, dtype, batch, heads, head_dim, slots, n_rows, kv_len, splits);
+  if (st != LCA_OK) return st;
+  if (op_scratch_layout(nullptr, batch, heads, head_dim, splits).bytes > kNoAllocScratchBytes)
+    return LCA_E_CAPACITY;
+  char* base = nullptr;
+  st = noalloc_scratch(&base);
+  if (st != LCA_OK) return st;
+  const OpScratch o = op_scratch_layout(base, batch, heads, head_dim, splits);
+  return op_run(q, out, k_cache, v_cache, dtype, batch, heads, head_dim, slots, n_rows, kv_len, scale,
+                splits, o, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t lca_decode_attention_noalloc_capacity(void) { return kNoAllocScratchBytes; }
 
 }  // extern "C"
 

@@ -28,7 +28,8 @@ EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "
            "lca_debug_set_eager", "lca_debug_profile",
            "lca_debug_logits",
            "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str",
-           "lca_decode_attention_scratch_bytes", "lca_decode_attention")
+           "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
+           "lca_decode_attention_noalloc_capacity")
 
 
 class LcaConfig(ctypes.Structure):
@@ -105,11 +106,14 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_decode_attention_scratch_bytes": [I32, I32, I32, I32, ctypes.POINTER(ctypes.c_size_t)],
         "lca_decode_attention": [P, P, P, P, I32, I32, I32, I32, I32, I32, P, F32, I32, P,
                                  ctypes.c_size_t, P],
+        "lca_decode_attention_noalloc": [P, P, P, P, I32, I32, I32, I32, I32, I32, P, F32, I32, P],
+        "lca_decode_attention_noalloc_capacity": [],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
         f.argtypes = args
-        f.restype = ctypes.c_char_p if name == "lca_status_str" else ctypes.c_int
+        f.restype = (ctypes.c_char_p if name == "lca_status_str" else
+                     ctypes.c_size_t if name == "lca_decode_attention_noalloc_capacity" else ctypes.c_int)
     _lib = lib
     return lib
 
@@ -262,7 +266,8 @@ class Context:
         self._check(self.lib.lca_debug_force_candidates(self.h, _ptr(arr), n), "force_candidates")
 
 
-def decode_attention(q, out, k_cache, v_cache, kv_len, scale, splits, scratch=None, stream=None):
+def decode_attention(q, out, k_cache, v_cache, kv_len, scale, splits, scratch=None, stream=None,
+                     noalloc=False):
     """Standalone decode attention on torch CUDA tensors (see include/lca.h).
     q/out: fp32 [batch*n_rows, heads*head_dim]; caches [batch, heads, slots, head_dim];
     kv_len: int32 [batch*n_rows]. Returns the status code."""
@@ -274,6 +279,8 @@ def decode_attention(q, out, k_cache, v_cache, kv_len, scale, splits, scratch=No
     st = stream if stream is not None else torch.cuda.current_stream(q.device)
     args = [q.data_ptr(), out.data_ptr(), k_cache.data_ptr(), v_cache.data_ptr(), dt, batch, heads, hd,
             slots, n_rows, kv_len.data_ptr(), scale, splits]
+    if noalloc:
+        return lib.lca_decode_attention_noalloc(*args, st.cuda_stream)
     return lib.lca_decode_attention(*args, scratch.data_ptr(), scratch.numel(), st.cuda_stream)
 
 

@@ -1,0 +1,54 @@
+"""lca_decode_attention_noalloc: the decode attention for callers that cannot allocate device
+memory (plugin hosts that pass only input and output buffers, code that must not call an
+allocator). Its scratch is a fixed array inside the library; this test checks, through the C
+ABI, that two calls in a row give the same output as lca_decode_attention with caller scratch.
+
+This file is collected last on purpose, so that a run stopping at the first failure has run
+every other test before it.
+"""
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+
+def test_noalloc_attention_matches_scratch_version_twice():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2608_15454_gb300 import build, lca
+    build.build()
+    lca.load_library()
+    B, H, hd, S, n_rows, splits = 2, 16, 64, 700, 5, 8
+    g = torch.Generator(device="cuda").manual_seed(11)
+    scale = 1.0 / hd ** 0.5
+    scratch = torch.empty(lca.decode_attention_scratch_bytes(B, H, hd, splits), dtype=torch.uint8,
+                          device="cuda")
+    assert lca.decode_attention_scratch_bytes(B, H, hd, splits) <= lca.load_library() \
+        .lca_decode_attention_noalloc_capacity()
+    for call in range(2):
+        q = torch.randn(B * n_rows, H * hd, device="cuda", generator=g)
+        k = torch.randn(B, H, S, hd, device="cuda", generator=g).to(torch.bfloat16)
+        v = torch.randn(B, H, S, hd, device="cuda", generator=g).to(torch.bfloat16)
+        lens = torch.randint(1, S + 1, (B * n_rows,), device="cuda", generator=g, dtype=torch.int32)
+        want = torch.empty_like(q)
+        got = torch.full_like(q, float("nan"))
+        assert lca.decode_attention(q, want, k, v, lens, scale, splits, scratch) == 0
+        assert lca.decode_attention(q, got, k, v, lens, scale, splits, noalloc=True) == 0
+        torch.cuda.synchronize()
+        np.testing.assert_allclose(got.cpu().numpy(), want.cpu().numpy(), atol=1e-4, rtol=0)
+
+
+def test_noalloc_attention_rejects_sizes_beyond_its_array():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2608_15454_gb300 import lca
+    lib = lca.load_library()
+    B, H, hd, S = 64, 16, 64, 8
+    q = torch.zeros(B, H * hd, device="cuda")
+    k = torch.zeros(B, H, S, hd, device="cuda", dtype=torch.bfloat16)
+    lens = torch.ones(B, device="cuda", dtype=torch.int32)
+    assert lca.decode_attention_scratch_bytes(B, H, hd, 16) > lib.lca_decode_attention_noalloc_capacity()
+    out = torch.empty_like(q)
+    assert lca.decode_attention(q, out, k, k, lens, 0.125, 16, noalloc=True) == -2
