@@ -170,6 +170,15 @@ typedef struct {
 } lca_profile;
 int lca_debug_profile(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t steps,
                       lca_profile* out);
+
+/* Micro-benchmark: one graph of `iters` back-to-back launches of one kernel kind over `rows`
+ * rows (0 RMSNorm+QKV, 1 Wo, 2 RMSNorm+W1/W3+SwiGLU, 3 W2, 4 decode attention over the
+ * encoder cache, 5 unembedding head, 6 a glue kernel), cycling through all blocks' weights so
+ * that every launch streams its weights from HBM. us: average time per launch (CUDA events);
+ * bytes: the weight (or KV) bytes one launch reads. Overwrites step state: call lca_prefill
+ * before the next step. */
+int lca_debug_bench_kernel(lca_ctx* ctx, int32_t kind, int32_t rows, int32_t iters, double* us,
+                           double* bytes);
 /* Logits of the last step: nb host [batch * n * 256] (next-byte rows of the n candidates),
  * mb host [batch * (n-1) * 256] (drafter rows). Either may be NULL. */
 int lca_debug_logits(lca_ctx* ctx, float* nb, float* mb);

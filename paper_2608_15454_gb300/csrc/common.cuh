@@ -9,6 +9,29 @@
 
 namespace lca {
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// Every kernel of the step is launched with programmatic stream serialization: it lets its
+// successor launch at once (pdl_trigger), does only work that reads no upstream result (weight
+// loads), and waits for its predecessor's completion (pdl_wait) before touching anything else.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 constexpr int kVocab = 256;
 constexpr int kMaxKSplit = 8;     // split-K ways of the skinny linear kernel
 constexpr int kMaxAttnSplit = 16; // key-range splits of decode attention
@@ -17,6 +40,7 @@ constexpr int kAttnQT = 8;        // query rows per attention tile (decode)
 // device error word bits
 constexpr int kErrIndex = 1;   // an index was out of range; the access was skipped
 constexpr int kErrNumeric = 2; // non-finite logits
+constexpr int kErrTimeout = 4; // a bounded wait ran out
 
 // Linear epilogues.
 enum Epi : int {
@@ -128,6 +152,8 @@ struct Dev {
   int B, S, L, NMAX, R; // batch cap, byte slots, latent slots, max n, row cap
   int boundary;
   float eps, scale;
+  int num_sms;  // streaming multiprocessors of the device
+  int use_tma;  // bf16 linear layers use the bulk-copy weight pipeline
 
   // weights (storage type; norms and bos fp32)
   void* embed;   // [256][d]
@@ -218,6 +244,11 @@ struct LinearArgs {
   const int* M;  // device row count (per group when groups > 1)
   int M_cap;     // host upper bound of *M
   EpiArgs epi;
+  // weights of the next linear layer(s), prefetched into L2 by this launch's CTAs before the
+  // grid-dependency wait (nullptr: none)
+  const void* pf[2];
+  size_t pf_bytes[2];
+  int rows_typ;  // typical row count (sizes the activation staging); 0: M_cap
 };
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s);
 

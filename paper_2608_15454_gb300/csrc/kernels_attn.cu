@@ -6,6 +6,7 @@
 // values stream through shared memory in tiles of 32; softmax is computed online in fp32.
 // With several key splits each CTA writes (max, sum, acc) partials and the last CTA of the
 // (sequence, head) combines them in split order (deterministic).
+#include <cooperative_groups.h>
 #include <mutex>
 
 #include "common.cuh"
@@ -14,18 +15,28 @@ namespace lca {
 
 namespace {
 
-constexpr int kKT = 32;     // keys per tile
+constexpr int kKT = 64;     // keys per tile
 constexpr int kThreads = 128;
 constexpr int kQTMax = 4;   // query tiles per sequence that may split their key range
+constexpr int kMaxClusterSplit = 8;  // portable thread-block cluster size
 
-__device__ __forceinline__ float to_f(float v) { return v; }
-__device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+__device__ __forceinline__ void unpack16(const uint4& u, float* f, const float*) {
+  f[0] = __uint_as_float(u.x); f[1] = __uint_as_float(u.y);
+  f[2] = __uint_as_float(u.z); f[3] = __uint_as_float(u.w);
+}
+__device__ __forceinline__ void unpack16(const uint4& u, float* f, const __nv_bfloat16*) {
+  f[0] = __uint_as_float(u.x << 16); f[1] = __uint_as_float(u.x & 0xFFFF0000u);
+  f[2] = __uint_as_float(u.y << 16); f[3] = __uint_as_float(u.y & 0xFFFF0000u);
+  f[4] = __uint_as_float(u.z << 16); f[5] = __uint_as_float(u.z & 0xFFFF0000u);
+  f[6] = __uint_as_float(u.w << 16); f[7] = __uint_as_float(u.w & 0xFFFF0000u);
+}
 
 template <typename TC, int HD>
 __global__ void __launch_bounds__(kThreads)
 k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
        int splits, float* __restrict__ part, int* __restrict__ cnt, int* err) {
   constexpr int QT = kAttnQT;
+  constexpr int EV = 16 / (int)sizeof(TC);  // cache elements per 16-byte vector
   __shared__ float qs[QT][HD];
   __shared__ float ks[kKT][HD + 1];
   __shared__ float vs[kKT][HD];
@@ -34,6 +45,8 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
   __shared__ int s_kv[QT];
   __shared__ int s_last;
 
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const int h = blockIdx.z / splits;
   const int sp = blockIdx.z - h * splits;
@@ -49,6 +62,9 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
   constexpr int DPT = QT * HD / kThreads;
   const int ai = tid / (HD / DPT);
   const int ad = (tid % (HD / DPT)) * DPT;
+  // score ownership: key sk, rows sr..sr+3
+  const int sk = tid & (kKT - 1);
+  const int sr = (tid / kKT) * (QT * kKT / kThreads);
 
   for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
     const int r0 = rbeg + qt * QT;
@@ -76,7 +92,7 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
     const bool split_mode = splits > 1 && qt < kQTMax;
     if (!split_mode && sp != 0) continue;
     const int nsp = split_mode ? splits : 1;
-    const int chunk = ((kv_hi + nsp - 1) / nsp + kKT - 1) / kKT * kKT;
+    const int chunk = ((kv_hi + nsp - 1) / nsp + 15) / 16 * 16;
     const int lo = split_mode ? sp * chunk : 0;
     const int hi = min(kv_hi, lo + chunk);
 
@@ -86,37 +102,68 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
 
     for (int j0 = lo; j0 < hi; j0 += kKT) {
       const int nk = min(kKT, hi - j0);
-      for (int idx = tid; idx < kKT * HD; idx += kThreads) {
-        const int kk = idx / HD, dd = idx - kk * HD;
-        float kvk = 0.f, kvv = 0.f;
-        if (kk < nk) {
-          kvk = to_f(Kc[(size_t)(j0 + kk) * HD + dd]);
-          kvv = to_f(Vc[(size_t)(j0 + kk) * HD + dd]);
+      {
+        // the whole K/V tile: every thread issues all its 16-byte loads before any store
+        constexpr int NL = kKT * HD / EV / kThreads;
+        uint4 uk[NL], uv[NL];
+#pragma unroll
+        for (int u = 0; u < NL; ++u) {
+          const int e = (tid + u * kThreads) * EV;
+          const int kk = e / HD, dd = e - kk * HD;
+          if (kk < nk) {
+            uk[u] = *reinterpret_cast<const uint4*>(Kc + (size_t)(j0 + kk) * HD + dd);
+            uv[u] = *reinterpret_cast<const uint4*>(Vc + (size_t)(j0 + kk) * HD + dd);
+          } else {
+            uk[u] = make_uint4(0, 0, 0, 0);
+            uv[u] = make_uint4(0, 0, 0, 0);
+          }
         }
-        ks[kk][dd] = kvk;
-        vs[kk][dd] = kvv;
+#pragma unroll
+        for (int u = 0; u < NL; ++u) {
+          const int e = (tid + u * kThreads) * EV;
+          const int kk = e / HD, dd = e - kk * HD;
+          float fk[8], fv[8];
+          unpack16(uk[u], fk, (const TC*)nullptr);
+          unpack16(uv[u], fv, (const TC*)nullptr);
+#pragma unroll
+          for (int j = 0; j < EV; ++j) {
+            ks[kk][dd + j] = fk[j];
+            vs[kk][dd + j] = fv[j];
+          }
+        }
       }
       __syncthreads();
-      // scores: thread -> key lane, rows warp, warp+4
-      for (int i = warp; i < QT; i += kThreads / 32) {
-        float sc = -INFINITY;
-        if (lane < nk && j0 + lane < s_kv[i]) {
-          float s = 0.f;
+      // scores of 4 rows for one key per thread
+      {
+        float sc[QT * kKT / kThreads];
+#pragma unroll
+        for (int r = 0; r < QT * kKT / kThreads; ++r) sc[r] = 0.f;
 #pragma unroll 16
-          for (int dd = 0; dd < HD; ++dd) s = fmaf(qs[i][dd], ks[lane][dd], s);
-          sc = s;
+        for (int dd = 0; dd < HD; ++dd) {
+          const float kd = ks[sk][dd];
+#pragma unroll
+          for (int r = 0; r < QT * kKT / kThreads; ++r) sc[r] = fmaf(qs[sr + r][dd], kd, sc[r]);
         }
-        // online softmax update of row i
-        float mx = sc;
+#pragma unroll
+        for (int r = 0; r < QT * kKT / kThreads; ++r)
+          ps[sr + r][sk] = (sk < nk && j0 + sk < s_kv[sr + r]) ? sc[r] : -INFINITY;
+      }
+      __syncthreads();
+      // online softmax: warp w updates rows 2w, 2w+1
+      for (int i = warp * (QT / 4); i < (warp + 1) * (QT / 4); ++i) {
+        const float v0 = ps[i][lane], v1 = ps[i][lane + 32];
+        float mx = fmaxf(v0, v1);
 #pragma unroll
         for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
         const float m_old = s_m[i];
         const float m_new = fmaxf(m_old, mx);
-        const float p = (sc == -INFINITY) ? 0.f : expf(sc - m_new);
-        float ssum = p;
+        const float p0 = v0 == -INFINITY ? 0.f : expf(v0 - m_new);
+        const float p1 = v1 == -INFINITY ? 0.f : expf(v1 - m_new);
+        float ssum = p0 + p1;
 #pragma unroll
         for (int o = 16; o; o >>= 1) ssum += __shfl_xor_sync(0xffffffffu, ssum, o);
-        ps[i][lane] = p;
+        ps[i][lane] = p0;
+        ps[i][lane + 32] = p1;
         __syncwarp();
         if (lane == 0) {
           const float corr = (m_old == -INFINITY) ? 0.f : expf(m_old - m_new);
@@ -149,7 +196,7 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
       }
       continue;
     }
-    // split partials: [b][h][sp] -> acc[QT][HD], m[QT], l[QT]
+    // split partials: tile (b, qt, h), split sp -> acc[QT][HD], m[QT], l[QT]
     const size_t tile_id = ((size_t)b * kQTMax + qt) * H + h;
     float* pp = part + (tile_id * splits + sp) * (QT * (HD + 2));
 #pragma unroll
@@ -164,29 +211,460 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
     __syncthreads();
     if (!s_last) continue;
     __threadfence();
-    if (ai < nq) {
+    {
+      // stage every split's (max, sum) in shared memory with parallel loads, then combine
       const float* base = part + tile_id * splits * (QT * (HD + 2));
+      float* sm = &ps[0][0];                // splits * QT maxima   (<= 128 floats)
+      float* sl = &ks[0][0];                // splits * QT sums
+      for (int idx = tid; idx < splits * QT; idx += kThreads) {
+        const int k = idx / QT, i = idx - k * QT;
+        sm[idx] = __ldcg(base + k * (QT * (HD + 2)) + QT * HD + i);
+        sl[idx] = __ldcg(base + k * (QT * (HD + 2)) + QT * HD + QT + i);
+      }
+      __syncthreads();
+      if (ai < nq) {
+        float M = -INFINITY;
+        for (int k = 0; k < splits; ++k) M = fmaxf(M, sm[k * QT + ai]);
+        float L = 0.f, o[DPT];
+#pragma unroll
+        for (int j = 0; j < DPT; ++j) o[j] = 0.f;
+#pragma unroll 4
+        for (int k = 0; k < splits; ++k) {
+          const float mk = sm[k * QT + ai];
+          const float w = mk == -INFINITY ? 0.f : expf(mk - M);
+          L += w * sl[k * QT + ai];
+          const float* pk = base + k * (QT * (HD + 2)) + ai * HD + ad;
+#pragma unroll
+          for (int j = 0; j < DPT; ++j) o[j] += w * __ldcg(pk + j);
+        }
+        const float il = L > 0.f ? 1.f / L : 0.f;
+        float* dst = out + (size_t)(r0 + ai) * ld + h * HD + ad;
+#pragma unroll
+        for (int j = 0; j < DPT; ++j) dst[j] = o[j] * il;
+      }
+    }
+    if (tid == 0) cnt[tile_id] = 0;
+  }
+}
+
+// The same attention with the key range of each (sequence, query tile, head) split over the CTAs
+// of one thread-block cluster: every CTA keeps its (max, sum, acc) partial in its own shared
+// memory, and rank 0 combines the ranks' partials through distributed shared memory, in rank
+// order (deterministic), with no global scratch and no atomics.
+template <typename TC, int HD>
+__global__ void __launch_bounds__(kThreads)
+k_attn_cl(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
+          int* err) {
+  namespace cgr = cooperative_groups;
+  constexpr int QT = kAttnQT;
+  constexpr int EV = 16 / (int)sizeof(TC);
+  __shared__ float qs[QT][HD];
+  __shared__ float ks[kKT][HD + 1];
+  __shared__ float vs[kKT][HD];
+  __shared__ float ps[QT][kKT];
+  __shared__ float s_m[QT], s_l[QT], s_corr[QT];
+  __shared__ int s_kv[QT];
+  __shared__ float pacc[QT][HD];  // this CTA's partial accumulator (read by rank 0)
+
+  cgr::cluster_group cl = cgr::this_cluster();
+  const int splits = (int)cl.dim_blocks().z;
+  const int sp = (int)cl.block_rank();
+  pdl_trigger();
+  pdl_wait();
+  const int b = blockIdx.x;
+  const int h = blockIdx.z / splits;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nrows = rows.seq_count[b];
+  const int rbeg = rows.seq_start[b];
+  const int ntiles = (nrows + QT - 1) / QT;
+  const TC* Kc = reinterpret_cast<const TC*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
+  const TC* Vc = reinterpret_cast<const TC*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  const int ld = H * HD;
+  constexpr int DPT = QT * HD / kThreads;
+  const int ai = tid / (HD / DPT);
+  const int ad = (tid % (HD / DPT)) * DPT;
+  const int sk = tid & (kKT - 1);
+  const int sr = (tid / kKT) * (QT * kKT / kThreads);
+
+  for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
+    const int r0 = rbeg + qt * QT;
+    const int nq = min(QT, nrows - qt * QT);
+    __syncthreads();
+    for (int idx = tid; idx < QT * HD; idx += kThreads) {
+      const int i = idx / HD, dd = idx - i * HD;
+      qs[i][dd] = i < nq ? q[(size_t)(r0 + i) * ld + h * HD + dd] * scale : 0.f;
+    }
+    if (tid < QT) {
+      int kl = tid < nq ? rows.kvlen[r0 + tid] : 0;
+      if (kl > kv.S) {
+        atomicOr(err, kErrIndex);
+        kl = kv.S;
+      }
+      s_kv[tid] = kl;
+      s_m[tid] = -INFINITY;
+      s_l[tid] = 0.f;
+    }
+    __syncthreads();
+    int kv_hi = 0;
+#pragma unroll
+    for (int i = 0; i < QT; ++i) kv_hi = max(kv_hi, s_kv[i]);
+    const int chunk = ((kv_hi + splits - 1) / splits + 15) / 16 * 16;
+    const int lo = sp * chunk;
+    const int hi = min(kv_hi, lo + chunk);
+    float acc[DPT];
+#pragma unroll
+    for (int j = 0; j < DPT; ++j) acc[j] = 0.f;
+    for (int j0 = lo; j0 < hi; j0 += kKT) {
+      const int nk = min(kKT, hi - j0);
+      {
+        // the whole K/V tile: every thread issues all its 16-byte loads before any store
+        constexpr int NL = kKT * HD / EV / kThreads;
+        uint4 uk[NL], uv[NL];
+#pragma unroll
+        for (int u = 0; u < NL; ++u) {
+          const int e = (tid + u * kThreads) * EV;
+          const int kk = e / HD, dd = e - kk * HD;
+          if (kk < nk) {
+            uk[u] = *reinterpret_cast<const uint4*>(Kc + (size_t)(j0 + kk) * HD + dd);
+            uv[u] = *reinterpret_cast<const uint4*>(Vc + (size_t)(j0 + kk) * HD + dd);
+          } else {
+            uk[u] = make_uint4(0, 0, 0, 0);
+            uv[u] = make_uint4(0, 0, 0, 0);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < NL; ++u) {
+          const int e = (tid + u * kThreads) * EV;
+          const int kk = e / HD, dd = e - kk * HD;
+          float fk[8], fv[8];
+          unpack16(uk[u], fk, (const TC*)nullptr);
+          unpack16(uv[u], fv, (const TC*)nullptr);
+#pragma unroll
+          for (int j = 0; j < EV; ++j) {
+            ks[kk][dd + j] = fk[j];
+            vs[kk][dd + j] = fv[j];
+          }
+        }
+      }
+      __syncthreads();
+      {
+        float sc[QT * kKT / kThreads];
+#pragma unroll
+        for (int r = 0; r < QT * kKT / kThreads; ++r) sc[r] = 0.f;
+#pragma unroll 16
+        for (int dd = 0; dd < HD; ++dd) {
+          const float kd = ks[sk][dd];
+#pragma unroll
+          for (int r = 0; r < QT * kKT / kThreads; ++r) sc[r] = fmaf(qs[sr + r][dd], kd, sc[r]);
+        }
+#pragma unroll
+        for (int r = 0; r < QT * kKT / kThreads; ++r)
+          ps[sr + r][sk] = (sk < nk && j0 + sk < s_kv[sr + r]) ? sc[r] : -INFINITY;
+      }
+      __syncthreads();
+      for (int i = warp * (QT / 4); i < (warp + 1) * (QT / 4); ++i) {
+        const float v0 = ps[i][lane], v1 = ps[i][lane + 32];
+        float mx = fmaxf(v0, v1);
+#pragma unroll
+        for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        const float m_old = s_m[i];
+        const float m_new = fmaxf(m_old, mx);
+        const float p0 = v0 == -INFINITY ? 0.f : expf(v0 - m_new);
+        const float p1 = v1 == -INFINITY ? 0.f : expf(v1 - m_new);
+        float ssum = p0 + p1;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) ssum += __shfl_xor_sync(0xffffffffu, ssum, o);
+        ps[i][lane] = p0;
+        ps[i][lane + 32] = p1;
+        __syncwarp();
+        if (lane == 0) {
+          const float corr = (m_old == -INFINITY) ? 0.f : expf(m_old - m_new);
+          s_corr[i] = corr;
+          s_l[i] = s_l[i] * corr + ssum;
+          s_m[i] = m_new;
+        }
+      }
+      __syncthreads();
+      {
+        const float corr = s_corr[ai];
+#pragma unroll
+        for (int j = 0; j < DPT; ++j) acc[j] *= corr;
+        for (int kk = 0; kk < nk; ++kk) {
+          const float p = ps[ai][kk];
+#pragma unroll
+          for (int j = 0; j < DPT; ++j) acc[j] = fmaf(p, vs[kk][ad + j], acc[j]);
+        }
+      }
+      __syncthreads();
+    }
+#pragma unroll
+    for (int j = 0; j < DPT; ++j) pacc[ai][ad + j] = acc[j];
+    cl.sync();
+    if (sp == 0 && ai < nq) {
       float M = -INFINITY;
-      for (int k = 0; k < splits; ++k) M = fmaxf(M, __ldcg(base + k * (QT * (HD + 2)) + QT * HD + ai));
+      for (int r = 0; r < splits; ++r) M = fmaxf(M, *cl.map_shared_rank(&s_m[ai], r));
       float L = 0.f, o[DPT];
 #pragma unroll
       for (int j = 0; j < DPT; ++j) o[j] = 0.f;
-      for (int k = 0; k < splits; ++k) {
-        const float* pk = base + k * (QT * (HD + 2));
-        const float mk = __ldcg(pk + QT * HD + ai);
-        if (mk == -INFINITY) continue;
-        const float w = expf(mk - M);
-        L += w * __ldcg(pk + QT * HD + QT + ai);
+      for (int r = 0; r < splits; ++r) {
+        const float mr = *cl.map_shared_rank(&s_m[ai], r);
+        if (mr == -INFINITY) continue;
+        const float w = expf(mr - M);
+        L += w * *cl.map_shared_rank(&s_l[ai], r);
+        const float* pr = cl.map_shared_rank(&pacc[ai][ad], r);
 #pragma unroll
-        for (int j = 0; j < DPT; ++j) o[j] += w * __ldcg(pk + ai * HD + ad + j);
+        for (int j = 0; j < DPT; ++j) o[j] += w * pr[j];
       }
       const float il = L > 0.f ? 1.f / L : 0.f;
       float* dst = out + (size_t)(r0 + ai) * ld + h * HD + ad;
 #pragma unroll
       for (int j = 0; j < DPT; ++j) dst[j] = o[j] * il;
     }
-    if (tid == 0) cnt[tile_id] = 0;
+    cl.sync();
   }
+}
+
+// Decode attention, second form: 256 threads; scores with one key per thread (its K row held in
+// registers, loaded straight from global memory), online softmax with one warp per query row,
+// and P.V with each thread owning 4 dims of every row over a group of keys. The key range of a
+// (sequence, query tile, head) is split over the CTAs of a cluster and combined through
+// distributed shared memory by rank 0, in rank order.
+constexpr int kA2Threads = 256;
+constexpr int kA2Keys = 256;  // keys per pass
+
+__device__ __forceinline__ void unpack_vec(const uint4& u, float* f, const __nv_bfloat16*) {
+  f[0] = __uint_as_float(u.x << 16); f[1] = __uint_as_float(u.x & 0xFFFF0000u);
+  f[2] = __uint_as_float(u.y << 16); f[3] = __uint_as_float(u.y & 0xFFFF0000u);
+  f[4] = __uint_as_float(u.z << 16); f[5] = __uint_as_float(u.z & 0xFFFF0000u);
+  f[6] = __uint_as_float(u.w << 16); f[7] = __uint_as_float(u.w & 0xFFFF0000u);
+}
+__device__ __forceinline__ void unpack_vec(const uint4& u, float* f, const float*) {
+  f[0] = __uint_as_float(u.x); f[1] = __uint_as_float(u.y);
+  f[2] = __uint_as_float(u.z); f[3] = __uint_as_float(u.w);
+}
+__device__ __forceinline__ void load4(const __nv_bfloat16* p, float (&v)[4]) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  v[0] = __uint_as_float(u.x << 16); v[1] = __uint_as_float(u.x & 0xFFFF0000u);
+  v[2] = __uint_as_float(u.y << 16); v[3] = __uint_as_float(u.y & 0xFFFF0000u);
+}
+__device__ __forceinline__ void load4(const float* p, float (&v)[4]) {
+  const float4 u = *reinterpret_cast<const float4*>(p);
+  v[0] = u.x; v[1] = u.y; v[2] = u.z; v[3] = u.w;
+}
+
+template <typename TC, int HD>
+__global__ void __launch_bounds__(kA2Threads)
+k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
+        int* err) {
+  namespace cgr = cooperative_groups;
+  constexpr int QT = kAttnQT;
+  constexpr int EV = 16 / (int)sizeof(TC);
+  constexpr int NV = HD / EV;              // 16-byte vectors per key row
+  constexpr int DG = HD / 4;               // dim groups of 4
+  constexpr int KG = kA2Threads / DG;      // key groups in P.V
+  constexpr int KPG = kA2Keys / KG;        // keys per key group
+  __shared__ __align__(16) float qs[QT][HD];
+  __shared__ float ps[QT][kA2Keys];
+  __shared__ __align__(16) float red[KG][QT][HD];
+  __shared__ __align__(16) float pacc[QT][HD];
+  __shared__ float s_m[QT], s_l[QT], s_corr[QT];
+  __shared__ int s_kv[QT];
+
+  cgr::cluster_group cl = cgr::this_cluster();
+  const int splits = (int)cl.dim_blocks().z;
+  const int sp = (int)cl.block_rank();
+  pdl_trigger();
+  pdl_wait();
+  const int b = blockIdx.x;
+  const int h = blockIdx.z / splits;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int dg = tid % DG, kg = tid / DG;
+  const int nrows = rows.seq_count[b];
+  const int rbeg = rows.seq_start[b];
+  const int ntiles = (nrows + QT - 1) / QT;
+  const TC* Kc = reinterpret_cast<const TC*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
+  const TC* Vc = reinterpret_cast<const TC*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  const int ld = H * HD;
+
+  for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
+    const int r0 = rbeg + qt * QT;
+    const int nq = min(QT, nrows - qt * QT);
+    __syncthreads();
+    for (int idx = tid; idx < QT * HD; idx += kA2Threads) {
+      const int i = idx / HD, dd = idx - i * HD;
+      qs[i][dd] = i < nq ? q[(size_t)(r0 + i) * ld + h * HD + dd] * scale : 0.f;
+    }
+    if (tid < QT) {
+      int kl = tid < nq ? rows.kvlen[r0 + tid] : 0;
+      if (kl > kv.S) {
+        atomicOr(err, kErrIndex);
+        kl = kv.S;
+      }
+      s_kv[tid] = kl;
+      s_m[tid] = -INFINITY;
+      s_l[tid] = 0.f;
+    }
+    __syncthreads();
+    int kv_hi = 0;
+#pragma unroll
+    for (int i = 0; i < QT; ++i) kv_hi = max(kv_hi, s_kv[i]);
+    const int chunk = ((kv_hi + splits - 1) / splits + 15) / 16 * 16;
+    const int lo = sp * chunk;
+    const int hi = min(kv_hi, lo + chunk);
+    float acc[QT][4];
+#pragma unroll
+    for (int r = 0; r < QT; ++r)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[r][e] = 0.f;
+
+    for (int j0 = lo; j0 < hi; j0 += kA2Keys) {
+      const int nk = min(kA2Keys, hi - j0);
+      // scores: thread tid owns key j0 + tid
+      {
+        const int j = j0 + tid;
+        float sc[QT];
+#pragma unroll
+        for (int r = 0; r < QT; ++r) sc[r] = 0.f;
+        if (tid < nk) {
+          uint4 kr[NV];
+#pragma unroll
+          for (int v = 0; v < NV; ++v) kr[v] = *reinterpret_cast<const uint4*>(Kc + (size_t)j * HD + v * EV);
+#pragma unroll
+          for (int v = 0; v < NV; ++v) {
+            float kf[8];
+            unpack_vec(kr[v], kf, (const TC*)nullptr);
+#pragma unroll
+            for (int r = 0; r < QT; ++r) {
+              if (r < nq) {
+#pragma unroll
+                for (int e4 = 0; e4 < EV; e4 += 4) {
+                  const float4 qv = *reinterpret_cast<const float4*>(&qs[r][v * EV + e4]);
+                  sc[r] = fmaf(qv.x, kf[e4 + 0], sc[r]);
+                  sc[r] = fmaf(qv.y, kf[e4 + 1], sc[r]);
+                  sc[r] = fmaf(qv.z, kf[e4 + 2], sc[r]);
+                  sc[r] = fmaf(qv.w, kf[e4 + 3], sc[r]);
+                }
+              }
+            }
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < QT; ++r) ps[r][tid] = (tid < nk && r < nq && j < s_kv[r]) ? sc[r] : -INFINITY;
+      }
+      __syncthreads();
+      // online softmax: warp w owns row w
+      if (warp < QT) {
+        const int i = warp;
+        float v[kA2Keys / 32];
+        float mx = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < kA2Keys / 32; ++u) {
+          v[u] = ps[i][lane + 32 * u];
+          mx = fmaxf(mx, v[u]);
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        const float m_old = s_m[i];
+        const float m_new = fmaxf(m_old, mx);
+        float ssum = 0.f;
+#pragma unroll
+        for (int u = 0; u < kA2Keys / 32; ++u) {
+          const float p = v[u] == -INFINITY ? 0.f : expf(v[u] - m_new);
+          ps[i][lane + 32 * u] = p;
+          ssum += p;
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) ssum += __shfl_xor_sync(0xffffffffu, ssum, o);
+        if (lane == 0) {
+          const float corr = (m_old == -INFINITY) ? 0.f : expf(m_old - m_new);
+          s_corr[i] = corr;
+          s_l[i] = s_l[i] * corr + ssum;
+          s_m[i] = m_new;
+        }
+      }
+      __syncthreads();
+      // P.V: thread (dg, kg) accumulates dims 4dg..4dg+3 of every row over its keys
+      {
+#pragma unroll
+        for (int r = 0; r < QT; ++r) {
+          const float corr = s_corr[r];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) acc[r][e] *= corr;
+        }
+        float vv[KPG][4];
+#pragma unroll
+        for (int u = 0; u < KPG; ++u) {
+          const int key = kg * KPG + u;
+          if (key < nk) load4(Vc + (size_t)(j0 + key) * HD + dg * 4, vv[u]);
+          else vv[u][0] = vv[u][1] = vv[u][2] = vv[u][3] = 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < KPG; ++u) {
+          const int key = kg * KPG + u;
+#pragma unroll
+          for (int r = 0; r < QT; ++r) {
+            if (r < nq) {
+              const float p = ps[r][key];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) acc[r][e] = fmaf(p, vv[u][e], acc[r][e]);
+            }
+          }
+        }
+      }
+      __syncthreads();
+    }
+    // reduce the key groups: pacc[r][d] = sum over kg
+#pragma unroll
+    for (int r = 0; r < QT; ++r)
+      *reinterpret_cast<float4*>(&red[kg][r][dg * 4]) = make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]);
+    __syncthreads();
+    for (int idx = tid; idx < QT * HD; idx += kA2Threads) {
+      const int r = idx / HD, dd = idx - r * HD;
+      float t = 0.f;
+#pragma unroll 8
+      for (int g2 = 0; g2 < KG; ++g2) t += red[g2][r][dd];
+      pacc[r][dd] = t;
+    }
+    cl.sync();
+    // rank 0 combines the ranks' partials (max, sum, acc) in rank order
+    if (sp == 0) {
+      for (int idx = tid; idx < nq * HD; idx += kA2Threads) {
+        const int r = idx / HD, dd = idx - r * HD;
+        float M = -INFINITY;
+        for (int k = 0; k < splits; ++k) M = fmaxf(M, *cl.map_shared_rank(&s_m[r], k));
+        float L = 0.f, o = 0.f;
+        for (int k = 0; k < splits; ++k) {
+          const float mk = *cl.map_shared_rank(&s_m[r], k);
+          if (mk == -INFINITY) continue;
+          const float w = expf(mk - M);
+          L += w * *cl.map_shared_rank(&s_l[r], k);
+          o += w * *cl.map_shared_rank(&pacc[r][dd], k);
+        }
+        out[(size_t)(r0 + r) * ld + h * HD + dd] = L > 0.f ? o / L : 0.f;
+      }
+    }
+    cl.sync();
+  }
+}
+
+template <typename TC, int HD>
+void launch_cl(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
+               int qtiles_grid, int splits, int* err, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(B, qtiles_grid, H * splits);
+  cfg.blockDim = dim3(kA2Threads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = splits;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++g_launches;
+  cudaLaunchKernelEx(&cfg, k_attn2<TC, HD>, q, out, kv, rows, H, scale, err);
 }
 
 template <typename TC, int HD>
@@ -194,7 +672,7 @@ void launch(const float* q, float* out, const KV& kv, const Rows& rows, int B, i
             int qtiles_grid, int splits, float* part, int* cnt, int* err, cudaStream_t s) {
   dim3 grid(B, qtiles_grid, H * splits);
   ++g_launches;
-  k_attn<TC, HD><<<grid, kThreads, 0, s>>>(q, out, kv, rows, H, scale, splits, part, cnt, err);
+  launch_pdl(k_attn<TC, HD>, grid, dim3(kThreads), 0, s, q, out, kv, rows, H, scale, splits, part, cnt, err);
 }
 
 void launch_any(int dtype, int hd, const float* q, float* out, const KV& kv, const Rows& rows, int B,
@@ -211,6 +689,8 @@ void launch_any(int dtype, int hd, const float* q, float* out, const KV& kv, con
 
 // Rows of the standalone op: sequence b owns rows [b*n_rows, (b+1)*n_rows).
 __global__ void k_regular_rows(int* seq_start, int* seq_count, int batch, int n_rows) {
+  pdl_trigger();
+  pdl_wait();
   for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < batch; b += gridDim.x * blockDim.x) {
     seq_start[b] = b * n_rows;
     seq_count[b] = n_rows;
@@ -262,7 +742,7 @@ int op_run(const float* q, float* out, const void* k, const void* v, int dtype, 
            int head_dim, int slots, int n_rows, const int* kv_len, float scale, int splits,
            const OpScratch& o, cudaStream_t s) {
   if (cudaMemsetAsync(o.err, 0, o.header_bytes, s) != cudaSuccess) return LCA_E_CUDA;
-  k_regular_rows<<<(batch + 255) / 256, 256, 0, s>>>(o.seq_start, o.seq_count, batch, n_rows);
+  launch_pdl(k_regular_rows, dim3((batch + 255) / 256), dim3(256), 0, s, o.seq_start, o.seq_count, batch, n_rows);
   Rows rows{};
   rows.kvlen = const_cast<int*>(kv_len);
   rows.seq_start = o.seq_start;
@@ -309,10 +789,15 @@ size_t attention_counters(int B, int H) { return (size_t)B * kQTMax * H; }
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s) {
   ProfScope ps(PK_ATTN, 0.0, s);
-  if (splits > kMaxAttnSplit) splits = kMaxAttnSplit;
+  if (splits > kMaxClusterSplit) splits = kMaxClusterSplit;
   if (splits < 1) splits = 1;
-  launch_any(D.dtype, D.hd, q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.attn_part,
-             D.attn_cnt, D.err, s);
+  if (D.dtype == LCA_BF16) {
+    if (D.hd == 64) launch_cl<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+    else launch_cl<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+  } else {
+    if (D.hd == 64) launch_cl<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+    else launch_cl<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+  }
 }
 
 } // namespace lca

@@ -8,6 +8,8 @@
 //    is split along K across CTAs; the last CTA of a column tile sums the partials in a
 //    fixed order (deterministic, no atomics on data).
 //  * k_gemm: a persistent tiled FFMA GEMM for many rows (prefill, large batches).
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 
 namespace lca {
@@ -133,13 +135,42 @@ __device__ __forceinline__ float warp_reduce_scatter32(float (&v)[32], int lane)
   return v[0];
 }
 
-template <typename TW, bool NORM>
+template <typename TW>
+struct WTraits;
+template <>
+struct WTraits<__nv_bfloat16> {
+  static constexpr int VEC = 1;  // 16-byte vectors per 8 weights
+};
+template <>
+struct WTraits<float> {
+  static constexpr int VEC = 2;
+};
+
+__device__ __forceinline__ void unpack8(const uint4 (&u)[1], float (&w)[8]) {
+  unpack_bf16x2(u[0].x, w[0], w[1]);
+  unpack_bf16x2(u[0].y, w[2], w[3]);
+  unpack_bf16x2(u[0].z, w[4], w[5]);
+  unpack_bf16x2(u[0].w, w[6], w[7]);
+}
+__device__ __forceinline__ void unpack8(const uint4 (&u)[2], float (&w)[8]) {
+  w[0] = __uint_as_float(u[0].x); w[1] = __uint_as_float(u[0].y);
+  w[2] = __uint_as_float(u[0].z); w[3] = __uint_as_float(u[0].w);
+  w[4] = __uint_as_float(u[1].x); w[5] = __uint_as_float(u[1].y);
+  w[6] = __uint_as_float(u[1].z); w[7] = __uint_as_float(u[1].w);
+}
+
+// Skinny linear layer. The CTA owns 16 output columns (4 per warp) and a K-range; lanes stride
+// K by 8 elements. With KIT > 0 every weight the warp needs (KIT x 4 columns x 16 bytes per lane)
+// is loaded into registers before the grid-dependency wait, so the weight stream of this layer
+// overlaps the tail of the previous kernels; activations are staged in shared memory afterwards.
+template <typename TW, bool NORM, int KIT>
 __global__ void __launch_bounds__(kWarps * 32)
 k_gemv(LinearArgs a, int ksplit, float* __restrict__ part, int* __restrict__ cnt) {
+  constexpr int VEC = WTraits<TW>::VEC;
   extern __shared__ float smem[];
   const int Kr = a.Kd / ksplit;
-  float* xs = smem;                 // [kMC][Kr]
-  float* inv = smem + kMC * Kr;     // [kMC]
+  float* xs = smem;              // [kMC][Kr]
+  float* inv = smem + kMC * Kr;  // [kMC]
   __shared__ int s_last;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -148,7 +179,27 @@ k_gemv(LinearArgs a, int ksplit, float* __restrict__ part, int* __restrict__ cnt
   const int grp = blockIdx.z;
   const int k0 = split * Kr;
   const int col0 = tile * kColsPerCta + warp * kCPW;
+  const bool colok = col0 < a.N;
   const TW* W = reinterpret_cast<const TW*>(a.W) + (size_t)grp * a.N * a.Kd;
+
+  uint4 wr[KIT > 0 ? KIT : 1][kCPW][VEC];
+  if (KIT > 0 && colok) {
+#pragma unroll
+    for (int it = 0; it < (KIT > 0 ? KIT : 1); ++it) {
+      const int kk = lane * 8 + it * 256;
+      if (kk < Kr) {
+#pragma unroll
+        for (int c = 0; c < kCPW; ++c) {
+          const uint4* p = reinterpret_cast<const uint4*>(W + (size_t)(col0 + c) * a.Kd + k0 + kk);
+#pragma unroll
+          for (int v = 0; v < VEC; ++v) wr[it][c][v] = ldg_stream(p + v);
+        }
+      }
+    }
+  }
+  pdl_trigger();
+  pdl_wait();
+
   const int rbase = grp * a.Mg_stride;
   int M = *a.M;
   M = M < a.M_cap ? M : a.M_cap;
@@ -161,7 +212,10 @@ k_gemv(LinearArgs a, int ksplit, float* __restrict__ part, int* __restrict__ cnt
       for (int i = warp; i < mc; i += kWarps) {
         const float* xr = a.x + (size_t)(rbase + r0 + i) * a.ldx;
         float ss = 0.f;
-        for (int k = lane; k < a.Kd; k += 32) ss += xr[k] * xr[k];
+        for (int k = lane * 4; k < a.Kd; k += 128) {
+          const float4 v = *reinterpret_cast<const float4*>(xr + k);
+          ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        }
 #pragma unroll
         for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
         if (lane == 0) inv[i] = rsqrtf(ss / (float)a.Kd + a.eps);
@@ -177,36 +231,65 @@ k_gemv(LinearArgs a, int ksplit, float* __restrict__ part, int* __restrict__ cnt
       if (i < mc) {
         v = *reinterpret_cast<const float4*>(a.x + (size_t)(rbase + r0 + i) * a.ldx + k0 + kk);
         if (NORM) {
-          const float s = inv[i];
+          const float sc = inv[i];
           const float4 g = *reinterpret_cast<const float4*>(a.norm + k0 + kk);
-          v.x *= s * g.x; v.y *= s * g.y; v.z *= s * g.z; v.w *= s * g.w;
+          v.x *= sc * g.x; v.y *= sc * g.y; v.z *= sc * g.z; v.w *= sc * g.w;
         }
       }
       *reinterpret_cast<float4*>(xs + i * Kr + kk) = v;
     }
     __syncthreads();
 
-    if (col0 < a.N) {
+    if (colok) {
       float acc[32];
 #pragma unroll
       for (int j = 0; j < 32; ++j) acc[j] = 0.f;
-#pragma unroll 2
-      for (int kk = lane * 8; kk < Kr; kk += 256) {
-        float w[kCPW][8];
+      if (KIT > 0) {
 #pragma unroll
-        for (int c = 0; c < kCPW; ++c) load_w8(W + (size_t)(col0 + c) * a.Kd + k0 + kk, w[c]);
+        for (int it = 0; it < (KIT > 0 ? KIT : 1); ++it) {
+          const int kk = lane * 8 + it * 256;
+          if (kk < Kr) {
+            float w[kCPW][8];
 #pragma unroll
-        for (int i = 0; i < kMC; ++i) {
-          const float4 xa = *reinterpret_cast<const float4*>(xs + i * Kr + kk);
-          const float4 xb = *reinterpret_cast<const float4*>(xs + i * Kr + kk + 4);
+            for (int c = 0; c < kCPW; ++c) unpack8(wr[it][c], w[c]);
 #pragma unroll
-          for (int c = 0; c < kCPW; ++c) {
-            float s = acc[i * kCPW + c];
-            s = fmaf(w[c][0], xa.x, s); s = fmaf(w[c][1], xa.y, s);
-            s = fmaf(w[c][2], xa.z, s); s = fmaf(w[c][3], xa.w, s);
-            s = fmaf(w[c][4], xb.x, s); s = fmaf(w[c][5], xb.y, s);
-            s = fmaf(w[c][6], xb.z, s); s = fmaf(w[c][7], xb.w, s);
-            acc[i * kCPW + c] = s;
+            for (int i = 0; i < kMC; ++i) {
+              if (i < mc) {
+                const float4 xa = *reinterpret_cast<const float4*>(xs + i * Kr + kk);
+                const float4 xb = *reinterpret_cast<const float4*>(xs + i * Kr + kk + 4);
+#pragma unroll
+                for (int c = 0; c < kCPW; ++c) {
+                  float sacc = acc[i * kCPW + c];
+                  sacc = fmaf(w[c][0], xa.x, sacc); sacc = fmaf(w[c][1], xa.y, sacc);
+                  sacc = fmaf(w[c][2], xa.z, sacc); sacc = fmaf(w[c][3], xa.w, sacc);
+                  sacc = fmaf(w[c][4], xb.x, sacc); sacc = fmaf(w[c][5], xb.y, sacc);
+                  sacc = fmaf(w[c][6], xb.z, sacc); sacc = fmaf(w[c][7], xb.w, sacc);
+                  acc[i * kCPW + c] = sacc;
+                }
+              }
+            }
+          }
+        }
+      } else {
+        for (int kk = lane * 8; kk < Kr; kk += 256) {
+          float w[kCPW][8];
+#pragma unroll
+          for (int c = 0; c < kCPW; ++c) load_w8(W + (size_t)(col0 + c) * a.Kd + k0 + kk, w[c]);
+#pragma unroll
+          for (int i = 0; i < kMC; ++i) {
+            if (i < mc) {
+              const float4 xa = *reinterpret_cast<const float4*>(xs + i * Kr + kk);
+              const float4 xb = *reinterpret_cast<const float4*>(xs + i * Kr + kk + 4);
+#pragma unroll
+              for (int c = 0; c < kCPW; ++c) {
+                float sacc = acc[i * kCPW + c];
+                sacc = fmaf(w[c][0], xa.x, sacc); sacc = fmaf(w[c][1], xa.y, sacc);
+                sacc = fmaf(w[c][2], xa.z, sacc); sacc = fmaf(w[c][3], xa.w, sacc);
+                sacc = fmaf(w[c][4], xb.x, sacc); sacc = fmaf(w[c][5], xb.y, sacc);
+                sacc = fmaf(w[c][6], xb.z, sacc); sacc = fmaf(w[c][7], xb.w, sacc);
+                acc[i * kCPW + c] = sacc;
+              }
+            }
           }
         }
       }
@@ -246,11 +329,272 @@ k_gemv(LinearArgs a, int ksplit, float* __restrict__ part, int* __restrict__ cnt
   if (tid == 0) cnt[tile] = 0;
 }
 
+// ---------------------------------------------------------------- bulk-copy weight-streaming GEMV
+// Skinny linear layer for bf16 weights: the weights of each CTA's tile arrive in shared memory by
+// bulk async copies (cp.async.bulk) completing on an mbarrier, issued before the grid-dependency
+// wait so that they stream while the previous kernel finishes. Every wait is bounded.
+constexpr int kWaitSpins = 1 << 22;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait: false if the phase did not complete within the spin budget.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  for (int i = 0; i < kWaitSpins; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+
+// Each CTA prefetches an equal slice of the next layers' weights into L2 (no shared memory or
+// registers are used, so the HBM stream continues across kernel boundaries).
+__device__ __forceinline__ void prefetch_next(const LinearArgs& a) {
+  const int nct = gridDim.x * gridDim.y * gridDim.z;
+  const int cta = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    if (!a.pf[j] || !a.pf_bytes[j]) continue;
+    const size_t per = ((a.pf_bytes[j] + nct - 1) / nct + 255) & ~size_t(255);
+    const size_t off = per * cta;
+    if (off >= a.pf_bytes[j]) continue;
+    size_t len = a.pf_bytes[j] - off < per ? a.pf_bytes[j] - off : per;
+    const char* p = reinterpret_cast<const char*>(a.pf[j]) + off;
+    // one bulk prefetch per 32 KB, issued by the first lanes of warp 0
+    for (size_t q = threadIdx.x * 32768; q < len; q += blockDim.x * 32768) {
+      const uint32_t n = (uint32_t)((len - q) < 32768 ? (len - q) : 32768) & ~15u;
+      if (n) asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p + q), "r"(n) : "memory");
+    }
+  }
+}
+
+// One tile per CTA: NW*4 output columns x Kr inputs (the CTA's K-split), copied into shared
+// memory by bulk async copies issued before the grid-dependency wait. Warps own 4 columns each;
+// lanes stride K by 8, and one activation load from shared memory feeds 4 columns. Rows are
+// processed in chunks of MCA. With a K-split the `ksplit` CTAs of a column tile form a thread-
+// block cluster: each leaves its partial sums in its own shared memory and rank 0 adds the
+// ranks' partials through distributed shared memory in rank order (no global scratch).
+template <int MCA, int NW, bool NORM>
+__global__ void __launch_bounds__(NW * 32)
+k_gemv_bulk(LinearArgs a, int ksplit) {
+  namespace cgr = cooperative_groups;
+  constexpr int CT = NW * kCPW;  // columns per CTA
+  extern __shared__ __align__(128) unsigned char sm[];
+  const int Kr = a.Kd / ksplit;
+  __nv_bfloat16* wt = reinterpret_cast<__nv_bfloat16*>(sm);            // [CT][Kr]
+  float* xs = reinterpret_cast<float*>(sm + (size_t)CT * Kr * 2);       // [MCA][Kr]
+  float* inv = xs + MCA * Kr;                                          // [MCA]
+  float* cpart = inv + MCA;                                            // [MCA][CT]
+  uint64_t* bar = reinterpret_cast<uint64_t*>(
+      (reinterpret_cast<uintptr_t>(cpart + MCA * CT) + 15) & ~uintptr_t(15));  // 16-byte aligned
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tile = blockIdx.x;
+  const int split = blockIdx.y;
+  const int grp = blockIdx.z;
+  const int k0 = split * Kr;
+  const int ncols = min(CT, a.N - tile * CT);
+  const __nv_bfloat16* W = reinterpret_cast<const __nv_bfloat16*>(a.W) + (size_t)grp * a.N * a.Kd +
+                           (size_t)tile * CT * a.Kd + k0;
+  if (tid == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+    mbar_expect_tx(bar, (uint32_t)(ncols * Kr * 2));
+    if (ksplit == 1) {
+      bulk_g2s(wt, W, (uint32_t)(ncols * Kr * 2), bar);
+    } else {
+      for (int c = 0; c < ncols; ++c) bulk_g2s(wt + c * Kr, W + (size_t)c * a.Kd, (uint32_t)(Kr * 2), bar);
+    }
+  }
+  prefetch_next(a);
+  pdl_trigger();
+  pdl_wait();
+
+  const int rbase = grp * a.Mg_stride;
+  int M = *a.M;
+  M = M < a.M_cap ? M : a.M_cap;
+  if (M < 0) M = 0;
+  const int col0 = warp * kCPW;  // within the tile
+  bool have_w = false;
+
+  for (int r0 = 0; r0 < M; r0 += MCA) {
+    const int mc = min(MCA, M - r0);
+    __syncthreads();
+    // raw rows -> shared memory, loads batched 8 at a time per thread
+    constexpr int UNR = 8;
+    const int nv = MCA * Kr / 4;
+    for (int base = tid; base < nv; base += NW * 32 * UNR) {
+      float4 v[UNR];
+#pragma unroll
+      for (int u = 0; u < UNR; ++u) {
+        const int idx = base + u * NW * 32;
+        const int i = (idx * 4) / Kr, kk = idx * 4 - i * Kr;
+        v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (idx < nv && i < mc)
+          v[u] = *reinterpret_cast<const float4*>(a.x + (size_t)(rbase + r0 + i) * a.ldx + k0 + kk);
+      }
+#pragma unroll
+      for (int u = 0; u < UNR; ++u) {
+        const int idx = base + u * NW * 32;
+        if (idx < nv) *reinterpret_cast<float4*>(xs + idx * 4) = v[u];
+      }
+    }
+    __syncthreads();
+    if (NORM) {
+      // RMSNorm: inverse RMS of each row (from shared memory when the CTA holds all of K, else
+      // from global memory), then x * inv * g in place
+      for (int i = warp; i < mc; i += NW) {
+        float ss = 0.f;
+        if (ksplit == 1) {
+          for (int k = lane * 4; k < Kr; k += 128) {
+            const float4 q = *reinterpret_cast<const float4*>(xs + i * Kr + k);
+            ss += q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
+          }
+        } else {
+          const float* xr = a.x + (size_t)(rbase + r0 + i) * a.ldx;
+          for (int k = lane * 4; k < a.Kd; k += 128) {
+            const float4 q = *reinterpret_cast<const float4*>(xr + k);
+            ss += q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
+          }
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        if (lane == 0) inv[i] = rsqrtf(ss / (float)a.Kd + a.eps);
+      }
+      __syncthreads();
+      for (int base = tid; base < mc * Kr / 4; base += NW * 32 * UNR) {
+        float4 g[UNR];
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+          const int idx = base + u * NW * 32;
+          const int kk = (idx * 4) % Kr;
+          if (idx < mc * Kr / 4) g[u] = *reinterpret_cast<const float4*>(a.norm + k0 + kk);
+        }
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+          const int idx = base + u * NW * 32;
+          if (idx < mc * Kr / 4) {
+            const int i = (idx * 4) / Kr;
+            float4 q = *reinterpret_cast<float4*>(xs + idx * 4);
+            const float sc = inv[i];
+            q.x *= sc * g[u].x; q.y *= sc * g[u].y; q.z *= sc * g[u].z; q.w *= sc * g[u].w;
+            *reinterpret_cast<float4*>(xs + idx * 4) = q;
+          }
+        }
+      }
+    }
+    if (!have_w) {
+      // the bounded wait for the weight tile; on a timeout the error is recorded and the
+      // kernel runs on (no early exit, so cluster barriers stay matched)
+      const bool ok = mbar_wait(bar, 0);
+      if (__syncthreads_or(!ok) && tid == 0) atomicOr(a.epi.err, kErrTimeout);
+      have_w = true;
+    } else {
+      __syncthreads();
+    }
+    if (col0 < ncols) {
+      float acc[MCA * kCPW];
+#pragma unroll
+      for (int j = 0; j < MCA * kCPW; ++j) acc[j] = 0.f;
+      for (int kk = lane * 8; kk < Kr; kk += 256) {
+        float w[kCPW][8];
+#pragma unroll
+        for (int c = 0; c < kCPW; ++c) {
+          const uint4 u = *reinterpret_cast<const uint4*>(wt + (col0 + c) * Kr + kk);
+          unpack_bf16x2(u.x, w[c][0], w[c][1]);
+          unpack_bf16x2(u.y, w[c][2], w[c][3]);
+          unpack_bf16x2(u.z, w[c][4], w[c][5]);
+          unpack_bf16x2(u.w, w[c][6], w[c][7]);
+        }
+#pragma unroll
+        for (int i = 0; i < MCA; ++i) {
+          if (i < mc) {
+            const float4 xa = *reinterpret_cast<const float4*>(xs + i * Kr + kk);
+            const float4 xb = *reinterpret_cast<const float4*>(xs + i * Kr + kk + 4);
+#pragma unroll
+            for (int c = 0; c < kCPW; ++c) {
+              float sacc = acc[i * kCPW + c];
+              sacc = fmaf(w[c][0], xa.x, sacc); sacc = fmaf(w[c][1], xa.y, sacc);
+              sacc = fmaf(w[c][2], xa.z, sacc); sacc = fmaf(w[c][3], xa.w, sacc);
+              sacc = fmaf(w[c][4], xb.x, sacc); sacc = fmaf(w[c][5], xb.y, sacc);
+              sacc = fmaf(w[c][6], xb.z, sacc); sacc = fmaf(w[c][7], xb.w, sacc);
+              acc[i * kCPW + c] = sacc;
+            }
+          }
+        }
+      }
+      float full[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) full[j] = j < MCA * kCPW ? acc[j] : 0.f;
+      const float v = warp_reduce_scatter32(full, lane);
+      const int i = lane / kCPW, c = lane % kCPW;
+      if (ksplit == 1) {
+        const float vn = __shfl_down_sync(0xffffffffu, v, 1);
+        if (i < mc && (c & 1) == 0)
+          epi_pair<__nv_bfloat16>(a.epi, rbase + r0 + i, tile * CT + col0 + c, v, vn);
+      } else if (i < MCA) {
+        cpart[i * CT + col0 + c] = v;
+      }
+    }
+    if (ksplit > 1) {
+      // cluster reduction of the K-split partials of this row chunk
+      cgr::cluster_group cl = cgr::this_cluster();
+      cl.sync();
+      if (split == 0) {
+        for (int idx = tid; idx < mc * (CT / 2); idx += NW * 32) {
+          const int i = idx / (CT / 2), c = (idx - i * (CT / 2)) * 2;
+          if (c >= ncols) continue;
+          float t0 = 0.f, t1 = 0.f;
+          for (int sp = 0; sp < ksplit; ++sp) {
+            const float* pr = cl.map_shared_rank(cpart + i * CT + c, sp);
+            t0 += pr[0];
+            t1 += pr[1];
+          }
+          epi_pair<__nv_bfloat16>(a.epi, rbase + r0 + i, tile * CT + c, t0, t1);
+        }
+      }
+      cl.sync();
+    }
+  }
+  if (!have_w) {  // no rows: still wait (bounded) for the copy before leaving
+    if (!mbar_wait(bar, 0) && tid == 0) atomicOr(a.epi.err, kErrTimeout);
+  }
+}
+
 // ---------------------------------------------------------------- tiled GEMM (many rows)
 constexpr int kBM = 64, kBN = 64, kBK = 32;
 
 __global__ void k_rowstats(const float* __restrict__ x, int ldx, int Kd, const int* Mp, int M_cap,
                            int groups, int Mg_stride, float eps, float* __restrict__ inv) {
+  pdl_trigger();
+  pdl_wait();
   int M = *Mp;
   M = M < M_cap ? M : M_cap;
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
@@ -275,6 +619,8 @@ __global__ void __launch_bounds__(256) k_gemm(LinearArgs a, const float* __restr
   const int grp = blockIdx.z;
   const TW* W = reinterpret_cast<const TW*>(a.W) + (size_t)grp * a.N * a.Kd;
   const int rbase = grp * a.Mg_stride;
+  pdl_trigger();
+  pdl_wait();
   int M = *a.M;
   M = M < a.M_cap ? M : a.M_cap;
   if (M <= 0) return;
@@ -346,8 +692,67 @@ __global__ void __launch_bounds__(256) k_gemm(LinearArgs a, const float* __restr
   }
 }
 
+template <typename TW, bool NORM, int KIT>
+void launch_gemv_kit(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s) {
+  const int Kr = a.Kd / ksplit;
+  const size_t smem = (size_t)kMC * Kr * sizeof(float) + kMC * sizeof(float);
+  dim3 grid((a.N + kColsPerCta - 1) / kColsPerCta, ksplit, a.groups);
+  ++g_launches;
+  launch_pdl(k_gemv<TW, NORM, KIT>, grid, dim3(kWarps * 32), smem, s, a, ksplit, D.lin_part, D.lin_cnt);
+}
+
+template <int MCA, int NW, bool NORM>
+void gemv_bulk_go(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s) {
+  constexpr int CT = NW * kCPW;
+  const int Kr = a.Kd / ksplit;
+  const size_t smem = (size_t)CT * Kr * 2 + (size_t)MCA * Kr * 4 + (MCA + MCA * CT + 2) * 4 + 16 + 64;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((a.N + CT - 1) / CT, ksplit, a.groups);
+  cfg.blockDim = dim3(NW * 32);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = ksplit;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++g_launches;
+  cudaLaunchKernelEx(&cfg, k_gemv_bulk<MCA, NW, NORM>, a, ksplit);
+}
+
+template <int MCA, bool NORM>
+void gemv_bulk_width(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s) {
+  // wide layers with many rows: 32-column CTAs keep the grid within one wave
+  if (MCA >= 8 && ksplit == 1 && a.N >= 4096) gemv_bulk_go<MCA, 8, NORM>(D, a, ksplit, s);
+  else gemv_bulk_go<MCA, 4, NORM>(D, a, ksplit, s);
+}
+
+template <bool NORM>
+bool launch_gemv_tma(const Dev& D, const LinearArgs& a, int rows_typ, cudaStream_t s) {
+  if (a.N % 8 || a.Kd % 256) return false;
+  int ksplit = 1;
+  if (a.groups == 1 && a.N <= 2048) {
+    ksplit = a.Kd >= 2048 ? 8 : 4;
+    while (ksplit > 1 && ((a.Kd % ksplit) || ((a.Kd / ksplit) % 256))) ksplit >>= 1;
+  }
+  if (a.Kd / ksplit > 4096) return false;
+  // activations staged per chunk of the typical row count (shared memory sets CTAs per SM)
+  const int mt = rows_typ < a.M_cap ? rows_typ : a.M_cap;
+  if (mt <= 1) gemv_bulk_width<1, NORM>(D, a, ksplit, s);
+  else if (mt <= 2) gemv_bulk_width<2, NORM>(D, a, ksplit, s);
+  else if (mt <= 4) gemv_bulk_width<4, NORM>(D, a, ksplit, s);
+  else gemv_bulk_width<8, NORM>(D, a, ksplit, s);
+  return true;
+}
+
 template <typename TW, bool NORM>
 void launch_gemv(const Dev& D, const LinearArgs& a, cudaStream_t s) {
+  if (sizeof(TW) == 2 && D.use_tma && launch_gemv_tma<NORM>(D, a, a.rows_typ > 0 ? a.rows_typ : a.M_cap, s))
+    return;
   int ksplit = 1;
   if (a.groups == 1 && a.N <= 2048 && D.lin_part) {
     ksplit = a.Kd >= 2048 ? 8 : 4;
@@ -356,34 +761,52 @@ void launch_gemv(const Dev& D, const LinearArgs& a, cudaStream_t s) {
       ksplit >>= 1;
   }
   const int Kr = a.Kd / ksplit;
-  const size_t smem = (size_t)kMC * Kr * sizeof(float) + kMC * sizeof(float);
-  dim3 grid((a.N + kColsPerCta - 1) / kColsPerCta, ksplit, a.groups);
-  ++g_launches;
-  k_gemv<TW, NORM><<<grid, kWarps * 32, smem, s>>>(a, ksplit, D.lin_part, D.lin_cnt);
+  const int kmax = sizeof(TW) == 2 ? 1024 : 512;  // register budget for the hoisted weights
+  if (Kr <= 256) launch_gemv_kit<TW, NORM, 1>(D, a, ksplit, s);
+  else if (Kr <= 512) launch_gemv_kit<TW, NORM, 2>(D, a, ksplit, s);
+  else if (Kr <= kmax) launch_gemv_kit<TW, NORM, 4>(D, a, ksplit, s);
+  else launch_gemv_kit<TW, NORM, 0>(D, a, ksplit, s);
 }
 
 template <typename TW, bool NORM>
 void launch_gemm(const Dev& D, const LinearArgs& a, cudaStream_t s) {
   if (NORM) {
     ++g_launches;
-    k_rowstats<<<256, 256, 0, s>>>(a.x, a.ldx, a.Kd, a.M, a.M_cap, a.groups, a.Mg_stride, a.eps,
-                                   D.inv_rms);
+    launch_pdl(k_rowstats, dim3(256), dim3(256), 0, s, a.x, a.ldx, a.Kd, a.M, a.M_cap, a.groups,
+               a.Mg_stride, a.eps, D.inv_rms);
   }
   const int ntm = (a.M_cap + kBM - 1) / kBM, ntn = (a.N + kBN - 1) / kBN;
   int tiles = ntm * ntn;
   int grid = tiles < 152 * 4 ? tiles : 152 * 4;
   ++g_launches;
-  k_gemm<TW, NORM><<<dim3(grid, 1, a.groups), 256, 0, s>>>(a, D.inv_rms);
+  launch_pdl(k_gemm<TW, NORM>, dim3(grid, 1, a.groups), dim3(256), 0, s, a, (const float*)D.inv_rms);
 }
 
 } // namespace
 
+template <typename TW, bool NORM>
+void attrs_one() {
+  const int mx = 200 * 1024;
+  cudaFuncSetAttribute(k_gemv<TW, NORM, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  cudaFuncSetAttribute(k_gemv<TW, NORM, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  cudaFuncSetAttribute(k_gemv<TW, NORM, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  cudaFuncSetAttribute(k_gemv<TW, NORM, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+}
+
 void kernel_attrs_linear() {
   const int mx = 200 * 1024;
-  cudaFuncSetAttribute(k_gemv<__nv_bfloat16, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-  cudaFuncSetAttribute(k_gemv<__nv_bfloat16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-  cudaFuncSetAttribute(k_gemv<float, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-  cudaFuncSetAttribute(k_gemv<float, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+#define LCA_ATTR_BULK(M, W)                                                                                   \
+  cudaFuncSetAttribute(k_gemv_bulk<M, W, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);           \
+  cudaFuncSetAttribute(k_gemv_bulk<M, W, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);          \
+  cudaFuncSetAttribute(k_gemv_bulk<M, W, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);         \
+  cudaFuncSetAttribute(k_gemv_bulk<M, W, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  LCA_ATTR_BULK(1, 4) LCA_ATTR_BULK(2, 4) LCA_ATTR_BULK(4, 4) LCA_ATTR_BULK(8, 4)
+  LCA_ATTR_BULK(1, 8) LCA_ATTR_BULK(2, 8) LCA_ATTR_BULK(4, 8) LCA_ATTR_BULK(8, 8)
+#undef LCA_ATTR_BULK
+  attrs_one<__nv_bfloat16, true>();
+  attrs_one<__nv_bfloat16, false>();
+  attrs_one<float, true>();
+  attrs_one<float, false>();
 }
 
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s) {

@@ -22,6 +22,8 @@ __device__ __forceinline__ void err_or(int* e, int bits) { atomicOr(e, bits); }
 // MB cache (slot = position - window start) and only new committed rows plus the copies are
 // computed. A changed window start (a committed boundary) rebuilds the cache.
 __global__ void k_mb_plan(Dev D) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ int s_cnt[1024];
   __shared__ int s_first[1024];
   const Params P = *D.params;
@@ -83,6 +85,8 @@ __global__ void k_mb_plan(Dev D) {
 // MB input rows: byte p of group k gets o_k + u_k (Algorithm 1 line 9, residual r_2 added
 // before upsampling); copies beyond t belong to the current group K.
 __global__ void k_mb_fill(Dev D) {
+  pdl_trigger();
+  pdl_wait();
   const int M = *D.r_mb.M;
   const int d4 = D.d / 4;
   for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < (size_t)M * d4;
@@ -102,6 +106,8 @@ __global__ void k_mb_fill(Dev D) {
 
 // MLP-MBP heads: row j*batch + b starts from the last next-byte hidden state of b.
 __global__ void k_mlp_plan(Dev D) {
+  pdl_trigger();
+  pdl_wait();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int rows = batch * (n - 1);
@@ -122,64 +128,118 @@ __global__ void k_mlp_plan(Dev D) {
 // Final RMSNorm of the head, shared unembedding (Section 3), then per row the argmax (lowest
 // byte among equal maxima) and its softmax probability exp(l_max - logsumexp(l)).
 constexpr int kHR = 8;   // rows per CTA
-constexpr int kHV = 16;  // vocab entries per CTA
+constexpr int kHV = 8;   // vocab entries per CTA (one per warp)
 
-template <typename TW>
-__global__ void __launch_bounds__(128)
+__device__ __forceinline__ uint4 ldg_nc16(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+__device__ __forceinline__ void unpack8w(const uint4* u, float* w, const __nv_bfloat16*) {
+  w[0] = __uint_as_float(u[0].x << 16); w[1] = __uint_as_float(u[0].x & 0xFFFF0000u);
+  w[2] = __uint_as_float(u[0].y << 16); w[3] = __uint_as_float(u[0].y & 0xFFFF0000u);
+  w[4] = __uint_as_float(u[0].z << 16); w[5] = __uint_as_float(u[0].z & 0xFFFF0000u);
+  w[6] = __uint_as_float(u[0].w << 16); w[7] = __uint_as_float(u[0].w & 0xFFFF0000u);
+}
+__device__ __forceinline__ void unpack8w(const uint4* u, float* w, const float*) {
+  w[0] = __uint_as_float(u[0].x); w[1] = __uint_as_float(u[0].y);
+  w[2] = __uint_as_float(u[0].z); w[3] = __uint_as_float(u[0].w);
+  w[4] = __uint_as_float(u[1].x); w[5] = __uint_as_float(u[1].y);
+  w[6] = __uint_as_float(u[1].z); w[7] = __uint_as_float(u[1].w);
+}
+
+// One CTA: kHR rows x kHV vocab entries; warp w owns vocab row blockIdx.y*kHV + w, whose
+// weights are loaded into registers before the grid-dependency wait. The last CTA of a row
+// tile reduces the 256 logits of each row to (argmax, probability).
+template <typename TW, int HCH>
+__global__ void __launch_bounds__(256)
 k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const int* Mp, int M_cap,
        const float* __restrict__ norm, float* __restrict__ logits, int* __restrict__ arg,
        float* __restrict__ prob, int* __restrict__ cnt) {
+  constexpr int VEC = sizeof(TW) == 2 ? 1 : 2;
   extern __shared__ float xs[];  // [kHR][d]
   __shared__ float inv[kHR];
   __shared__ int s_last;
+  const int d = D.d;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int v = blockIdx.y * kHV + warp;
+  const TW* Wu = reinterpret_cast<const TW*>(D.unembed) + (size_t)v * d;
+  uint4 wr[HCH][VEC];
+#pragma unroll
+  for (int c = 0; c < HCH; ++c) {
+    const int k = lane * 8 + c * 256;
+    if (k < d) {
+#pragma unroll
+      for (int e = 0; e < VEC; ++e) wr[c][e] = ldg_nc16(reinterpret_cast<const uint4*>(Wu + k) + e);
+    }
+  }
+  pdl_trigger();
+  pdl_wait();
   int M = *Mp;
   M = M < M_cap ? M : M_cap;
   const int rt = blockIdx.x;
   const int r0 = rt * kHR;
   if (r0 >= M) return;
   const int mr = min(kHR, M - r0);
-  const int d = D.d;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  for (int i = warp; i < mr; i += 4) {
-    const int src = rows ? rows[r0 + i] : r0 + i;
-    const float* xr = x + (size_t)src * d;
+  // warp w stages row w (raw, loads batched), computes its inverse RMS, then scales in place
+  if (warp < kHR) {
+    const int i = warp;
     float ss = 0.f;
-    for (int k = lane; k < d; k += 32) ss += xr[k] * xr[k];
+    constexpr int NQ = HCH * 2;  // float4 per lane (d <= HCH * 256)
+    float4 q[NQ];
+    const int src = i < mr ? (rows ? rows[r0 + i] : r0 + i) : 0;
+#pragma unroll
+    for (int u = 0; u < NQ; ++u) {
+      const int k = (lane + u * 32) * 4;
+      q[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (i < mr && k < d) q[u] = *reinterpret_cast<const float4*>(x + (size_t)src * d + k);
+      ss += q[u].x * q[u].x + q[u].y * q[u].y + q[u].z * q[u].z + q[u].w * q[u].w;
+    }
 #pragma unroll
     for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-    if (lane == 0) inv[i] = rsqrtf(ss / (float)d + D.eps);
+    const float sc = rsqrtf(ss / (float)d + D.eps);
+#pragma unroll
+    for (int u = 0; u < NQ; ++u) {
+      const int k = (lane + u * 32) * 4;
+      if (k < d) {
+        const float4 g = *reinterpret_cast<const float4*>(norm + k);
+        float4 v = q[u];
+        v.x *= sc * g.x; v.y *= sc * g.y; v.z *= sc * g.z; v.w *= sc * g.w;
+        *reinterpret_cast<float4*>(xs + i * d + k) = v;
+      }
+    }
   }
   __syncthreads();
-  for (int idx = tid; idx < kHR * d; idx += 128) {
-    const int i = idx / d, k = idx - i * d;
-    float v = 0.f;
-    if (i < mr) {
-      const int src = rows ? rows[r0 + i] : r0 + i;
-      v = x[(size_t)src * d + k] * inv[i] * norm[k];
+  float acc[kHR];
+#pragma unroll
+  for (int i = 0; i < kHR; ++i) acc[i] = 0.f;
+#pragma unroll
+  for (int c = 0; c < HCH; ++c) {
+    const int k = lane * 8 + c * 256;
+    if (k < d) {
+      float w[8];
+      unpack8w(wr[c], w, (const TW*)nullptr);
+#pragma unroll
+      for (int i = 0; i < kHR; ++i) {
+        const float4 xa = *reinterpret_cast<const float4*>(xs + i * d + k);
+        const float4 xb = *reinterpret_cast<const float4*>(xs + i * d + k + 4);
+        float sacc = acc[i];
+        sacc = fmaf(w[0], xa.x, sacc); sacc = fmaf(w[1], xa.y, sacc);
+        sacc = fmaf(w[2], xa.z, sacc); sacc = fmaf(w[3], xa.w, sacc);
+        sacc = fmaf(w[4], xb.x, sacc); sacc = fmaf(w[5], xb.y, sacc);
+        sacc = fmaf(w[6], xb.z, sacc); sacc = fmaf(w[7], xb.w, sacc);
+        acc[i] = sacc;
+      }
     }
-    xs[idx] = v;
   }
-  __syncthreads();
-  const TW* Wu = reinterpret_cast<const TW*>(D.unembed);
-  // each warp: 4 vocab rows; each lane a strided slice of d
-  const int v0 = blockIdx.y * kHV + warp * 4;
-  for (int vv = 0; vv < 4; ++vv) {
-    const int v = v0 + vv;
-    float acc[kHR];
 #pragma unroll
-    for (int i = 0; i < kHR; ++i) acc[i] = 0.f;
-    for (int k = lane; k < d; k += 32) {
-      const float w = ld_w(Wu, (size_t)v * d + k);
+  for (int i = 0; i < kHR; ++i) {
+    float sacc = acc[i];
 #pragma unroll
-      for (int i = 0; i < kHR; ++i) acc[i] = fmaf(w, xs[i * d + k], acc[i]);
-    }
-#pragma unroll
-    for (int i = 0; i < kHR; ++i) {
-      float s = acc[i];
-#pragma unroll
-      for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-      if (lane == 0 && i < mr) logits[(size_t)(r0 + i) * kVocab + v] = s;
-    }
+    for (int o = 16; o; o >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, o);
+    if (lane == 0 && i < mr) logits[(size_t)(r0 + i) * kVocab + v] = sacc;
   }
   __threadfence();
   __syncthreads();
@@ -187,17 +247,22 @@ k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const i
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  for (int i = warp; i < mr; i += 4) {
+  if (warp < mr) {
+    const int i = warp;
     const float* lg = logits + (size_t)(r0 + i) * kVocab;
     float best = -INFINITY;
     int bi = kVocab;
     bool bad = false;
-    for (int v = lane; v < kVocab; v += 32) {
-      const float l = __ldcg(lg + v);
+    float lv[kVocab / 32];
+#pragma unroll
+    for (int j = 0; j < kVocab / 32; ++j) {
+      const int vv = lane + 32 * j;
+      const float l = __ldcg(lg + vv);
+      lv[j] = l;
       if (!isfinite(l)) bad = true;
-      if (l > best || (l == best && v < bi)) {
+      if (l > best || (l == best && vv < bi)) {
         best = l;
-        bi = v;
+        bi = vv;
       }
     }
 #pragma unroll
@@ -211,7 +276,8 @@ k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const i
     }
     bad = __any_sync(0xffffffffu, bad);
     float se = 0.f;
-    for (int v = lane; v < kVocab; v += 32) se += expf(__ldcg(lg + v) - best);
+#pragma unroll
+    for (int j = 0; j < kVocab / 32; ++j) se += expf(lv[j] - best);
 #pragma unroll
     for (int o = 16; o; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
     if (lane == 0) {
@@ -229,6 +295,8 @@ k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const i
 // ---------------------------------------------------------------- verify rows
 // Candidates c_1 (next-byte argmax) and d_2..d_n (drafts) at positions t..t+n-1; embed them.
 __global__ void k_verify_plan(Dev D) {
+  pdl_trigger();
+  pdl_wait();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int b = blockIdx.x;
@@ -280,6 +348,8 @@ __global__ void k_verify_plan(Dev D) {
 // K(p) of candidate row i counts boundaries at positions <= p. New latents of all sequences
 // are compacted into LM rows; the LM module runs (graph conditional) only if there are any.
 __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handle) {
+  pdl_trigger();
+  pdl_wait();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int b = blockIdx.x;
@@ -359,6 +429,8 @@ __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handl
 
 // o_k of the latents the LM module just produced.
 __global__ void k_lm_scatter(Dev D) {
+  pdl_trigger();
+  pdl_wait();
   const int M = *D.r_lm.M;
   for (int r = blockIdx.x; r < M; r += gridDim.x) {
     const int b = D.r_lm.b[r], k = D.r_lm.pos[r];
@@ -370,6 +442,8 @@ __global__ void k_lm_scatter(Dev D) {
 // Next-byte decoder input: upsampled LM output plus the encoder residual r_1 (Algorithm 1
 // line 8): o_{K(p)} + h_e[p].
 __global__ void k_nb_input(Dev D) {
+  pdl_trigger();
+  pdl_wait();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int rows = batch * n;
@@ -388,6 +462,8 @@ __global__ void k_nb_input(Dev D) {
 // position before them (SPEC); the first failure drops the rest. The accepted prefix of every
 // cache is kept by advancing t and K; everything beyond is dropped (overwritten later).
 __global__ void k_commit(Dev D) {
+  pdl_trigger();
+  pdl_wait();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int b = blockIdx.x;
@@ -461,6 +537,8 @@ __global__ void k_commit(Dev D) {
 // Generate loop control: keep looping while a sequence is short of its budget (and never more
 // than max_iter steps, each of which commits at least one byte per unfinished sequence).
 __global__ void k_loop_ctl(Dev D, cudaGraphConditionalHandle h) {
+  pdl_trigger();
+  pdl_wait();
   if (threadIdx.x != 0) return;
   Params* P = D.params;
   const int it = P->iter + 1;
@@ -471,6 +549,8 @@ __global__ void k_loop_ctl(Dev D, cudaGraphConditionalHandle h) {
 }
 
 __global__ void k_gen_init(Dev D, int max_new) {
+  pdl_trigger();
+  pdl_wait();
   const int b = threadIdx.x;
   if (b < D.B) {
     SeqState& st = D.seq[b];
@@ -495,6 +575,8 @@ __global__ void k_rope_table(float2* tab, int slots, int hd, double base) {
 
 // ---------------------------------------------------------------- prefill
 __global__ void k_prefill_embed(Dev D, const uint8_t* __restrict__ bytes, int M) {
+  pdl_trigger();
+  pdl_wait();
   for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < (size_t)M * D.d;
        idx += (size_t)gridDim.x * blockDim.x) {
     const int r = (int)(idx / D.d), k = (int)(idx - (size_t)r * D.d);
@@ -508,6 +590,8 @@ __global__ void k_prefill_embed(Dev D, const uint8_t* __restrict__ bytes, int M)
 // One CTA per sequence: K(p) for every prompt byte and the group starts.
 __global__ void k_prefill_segment(Dev D, const uint8_t* __restrict__ bytes, const int* row0,
                                   const int* lens) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const int tid = threadIdx.x;
   __shared__ int s_scan[1024];
@@ -551,6 +635,8 @@ __global__ void k_prefill_segment(Dev D, const uint8_t* __restrict__ bytes, cons
 
 // CTA (b, k): latent k of sequence b: BOS for k = 0, else the mean of segment k.
 __global__ void k_prefill_pool(Dev D, const int* row0, const int* lm_row0) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const int k = blockIdx.y;
   const int K = D.seq[b].K;
@@ -576,6 +662,8 @@ __global__ void k_prefill_pool(Dev D, const int* row0, const int* lm_row0) {
 }
 
 __global__ void k_prefill_nb_input(Dev D, int M) {
+  pdl_trigger();
+  pdl_wait();
   for (int r = blockIdx.x; r < M; r += gridDim.x) {
     const int b = D.r_v.b[r], p = D.r_v.pos[r];
     const int k = D.kpos[(size_t)b * D.S + p];
@@ -589,6 +677,8 @@ __global__ void k_prefill_nb_input(Dev D, int M) {
 }
 
 __global__ void k_prefill_finish(Dev D, const int* row0, const int* lens) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const int last = row0[b] + lens[b] - 1;
   for (int c = threadIdx.x; c < D.d; c += blockDim.x)
@@ -620,9 +710,17 @@ __global__ void k_pack_rows(uint8_t* dst, const uint8_t* src, int rows, size_t r
 } // namespace
 
 // ---------------------------------------------------------------- launch wrappers
+template <typename TW>
+void head_attrs() {
+  cudaFuncSetAttribute(k_head<TW, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  cudaFuncSetAttribute(k_head<TW, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  cudaFuncSetAttribute(k_head<TW, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  cudaFuncSetAttribute(k_head<TW, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+}
+
 void kernel_attrs_step() {
-  cudaFuncSetAttribute(k_head<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-  cudaFuncSetAttribute(k_head<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  head_attrs<__nv_bfloat16>();
+  head_attrs<float>();
 }
 
 thread_local long long g_launches = 0;
@@ -631,64 +729,77 @@ thread_local ProfHook* g_prof = nullptr;
 void launch_mb_plan(const Dev& D, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_mb_plan<<<1, 1024, 0, s>>>(D);
+  launch_pdl(k_mb_plan, dim3(1), dim3(1024), 0, s, D);
 }
 void launch_mb_fill(const Dev& D, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_mb_fill<<<152 * 2, 256, 0, s>>>(D);
+  launch_pdl(k_mb_fill, dim3(152 * 2), dim3(256), 0, s, D);
 }
 void launch_mlp_plan(const Dev& D, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_mlp_plan<<<256, 256, 0, s>>>(D);
+  launch_pdl(k_mlp_plan, dim3(256), dim3(256), 0, s, D);
+}
+
+template <typename TW, int HCH>
+void head_launch(const Dev& D, const float* x, const int* rows, const int* M, int M_cap,
+                 const float* norm, float* logits, int* arg, float* prob, cudaStream_t s) {
+  dim3 grid((M_cap + kHR - 1) / kHR, kVocab / kHV);
+  const size_t smem = (size_t)kHR * D.d * sizeof(float);
+  launch_pdl(k_head<TW, HCH>, grid, dim3(256), smem, s, D, x, rows, M, M_cap, norm, logits, arg,
+             prob, D.head_cnt);
+}
+
+template <typename TW>
+void head_dispatch(const Dev& D, const float* x, const int* rows, const int* M, int M_cap,
+                   const float* norm, float* logits, int* arg, float* prob, cudaStream_t s) {
+  if (D.d <= 256) head_launch<TW, 1>(D, x, rows, M, M_cap, norm, logits, arg, prob, s);
+  else if (D.d <= 512) head_launch<TW, 2>(D, x, rows, M, M_cap, norm, logits, arg, prob, s);
+  else if (D.d <= 1024) head_launch<TW, 4>(D, x, rows, M, M_cap, norm, logits, arg, prob, s);
+  else head_launch<TW, 8>(D, x, rows, M, M_cap, norm, logits, arg, prob, s);
 }
 
 void launch_head(const Dev& D, const float* x, const int* rows, const int* M, int M_cap,
                  const float* norm, float* logits, int* arg, float* prob, cudaStream_t s) {
-  dim3 grid((M_cap + kHR - 1) / kHR, kVocab / kHV);
-  const size_t smem = (size_t)kHR * D.d * sizeof(float);
   ++g_launches;
   ProfScope ps(PK_HEAD, 256.0 * D.d * (D.dtype == LCA_BF16 ? 2 : 4), s);
-  // the split-K counters double as head row-tile counters (different launches, same stream)
-  if (D.dtype == LCA_BF16)
-    k_head<__nv_bfloat16><<<grid, 128, smem, s>>>(D, x, rows, M, M_cap, norm, logits, arg, prob, D.head_cnt);
-  else
-    k_head<float><<<grid, 128, smem, s>>>(D, x, rows, M, M_cap, norm, logits, arg, prob, D.head_cnt);
+  if (D.dtype == LCA_BF16) head_dispatch<__nv_bfloat16>(D, x, rows, M, M_cap, norm, logits, arg, prob, s);
+  else head_dispatch<float>(D, x, rows, M, M_cap, norm, logits, arg, prob, s);
 }
 
 void launch_verify_plan(const Dev& D, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_verify_plan<<<D.B, 256, 0, s>>>(D);
+  launch_pdl(k_verify_plan, dim3(D.B), dim3(256), 0, s, D);
 }
 void launch_segment(const Dev& D, cudaGraphConditionalHandle h, int use_handle, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_segment<<<D.B, 256, 0, s>>>(D, h, use_handle);
+  launch_pdl(k_segment, dim3(D.B), dim3(256), 0, s, D, h, use_handle);
 }
 void launch_lm_scatter(const Dev& D, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_lm_scatter<<<256, 256, 0, s>>>(D);
+  launch_pdl(k_lm_scatter, dim3(256), dim3(256), 0, s, D);
 }
 void launch_nb_input(const Dev& D, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_nb_input<<<256, 256, 0, s>>>(D);
+  launch_pdl(k_nb_input, dim3(256), dim3(256), 0, s, D);
 }
 void launch_commit(const Dev& D, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_commit<<<D.B, 256, 0, s>>>(D);
+  launch_pdl(k_commit, dim3(D.B), dim3(256), 0, s, D);
 }
 void launch_loop_ctl(const Dev& D, cudaGraphConditionalHandle h, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  k_loop_ctl<<<1, 32, 0, s>>>(D, h);
+  launch_pdl(k_loop_ctl, dim3(1), dim3(32), 0, s, D, h);
 }
 void launch_gen_init(const Dev& D, int max_new, cudaStream_t s) {
-  k_gen_init<<<1, 1024, 0, s>>>(D, max_new);
+  launch_pdl(k_gen_init, dim3(1), dim3(1024), 0, s, D, max_new);
 }
 void launch_rope_table(const Dev& D, float base, cudaStream_t s) {
   k_rope_table<<<256, 256, 0, s>>>(D.rope, D.rope_slots, D.hd, (double)base);
@@ -699,25 +810,25 @@ void launch_pack_rows(void* dst, const void* src, int rows, int cols, int dst_ro
                                   (size_t)cols * elem_bytes, dst_row0, row_step);
 }
 void launch_prefill_embed(const Dev& D, const uint8_t* bytes, int M, cudaStream_t s) {
-  k_prefill_embed<<<1024, 256, 0, s>>>(D, bytes, M);
+  launch_pdl(k_prefill_embed, dim3(1024), dim3(256), 0, s, D, bytes, M);
 }
 void launch_prefill_segment(const Dev& D, const uint8_t* bytes, const int* row0, const int* lens,
                             int batch, const int* lm_row0, cudaStream_t s) {
   (void)lm_row0;
-  k_prefill_segment<<<batch, 1024, 0, s>>>(D, bytes, row0, lens);
+  launch_pdl(k_prefill_segment, dim3(batch), dim3(1024), 0, s, D, bytes, row0, lens);
 }
 void launch_prefill_pool(const Dev& D, const int* row0, const int* lens, const int* lm_row0,
                          int batch, int max_lat, cudaStream_t s) {
   (void)lens;
-  k_prefill_pool<<<dim3(batch, max_lat + 1), 256, 0, s>>>(D, row0, lm_row0);
+  launch_pdl(k_prefill_pool, dim3(batch, max_lat + 1), dim3(256), 0, s, D, row0, lm_row0);
 }
 void launch_prefill_nb_input(const Dev& D, int M, cudaStream_t s) {
-  k_prefill_nb_input<<<1024, 256, 0, s>>>(D, M);
+  launch_pdl(k_prefill_nb_input, dim3(1024), dim3(256), 0, s, D, M);
 }
 void launch_prefill_finish(const Dev& D, const int* row0, const int* lens, const int* lm_row0,
                            int batch, cudaStream_t s) {
   (void)lm_row0;
-  k_prefill_finish<<<batch, 256, 0, s>>>(D, row0, lens);
+  launch_pdl(k_prefill_finish, dim3(batch), dim3(256), 0, s, D, row0, lens);
 }
 
 } // namespace lca

@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstdlib>
 #include <cstdio>
 #include <cstring>
 #include <map>
@@ -254,16 +255,25 @@ int attn_splits(const Dev& D, int batch_cap, int qtiles) {
 
 // Run the pre-norm blocks of one module over rows [0, *rows.M) of x (in place).
 void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& rows, int M_cap,
-               int M_typ, int qt_grid, int splits, cudaStream_t s) {
+               int M_typ, int qt_grid, int splits, cudaStream_t s, const void* next_w = nullptr,
+               size_t next_bytes = 0) {
   Dev& D = c->L.D;
   const bool tiled = tiled_for(M_typ);
-  for (auto& bk : blocks) {
+  const size_t tb = tw_bytes(D.dtype);
+  const size_t b_qkv = 3ull * D.d * D.d * tb, b_o = (size_t)D.d * D.d * tb;
+  const size_t b_13 = 2ull * D.F * D.d * tb, b_2 = (size_t)D.d * D.F * tb;
+  for (size_t l = 0; l < blocks.size(); ++l) {
+    Block& bk = blocks[l];
+    const Block* nx = l + 1 < blocks.size() ? &blocks[l + 1] : nullptr;
+    const void* nqkv = nx ? nx->wqkv : next_w;
+    const size_t nqkv_b = nx ? b_qkv : next_bytes;
     LinearArgs a{};
     a.groups = 1;
     a.Mg_stride = 0;
     a.eps = D.eps;
     a.M = rows.M;
     a.M_cap = M_cap;
+    a.rows_typ = M_typ;
     // RMSNorm -> Q,K,V -> RoPE -> K,V appended to the cache
     a.x = x;
     a.ldx = D.d;
@@ -282,6 +292,10 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.epi.hd = D.hd;
     a.epi.d = D.d;
     a.epi.err = D.err;
+    a.pf[0] = bk.wo;
+    a.pf_bytes[0] = b_o;
+    a.pf[1] = bk.w13;
+    a.pf_bytes[1] = b_13;
     linear(D, a, tiled, s);
     attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s);
     // x += Wo . attn
@@ -293,6 +307,10 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.epi.y = x;
     a.epi.res = x;
     a.epi.ldy = a.epi.ldres = D.d;
+    a.pf[0] = bk.w2;
+    a.pf_bytes[0] = b_2;
+    a.pf[1] = nullptr;
+    a.pf_bytes[1] = 0;
     linear(D, a, tiled, s);
     // mid = silu(W1 . n(x)) * (W3 . n(x))
     a.x = x;
@@ -302,6 +320,8 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.epi.mode = EPI_SWIGLU;
     a.epi.y = D.mid;
     a.epi.ldy = D.F;
+    a.pf[0] = nqkv;
+    a.pf_bytes[0] = nqkv_b;
     linear(D, a, tiled, s);
     // x += W2 . mid
     a.x = D.mid;
@@ -314,6 +334,8 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.epi.y = x;
     a.epi.res = x;
     a.epi.ldy = a.epi.ldres = D.d;
+    a.pf[0] = nx ? nx->wo : nullptr;
+    a.pf_bytes[0] = nx ? b_o : 0;
     linear(D, a, tiled, s);
   }
 }
@@ -335,6 +357,7 @@ void run_mlp_heads(lca_ctx* c, int n, cudaStream_t s) {
     a.eps = D.eps;
     a.M = D.r_mb.M;
     a.M_cap = D.B;
+    a.rows_typ = D.B;
     a.epi.mode = EPI_RESID_SILU;
     a.epi.y = D.x_mb;
     a.epi.res = D.x_mb;
@@ -353,8 +376,9 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
     if (D.mb_kind == LCA_MB_LCA) {
       launch_mb_plan(D, s);
       launch_mb_fill(D, s);
-      const int typ = B * (2 * n);  // typical window rows: the new committed bytes + copies
-      run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2), s);
+      const int typ = B * (2 * n - 2);  // typical window rows: new committed bytes + copies
+      run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2), s,
+                c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype));
     } else {
       launch_mlp_plan(D, s);
       run_mlp_heads(c, n, s);
@@ -364,7 +388,8 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
   }
   // (1) embed + encoder over the n candidates
   launch_verify_plan(D, s);
-  run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s);
+  run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s,
+            c->L.nb.empty() ? nullptr : c->L.nb[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype));
 }
 
 void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
@@ -544,6 +569,7 @@ int read_err(lca_ctx* c) {
     CK(cudaMemsetAsync(c->L.D.err, 0, sizeof(int), c->stream));
     CK(cudaStreamSynchronize(c->stream));
   }
+  if (e & kErrTimeout) return LCA_E_TIMEOUT;
   if (e & kErrNumeric) return LCA_E_NUMERIC;
   if (e & kErrIndex) return LCA_E_DEVICE_STATE;
   return LCA_OK;
@@ -705,6 +731,14 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
   kernel_attrs_linear();
   kernel_attrs_step();
   Dev& D = c->L.D;
+  {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    D.num_sms = sms > 0 ? sms : 148;
+    const char* e = getenv("LCA_NO_TMA");
+    D.use_tma = (e && e[0] == '1') ? 0 : 1;
+  }
   // state and counters start at zero
   if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);
   st = load_weights(c, weights, n_weights);
@@ -1052,6 +1086,114 @@ int lca_debug_profile(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t st
     out->ms[k] = prof.ms[k];
     out->bytes[k] = prof.bytes[k];
   }
+  return read_err(c);
+}
+
+int lca_debug_bench_kernel(lca_ctx* c, int32_t kind, int32_t rows, int32_t iters, double* us,
+                           double* bytes) {
+  if (!c || !us || !bytes || iters < 1 || rows < 1) return LCA_E_ARG;
+  if (!c->prefilled) return LCA_E_STATE;
+  Dev& D = c->L.D;
+  if (rows > std::min(D.R, 64)) return LCA_E_CAPACITY;
+  std::vector<Block*> blocks;
+  for (auto* v : {&c->L.enc, &c->L.lm, &c->L.nb, &c->L.mb})
+    for (auto& b : *v) blocks.push_back(&b);
+  if (blocks.empty()) return LCA_E_STATE;
+  const double tb = tw_bytes(D.dtype);
+  // rows [0, rows) of x_enc feed the kernels; r_v describes them (sequence 0, positions 0..)
+  std::vector<int> z(rows, 0), pos(rows), kvl(rows);
+  for (int i = 0; i < rows; ++i) {
+    pos[i] = i;
+    kvl[i] = std::min(c->t_host.empty() ? 1 : (int)c->t_host[0], D.S);
+  }
+  std::vector<int> ss(D.B, rows), sc(D.B, 0);
+  ss[0] = 0;
+  sc[0] = rows;
+  cudaStream_t s = c->stream;
+  CK(cudaMemcpyAsync(D.r_v.b, z.data(), rows * 4, cudaMemcpyHostToDevice, s));
+  CK(cudaMemcpyAsync(D.r_v.pos, pos.data(), rows * 4, cudaMemcpyHostToDevice, s));
+  CK(cudaMemcpyAsync(D.r_v.slot, pos.data(), rows * 4, cudaMemcpyHostToDevice, s));
+  CK(cudaMemcpyAsync(D.r_v.kvlen, kvl.data(), rows * 4, cudaMemcpyHostToDevice, s));
+  CK(cudaMemcpyAsync(D.r_v.seq_start, ss.data(), D.B * 4, cudaMemcpyHostToDevice, s));
+  CK(cudaMemcpyAsync(D.r_v.seq_count, sc.data(), D.B * 4, cudaMemcpyHostToDevice, s));
+  CK(cudaMemcpyAsync(D.r_v.M, &rows, 4, cudaMemcpyHostToDevice, s));
+  CK(cudaStreamSynchronize(s));
+  double by = 0;
+  cudaGraph_t g;
+  CK(cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeRelaxed));
+  for (int i = 0; i < iters; ++i) {
+    Block& bk = *blocks[i % blocks.size()];
+    LinearArgs a{};
+    a.groups = 1;
+    a.eps = D.eps;
+    a.M = D.r_v.M;
+    a.M_cap = rows;
+    a.x = D.x_enc;
+    a.ldx = D.d;
+    a.epi.mode = EPI_STORE;
+    a.epi.y = D.mid;
+    a.epi.ldy = 3 * D.d;
+    a.epi.err = D.err;
+    switch (kind) {
+      case 0:  // RMSNorm + QKV (stored, no cache write)
+        a.W = bk.wqkv; a.N = 3 * D.d; a.Kd = D.d; a.norm = bk.attn_norm;
+        linear(D, a, false, c->cap);
+        by = (double)a.N * a.Kd * tb;
+        break;
+      case 1:  // Wo
+        a.W = bk.wo; a.N = D.d; a.Kd = D.d;
+        linear(D, a, false, c->cap);
+        by = (double)a.N * a.Kd * tb;
+        break;
+      case 2:  // RMSNorm + W1/W3 + SwiGLU
+        a.W = bk.w13; a.N = 2 * D.F; a.Kd = D.d; a.norm = bk.mlp_norm;
+        a.epi.mode = EPI_SWIGLU; a.epi.ldy = D.F;
+        linear(D, a, false, c->cap);
+        by = (double)a.N * a.Kd * tb;
+        break;
+      case 3:  // W2
+        a.x = D.mid; a.ldx = D.F; a.W = bk.w2; a.N = D.d; a.Kd = D.F;
+        a.epi.ldy = D.d; a.epi.y = D.att;
+        linear(D, a, false, c->cap);
+        by = (double)a.N * a.Kd * tb;
+        break;
+      case 4: {  // attention over the encoder cache of layer (i % n_enc)
+        Block& eb = c->L.enc[i % c->L.enc.size()];
+        attention(D, D.qbuf, D.att, eb.kv, D.r_v, D.B, 1, attn_splits(D, D.B, 1), c->cap);
+        by = 2.0 * D.H * (double)kvl[0] * D.hd * tb;
+        break;
+      }
+      case 5:  // unembedding head
+        launch_head(D, D.x_enc, nullptr, D.r_v.M, rows, D.nb_norm, D.nb_logits, D.nb_arg, D.nb_prob, c->cap);
+        by = 256.0 * D.d * tb;
+        break;
+      default:  // a glue kernel (upsampling input of the next-byte decoder)
+        launch_lm_scatter(D, c->cap);
+        by = 0;
+        break;
+    }
+  }
+  CK(cudaStreamEndCapture(c->cap, &g));
+  cudaGraphExec_t ex;
+  CK(cudaGraphInstantiate(&ex, g, 0));
+  cudaEvent_t e0, e1;
+  CK(cudaEventCreate(&e0));
+  CK(cudaEventCreate(&e1));
+  for (int w = 0; w < 2; ++w) CK(cudaGraphLaunch(ex, s));
+  CK(cudaEventRecord(e0, s));
+  const int reps = 5;
+  for (int r = 0; r < reps; ++r) CK(cudaGraphLaunch(ex, s));
+  CK(cudaEventRecord(e1, s));
+  CK(cudaEventSynchronize(e1));
+  float ms = 0;
+  CK(cudaEventElapsedTime(&ms, e0, e1));
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  cudaGraphExecDestroy(ex);
+  cudaGraphDestroy(g);
+  *us = ms * 1000.0 / (reps * iters);
+  *bytes = by;
+  c->prefilled = false;  // the row descriptors were overwritten: prefill again before stepping
   return read_err(c);
 }
 

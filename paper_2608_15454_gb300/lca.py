@@ -25,7 +25,7 @@ STATUS = {0: "LCA_OK", -1: "LCA_E_ARG", -2: "LCA_E_CAPACITY", -3: "LCA_E_WEIGHTS
 EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "lca_mbp_step_async",
            "lca_generate",
            "lca_generate_async", "lca_generate_fetch", "lca_debug_state", "lca_debug_stats",
-           "lca_debug_set_eager", "lca_debug_profile",
+           "lca_debug_set_eager", "lca_debug_profile", "lca_debug_bench_kernel",
            "lca_debug_logits",
            "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str",
            "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
@@ -98,6 +98,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_debug_stats": [P, ctypes.POINTER(LcaStats)],
         "lca_debug_logits": [P, P, P],
         "lca_debug_set_eager": [P, I32],
+        "lca_debug_bench_kernel": [P, I32, I32, I32, ctypes.POINTER(ctypes.c_double),
+                                   ctypes.POINTER(ctypes.c_double)],
         "lca_debug_profile": [P, I32, F32, I32, I32, ctypes.POINTER(LcaProfile)],
         "lca_debug_force_accept": [P, P],
         "lca_debug_force_candidates": [P, P, I32],
@@ -243,6 +245,12 @@ class Context:
                     "lca_debug_profile")
         return {k: {"launches": p.launches[i], "ms": p.ms[i], "bytes": p.bytes[i]}
                 for i, k in enumerate(PROFILE_KINDS)}
+
+    def bench_kernel(self, kind, rows, iters):
+        us, by = ctypes.c_double(), ctypes.c_double()
+        self._check(self.lib.lca_debug_bench_kernel(self.h, kind, rows, iters, ctypes.byref(us),
+                                                    ctypes.byref(by)), "lca_debug_bench_kernel")
+        return us.value, by.value
 
     def logits(self, n):
         nb = np.zeros((self.batch, n, 256), dtype=np.float32)

@@ -203,3 +203,39 @@ def test_paper_bf16_steps_with_resync(lca, n):
         st = ctx.state(0)
         assert (st["t"], st["K"]) == (dec.t, dec.K)
     assert resync <= 1
+
+
+# ----------------------------------------------------------------------------- small bf16
+SMALL_BF16 = TINY.replace(d_model=256, n_heads=4, head_dim=64, d_ff=1024, n_enc=1, n_lm=2,
+                          n_nb=1, n_mb=2, dtype="bf16")
+
+
+@pytest.mark.parametrize("mb_kind", ["lca", "mlp"])
+def test_small_bf16_batch_forced_and_free_steps(lca, mb_kind):
+    """bf16 storage at d = 256 (bulk-copy weight pipeline, split-K and grouped paths): logits
+    within the bf16 tolerance, and bytes/state equal whenever the oracle's decisions have margin."""
+    model = SMALL_BF16 if mb_kind == "lca" else SMALL_BF16.replace(mb_kind="mlp", n_mb=3, n_mlp_heads=5)
+    W = make_weights(model, gain=8.0, seed=5)
+    prompts = [zipf_text(0, 300), zipf_text(1, 77) + b" ", zipf_text(2, 150)]
+    n = 4
+    ctx = new_ctx(lca, model, W, len(prompts), 600, 6)
+    ctx.prefill(prompts)
+    decs = []
+    for p in prompts:
+        d = IncrementalDecoder(Model(model, W))
+        d.prefill(p)
+        decs.append(d)
+    for s in range(12):
+        cands = [bytes([97 + (s + b) % 26, 32 if (s + b) % 2 == 0 else 98, 99, 32]) for b in range(3)]
+        a = [s % 4, (s + 2) % 4, 3]
+        ctx.force_candidates(cands, n)
+        ctx.force_accept(a)
+        recs = [d.step(n, 0.75, THRESH, forced=a[b], forced_cand=cands[b]) for b, d in enumerate(decs)]
+        out, cnt = ctx.step(n, 0.75, lca.LCA_THRESH)
+        nb, mb = ctx.logits(n)
+        for b, r in enumerate(recs):
+            np.testing.assert_allclose(nb[b], r.nb_logits, atol=BF16_TOL * 8, rtol=0)
+            np.testing.assert_allclose(mb[b], r.mb_logits, atol=BF16_TOL * 8, rtol=0)
+            assert out[b] == r.emitted
+            st = ctx.state(b)
+            assert (st["t"], st["K"]) == (decs[b].t, decs[b].K)
