@@ -171,6 +171,14 @@ typedef struct {
 int lca_debug_profile(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t steps,
                       lca_profile* out);
 
+/* Run `steps` step graphs with launch tracing on: thread 0 of every CTA of every kernel records
+ * {u64 start_ns, u64 end_ns, u64 wait_done_ns, i32 kernel tag, i32 cta, i32 sm, i32 pad}
+ * (40 bytes) into `out`
+ * (host, room for `cap` records); count = records written. Needs a bf16 context (the trace
+ * buffer borrows scratch that the bf16 step does not use). */
+int lca_debug_trace(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t steps,
+                    void* out, int32_t cap, int32_t* count);
+
 /* Micro-benchmark: one graph of `iters` back-to-back launches of one kernel kind over `rows`
  * rows (0 RMSNorm+QKV, 1 Wo, 2 RMSNorm+W1/W3+SwiGLU, 3 W2, 4 decode attention over the
  * encoder cache, 5 unembedding head, 6 a glue kernel), cycling through all blocks' weights so

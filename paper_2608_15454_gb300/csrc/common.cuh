@@ -32,6 +32,73 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
+// ---------------------------------------------------------------- optional launch trace
+// When enabled, thread 0 of every CTA records (kernel tag, globaltimer at entry and exit) in a
+// device buffer, so the timeline of the kernels inside a graph can be rebuilt on the host.
+// The pointers are per translation unit (no relocatable device code); trace_set() fills them.
+struct TraceRec {
+  unsigned long long t0, t1, tw;  // entry, exit, grid-dependency wait returned
+  int tag, cta, sm, pad;
+};
+enum TraceTag : int {
+  TT_GEMV = 1, TT_GEMV_F32, TT_GEMM, TT_ROWSTATS, TT_ATTN, TT_HEAD, TT_MB_PLAN, TT_MB_FILL,
+  TT_MLP_PLAN, TT_VERIFY_PLAN, TT_SEGMENT, TT_LM_SCATTER, TT_NB_INPUT, TT_COMMIT, TT_LOOP_CTL,
+  TT_OTHER
+};
+static __device__ TraceRec* g_trace = nullptr;
+static __device__ unsigned int* g_trace_n = nullptr;
+static __device__ unsigned int g_trace_cap = 0;
+__device__ __forceinline__ unsigned long long gtimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ unsigned smid() {
+  unsigned r;
+  asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+  return r;
+}
+struct TraceScope {
+  unsigned long long t0, tw;
+  int tag;
+  bool on;
+  __device__ __forceinline__ explicit TraceScope(int t) : t0(0), tw(0), tag(t), on(false) {
+    if (threadIdx.x == 0 && threadIdx.y == 0 && g_trace) {
+      on = true;
+      t0 = gtimer();
+      tw = t0;
+    }
+  }
+  __device__ __forceinline__ void waited() {
+    if (on) tw = gtimer();
+  }
+  __device__ __forceinline__ ~TraceScope() {
+    if (on) {
+      const unsigned i = atomicAdd(g_trace_n, 1u);
+      if (i < g_trace_cap) {
+        TraceRec r;
+        r.t0 = t0;
+        r.t1 = gtimer();
+        r.tw = tw;
+        r.tag = tag;
+        r.cta = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+        r.sm = (int)smid();
+        r.pad = 0;
+        g_trace[i] = r;
+      }
+    }
+  }
+};
+#define LCA_TRACE_SETTER(name)                                                         \
+  void name(TraceRec* buf, unsigned* counter, unsigned cap) {                          \
+    cudaMemcpyToSymbol(g_trace, &buf, sizeof(buf));                                    \
+    cudaMemcpyToSymbol(g_trace_n, &counter, sizeof(counter));                          \
+    cudaMemcpyToSymbol(g_trace_cap, &cap, sizeof(cap));                                \
+  }
+void trace_set_linear(TraceRec* buf, unsigned* counter, unsigned cap);
+void trace_set_attn(TraceRec* buf, unsigned* counter, unsigned cap);
+void trace_set_step(TraceRec* buf, unsigned* counter, unsigned cap);
+
 constexpr int kVocab = 256;
 constexpr int kMaxKSplit = 8;     // split-K ways of the skinny linear kernel
 constexpr int kMaxAttnSplit = 16; // key-range splits of decode attention
@@ -154,6 +221,7 @@ struct Dev {
   float eps, scale;
   int num_sms;  // streaming multiprocessors of the device
   int use_tma;  // bf16 linear layers use the bulk-copy weight pipeline
+  int attn_split_cap;  // largest cluster (key split) of decode attention
 
   // weights (storage type; norms and bos fp32)
   void* embed;   // [256][d]
@@ -257,8 +325,11 @@ size_t attention_counters(int B, int H);
 void kernel_attrs_linear();
 void kernel_attrs_step();
 // Attention of query rows over a KV-cache layer (keys [0, kvlen[r]) of sequence b[r]).
+// stable: optional per-sequence committed length (stride in ints) whose cache prefix does not
+// change during a step, prefetched into L2 before the dependency wait; stable_extra: rows added.
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
-               int qtiles_grid, int splits, cudaStream_t s);
+               int qtiles_grid, int splits, cudaStream_t s, const int* stable = nullptr,
+               int stable_extra = 0);
 
 // Step / prefill glue kernels (kernels_step.cu).
 void launch_mb_plan(const Dev& D, cudaStream_t s);

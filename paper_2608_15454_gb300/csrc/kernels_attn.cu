@@ -35,6 +35,7 @@ template <typename TC, int HD>
 __global__ void __launch_bounds__(kThreads)
 k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
        int splits, float* __restrict__ part, int* __restrict__ cnt, int* err) {
+  TraceScope _trace(TT_ATTN);
   constexpr int QT = kAttnQT;
   constexpr int EV = 16 / (int)sizeof(TC);  // cache elements per 16-byte vector
   __shared__ float qs[QT][HD];
@@ -47,6 +48,7 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
 
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const int b = blockIdx.x;
   const int h = blockIdx.z / splits;
   const int sp = blockIdx.z - h * splits;
@@ -247,183 +249,6 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
   }
 }
 
-// The same attention with the key range of each (sequence, query tile, head) split over the CTAs
-// of one thread-block cluster: every CTA keeps its (max, sum, acc) partial in its own shared
-// memory, and rank 0 combines the ranks' partials through distributed shared memory, in rank
-// order (deterministic), with no global scratch and no atomics.
-template <typename TC, int HD>
-__global__ void __launch_bounds__(kThreads)
-k_attn_cl(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
-          int* err) {
-  namespace cgr = cooperative_groups;
-  constexpr int QT = kAttnQT;
-  constexpr int EV = 16 / (int)sizeof(TC);
-  __shared__ float qs[QT][HD];
-  __shared__ float ks[kKT][HD + 1];
-  __shared__ float vs[kKT][HD];
-  __shared__ float ps[QT][kKT];
-  __shared__ float s_m[QT], s_l[QT], s_corr[QT];
-  __shared__ int s_kv[QT];
-  __shared__ float pacc[QT][HD];  // this CTA's partial accumulator (read by rank 0)
-
-  cgr::cluster_group cl = cgr::this_cluster();
-  const int splits = (int)cl.dim_blocks().z;
-  const int sp = (int)cl.block_rank();
-  pdl_trigger();
-  pdl_wait();
-  const int b = blockIdx.x;
-  const int h = blockIdx.z / splits;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int nrows = rows.seq_count[b];
-  const int rbeg = rows.seq_start[b];
-  const int ntiles = (nrows + QT - 1) / QT;
-  const TC* Kc = reinterpret_cast<const TC*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
-  const TC* Vc = reinterpret_cast<const TC*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
-  const int ld = H * HD;
-  constexpr int DPT = QT * HD / kThreads;
-  const int ai = tid / (HD / DPT);
-  const int ad = (tid % (HD / DPT)) * DPT;
-  const int sk = tid & (kKT - 1);
-  const int sr = (tid / kKT) * (QT * kKT / kThreads);
-
-  for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
-    const int r0 = rbeg + qt * QT;
-    const int nq = min(QT, nrows - qt * QT);
-    __syncthreads();
-    for (int idx = tid; idx < QT * HD; idx += kThreads) {
-      const int i = idx / HD, dd = idx - i * HD;
-      qs[i][dd] = i < nq ? q[(size_t)(r0 + i) * ld + h * HD + dd] * scale : 0.f;
-    }
-    if (tid < QT) {
-      int kl = tid < nq ? rows.kvlen[r0 + tid] : 0;
-      if (kl > kv.S) {
-        atomicOr(err, kErrIndex);
-        kl = kv.S;
-      }
-      s_kv[tid] = kl;
-      s_m[tid] = -INFINITY;
-      s_l[tid] = 0.f;
-    }
-    __syncthreads();
-    int kv_hi = 0;
-#pragma unroll
-    for (int i = 0; i < QT; ++i) kv_hi = max(kv_hi, s_kv[i]);
-    const int chunk = ((kv_hi + splits - 1) / splits + 15) / 16 * 16;
-    const int lo = sp * chunk;
-    const int hi = min(kv_hi, lo + chunk);
-    float acc[DPT];
-#pragma unroll
-    for (int j = 0; j < DPT; ++j) acc[j] = 0.f;
-    for (int j0 = lo; j0 < hi; j0 += kKT) {
-      const int nk = min(kKT, hi - j0);
-      {
-        // the whole K/V tile: every thread issues all its 16-byte loads before any store
-        constexpr int NL = kKT * HD / EV / kThreads;
-        uint4 uk[NL], uv[NL];
-#pragma unroll
-        for (int u = 0; u < NL; ++u) {
-          const int e = (tid + u * kThreads) * EV;
-          const int kk = e / HD, dd = e - kk * HD;
-          if (kk < nk) {
-            uk[u] = *reinterpret_cast<const uint4*>(Kc + (size_t)(j0 + kk) * HD + dd);
-            uv[u] = *reinterpret_cast<const uint4*>(Vc + (size_t)(j0 + kk) * HD + dd);
-          } else {
-            uk[u] = make_uint4(0, 0, 0, 0);
-            uv[u] = make_uint4(0, 0, 0, 0);
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < NL; ++u) {
-          const int e = (tid + u * kThreads) * EV;
-          const int kk = e / HD, dd = e - kk * HD;
-          float fk[8], fv[8];
-          unpack16(uk[u], fk, (const TC*)nullptr);
-          unpack16(uv[u], fv, (const TC*)nullptr);
-#pragma unroll
-          for (int j = 0; j < EV; ++j) {
-            ks[kk][dd + j] = fk[j];
-            vs[kk][dd + j] = fv[j];
-          }
-        }
-      }
-      __syncthreads();
-      {
-        float sc[QT * kKT / kThreads];
-#pragma unroll
-        for (int r = 0; r < QT * kKT / kThreads; ++r) sc[r] = 0.f;
-#pragma unroll 16
-        for (int dd = 0; dd < HD; ++dd) {
-          const float kd = ks[sk][dd];
-#pragma unroll
-          for (int r = 0; r < QT * kKT / kThreads; ++r) sc[r] = fmaf(qs[sr + r][dd], kd, sc[r]);
-        }
-#pragma unroll
-        for (int r = 0; r < QT * kKT / kThreads; ++r)
-          ps[sr + r][sk] = (sk < nk && j0 + sk < s_kv[sr + r]) ? sc[r] : -INFINITY;
-      }
-      __syncthreads();
-      for (int i = warp * (QT / 4); i < (warp + 1) * (QT / 4); ++i) {
-        const float v0 = ps[i][lane], v1 = ps[i][lane + 32];
-        float mx = fmaxf(v0, v1);
-#pragma unroll
-        for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        const float m_old = s_m[i];
-        const float m_new = fmaxf(m_old, mx);
-        const float p0 = v0 == -INFINITY ? 0.f : expf(v0 - m_new);
-        const float p1 = v1 == -INFINITY ? 0.f : expf(v1 - m_new);
-        float ssum = p0 + p1;
-#pragma unroll
-        for (int o = 16; o; o >>= 1) ssum += __shfl_xor_sync(0xffffffffu, ssum, o);
-        ps[i][lane] = p0;
-        ps[i][lane + 32] = p1;
-        __syncwarp();
-        if (lane == 0) {
-          const float corr = (m_old == -INFINITY) ? 0.f : expf(m_old - m_new);
-          s_corr[i] = corr;
-          s_l[i] = s_l[i] * corr + ssum;
-          s_m[i] = m_new;
-        }
-      }
-      __syncthreads();
-      {
-        const float corr = s_corr[ai];
-#pragma unroll
-        for (int j = 0; j < DPT; ++j) acc[j] *= corr;
-        for (int kk = 0; kk < nk; ++kk) {
-          const float p = ps[ai][kk];
-#pragma unroll
-          for (int j = 0; j < DPT; ++j) acc[j] = fmaf(p, vs[kk][ad + j], acc[j]);
-        }
-      }
-      __syncthreads();
-    }
-#pragma unroll
-    for (int j = 0; j < DPT; ++j) pacc[ai][ad + j] = acc[j];
-    cl.sync();
-    if (sp == 0 && ai < nq) {
-      float M = -INFINITY;
-      for (int r = 0; r < splits; ++r) M = fmaxf(M, *cl.map_shared_rank(&s_m[ai], r));
-      float L = 0.f, o[DPT];
-#pragma unroll
-      for (int j = 0; j < DPT; ++j) o[j] = 0.f;
-      for (int r = 0; r < splits; ++r) {
-        const float mr = *cl.map_shared_rank(&s_m[ai], r);
-        if (mr == -INFINITY) continue;
-        const float w = expf(mr - M);
-        L += w * *cl.map_shared_rank(&s_l[ai], r);
-        const float* pr = cl.map_shared_rank(&pacc[ai][ad], r);
-#pragma unroll
-        for (int j = 0; j < DPT; ++j) o[j] += w * pr[j];
-      }
-      const float il = L > 0.f ? 1.f / L : 0.f;
-      float* dst = out + (size_t)(r0 + ai) * ld + h * HD + ad;
-#pragma unroll
-      for (int j = 0; j < DPT; ++j) dst[j] = o[j] * il;
-    }
-    cl.sync();
-  }
-}
-
 // Decode attention, second form: 256 threads; scores with one key per thread (its K row held in
 // registers, loaded straight from global memory), online softmax with one warp per query row,
 // and P.V with each thread owning 4 dims of every row over a group of keys. The key range of a
@@ -455,7 +280,7 @@ __device__ __forceinline__ void load4(const float* p, float (&v)[4]) {
 template <typename TC, int HD>
 __global__ void __launch_bounds__(kA2Threads)
 k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
-        int* err) {
+        int* err, const int* __restrict__ stable, int stable_stride, int stable_extra) {
   namespace cgr = cooperative_groups;
   constexpr int QT = kAttnQT;
   constexpr int EV = 16 / (int)sizeof(TC);
@@ -470,11 +295,27 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
   __shared__ float s_m[QT], s_l[QT], s_corr[QT];
   __shared__ int s_kv[QT];
 
+  TraceScope _trace(TT_ATTN);
   cgr::cluster_group cl = cgr::this_cluster();
   const int splits = (int)cl.dim_blocks().z;
   const int sp = (int)cl.block_rank();
+  if (stable && threadIdx.x < 2) {
+    // Cache slots below the committed length do not change during a step: prefetch this CTA's
+    // approximate K (thread 0) and V (thread 1) range into L2 before the dependency wait.
+    const int bb = blockIdx.x, hh = blockIdx.z / splits;
+    const int t = stable[(size_t)bb * stable_stride];
+    const int est = ((t + stable_extra + splits - 1) / splits + 15) / 16 * 16;
+    const int lo = sp * est, hi = min(t, lo + est);
+    if (hi > lo) {
+      const TC* base = reinterpret_cast<const TC*>(threadIdx.x == 0 ? kv.k : kv.v) +
+                       (((size_t)bb * H + hh) * kv.S + lo) * HD;
+      const uint32_t bytes = (uint32_t)((hi - lo) * HD * sizeof(TC));
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"(bytes & ~15u) : "memory");
+    }
+  }
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const int b = blockIdx.x;
   const int h = blockIdx.z / splits;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -626,19 +467,35 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
       pacc[r][dd] = t;
     }
     cl.sync();
-    // rank 0 combines the ranks' partials (max, sum, acc) in rank order
-    if (sp == 0) {
-      for (int idx = tid; idx < nq * HD; idx += kA2Threads) {
-        const int r = idx / HD, dd = idx - r * HD;
+    // every rank combines its slice of the head dims over all ranks, in rank order; the
+    // remote (max, sum, acc) values are requested before any is used
+    {
+      const int dpr = (HD + splits - 1) / splits;  // dims per rank
+      const int d0 = sp * dpr;
+      const int nd = min(dpr, HD - d0);
+      for (int idx = tid; idx < nq * nd; idx += kA2Threads) {
+        const int r = idx / nd, dd = d0 + (idx - r * nd);
+        float mr[kMaxClusterSplit], lr[kMaxClusterSplit], ar[kMaxClusterSplit];
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
+          if (k < splits) {
+            mr[k] = *cl.map_shared_rank(&s_m[r], k);
+            lr[k] = *cl.map_shared_rank(&s_l[r], k);
+            ar[k] = *cl.map_shared_rank(&pacc[r][dd], k);
+          }
+        }
         float M = -INFINITY;
-        for (int k = 0; k < splits; ++k) M = fmaxf(M, *cl.map_shared_rank(&s_m[r], k));
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k)
+          if (k < splits) M = fmaxf(M, mr[k]);
         float L = 0.f, o = 0.f;
-        for (int k = 0; k < splits; ++k) {
-          const float mk = *cl.map_shared_rank(&s_m[r], k);
-          if (mk == -INFINITY) continue;
-          const float w = expf(mk - M);
-          L += w * *cl.map_shared_rank(&s_l[r], k);
-          o += w * *cl.map_shared_rank(&pacc[r][dd], k);
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
+          if (k < splits && mr[k] != -INFINITY) {
+            const float w = expf(mr[k] - M);
+            L += w * lr[k];
+            o += w * ar[k];
+          }
         }
         out[(size_t)(r0 + r) * ld + h * HD + dd] = L > 0.f ? o / L : 0.f;
       }
@@ -649,7 +506,8 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
 
 template <typename TC, int HD>
 void launch_cl(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-               int qtiles_grid, int splits, int* err, cudaStream_t s) {
+               int qtiles_grid, int splits, int* err, const int* stable, int stable_stride,
+               int stable_extra, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA2Threads);
@@ -664,7 +522,8 @@ void launch_cl(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn2<TC, HD>, q, out, kv, rows, H, scale, err);
+  cudaLaunchKernelEx(&cfg, k_attn2<TC, HD>, q, out, kv, rows, H, scale, err, stable, stable_stride,
+                     stable_extra);
 }
 
 template <typename TC, int HD>
@@ -787,16 +646,17 @@ size_t attention_scratch_floats(int B, int H, int hd) {
 size_t attention_counters(int B, int H) { return (size_t)B * kQTMax * H; }
 
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
-               int qtiles_grid, int splits, cudaStream_t s) {
+               int qtiles_grid, int splits, cudaStream_t s, const int* stable, int stable_extra) {
   ProfScope ps(PK_ATTN, 0.0, s);
   if (splits > kMaxClusterSplit) splits = kMaxClusterSplit;
   if (splits < 1) splits = 1;
+  const int ss = (int)(sizeof(SeqState) / sizeof(int));
   if (D.dtype == LCA_BF16) {
-    if (D.hd == 64) launch_cl<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
-    else launch_cl<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+    if (D.hd == 64) launch_cl<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+    else launch_cl<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
   } else {
-    if (D.hd == 64) launch_cl<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
-    else launch_cl<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+    if (D.hd == 64) launch_cl<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+    else launch_cl<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
   }
 }
 
@@ -849,5 +709,7 @@ size_t lca_decode_attention_noalloc_capacity(void) { return kNoAllocScratchBytes
 }  // extern "C"
 
 namespace lca {
+
+LCA_TRACE_SETTER(trace_set_attn)
 
 } // namespace lca

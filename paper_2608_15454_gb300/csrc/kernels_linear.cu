@@ -119,6 +119,89 @@ __device__ __forceinline__ void epi_pair(const EpiArgs& e, int r, int c, float a
   }
 }
 
+// Epilogue operands that do not depend on the dot products (residual values, RoPE angle,
+// cache slot), loaded early so that their latency overlaps the main loop.
+struct EpiPre {
+  float r0, r1;  // residual pair
+  float2 cs;     // RoPE cos/sin
+  int b, slot;
+};
+
+__device__ __forceinline__ EpiPre epi_load(const EpiArgs& e, int r, int c) {
+  EpiPre p;
+  p.r0 = p.r1 = 0.f;
+  p.cs = make_float2(1.f, 0.f);
+  p.b = p.slot = 0;
+  if (e.mode == EPI_RESID || e.mode == EPI_RESID_SILU) {
+    const float2 q = *reinterpret_cast<const float2*>(e.res + (size_t)r * e.ldres + c);
+    p.r0 = q.x;
+    p.r1 = q.y;
+  } else if (e.mode == EPI_QKV) {
+    const int part = c / e.d;
+    const int cc = c - part * e.d;
+    const int dd = cc % e.hd;
+    if (part < 2) {
+      const int pos = e.rows.pos[r];
+      p.cs = e.rope[(size_t)pos * (e.hd >> 1) + (dd >> 1)];
+    }
+    if (part > 0) {
+      p.b = e.rows.b[r];
+      p.slot = e.rows.slot[r];
+    }
+  }
+  return p;
+}
+
+template <typename TC>
+__device__ __forceinline__ void epi_store(const EpiArgs& e, const EpiPre& p, int r, int c, float a0, float a1) {
+  switch (e.mode) {
+    case EPI_STORE: {
+      float* y = e.y + (size_t)r * e.ldy + c;
+      *reinterpret_cast<float2*>(y) = make_float2(a0, a1);
+      break;
+    }
+    case EPI_RESID: {
+      float* y = e.y + (size_t)r * e.ldy + c;
+      *reinterpret_cast<float2*>(y) = make_float2(p.r0 + a0, p.r1 + a1);
+      break;
+    }
+    case EPI_RESID_SILU: {
+      float* y = e.y + (size_t)r * e.ldy + c;
+      *reinterpret_cast<float2*>(y) = make_float2(p.r0 + silu_f(a0), p.r1 + silu_f(a1));
+      break;
+    }
+    case EPI_SWIGLU: {
+      e.y[(size_t)r * e.ldy + (c >> 1)] = silu_f(a0) * a1;
+      break;
+    }
+    case EPI_QKV: {
+      const int part = c / e.d;
+      const int cc = c - part * e.d;
+      const int h = cc / e.hd;
+      const int dd = cc - h * e.hd;
+      if (part < 2) {
+        const float x0 = a0 * p.cs.x - a1 * p.cs.y;
+        const float x1 = a0 * p.cs.y + a1 * p.cs.x;
+        a0 = x0;
+        a1 = x1;
+      }
+      if (part == 0) {
+        *reinterpret_cast<float2*>(e.y + (size_t)r * e.ldy + cc) = make_float2(a0, a1);
+      } else {
+        if (p.slot < 0 || p.slot >= e.kv.S) {
+          atomicOr(e.err, kErrIndex);
+          return;
+        }
+        TC* base = reinterpret_cast<TC*>(part == 1 ? e.kv.k : e.kv.v);
+        TC* q = base + (((size_t)p.b * e.H + h) * e.kv.S + p.slot) * e.hd + dd;
+        store_cache(q, a0);
+        store_cache(q + 1, a1);
+      }
+      break;
+    }
+  }
+}
+
 // Reduce-scatter of 32 per-lane partial sums: afterwards lane L holds the warp total of
 // value index L (row L / kCPW, column L % kCPW). 31 shuffles.
 __device__ __forceinline__ float warp_reduce_scatter32(float (&v)[32], int lane) {
@@ -166,6 +249,7 @@ __device__ __forceinline__ void unpack8(const uint4 (&u)[2], float (&w)[8]) {
 template <typename TW, bool NORM, int KIT>
 __global__ void __launch_bounds__(kWarps * 32)
 k_gemv(LinearArgs a, int ksplit, float* __restrict__ part, int* __restrict__ cnt) {
+  TraceScope _trace(TT_GEMV_F32);
   constexpr int VEC = WTraits<TW>::VEC;
   extern __shared__ float smem[];
   const int Kr = a.Kd / ksplit;
@@ -199,6 +283,7 @@ k_gemv(LinearArgs a, int ksplit, float* __restrict__ part, int* __restrict__ cnt
   }
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
 
   const int rbase = grp * a.Mg_stride;
   int M = *a.M;
@@ -396,24 +481,29 @@ __device__ __forceinline__ void prefetch_next(const LinearArgs& a) {
 }
 
 // One tile per CTA: NW*4 output columns x Kr inputs (the CTA's K-split), copied into shared
-// memory by bulk async copies issued before the grid-dependency wait. Warps own 4 columns each;
-// lanes stride K by 8, and one activation load from shared memory feeds 4 columns. Rows are
+// memory by bulk async copies issued before the grid-dependency wait, together with the RMSNorm
+// gain of the K-range. Warps own 4 columns each; lanes stride K by 8, and one activation load
+// from shared memory feeds 4 columns. RMSNorm is folded in: rows are staged as x * g while their
+// sums of squares accumulate, and the per-row inverse RMS scales the dot products. Rows are
 // processed in chunks of MCA. With a K-split the `ksplit` CTAs of a column tile form a thread-
-// block cluster: each leaves its partial sums in its own shared memory and rank 0 adds the
-// ranks' partials through distributed shared memory in rank order (no global scratch).
+// block cluster: each leaves its partial sums in its own shared memory and rank 0 adds the ranks'
+// partials through distributed shared memory in rank order (no global scratch).
 template <int MCA, int NW, bool NORM>
-__global__ void __launch_bounds__(NW * 32)
+__global__ void __launch_bounds__(NW * 32, 1)
 k_gemv_bulk(LinearArgs a, int ksplit) {
+  TraceScope _trace(TT_GEMV);
   namespace cgr = cooperative_groups;
   constexpr int CT = NW * kCPW;  // columns per CTA
+  constexpr int NT = NW * 32;
   extern __shared__ __align__(128) unsigned char sm[];
   const int Kr = a.Kd / ksplit;
-  __nv_bfloat16* wt = reinterpret_cast<__nv_bfloat16*>(sm);            // [CT][Kr]
-  float* xs = reinterpret_cast<float*>(sm + (size_t)CT * Kr * 2);       // [MCA][Kr]
-  float* inv = xs + MCA * Kr;                                          // [MCA]
-  float* cpart = inv + MCA;                                            // [MCA][CT]
+  __nv_bfloat16* wt = reinterpret_cast<__nv_bfloat16*>(sm);             // [CT][Kr]
+  float* gs = reinterpret_cast<float*>(sm + (size_t)CT * Kr * 2);        // [Kr] (NORM)
+  float* xs = gs + Kr;                                                   // [MCA][Kr]
+  float* rs = xs + MCA * Kr;                                             // [MCA] sums of squares
+  float* cpart = rs + MCA;                                               // [MCA][CT]
   uint64_t* bar = reinterpret_cast<uint64_t*>(
-      (reinterpret_cast<uintptr_t>(cpart + MCA * CT) + 15) & ~uintptr_t(15));  // 16-byte aligned
+      (reinterpret_cast<uintptr_t>(cpart + MCA * CT) + 15) & ~uintptr_t(15));
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int tile = blockIdx.x;
@@ -426,16 +516,18 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   if (tid == 0) {
     mbar_init(bar, 1);
     fence_mbar_init();
-    mbar_expect_tx(bar, (uint32_t)(ncols * Kr * 2));
+    mbar_expect_tx(bar, (uint32_t)(ncols * Kr * 2 + (NORM ? Kr * 4 : 0)));
     if (ksplit == 1) {
       bulk_g2s(wt, W, (uint32_t)(ncols * Kr * 2), bar);
     } else {
       for (int c = 0; c < ncols; ++c) bulk_g2s(wt + c * Kr, W + (size_t)c * a.Kd, (uint32_t)(Kr * 2), bar);
     }
+    if (NORM) bulk_g2s(gs, a.norm + k0, (uint32_t)(Kr * 4), bar);
   }
   prefetch_next(a);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
 
   const int rbase = grp * a.Mg_stride;
   int M = *a.M;
@@ -443,71 +535,60 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   if (M < 0) M = 0;
   const int col0 = warp * kCPW;  // within the tile
   bool have_w = false;
+  const int ei = lane / kCPW, ec = lane % kCPW;  // this lane's (row, column) after the reduction
 
   for (int r0 = 0; r0 < M; r0 += MCA) {
     const int mc = min(MCA, M - r0);
+    // epilogue operands of this lane, loaded while the rows are staged and multiplied
+    EpiPre pre{};
+    const bool epi_lane = ksplit == 1 && col0 < ncols && ei < mc && (ec & 1) == 0;
+    if (epi_lane) pre = epi_load(a.epi, rbase + r0 + ei, tile * CT + col0 + ec);
     __syncthreads();
-    // raw rows -> shared memory, loads batched 8 at a time per thread
+    if (NORM && tid < MCA) rs[tid] = 0.f;
+    // raw rows -> registers (loads batched), then x * g -> shared memory with sums of squares
     constexpr int UNR = 8;
     const int nv = MCA * Kr / 4;
-    for (int base = tid; base < nv; base += NW * 32 * UNR) {
+    float ss[MCA];
+#pragma unroll
+    for (int i = 0; i < MCA; ++i) ss[i] = 0.f;
+    for (int base = tid; base < nv; base += NT * UNR) {
       float4 v[UNR];
 #pragma unroll
       for (int u = 0; u < UNR; ++u) {
-        const int idx = base + u * NW * 32;
+        const int idx = base + u * NT;
         const int i = (idx * 4) / Kr, kk = idx * 4 - i * Kr;
         v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
         if (idx < nv && i < mc)
           v[u] = *reinterpret_cast<const float4*>(a.x + (size_t)(rbase + r0 + i) * a.ldx + k0 + kk);
       }
+      if (NORM && !have_w) {
+        const bool ok = mbar_wait(bar, 0);  // the gain slice travels with the weights
+        if (!ok) atomicOr(a.epi.err, kErrTimeout);
+      }
 #pragma unroll
       for (int u = 0; u < UNR; ++u) {
-        const int idx = base + u * NW * 32;
-        if (idx < nv) *reinterpret_cast<float4*>(xs + idx * 4) = v[u];
+        const int idx = base + u * NT;
+        if (idx < nv) {
+          float4 q = v[u];
+          if (NORM) {
+            const int i = (idx * 4) / Kr, kk = idx * 4 - i * Kr;
+#pragma unroll
+            for (int r = 0; r < MCA; ++r)
+              if (r == i) ss[r] += q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
+            const float4 g = *reinterpret_cast<const float4*>(gs + kk);
+            q.x *= g.x; q.y *= g.y; q.z *= g.z; q.w *= g.w;
+          }
+          *reinterpret_cast<float4*>(xs + idx * 4) = q;
+        }
       }
     }
-    __syncthreads();
-    if (NORM) {
-      // RMSNorm: inverse RMS of each row (from shared memory when the CTA holds all of K, else
-      // from global memory), then x * inv * g in place
-      for (int i = warp; i < mc; i += NW) {
-        float ss = 0.f;
-        if (ksplit == 1) {
-          for (int k = lane * 4; k < Kr; k += 128) {
-            const float4 q = *reinterpret_cast<const float4*>(xs + i * Kr + k);
-            ss += q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
-          }
-        } else {
-          const float* xr = a.x + (size_t)(rbase + r0 + i) * a.ldx;
-          for (int k = lane * 4; k < a.Kd; k += 128) {
-            const float4 q = *reinterpret_cast<const float4*>(xr + k);
-            ss += q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
-          }
-        }
+    if (NORM && ksplit == 1) {
 #pragma unroll
-        for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-        if (lane == 0) inv[i] = rsqrtf(ss / (float)a.Kd + a.eps);
-      }
-      __syncthreads();
-      for (int base = tid; base < mc * Kr / 4; base += NW * 32 * UNR) {
-        float4 g[UNR];
+      for (int i = 0; i < MCA; ++i) {
+        float t = ss[i];
 #pragma unroll
-        for (int u = 0; u < UNR; ++u) {
-          const int idx = base + u * NW * 32;
-          const int kk = (idx * 4) % Kr;
-          if (idx < mc * Kr / 4) g[u] = *reinterpret_cast<const float4*>(a.norm + k0 + kk);
-        }
-#pragma unroll
-        for (int u = 0; u < UNR; ++u) {
-          const int idx = base + u * NW * 32;
-          if (idx < mc * Kr / 4) {
-            const int i = (idx * 4) / Kr;
-            float4 q = *reinterpret_cast<float4*>(xs + idx * 4);
-            const float sc = inv[i];
-            q.x *= sc * g[u].x; q.y *= sc * g[u].y; q.z *= sc * g[u].z; q.w *= sc * g[u].w;
-            *reinterpret_cast<float4*>(xs + idx * 4) = q;
-          }
-        }
+        for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0 && i < mc) atomicAdd(&rs[i], t);
       }
     }
     if (!have_w) {
@@ -517,6 +598,21 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       if (__syncthreads_or(!ok) && tid == 0) atomicOr(a.epi.err, kErrTimeout);
       have_w = true;
     } else {
+      __syncthreads();
+    }
+    if (NORM && ksplit > 1) {
+      // a K-split CTA sees part of each row: the full-row sums come from global memory
+      for (int i = warp; i < mc; i += NW) {
+        const float* xr = a.x + (size_t)(rbase + r0 + i) * a.ldx;
+        float t = 0.f;
+        for (int k = lane * 4; k < a.Kd; k += 128) {
+          const float4 q = *reinterpret_cast<const float4*>(xr + k);
+          t += q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) rs[i] = t;
+      }
       __syncthreads();
     }
     if (col0 < ncols) {
@@ -553,22 +649,31 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       float full[32];
 #pragma unroll
       for (int j = 0; j < 32; ++j) full[j] = j < MCA * kCPW ? acc[j] : 0.f;
-      const float v = warp_reduce_scatter32(full, lane);
-      const int i = lane / kCPW, c = lane % kCPW;
+      float v = warp_reduce_scatter32(full, lane);
       if (ksplit == 1) {
+        if (NORM && ei < mc) v *= rsqrtf(rs[ei] / (float)a.Kd + a.eps);
         const float vn = __shfl_down_sync(0xffffffffu, v, 1);
-        if (i < mc && (c & 1) == 0)
-          epi_pair<__nv_bfloat16>(a.epi, rbase + r0 + i, tile * CT + col0 + c, v, vn);
-      } else if (i < MCA) {
-        cpart[i * CT + col0 + c] = v;
+        if (epi_lane) epi_store<__nv_bfloat16>(a.epi, pre, rbase + r0 + ei, tile * CT + col0 + ec, v, vn);
+      } else if (ei < MCA) {
+        cpart[ei * CT + col0 + ec] = v;
       }
     }
     if (ksplit > 1) {
       // cluster reduction of the K-split partials of this row chunk
       cgr::cluster_group cl = cgr::this_cluster();
+      EpiPre pp[2];
+      int pi[2], pc[2], np = 0;
+      if (split == 0)
+        for (int idx = tid; idx < mc * (CT / 2) && np < 2; idx += NT) {
+          pi[np] = idx / (CT / 2);
+          pc[np] = (idx - pi[np] * (CT / 2)) * 2;
+          if (pc[np] < ncols) pp[np] = epi_load(a.epi, rbase + r0 + pi[np], tile * CT + pc[np]);
+          ++np;
+        }
       cl.sync();
       if (split == 0) {
-        for (int idx = tid; idx < mc * (CT / 2); idx += NW * 32) {
+        int j = 0;
+        for (int idx = tid; idx < mc * (CT / 2); idx += NT, ++j) {
           const int i = idx / (CT / 2), c = (idx - i * (CT / 2)) * 2;
           if (c >= ncols) continue;
           float t0 = 0.f, t1 = 0.f;
@@ -577,7 +682,13 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
             t0 += pr[0];
             t1 += pr[1];
           }
-          epi_pair<__nv_bfloat16>(a.epi, rbase + r0 + i, tile * CT + c, t0, t1);
+          if (NORM) {
+            const float sc = rsqrtf(rs[i] / (float)a.Kd + a.eps);
+            t0 *= sc;
+            t1 *= sc;
+          }
+          const EpiPre q = j < 2 ? pp[j] : epi_load(a.epi, rbase + r0 + i, tile * CT + c);
+          epi_store<__nv_bfloat16>(a.epi, q, rbase + r0 + i, tile * CT + c, t0, t1);
         }
       }
       cl.sync();
@@ -593,8 +704,10 @@ constexpr int kBM = 64, kBN = 64, kBK = 32;
 
 __global__ void k_rowstats(const float* __restrict__ x, int ldx, int Kd, const int* Mp, int M_cap,
                            int groups, int Mg_stride, float eps, float* __restrict__ inv) {
+  TraceScope _trace(TT_ROWSTATS);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   int M = *Mp;
   M = M < M_cap ? M : M_cap;
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
@@ -613,6 +726,7 @@ __global__ void k_rowstats(const float* __restrict__ x, int ldx, int Kd, const i
 
 template <typename TW, bool NORM>
 __global__ void __launch_bounds__(256) k_gemm(LinearArgs a, const float* __restrict__ inv) {
+  TraceScope _trace(TT_GEMM);
   __shared__ float As[kBK][kBM + 4];
   __shared__ float Bs[kBK][kBN + 4];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
@@ -621,6 +735,7 @@ __global__ void __launch_bounds__(256) k_gemm(LinearArgs a, const float* __restr
   const int rbase = grp * a.Mg_stride;
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   int M = *a.M;
   M = M < a.M_cap ? M : a.M_cap;
   if (M <= 0) return;
@@ -705,7 +820,7 @@ template <int MCA, int NW, bool NORM>
 void gemv_bulk_go(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s) {
   constexpr int CT = NW * kCPW;
   const int Kr = a.Kd / ksplit;
-  const size_t smem = (size_t)CT * Kr * 2 + (size_t)MCA * Kr * 4 + (MCA + MCA * CT + 2) * 4 + 16 + 64;
+  const size_t smem = (size_t)CT * Kr * 2 + (size_t)Kr * 4 + (size_t)MCA * Kr * 4 + (MCA + MCA * CT) * 4 + 16 + 64;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((a.N + CT - 1) / CT, ksplit, a.groups);
   cfg.blockDim = dim3(NW * 32);
@@ -820,5 +935,7 @@ void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s) {
     else norm ? launch_gemv<float, true>(D, a, s) : launch_gemv<float, false>(D, a, s);
   }
 }
+
+LCA_TRACE_SETTER(trace_set_linear)
 
 } // namespace lca

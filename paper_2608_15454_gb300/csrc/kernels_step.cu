@@ -22,8 +22,10 @@ __device__ __forceinline__ void err_or(int* e, int bits) { atomicOr(e, bits); }
 // MB cache (slot = position - window start) and only new committed rows plus the copies are
 // computed. A changed window start (a committed boundary) rebuilds the cache.
 __global__ void k_mb_plan(Dev D) {
+  TraceScope _trace(TT_MB_PLAN);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   __shared__ int s_cnt[1024];
   __shared__ int s_first[1024];
   const Params P = *D.params;
@@ -80,13 +82,30 @@ __global__ void k_mb_plan(Dev D) {
     for (int j = lane; j < n - 1; j += 32)
       D.head_rows_mb[b * (n - 1) + j] = cnt > 0 ? st0 + cnt - (n - 1) + j : 0;
   }
+  __syncthreads();
+  // window rows: byte p of group k gets o_k + u_k (Algorithm 1 line 9, residual r_2 added before
+  // upsampling); copies beyond t belong to the current group K
+  const int M = *D.r_mb.M;
+  const int d4 = D.d / 4;
+  for (int idx = tid; idx < M * d4; idx += blockDim.x) {
+    const int r = idx / d4, c4 = idx - r * d4;
+    const int b = D.r_mb.b[r], p = D.r_mb.pos[r];
+    const int g = D.seq[b].K;
+    const int gs = D.gstart[(size_t)b * D.L + g];
+    const int k = (g >= 1 && p < gs) ? g - 1 : g;
+    const float4 o = reinterpret_cast<const float4*>(D.o_tab + ((size_t)b * D.L + k) * D.d)[c4];
+    const float4 u = reinterpret_cast<const float4*>(D.u_tab + ((size_t)b * D.L + k) * D.d)[c4];
+    reinterpret_cast<float4*>(D.x_mb + (size_t)r * D.d)[c4] = make_float4(o.x + u.x, o.y + u.y, o.z + u.z, o.w + u.w);
+  }
 }
 
 // MB input rows: byte p of group k gets o_k + u_k (Algorithm 1 line 9, residual r_2 added
 // before upsampling); copies beyond t belong to the current group K.
 __global__ void k_mb_fill(Dev D) {
+  TraceScope _trace(TT_MB_FILL);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const int M = *D.r_mb.M;
   const int d4 = D.d / 4;
   for (size_t idx = blockIdx.x * (size_t)blockDim.x + threadIdx.x; idx < (size_t)M * d4;
@@ -106,8 +125,10 @@ __global__ void k_mb_fill(Dev D) {
 
 // MLP-MBP heads: row j*batch + b starts from the last next-byte hidden state of b.
 __global__ void k_mlp_plan(Dev D) {
+  TraceScope _trace(TT_MLP_PLAN);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int rows = batch * (n - 1);
@@ -158,6 +179,7 @@ __global__ void __launch_bounds__(256)
 k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const int* Mp, int M_cap,
        const float* __restrict__ norm, float* __restrict__ logits, int* __restrict__ arg,
        float* __restrict__ prob, int* __restrict__ cnt) {
+  TraceScope _trace(TT_HEAD);
   constexpr int VEC = sizeof(TW) == 2 ? 1 : 2;
   extern __shared__ float xs[];  // [kHR][d]
   __shared__ float inv[kHR];
@@ -177,6 +199,7 @@ k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const i
   }
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   int M = *Mp;
   M = M < M_cap ? M : M_cap;
   const int rt = blockIdx.x;
@@ -295,8 +318,11 @@ k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const i
 // ---------------------------------------------------------------- verify rows
 // Candidates c_1 (next-byte argmax) and d_2..d_n (drafts) at positions t..t+n-1; embed them.
 __global__ void k_verify_plan(Dev D) {
+  TraceScope _trace(TT_VERIFY_PLAN);
+  __shared__ int s_c[64];
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int b = blockIdx.x;
@@ -308,13 +334,15 @@ __global__ void k_verify_plan(Dev D) {
     }
     return;
   }
-  const int t = D.seq[b].t;
-  if (b == 0 && tid == 0) *D.r_v.M = batch * n;
-  for (int i = tid; i < n; i += blockDim.x) {
+  if (tid < n) {
+    const int i = tid;
+    const int t = D.seq[b].t;
     int c;
     if (P.force_cand) c = D.forced_cand[b * D.NMAX + i];
     else c = i == 0 ? D.seq[b].next_c1 : D.mb_arg[b * (n - 1) + i - 1];
-    D.cand[b * D.NMAX + i] = c & 255;
+    c &= 255;
+    s_c[i] = c;
+    D.cand[b * D.NMAX + i] = c;
     const int r = b * n + i;
     int p = t + i;
     if (p >= D.S) {
@@ -329,15 +357,42 @@ __global__ void k_verify_plan(Dev D) {
   if (tid == 0) {
     D.r_v.seq_start[b] = b * n;
     D.r_v.seq_count[b] = n;
+    if (b == 0) *D.r_v.M = batch * n;
   }
   __syncthreads();
-  for (int idx = tid; idx < n * D.d; idx += blockDim.x) {
-    const int i = idx / D.d, k = idx - i * D.d;
-    const int c = D.cand[b * D.NMAX + i];
-    const float e = D.dtype == LCA_BF16
-                        ? ld_w(reinterpret_cast<const __nv_bfloat16*>(D.embed), (size_t)c * D.d + k)
-                        : ld_w(reinterpret_cast<const float*>(D.embed), (size_t)c * D.d + k);
-    D.x_enc[(size_t)(b * n + i) * D.d + k] = e;
+  // embedding rows of the candidates, 16-byte vectors, loads issued before the stores
+  const int ev = D.dtype == LCA_BF16 ? 8 : 4;  // elements per 16-byte vector
+  const int per_row = D.d / ev;
+  const int total = n * per_row;
+  constexpr int UNR = 4;
+  for (int base = tid; base < total; base += blockDim.x * UNR) {
+    uint4 u[UNR];
+#pragma unroll
+    for (int k = 0; k < UNR; ++k) {
+      const int idx = base + k * blockDim.x;
+      if (idx < total) {
+        const int i = idx / per_row, j = idx - i * per_row;
+        const char* row = reinterpret_cast<const char*>(D.embed) + (size_t)s_c[i] * D.d * (ev == 8 ? 2 : 4);
+        u[k] = *reinterpret_cast<const uint4*>(row + (size_t)j * 16);
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < UNR; ++k) {
+      const int idx = base + k * blockDim.x;
+      if (idx < total) {
+        const int i = idx / per_row, j = idx - i * per_row;
+        float* dst = D.x_enc + (size_t)(b * n + i) * D.d + (size_t)j * ev;
+        if (ev == 8) {
+          float f[8];
+          unpack8w(&u[k], f, (const __nv_bfloat16*)nullptr);
+          reinterpret_cast<float4*>(dst)[0] = make_float4(f[0], f[1], f[2], f[3]);
+          reinterpret_cast<float4*>(dst)[1] = make_float4(f[4], f[5], f[6], f[7]);
+        } else {
+          reinterpret_cast<float4*>(dst)[0] = make_float4(__uint_as_float(u[k].x), __uint_as_float(u[k].y),
+                                                          __uint_as_float(u[k].z), __uint_as_float(u[k].w));
+        }
+      }
+    }
   }
 }
 
@@ -348,14 +403,18 @@ __global__ void k_verify_plan(Dev D) {
 // K(p) of candidate row i counts boundaries at positions <= p. New latents of all sequences
 // are compacted into LM rows; the LM module runs (graph conditional) only if there are any.
 __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handle) {
+  TraceScope _trace(TT_SEGMENT);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int b = blockIdx.x;
   const int tid = threadIdx.x;
+  __shared__ int s_c[64];
   __shared__ int s_sp[64];
-  __shared__ int s_nsp, s_off;
+  __shared__ int s_nsp;
+  __shared__ SeqState s_st;
   if (b >= batch) {
     if (tid == 0) {
       D.r_lm.seq_start[b] = 0;
@@ -363,19 +422,25 @@ __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handl
     }
     return;
   }
+  // boundaries among the candidates of earlier sequences (compaction offset) and of all
+  int off = 0, total = 0;
+  for (int base = 0; base < batch * n; base += blockDim.x) {
+    const int idx = base + tid;
+    const int bb = idx / n, i = idx - bb * n;
+    const bool sp = idx < batch * n && D.cand[bb * D.NMAX + i] == D.boundary;
+    off += __syncthreads_count(sp && bb < b);
+    if (b == 0) total += __syncthreads_count(sp);
+  }
+  if (tid < n) s_c[tid] = D.cand[b * D.NMAX + tid];
+  if (tid == 0) s_st = D.seq[b];
+  __syncthreads();
   if (tid == 0) {
-    int off = 0, total = 0;
-    for (int bb = 0; bb < batch; ++bb) {
-      int c = 0;
-      for (int i = 0; i < n; ++i) c += D.cand[bb * D.NMAX + i] == D.boundary;
-      if (bb < b) off += c;
-      total += c;
-    }
-    s_off = off;
     int m = 0;
     for (int i = 0; i < n; ++i)
-      if (D.cand[b * D.NMAX + i] == D.boundary) s_sp[m++] = i;
+      if (s_c[i] == D.boundary) s_sp[m++] = i;
     s_nsp = m;
+    D.r_lm.seq_start[b] = off;
+    D.r_lm.seq_count[b] = m;
     if (b == 0) {
       *D.r_lm.M = total;
       if (use_handle) cudaGraphSetConditional(hcond, total > 0 ? 1u : 0u);
@@ -384,23 +449,19 @@ __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handl
       D.stats->lm_rows += total;
     }
   }
-  __syncthreads();
-  const SeqState st = D.seq[b];
-  const int t = st.t, K = st.K;
-  const int m = s_nsp, off = s_off;
+  const int t = s_st.t, K = s_st.K;
   if (tid < n) {
     int k = K;
-    for (int i = 0; i <= tid; ++i) k += D.cand[b * D.NMAX + i] == D.boundary;
+    for (int i = 0; i <= tid; ++i) k += s_c[i] == D.boundary;
     D.kc[b * D.NMAX + tid] = k;
   }
-  if (tid == 0) {
-    D.r_lm.seq_start[b] = off;
-    D.r_lm.seq_count[b] = m;
-  }
+  __syncthreads();
+  const int m = s_nsp;
+  const int d4 = D.d / 4;
   for (int j = 0; j < m; ++j) {
     const int i = s_sp[j];
     const int k = K + 1 + j;
-    const int seg0 = j == 0 ? st.open_start : t + s_sp[j - 1] + 1;
+    const int seg0 = j == 0 ? s_st.open_start : t + s_sp[j - 1] + 1;
     const int seg1 = t + i;  // inclusive
     const int row = off + j;
     if (k >= D.L) {
@@ -408,14 +469,31 @@ __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handl
       continue;
     }
     const float inv_cnt = 1.f / (float)(seg1 - seg0 + 1);
-    for (int c = tid; c < D.d; c += blockDim.x) {
-      float s = 0.f;
-      for (int p = seg0; p <= seg1; ++p)
-        s += p < t ? D.h_store[((size_t)b * D.S + p) * D.d + c]
-                   : D.x_enc[(size_t)(b * n + p - t) * D.d + c];
-      const float z = s * inv_cnt;
-      D.x_lm[(size_t)row * D.d + c] = z;
-      D.u_tab[((size_t)b * D.L + k) * D.d + c] = z;
+    for (int c4 = tid; c4 < d4; c4 += blockDim.x) {
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      int p = seg0;
+      // four positions per round, loads issued together
+      for (; p + 3 <= seg1; p += 4) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int q = p + u;
+          v[u] = q < t ? reinterpret_cast<const float4*>(D.h_store + ((size_t)b * D.S + q) * D.d)[c4]
+                       : reinterpret_cast<const float4*>(D.x_enc + (size_t)(b * n + q - t) * D.d)[c4];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          acc.x += v[u].x; acc.y += v[u].y; acc.z += v[u].z; acc.w += v[u].w;
+        }
+      }
+      for (; p <= seg1; ++p) {
+        const float4 v = p < t ? reinterpret_cast<const float4*>(D.h_store + ((size_t)b * D.S + p) * D.d)[c4]
+                               : reinterpret_cast<const float4*>(D.x_enc + (size_t)(b * n + p - t) * D.d)[c4];
+        acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+      }
+      const float4 z = make_float4(acc.x * inv_cnt, acc.y * inv_cnt, acc.z * inv_cnt, acc.w * inv_cnt);
+      reinterpret_cast<float4*>(D.x_lm + (size_t)row * D.d)[c4] = z;
+      reinterpret_cast<float4*>(D.u_tab + ((size_t)b * D.L + k) * D.d)[c4] = z;
     }
     if (tid == 0) {
       D.gstart[(size_t)b * D.L + k] = seg1;
@@ -429,8 +507,10 @@ __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handl
 
 // o_k of the latents the LM module just produced.
 __global__ void k_lm_scatter(Dev D) {
+  TraceScope _trace(TT_LM_SCATTER);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const int M = *D.r_lm.M;
   for (int r = blockIdx.x; r < M; r += gridDim.x) {
     const int b = D.r_lm.b[r], k = D.r_lm.pos[r];
@@ -442,8 +522,10 @@ __global__ void k_lm_scatter(Dev D) {
 // Next-byte decoder input: upsampled LM output plus the encoder residual r_1 (Algorithm 1
 // line 8): o_{K(p)} + h_e[p].
 __global__ void k_nb_input(Dev D) {
+  TraceScope _trace(TT_NB_INPUT);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int rows = batch * n;
@@ -462,73 +544,97 @@ __global__ void k_nb_input(Dev D) {
 // position before them (SPEC); the first failure drops the rest. The accepted prefix of every
 // cache is kept by advancing t and K; everything beyond is dropped (overwritten later).
 __global__ void k_commit(Dev D) {
+  TraceScope _trace(TT_COMMIT);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int b = blockIdx.x;
   if (b >= batch) return;
   const int tid = threadIdx.x;
-  __shared__ int s_e, s_a, s_t, s_skip;
-  SeqState& st = D.seq[b];
+  __shared__ int s_c[64], s_kc[64], s_nb[64], s_ok[64];
+  __shared__ SeqState s_st;
+  __shared__ int s_e, s_a;
+  if (tid < n) {
+    s_c[tid] = D.cand[b * D.NMAX + tid];
+    s_kc[tid] = D.kc[b * D.NMAX + tid];
+    s_nb[tid] = D.nb_arg[b * n + tid];
+  }
+  if (tid < n - 1) {
+    s_ok[tid] = P.accept == LCA_SPEC ? D.cand[b * D.NMAX + tid + 1] == D.nb_arg[b * n + tid]
+                                     : D.mb_prob[b * (n - 1) + tid] >= P.tau;
+  }
+  if (tid == 0) s_st = D.seq[b];
+  __syncthreads();
   if (tid == 0) {
-    s_skip = 0;
-    s_t = st.t;
-    if (P.gen && st.done) {
-      D.out_cnt[b] = 0;
-      s_skip = 1;
-    } else {
-      const int* cand = D.cand + b * D.NMAX;
-      int a = 0;
+    int a = 0, e = 0;
+    if (!(P.gen && s_st.done)) {
       if (P.force_accept) {
         a = D.forced_a[b];
         a = a < 0 ? 0 : (a > n - 1 ? n - 1 : a);
       } else {
-        for (int j = 0; j < n - 1; ++j) {
-          const bool ok = P.accept == LCA_SPEC ? cand[j + 1] == D.nb_arg[b * n + j]
-                                               : D.mb_prob[b * (n - 1) + j] >= P.tau;
-          if (!ok) break;
-          ++a;
-        }
+        while (a < n - 1 && s_ok[a]) ++a;
       }
-      int e = 1 + a;
+      e = 1 + a;
       if (P.gen) {
-        const int rem = st.budget - st.generated;
+        const int rem = s_st.budget - s_st.generated;
         e = e < rem ? e : rem;
       }
-      s_e = e;
-      s_a = a;
     }
+    s_e = e;
+    s_a = a;
   }
   __syncthreads();
-  if (s_skip) return;
-  const int e = s_e, t = s_t;
-  // encoder outputs of the committed candidates join the pooled history
-  for (int idx = tid; idx < e * D.d; idx += blockDim.x) {
-    const int i = idx / D.d, c = idx - i * D.d;
-    D.h_store[((size_t)b * D.S + t + i) * D.d + c] = D.x_enc[(size_t)(b * n + i) * D.d + c];
+  const int e = s_e, t = s_st.t;
+  if (e == 0) {
+    if (tid == 0) D.out_cnt[b] = 0;
+    return;
   }
-  for (int c = tid; c < D.d; c += blockDim.x)
-    D.y_last[(size_t)b * D.d + c] = D.x_nb[(size_t)(b * n + e - 1) * D.d + c];
-  if (tid == 0) {
-    const int* cand = D.cand + b * D.NMAX;
-    int last_sp = -1;
-    const int gen0 = st.generated;
-    for (int i = 0; i < n; ++i) {
-      const int c = cand[i];
-      D.out_step[b * D.NMAX + i] = (uint8_t)(i < e ? c : 0);
-      if (i < e) {
-        if (c == D.boundary) last_sp = i;
-        if (P.gen && gen0 + i < D.S) D.out_gen[(size_t)b * D.S + gen0 + i] = (uint8_t)c;
+  // encoder outputs of the committed candidates join the pooled history; the last next-byte
+  // hidden state feeds the MLP heads (float4 copies, loads before stores)
+  const int d4 = D.d / 4;
+  const int tot = e * d4 + d4;
+  for (int base = tid; base < tot; base += blockDim.x * 4) {
+    float4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int idx = base + u * blockDim.x;
+      if (idx < e * d4) {
+        const int i = idx / d4, c4 = idx - i * d4;
+        v[u] = reinterpret_cast<const float4*>(D.x_enc + (size_t)(b * n + i) * D.d)[c4];
+      } else if (idx < tot) {
+        v[u] = reinterpret_cast<const float4*>(D.x_nb + (size_t)(b * n + e - 1) * D.d)[idx - e * d4];
       }
     }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int idx = base + u * blockDim.x;
+      if (idx < e * d4) {
+        const int i = idx / d4, c4 = idx - i * d4;
+        reinterpret_cast<float4*>(D.h_store + ((size_t)b * D.S + t + i) * D.d)[c4] = v[u];
+      } else if (idx < tot) {
+        reinterpret_cast<float4*>(D.y_last + (size_t)b * D.d)[idx - e * d4] = v[u];
+      }
+    }
+  }
+  if (tid < n) {
+    const int i = tid;
+    D.out_step[b * D.NMAX + i] = (uint8_t)(i < e ? s_c[i] : 0);
+    if (P.gen && i < e && s_st.generated + i < D.S) D.out_gen[(size_t)b * D.S + s_st.generated + i] = (uint8_t)s_c[i];
+  }
+  if (tid == 0) {
+    int last_sp = -1;
+    for (int i = 0; i < e; ++i)
+      if (s_c[i] == D.boundary) last_sp = i;
+    SeqState& st = D.seq[b];
     D.out_cnt[b] = e;
     st.t = t + e;
-    st.K = D.kc[b * D.NMAX + e - 1];
+    st.K = s_kc[e - 1];
     if (last_sp >= 0) st.open_start = t + last_sp + 1;
-    st.next_c1 = D.nb_arg[b * n + e - 1];
-    st.generated = gen0 + e;
-    if (P.gen && st.generated >= st.budget) st.done = 1;
+    st.next_c1 = s_nb[e - 1];
+    st.generated = s_st.generated + e;
+    if (P.gen && st.generated >= s_st.budget) st.done = 1;
     atomicAdd(D.hist + s_a, 1);
     atomicAdd(&D.stats->committed, (unsigned long long)e);
   }
@@ -537,8 +643,10 @@ __global__ void k_commit(Dev D) {
 // Generate loop control: keep looping while a sequence is short of its budget (and never more
 // than max_iter steps, each of which commits at least one byte per unfinished sequence).
 __global__ void k_loop_ctl(Dev D, cudaGraphConditionalHandle h) {
+  TraceScope _trace(TT_LOOP_CTL);
   pdl_trigger();
   pdl_wait();
+  _trace.waited();
   if (threadIdx.x != 0) return;
   Params* P = D.params;
   const int it = P->iter + 1;
@@ -830,5 +938,7 @@ void launch_prefill_finish(const Dev& D, const int* row0, const int* lens, const
   (void)lm_row0;
   launch_pdl(k_prefill_finish, dim3(batch), dim3(256), 0, s, D, row0, lens);
 }
+
+LCA_TRACE_SETTER(trace_set_step)
 
 } // namespace lca

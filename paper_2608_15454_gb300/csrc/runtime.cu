@@ -250,13 +250,13 @@ bool tiled_for(int rows) { return rows > 64; }
 
 int attn_splits(const Dev& D, int batch_cap, int qtiles) {
   int s = (2 * 152) / std::max(1, batch_cap * D.H * qtiles);
-  return std::max(1, std::min(s, kMaxAttnSplit));
+  return std::max(1, std::min(std::min(s, kMaxAttnSplit), D.attn_split_cap));
 }
 
 // Run the pre-norm blocks of one module over rows [0, *rows.M) of x (in place).
 void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& rows, int M_cap,
                int M_typ, int qt_grid, int splits, cudaStream_t s, const void* next_w = nullptr,
-               size_t next_bytes = 0) {
+               size_t next_bytes = 0, const int* stable = nullptr, int stable_extra = 0) {
   Dev& D = c->L.D;
   const bool tiled = tiled_for(M_typ);
   const size_t tb = tw_bytes(D.dtype);
@@ -297,7 +297,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.pf[1] = bk.w13;
     a.pf_bytes[1] = b_13;
     linear(D, a, tiled, s);
-    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s);
+    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra);
     // x += Wo . attn
     a.x = D.att;
     a.W = bk.wo;
@@ -375,7 +375,6 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
   if (n >= 2) {
     if (D.mb_kind == LCA_MB_LCA) {
       launch_mb_plan(D, s);
-      launch_mb_fill(D, s);
       const int typ = B * (2 * n - 2);  // typical window rows: new committed bytes + copies
       run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2), s,
                 c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype));
@@ -389,7 +388,8 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
   // (1) embed + encoder over the n candidates
   launch_verify_plan(D, s);
   run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s,
-            c->L.nb.empty() ? nullptr : c->L.nb[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype));
+            c->L.nb.empty() ? nullptr : c->L.nb[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype),
+            &D.seq[0].t, n);
 }
 
 void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
@@ -404,7 +404,8 @@ void enqueue_verify_commit(lca_ctx* c, int n, cudaStream_t s) {
   const int B = D.B;
   // (4) upsample + next-byte decoder over the n candidates, head
   launch_nb_input(D, s);
-  run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s);
+  run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s, nullptr, 0,
+            &D.seq[0].t, n);
   launch_head(D, D.x_nb, nullptr, D.r_v.M, B * n, D.nb_norm, D.nb_logits, D.nb_arg, D.nb_prob, s);
   // (5) accept + commit
   launch_commit(D, s);
@@ -738,6 +739,8 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.num_sms = sms > 0 ? sms : 148;
     const char* e = getenv("LCA_NO_TMA");
     D.use_tma = (e && e[0] == '1') ? 0 : 1;
+    const char* sc = getenv("LCA_ATTN_SPLIT_CAP");
+    D.attn_split_cap = sc ? std::max(1, std::min(8, atoi(sc))) : 4;
   }
   // state and counters start at zero
   if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);
@@ -1194,6 +1197,52 @@ int lca_debug_bench_kernel(lca_ctx* c, int32_t kind, int32_t rows, int32_t iters
   *us = ms * 1000.0 / (reps * iters);
   *bytes = by;
   c->prefilled = false;  // the row descriptors were overwritten: prefill again before stepping
+  return read_err(c);
+}
+
+int lca_debug_trace(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t steps, void* out,
+                    int32_t cap, int32_t* count) {
+  if (!out || !count || cap < 1 || steps < 1) return LCA_E_ARG;
+  int st = step_prep(c, n, tau, mode);
+  if (st != LCA_OK) return st;
+  for (int b = 0; b < c->batch; ++b)
+    if (c->t_host[b] + (long long)steps * n > c->cfg.max_bytes) return LCA_E_CAPACITY;
+  cudaGraphExec_t ex;
+  st = get_step_exec(c, n, &ex);
+  if (st != LCA_OK) return st;
+  // the trace buffer borrows the split-K scratch (unused by the bf16 step)
+  Dev& D = c->L.D;
+  const size_t rec_cap = D.lin_part_floats * sizeof(float) / sizeof(TraceRec);
+  const unsigned capu = (unsigned)std::min<size_t>(rec_cap, (size_t)cap);
+  if (capu == 0) return LCA_E_CAPACITY;
+  TraceRec* buf = reinterpret_cast<TraceRec*>(D.lin_part);
+  unsigned* counter = reinterpret_cast<unsigned*>(D.lin_cnt);
+  CK(cudaMemsetAsync(counter, 0, sizeof(unsigned), c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  trace_set_linear(buf, counter, capu);
+  trace_set_attn(buf, counter, capu);
+  trace_set_step(buf, counter, capu);
+  Params& P = c->host_params;
+  P.gen = 0;
+  P.force_accept = 0;
+  P.force_cand = 0;
+  st = upload_params(c);
+  if (st != LCA_OK) return st;
+  for (int i = 0; i < steps; ++i) CK(cudaGraphLaunch(ex, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  trace_set_linear(nullptr, nullptr, 0);
+  trace_set_attn(nullptr, nullptr, 0);
+  trace_set_step(nullptr, nullptr, 0);
+  unsigned got = 0;
+  CK(cudaMemcpy(&got, counter, sizeof(unsigned), cudaMemcpyDeviceToHost));
+  got = std::min(got, capu);
+  CK(cudaMemcpy(out, buf, sizeof(TraceRec) * got, cudaMemcpyDeviceToHost));
+  CK(cudaMemset(counter, 0, sizeof(unsigned)));
+  *count = (int32_t)got;
+  c->last_n = n;
+  std::vector<SeqState> all(c->batch);
+  CK(cudaMemcpy(all.data(), D.seq, sizeof(SeqState) * c->batch, cudaMemcpyDeviceToHost));
+  for (int i = 0; i < c->batch; ++i) c->t_host[i] = all[i].t;
   return read_err(c);
 }
 

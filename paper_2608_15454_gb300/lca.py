@@ -25,7 +25,7 @@ STATUS = {0: "LCA_OK", -1: "LCA_E_ARG", -2: "LCA_E_CAPACITY", -3: "LCA_E_WEIGHTS
 EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "lca_mbp_step_async",
            "lca_generate",
            "lca_generate_async", "lca_generate_fetch", "lca_debug_state", "lca_debug_stats",
-           "lca_debug_set_eager", "lca_debug_profile", "lca_debug_bench_kernel",
+           "lca_debug_set_eager", "lca_debug_profile", "lca_debug_bench_kernel", "lca_debug_trace",
            "lca_debug_logits",
            "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str",
            "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
@@ -98,6 +98,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_debug_stats": [P, ctypes.POINTER(LcaStats)],
         "lca_debug_logits": [P, P, P],
         "lca_debug_set_eager": [P, I32],
+        "lca_debug_trace": [P, I32, F32, I32, I32, P, I32, ctypes.POINTER(I32)],
         "lca_debug_bench_kernel": [P, I32, I32, I32, ctypes.POINTER(ctypes.c_double),
                                    ctypes.POINTER(ctypes.c_double)],
         "lca_debug_profile": [P, I32, F32, I32, I32, ctypes.POINTER(LcaProfile)],
@@ -245,6 +246,18 @@ class Context:
                     "lca_debug_profile")
         return {k: {"launches": p.launches[i], "ms": p.ms[i], "bytes": p.bytes[i]}
                 for i, k in enumerate(PROFILE_KINDS)}
+
+    TRACE_TAGS = {1: "gemv", 2: "gemv_f32", 3: "gemm", 4: "rowstats", 5: "attn", 6: "head",
+                  7: "mb_plan", 8: "mb_fill", 9: "mlp_plan", 10: "verify_plan", 11: "segment",
+                  12: "lm_scatter", 13: "nb_input", 14: "commit", 15: "loop_ctl", 16: "other"}
+
+    def trace(self, n, tau, mode, steps, cap=1 << 18):
+        rec = np.zeros(cap, dtype=[("t0", "<u8"), ("t1", "<u8"), ("tw", "<u8"), ("tag", "<i4"),
+                                   ("cta", "<i4"), ("sm", "<i4"), ("pad", "<i4")])
+        cnt = ctypes.c_int32()
+        self._check(self.lib.lca_debug_trace(self.h, n, tau, mode, steps, _ptr(rec), cap, ctypes.byref(cnt)),
+                    "lca_debug_trace")
+        return rec[:cnt.value]
 
     def bench_kernel(self, kind, rows, iters):
         us, by = ctypes.c_double(), ctypes.c_double()
