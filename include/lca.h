@@ -179,6 +179,13 @@ int lca_debug_profile(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, i
 int lca_debug_trace(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t steps,
                     void* out, int32_t cap, int32_t* count);
 
+/* The tensor-core linear layer alone: y[0:*M_dev] = bf16(x) . W^T (fp32 accumulation, tcgen05).
+ * x: device fp32 [M][K]; W: device bf16 [N][K]; y: device fp32 [M][N]; M_dev: device int32 rows
+ * to compute (<= M); err_dev: device int32 error word (bit 4: a bounded wait ran out). N and K must
+ * be multiples of 64. Asynchronous on `stream`. */
+int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N, int32_t K,
+                   const int32_t* M_dev, int32_t* err_dev, void* stream);
+
 /* Micro-benchmark: one graph of `iters` back-to-back launches of one kernel kind over `rows`
  * rows (0 RMSNorm+QKV, 1 Wo, 2 RMSNorm+W1/W3+SwiGLU, 3 W2, 4 decode attention over the
  * encoder cache, 5 unembedding head, 6 a glue kernel), cycling through all blocks' weights so

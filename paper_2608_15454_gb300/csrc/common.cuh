@@ -222,6 +222,7 @@ struct Dev {
   int num_sms;  // streaming multiprocessors of the device
   int use_tma;  // bf16 linear layers use the bulk-copy weight pipeline
   int attn_split_cap;  // largest cluster (key split) of decode attention
+  int use_umma;        // many-row bf16 layers run on the tensor cores (tcgen05)
 
   // weights (storage type; norms and bos fp32)
   void* embed;   // [256][d]
@@ -317,8 +318,13 @@ struct LinearArgs {
   const void* pf[2];
   size_t pf_bytes[2];
   int rows_typ;  // typical row count (sizes the activation staging); 0: M_cap
+  const void* tmap;  // host copy of the weight's TMA tensor map (tensor-core path), or nullptr
 };
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s);
+bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s);
+int make_weight_tmap(void* out, const void* W, long long rows, long long K);
+void kernel_attrs_umma();
+void trace_set_umma(TraceRec* buf, unsigned* counter, unsigned cap);
 
 size_t attention_scratch_floats(int B, int H, int hd);
 size_t attention_counters(int B, int H);

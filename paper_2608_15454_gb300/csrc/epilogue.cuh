@@ -1,0 +1,161 @@
+// Epilogues of the linear layers, shared by the CUDA-core and tensor-core kernels: residual add,
+// SwiGLU, residual SiLU (MLP head), and Q/K/V with rotary embedding and the KV-cache append.
+#pragma once
+#include "common.cuh"
+
+namespace lca {
+
+static __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
+
+static __device__ __forceinline__ void store_cache(float* p, float v) { *p = v; }
+static __device__ __forceinline__ void store_cache(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
+
+// Epilogue of one pair of adjacent output columns (c even) of row r.
+template <typename TC>
+static __device__ __forceinline__ void epi_pair(const EpiArgs& e, int r, int c, float a0, float a1) {
+  switch (e.mode) {
+    case EPI_STORE: {
+      float* y = e.y + (size_t)r * e.ldy + c;
+      y[0] = a0;
+      y[1] = a1;
+      break;
+    }
+    case EPI_RESID: {
+      const float* rr = e.res + (size_t)r * e.ldres + c;
+      float r0 = rr[0], r1 = rr[1];
+      float* y = e.y + (size_t)r * e.ldy + c;
+      y[0] = r0 + a0;
+      y[1] = r1 + a1;
+      break;
+    }
+    case EPI_RESID_SILU: {
+      const float* rr = e.res + (size_t)r * e.ldres + c;
+      float r0 = rr[0], r1 = rr[1];
+      float* y = e.y + (size_t)r * e.ldy + c;
+      y[0] = r0 + silu_f(a0);
+      y[1] = r1 + silu_f(a1);
+      break;
+    }
+    case EPI_SWIGLU: {
+      e.y[(size_t)r * e.ldy + (c >> 1)] = silu_f(a0) * a1;
+      break;
+    }
+    case EPI_QKV: {
+      const int part = c / e.d;
+      const int cc = c - part * e.d;
+      const int h = cc / e.hd;
+      const int dd = cc - h * e.hd;
+      if (part < 2) {
+        const int pos = e.rows.pos[r];
+        const float2 cs = e.rope[(size_t)pos * (e.hd >> 1) + (dd >> 1)];
+        const float r0 = a0 * cs.x - a1 * cs.y;
+        const float r1 = a0 * cs.y + a1 * cs.x;
+        a0 = r0;
+        a1 = r1;
+      }
+      if (part == 0) {
+        float* y = e.y + (size_t)r * e.ldy + cc;
+        y[0] = a0;
+        y[1] = a1;
+      } else {
+        const int b = e.rows.b[r];
+        const int slot = e.rows.slot[r];
+        if (slot < 0 || slot >= e.kv.S) {
+          atomicOr(e.err, kErrIndex);
+          return;
+        }
+        TC* base = reinterpret_cast<TC*>(part == 1 ? e.kv.k : e.kv.v);
+        TC* p = base + (((size_t)b * e.H + h) * e.kv.S + slot) * e.hd + dd;
+        store_cache(p, a0);
+        store_cache(p + 1, a1);
+      }
+      break;
+    }
+  }
+}
+
+// Epilogue operands that do not depend on the dot products (residual values, RoPE angle,
+// cache slot), loaded early so that their latency overlaps the main loop.
+struct EpiPre {
+  float r0, r1;  // residual pair
+  float2 cs;     // RoPE cos/sin
+  int b, slot;
+};
+
+static __device__ __forceinline__ EpiPre epi_load(const EpiArgs& e, int r, int c) {
+  EpiPre p;
+  p.r0 = p.r1 = 0.f;
+  p.cs = make_float2(1.f, 0.f);
+  p.b = p.slot = 0;
+  if (e.mode == EPI_RESID || e.mode == EPI_RESID_SILU) {
+    const float2 q = *reinterpret_cast<const float2*>(e.res + (size_t)r * e.ldres + c);
+    p.r0 = q.x;
+    p.r1 = q.y;
+  } else if (e.mode == EPI_QKV) {
+    const int part = c / e.d;
+    const int cc = c - part * e.d;
+    const int dd = cc % e.hd;
+    if (part < 2) {
+      const int pos = e.rows.pos[r];
+      p.cs = e.rope[(size_t)pos * (e.hd >> 1) + (dd >> 1)];
+    }
+    if (part > 0) {
+      p.b = e.rows.b[r];
+      p.slot = e.rows.slot[r];
+    }
+  }
+  return p;
+}
+
+template <typename TC>
+static __device__ __forceinline__ void epi_store(const EpiArgs& e, const EpiPre& p, int r, int c, float a0, float a1) {
+  switch (e.mode) {
+    case EPI_STORE: {
+      float* y = e.y + (size_t)r * e.ldy + c;
+      *reinterpret_cast<float2*>(y) = make_float2(a0, a1);
+      break;
+    }
+    case EPI_RESID: {
+      float* y = e.y + (size_t)r * e.ldy + c;
+      *reinterpret_cast<float2*>(y) = make_float2(p.r0 + a0, p.r1 + a1);
+      break;
+    }
+    case EPI_RESID_SILU: {
+      float* y = e.y + (size_t)r * e.ldy + c;
+      *reinterpret_cast<float2*>(y) = make_float2(p.r0 + silu_f(a0), p.r1 + silu_f(a1));
+      break;
+    }
+    case EPI_SWIGLU: {
+      e.y[(size_t)r * e.ldy + (c >> 1)] = silu_f(a0) * a1;
+      break;
+    }
+    case EPI_QKV: {
+      const int part = c / e.d;
+      const int cc = c - part * e.d;
+      const int h = cc / e.hd;
+      const int dd = cc - h * e.hd;
+      if (part < 2) {
+        const float x0 = a0 * p.cs.x - a1 * p.cs.y;
+        const float x1 = a0 * p.cs.y + a1 * p.cs.x;
+        a0 = x0;
+        a1 = x1;
+      }
+      if (part == 0) {
+        *reinterpret_cast<float2*>(e.y + (size_t)r * e.ldy + cc) = make_float2(a0, a1);
+      } else {
+        if (p.slot < 0 || p.slot >= e.kv.S) {
+          atomicOr(e.err, kErrIndex);
+          return;
+        }
+        TC* base = reinterpret_cast<TC*>(part == 1 ? e.kv.k : e.kv.v);
+        TC* q = base + (((size_t)p.b * e.H + h) * e.kv.S + p.slot) * e.hd + dd;
+        store_cache(q, a0);
+        store_cache(q + 1, a1);
+      }
+      break;
+    }
+  }
+}
+
+
+}  // namespace lca

@@ -174,7 +174,12 @@ struct Staging {
 
 }  // namespace
 
+struct alignas(64) TMapBlob {
+  unsigned char b[128];
+};
+
 struct lca_ctx {
+  std::map<const void*, TMapBlob> tmaps;  // TMA tensor maps of the bf16 weights
   lca_config cfg{};
   Layout L;
   Staging stg{};
@@ -248,6 +253,11 @@ int upload_params(lca_ctx* c) {
 
 bool tiled_for(int rows) { return rows > 64; }
 
+const void* tmap_of(lca_ctx* c, const void* W) {
+  auto it = c->tmaps.find(W);
+  return it == c->tmaps.end() ? nullptr : it->second.b;
+}
+
 int attn_splits(const Dev& D, int batch_cap, int qtiles) {
   int s = (2 * 152) / std::max(1, batch_cap * D.H * qtiles);
   return std::max(1, std::min(std::min(s, kMaxAttnSplit), D.attn_split_cap));
@@ -296,6 +306,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.pf_bytes[0] = b_o;
     a.pf[1] = bk.w13;
     a.pf_bytes[1] = b_13;
+    a.tmap = tmap_of(c, a.W);
     linear(D, a, tiled, s);
     attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra);
     // x += Wo . attn
@@ -311,6 +322,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.pf_bytes[0] = b_2;
     a.pf[1] = nullptr;
     a.pf_bytes[1] = 0;
+    a.tmap = tmap_of(c, a.W);
     linear(D, a, tiled, s);
     // mid = silu(W1 . n(x)) * (W3 . n(x))
     a.x = x;
@@ -322,6 +334,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.epi.ldy = D.F;
     a.pf[0] = nqkv;
     a.pf_bytes[0] = nqkv_b;
+    a.tmap = tmap_of(c, a.W);
     linear(D, a, tiled, s);
     // x += W2 . mid
     a.x = D.mid;
@@ -336,6 +349,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.epi.ldy = a.epi.ldres = D.d;
     a.pf[0] = nx ? nx->wo : nullptr;
     a.pf_bytes[0] = nx ? b_o : 0;
+    a.tmap = tmap_of(c, a.W);
     linear(D, a, tiled, s);
   }
 }
@@ -363,6 +377,7 @@ void run_mlp_heads(lca_ctx* c, int n, cudaStream_t s) {
     a.epi.res = D.x_mb;
     a.epi.ldy = a.epi.ldres = D.d;
     a.epi.err = D.err;
+    a.tmap = tmap_of(c, a.W);
     linear(D, a, tiled_for(D.B), s);
   }
 }
@@ -731,6 +746,7 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     return fail(LCA_E_CUDA);
   kernel_attrs_linear();
   kernel_attrs_step();
+  kernel_attrs_umma();
   Dev& D = c->L.D;
   {
     int dev = 0, sms = 0;
@@ -739,6 +755,8 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.num_sms = sms > 0 ? sms : 148;
     const char* e = getenv("LCA_NO_TMA");
     D.use_tma = (e && e[0] == '1') ? 0 : 1;
+    const char* um = getenv("LCA_NO_UMMA");
+    D.use_umma = (um && um[0] == '1') ? 0 : 1;
     const char* sc = getenv("LCA_ATTN_SPLIT_CAP");
     D.attn_split_cap = sc ? std::max(1, std::min(8, atoi(sc))) : 4;
   }
@@ -746,6 +764,22 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
   if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);
   st = load_weights(c, weights, n_weights);
   if (st != LCA_OK) return fail(st);
+  if (cfg->dtype == LCA_BF16) {
+    auto add = [&](const void* W, long long rows, long long K) {
+      TMapBlob blob;
+      if (make_weight_tmap(blob.b, W, rows, K) == LCA_OK) c->tmaps[W] = blob;
+    };
+    for (auto* v : {&c->L.enc, &c->L.lm, &c->L.nb, &c->L.mb})
+      for (auto& bk : *v) {
+        add(bk.wqkv, 3LL * D.d, D.d);
+        add(bk.wo, D.d, D.d);
+        add(bk.w13, 2LL * D.F, D.d);
+        add(bk.w2, D.d, D.F);
+      }
+    if (D.mlp_w)
+      for (int l = 0; l < D.n_mb; ++l)
+        add((char*)D.mlp_w + (size_t)l * D.n_mlp_heads * D.d * D.d * 2, (long long)D.n_mlp_heads * D.d, D.d);
+  }
   launch_rope_table(D, cfg->rope_base, c->stream);
   if (check(cudaGetLastError(), "rope") || check(cudaStreamSynchronize(c->stream), "create sync"))
     return fail(LCA_E_CUDA);
@@ -1222,6 +1256,7 @@ int lca_debug_trace(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t step
   trace_set_linear(buf, counter, capu);
   trace_set_attn(buf, counter, capu);
   trace_set_step(buf, counter, capu);
+  trace_set_umma(buf, counter, capu);
   Params& P = c->host_params;
   P.gen = 0;
   P.force_accept = 0;
@@ -1233,6 +1268,7 @@ int lca_debug_trace(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t step
   trace_set_linear(nullptr, nullptr, 0);
   trace_set_attn(nullptr, nullptr, 0);
   trace_set_step(nullptr, nullptr, 0);
+  trace_set_umma(nullptr, nullptr, 0);
   unsigned got = 0;
   CK(cudaMemcpy(&got, counter, sizeof(unsigned), cudaMemcpyDeviceToHost));
   got = std::min(got, capu);

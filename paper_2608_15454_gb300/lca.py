@@ -28,6 +28,7 @@ EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "
            "lca_debug_set_eager", "lca_debug_profile", "lca_debug_bench_kernel", "lca_debug_trace",
            "lca_debug_logits",
            "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str",
+           "lca_debug_gemm",
            "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
            "lca_decode_attention_noalloc_capacity")
 
@@ -106,6 +107,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_debug_force_candidates": [P, P, I32],
         "lca_destroy": [P],
         "lca_status_str": [ctypes.c_int],
+        "lca_debug_gemm": [P, P, P, I32, I32, I32, P, P, P],
         "lca_decode_attention_scratch_bytes": [I32, I32, I32, I32, ctypes.POINTER(ctypes.c_size_t)],
         "lca_decode_attention": [P, P, P, P, I32, I32, I32, I32, I32, I32, P, F32, I32, P,
                                  ctypes.c_size_t, P],
@@ -303,6 +305,15 @@ def decode_attention(q, out, k_cache, v_cache, kv_len, scale, splits, scratch=No
     if noalloc:
         return lib.lca_decode_attention_noalloc(*args, st.cuda_stream)
     return lib.lca_decode_attention(*args, scratch.data_ptr(), scratch.numel(), st.cuda_stream)
+
+
+def debug_gemm(x, W, y, M_dev, err_dev, stream=None):
+    """y[:M] = bf16(x[:M]) . W^T on the tensor cores (tcgen05). x fp32 [M,K], W bf16 [N,K],
+    y fp32 [M,N], M_dev int32 [1] (rows actually used), err_dev int32 [1]. Returns the status."""
+    import torch
+    st = stream if stream is not None else torch.cuda.current_stream(x.device)
+    return load_library().lca_debug_gemm(x.data_ptr(), W.data_ptr(), y.data_ptr(), x.shape[0], W.shape[0],
+                                         W.shape[1], M_dev.data_ptr(), err_dev.data_ptr(), st.cuda_stream)
 
 
 def decode_attention_scratch_bytes(batch, heads, head_dim, splits):

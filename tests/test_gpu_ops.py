@@ -67,3 +67,25 @@ def test_decode_attention_rejects_bad_arguments(lca):
     small = torch.empty(256, dtype=torch.uint8, device="cuda")
     assert lca.decode_attention(q, out, k, v, lens, 0.1, 4, small) == -2
     assert lca.decode_attention(q, out, k, v, lens, 0.1, 99, small) == -1
+
+
+@pytest.mark.parametrize("M,Mused,N,K", [(128, 128, 64, 64), (200, 200, 128, 1024), (300, 257, 1024, 1024),
+                                         (64, 17, 192, 4096), (1024, 1000, 3072, 1024)])
+def test_tensor_core_gemm_matches_reference(lca, M, Mused, N, K):
+    """tcgen05 GEMM (TMA weight tiles, 128-byte swizzle, TMEM accumulator) against a PyTorch
+    fp32 product of the same bf16-rounded operands."""
+    import torch
+    g = torch.Generator(device="cuda").manual_seed(M + N + K)
+    x = torch.randn(M, K, device="cuda", generator=g)
+    W = (torch.randn(N, K, device="cuda", generator=g) * 0.05).to(torch.bfloat16)
+    y = torch.full((M, N), float("nan"), device="cuda")
+    Md = torch.tensor([Mused], dtype=torch.int32, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    assert lca.debug_gemm(x, W, y, Md, err) == 0
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    want = x[:Mused].to(torch.bfloat16).float() @ W.float().t()
+    got = y[:Mused]
+    tol = 2e-3 * float(want.abs().max())
+    np.testing.assert_allclose(got.cpu().numpy(), want.cpu().numpy(), atol=tol, rtol=0)
+    assert torch.isnan(y[Mused:]).all()
