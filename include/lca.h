@@ -5,14 +5,14 @@
  *
  * One decode step (Algorithm 1, one iteration of its loop) does, per sequence:
  *   (1) draft n-1 bytes with the multi-byte head over the previous and current latent
- *       group (Algorithm 1 lines 9-14; Section 3), or with independent MLP heads
+ *       group (Algorithm 1, drafting step; Section 3), or with independent MLP heads
  *       (MLP-MBP, Section 4.1);
  *   (2) embed the n candidates (next-byte byte c_1 plus the drafts) and run the encoder
  *       module (Section 2.2 "Encoder Module") with its byte KV cache;
  *   (3) split at space boundaries, mean-pool closed segments and run the LM module over
  *       the new latents with its KV cache, only when a segment closes (Algorithm 1
- *       lines 4-7; Eff-FxT rule, Section 4.1);
- *   (4) run the next-byte decoder over all n candidates (Algorithm 1 line 8);
+ *       LM-module branch; Eff-FxT rule, Section 4.1);
+ *   (4) run the next-byte decoder over all n candidates (Algorithm 1, next-byte step);
  *   (5) accept: c_1 always, drafts left to right while their probability is >= tau
  *       (Section 3.1 "Byte Acceptance"; LCA_THRESH), or while they equal the next-byte
  *       argmax (speculative acceptance, Section 5.2 (ii); LCA_SPEC); then keep the
@@ -206,7 +206,7 @@ int lca_debug_force_candidates(lca_ctx* ctx, const uint8_t* cand, int32_t n);
 
 /* Decode attention as a standalone call: the attention every module of the decode step
  * runs (causal softmax attention, Section 2.2; inside the multi-byte window of Algorithm 1
- * line 12 the LCA mask reduces to the same causal form). Query row r of sequence b sees the
+ * (drafting step) the LCA mask reduces to the same causal form). Query row r of sequence b sees the
  * cache slots [0, kv_len[r]) of its sequence; softmax scale `scale`; fp32 arithmetic.
  *   q, out:   device fp32 [batch * n_rows][heads * head_dim] (RoPE already applied to q).
  *   k_cache, v_cache: device [batch][heads][slots][head_dim] of `dtype` (LCA_F32|LCA_BF16).

@@ -12,7 +12,7 @@ the multi-byte head of Section 3 (LCA mask, residual r_2 added before
 upsampling, shared unembedding). Blocks follow Llama 3 (Section 4.2): pre-norm
 RMSNorm (eps 1e-6), rotary embeddings (base 1e5), SwiGLU MLP, no biases.
 
-Readings taken where the paper is silent (each is listed in the design doc):
+Readings taken where the paper is silent (each is also listed with the design notes):
   * K(p) counts boundaries at positions <= p, so a boundary byte receives the
     latent of the segment it closes (Algorithm 1 runs the LM module before the
     next-byte layers in the same iteration).
@@ -178,7 +178,7 @@ def pool(h_e, segs):
 
 
 def window_draft_inputs(cfg: ModelConfig, Kp, o, u, t, n, x):
-    """Rows of the MB window of Algorithm 1 (lines 9-12) at committed length t:
+    """Rows of the MB window of Algorithm 1 (drafting step) at committed length t:
     the previous and the current group (from the first byte of group K(t-1)-1, or
     of group 0) then n-2 copies of the last row at positions t..t+n-3.
     Returns (inputs [W,d], positions [W], groups [W])."""
@@ -192,7 +192,7 @@ def window_draft_inputs(cfg: ModelConfig, Kp, o, u, t, n, x):
 
 def mb_draft_logits(model: Model, Kp, o, u, t, n, x, y_last=None):
     """Logits [n-1, V] of the n-1 drafted bytes d_2..d_n (predicting x_{t+1}..x_{t+n-1}).
-    LCA head (Section 3, Algorithm 1 lines 9-14): MB blocks over the window with the
+    LCA head (Section 3, Algorithm 1 drafting step): MB blocks over the window with the
     LCA mask, final RMSNorm, shared unembedding; only the last n-1 rows are kept.
     MLP head (Section 4.1, MLP-MBP): head j maps the last next-byte hidden state y_last
     through residual SiLU layers, then the MB norm and the unembedding."""
@@ -231,7 +231,7 @@ class Forward:
 
 
 def forward_full(model: Model, x, keep_caches=False):
-    """Definition of the forward over bytes x (Section 2.2 and Algorithm 1 lines 2-8):
+    """Definition of the forward over bytes x (Section 2.2 and the forward part of Algorithm 1):
     embed, encoder (causal, RoPE at byte position) -> h_e; space boundaries; mean-pool
     closed segments -> z_1..z_K; LM module over [BOS, z_1..z_K] (causal, RoPE at latent
     index) -> o_0..o_K; next-byte decoder over o_{K(p)} + h_e[p] (causal) -> y; final

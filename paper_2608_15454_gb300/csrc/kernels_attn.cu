@@ -1,5 +1,5 @@
 // Causal softmax attention of query rows over a KV-cache layer (Section 2.2 causal masks;
-// inside the multi-byte window of Algorithm 1 line 12 the LCA mask is causal as well, so
+// inside the multi-byte window of Algorithm 1 (its drafting window) the LCA mask is causal as well, so
 // every attention of the decode step is "query row r sees cache slots [0, kvlen[r])").
 //
 // One CTA serves one (sequence, query tile of up to 8 rows, head, key split). Keys and

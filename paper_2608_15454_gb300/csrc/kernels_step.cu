@@ -15,7 +15,7 @@ __device__ __forceinline__ float ld_w(const __nv_bfloat16* p, size_t i) { return
 __device__ __forceinline__ void err_or(int* e, int bits) { atomicOr(e, bits); }
 
 // ---------------------------------------------------------------- multi-byte window plan
-// Algorithm 1 lines 9-12: the window of sequence b is the previous and the current latent
+// Algorithm 1, drafting: the window of sequence b is the previous and the current latent
 // group, then n-2 copies of the last row. Inside the window the LCA mask is causal, and a
 // row depends only on the window start and the rows before it, so rows computed in earlier
 // steps stay valid while the window start is unchanged: their keys/values are kept in the
@@ -83,7 +83,7 @@ __global__ void k_mb_plan(Dev D) {
       D.head_rows_mb[b * (n - 1) + j] = cnt > 0 ? st0 + cnt - (n - 1) + j : 0;
   }
   __syncthreads();
-  // window rows: byte p of group k gets o_k + u_k (Algorithm 1 line 9, residual r_2 added before
+  // window rows: byte p of group k gets o_k + u_k (Algorithm 1, drafting input; residual r_2 added before
   // upsampling); copies beyond t belong to the current group K
   const int M = *D.r_mb.M;
   const int d4 = D.d / 4;
@@ -99,7 +99,7 @@ __global__ void k_mb_plan(Dev D) {
   }
 }
 
-// MB input rows: byte p of group k gets o_k + u_k (Algorithm 1 line 9, residual r_2 added
+// MB input rows: byte p of group k gets o_k + u_k (Algorithm 1, drafting input; residual r_2 added
 // before upsampling); copies beyond t belong to the current group K.
 __global__ void k_mb_fill(Dev D) {
   TraceScope _trace(TT_MB_FILL);
@@ -519,8 +519,8 @@ __global__ void k_lm_scatter(Dev D) {
   }
 }
 
-// Next-byte decoder input: upsampled LM output plus the encoder residual r_1 (Algorithm 1
-// line 8): o_{K(p)} + h_e[p].
+// Next-byte decoder input: upsampled LM output plus the encoder residual r_1 (Algorithm 1,
+// next-byte step): o_{K(p)} + h_e[p].
 __global__ void k_nb_input(Dev D) {
   TraceScope _trace(TT_NB_INPUT);
   pdl_trigger();

@@ -1,7 +1,7 @@
 // Host runtime behind include/lca.h: workspace layout, weight repacking, prefill, and the
 // decode step as a CUDA graph. One step is one graph replay with no host round trip; the
 // LM module sits in an IF conditional node that the segmentation kernel switches on only
-// when a segment closes (Algorithm 1 lines 4-7). lca_generate wraps the step in a WHILE
+// when a segment closes (Algorithm 1, LM-module branch). lca_generate wraps the step in a WHILE
 // conditional node whose control kernel stops once every sequence has its bytes.
 #include <cuda_runtime.h>
 

@@ -1,0 +1,95 @@
+"""GPU parity at the workloads' full sizes, in the bench's launch configuration (full batch,
+full prompts, the bench's context size and its n, tau and unembedding gain).
+
+The oracle cannot replay a whole batch, so it replays the sampled sequences of each
+workload (``oracle_seqs``) one by one, and the GPU rows of those sequences inside the full
+batch are compared with it: next-byte and drafter logits within the bf16 tolerance (times
+the gain), emitted bytes and t, K equal. A decision may differ only where the oracle's
+margin is inside the tolerance (a near-tie of the top two logits, or a drafter probability
+next to tau); the sequence is then no longer followed. That the sampled rows equal the
+oracle's single-sequence run also shows that sequences of a batch do not interact.
+"""
+import numpy as np
+import pytest
+
+import bench
+from oracle import THRESH, IncrementalDecoder, Model
+from synth import WORKLOADS, cached_weights, gain_for, prompts
+from synth.configs import load_gains
+
+pytestmark = pytest.mark.gpu
+
+BF16_TOL = 2e-2
+STEPS = 6
+
+
+@pytest.fixture(scope="module")
+def lca():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2608_15454_gb300 import build, lca as mod
+    build.build()
+    mod.load_library()
+    return mod
+
+
+def _decision_margin(rec, tau):
+    """Smallest distance, in logit units, of any decision of the step from flipping: half
+    the top-two gap of every row, and for each draft half the distance of
+    l_max - LSE from log(tau)."""
+    m = np.inf
+    rows = [rec.nb_logits] + ([rec.mb_logits] if rec.mb_logits is not None and len(rec.mb_logits) else [])
+    for blk in rows:
+        for r in np.atleast_2d(blk):
+            s = np.sort(r)
+            m = min(m, 0.5 * (s[-1] - s[-2]))
+    if rec.mb_logits is not None:
+        for r in np.atleast_2d(rec.mb_logits):
+            mx = r.max()
+            lse = mx + np.log(np.exp(r - mx).sum())
+            m = min(m, 0.5 * abs(mx - lse - np.log(tau)))
+    return m
+
+
+@pytest.mark.parametrize("name", ["paper_b32", "paper_long_b8", "mlp_b128"])
+def test_full_size_sampled_sequences(lca, name):
+    w = WORKLOADS[name]
+    n, tau = w.n_list[0], w.tau_list[0]
+    gain = gain_for(w, calibrated=w.gain_key in load_gains())
+    W = cached_weights(w.model, gain)
+    P = prompts(w, seqs=list(range(w.batch)))
+    max_bytes = bench.context_bytes(w, n, bench.DEFAULT_STEPS, bench.DEFAULT_WARMUP,
+                                    bench.DEFAULT_PROFILE_STEPS)
+    ctx = lca.Context(w.model, W, max_batch=w.batch, max_bytes=max_bytes, max_n=max(n, w.max_n))
+    ctx.prefill(P)
+    M = Model(w.model, W)
+    decs = {}
+    for b in w.oracle_seqs:
+        d = IncrementalDecoder(M)
+        d.prefill(P[b])
+        decs[b] = d
+    tol = BF16_TOL * gain
+    followed = {b: 0 for b in decs}
+    for _ in range(STEPS):
+        recs = {b: d.step(n, tau, THRESH) for b, d in decs.items()}
+        out, cnt = ctx.step(n, tau, lca.LCA_THRESH)
+        nb, mb = ctx.logits(n)
+        for b, r in recs.items():
+            np.testing.assert_allclose(nb[b], r.nb_logits, atol=tol, rtol=0)
+            if n > 1:
+                np.testing.assert_allclose(mb[b], r.mb_logits, atol=tol, rtol=0)
+            if out[b] != r.emitted:
+                assert _decision_margin(r, tau) < tol, (b, out[b], r.emitted)
+                del decs[b]
+                continue
+            st = ctx.state(b)
+            assert (st["t"], st["K"]) == (r.t, r.K)
+            followed[b] += 1
+        if not decs:
+            break
+    assert max(followed.values()) >= 2, followed
+    # every sequence of the batch advanced by 1..n bytes per step
+    for b in range(w.batch):
+        assert ctx.state(b)["t"] >= len(P[b]) + min(STEPS, max(followed.values()))
+    ctx.close()

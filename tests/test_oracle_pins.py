@@ -210,7 +210,7 @@ def test_zero_layer_next_byte_logits_use_the_latent_of_the_closing_segment():
 
 def test_zero_layer_mb_input_adds_r2_before_upsampling():
     """With empty stacks every draft row of group g decodes o_g + u_g = 2 u_g, whose
-    RMSNorm equals that of u_g (Algorithm 1 line 9)."""
+    RMSNorm equals that of u_g (Algorithm 1, drafting input)."""
     M = _zero_layer_model()
     x = b"ab cd ef"
     F = om.forward_full(M, x)
@@ -244,7 +244,7 @@ def test_lca_inside_the_window_is_plain_causal():
 
 
 def test_one_layer_window_equals_full_sequence_lca_forward():
-    """With one MB layer the slice of Algorithm 1 line 12 loses nothing: the LCA mask
+    """With one MB layer the window slice of Algorithm 1 loses nothing: the LCA mask
     already hides everything before the previous group."""
     M = micro_model(n_mb=1)
     x = b"ab cde fg hij k"
