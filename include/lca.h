@@ -179,12 +179,14 @@ int lca_debug_profile(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, i
 int lca_debug_trace(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t steps,
                     void* out, int32_t cap, int32_t* count);
 
-/* The tensor-core linear layer alone: y[0:*M_dev] = bf16(x) . W^T (fp32 accumulation, tcgen05).
- * x: device fp32 [M][K]; W: device bf16 [N][K]; y: device fp32 [M][N]; M_dev: device int32 rows
- * to compute (<= M); err_dev: device int32 error word (bit 4: a bounded wait ran out). N and K must
- * be multiples of 64. Asynchronous on `stream`. */
+/* The tensor-core linear layer alone: y[0:*M_dev] = x . W^T on tcgen05, with x split into two
+ * bf16 halves (x = hi + lo) so that about 16 bits of each activation enter the product, fp32
+ * accumulation. x: device fp32 [M][K]; W: device bf16 [N][K]; y: device fp32 [M][N]; M_dev:
+ * device int32 rows to compute (<= M); rows_typ: the row count the launch shape is chosen for
+ * (0 = M; a smaller value makes CTAs walk several row passes); err_dev: device int32 error word
+ * (bit 4: a bounded wait ran out). N and K must be multiples of 64. Asynchronous on `stream`. */
 int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N, int32_t K,
-                   const int32_t* M_dev, int32_t* err_dev, void* stream);
+                   const int32_t* M_dev, int32_t rows_typ, int32_t* err_dev, void* stream);
 
 /* Micro-benchmark: one graph of `iters` back-to-back launches of one kernel kind over `rows`
  * rows (0 RMSNorm+QKV, 1 Wo, 2 RMSNorm+W1/W3+SwiGLU, 3 W2, 4 decode attention over the

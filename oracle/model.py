@@ -61,13 +61,17 @@ def rope(x, pos, base):
 
 
 def attend(q, k, v, mask, scale):
-    """Softmax attention. q [T,H,h_d], k/v [S,H,h_d], mask [T,S] (True = key visible)."""
-    s = np.einsum("thd,shd->hts", q, k) * scale
-    s = np.where(mask[None, :, :], s, -np.inf)
-    s = s - s.max(axis=-1, keepdims=True)
-    p = np.exp(s)
-    p /= p.sum(axis=-1, keepdims=True)
-    return np.einsum("hts,shd->thd", p, v)
+    """Softmax attention. q [T,H,h_d], k/v [S,H,h_d], mask [T,S] (True = key visible).
+    One head at a time: scores q_h k_h^T * scale, masked softmax over keys, times v_h."""
+    out = np.empty_like(q)
+    for h in range(q.shape[1]):
+        s = (q[:, h, :] @ k[:, h, :].T) * scale
+        s = np.where(mask, s, -np.inf)
+        s = s - s.max(axis=-1, keepdims=True)
+        p = np.exp(s)
+        p /= p.sum(axis=-1, keepdims=True)
+        out[:, h, :] = p @ v[:, h, :]
+    return out
 
 
 def causal_mask(n_prev, n_new):

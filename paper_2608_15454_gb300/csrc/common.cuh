@@ -43,7 +43,7 @@ struct TraceRec {
 enum TraceTag : int {
   TT_GEMV = 1, TT_GEMV_F32, TT_GEMM, TT_ROWSTATS, TT_ATTN, TT_HEAD, TT_MB_PLAN, TT_MB_FILL,
   TT_MLP_PLAN, TT_VERIFY_PLAN, TT_SEGMENT, TT_LM_SCATTER, TT_NB_INPUT, TT_COMMIT, TT_LOOP_CTL,
-  TT_OTHER
+  TT_OTHER, TT_UMMA
 };
 static __device__ TraceRec* g_trace = nullptr;
 static __device__ unsigned int* g_trace_n = nullptr;
@@ -222,6 +222,8 @@ struct Dev {
   int num_sms;  // streaming multiprocessors of the device
   int use_tma;  // bf16 linear layers use the bulk-copy weight pipeline
   int attn_split_cap;  // largest cluster (key split) of decode attention
+  int tiled_min_rows;  // layers with more typical rows than this run on the tensor cores
+  int attn_pipe;       // decode attention: 1 = bulk-copy pipelined kernel, 0 = register-tiled kernel
   int use_umma;        // many-row bf16 layers run on the tensor cores (tcgen05)
 
   // weights (storage type; norms and bos fp32)
@@ -330,6 +332,7 @@ size_t attention_scratch_floats(int B, int H, int hd);
 size_t attention_counters(int B, int H);
 void kernel_attrs_linear();
 void kernel_attrs_step();
+void kernel_attrs_attn();
 // Attention of query rows over a KV-cache layer (keys [0, kvlen[r]) of sequence b[r]).
 // stable: optional per-sequence committed length (stride in ints) whose cache prefix does not
 // change during a step, prefetched into L2 before the dependency wait; stable_extra: rows added.

@@ -504,6 +504,343 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
   }
 }
 
+// ---------------------------------------------------------------- pipelined decode attention
+// One CTA of 128 threads serves (sequence, query tile of up to 8 rows, head, key split). Its key
+// range streams in chunks of 64 keys through a ring of shared-memory stages filled by bulk
+// asynchronous copies (the cache of one (sequence, head) is contiguous, so a chunk of K or V is
+// one copy), several chunks ahead of the arithmetic. Per chunk: one key per thread for the
+// scores (16-byte reads rotated per key, so a warp's reads spread over all banks), one warp per
+// query row for the online softmax (fp32), a pair of head dims per thread for P.V with the
+// probabilities broadcast from shared memory. Key splits of one (sequence, head) form a
+// thread-block cluster and combine (max, sum, accumulator) through distributed shared memory.
+constexpr int kA3Threads = 128;
+constexpr int kA3Keys = 64;     // keys per chunk
+constexpr int kA3Stages = 4;
+constexpr int kA3Spins = 1 << 22;
+
+__device__ __forceinline__ uint32_t a3_su32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void a3_expect(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a3_su32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void a3_copy(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          a3_su32(dst)),
+      "l"(src), "r"(bytes), "r"(a3_su32(bar))
+      : "memory");
+}
+__device__ __forceinline__ bool a3_wait(uint64_t* bar, uint32_t parity) {
+  for (int i = 0; i < kA3Spins; ++i) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(a3_su32(bar)), "r"(parity)
+        : "memory");
+    if (ok) return true;
+  }
+  return false;
+}
+__device__ __forceinline__ void a3_v2(const float* p, float& a, float& b) {
+  const float2 v = *reinterpret_cast<const float2*>(p);
+  a = v.x;
+  b = v.y;
+}
+__device__ __forceinline__ void a3_v2(const __nv_bfloat16* p, float& a, float& b) {
+  const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
+  a = __uint_as_float(u << 16);
+  b = __uint_as_float(u & 0xFFFF0000u);
+}
+
+template <typename TC, int HD>
+__global__ void __launch_bounds__(kA3Threads, 3)
+k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
+        int* err, const int* __restrict__ stable, int stable_stride, int stable_extra) {
+  namespace cgr = cooperative_groups;
+  constexpr int QT = kAttnQT;                     // query rows per tile (8)
+  constexpr int KC = kA3Keys;
+  constexpr int EV = 16 / (int)sizeof(TC);        // elements per 16-byte vector
+  constexpr int NV = HD / EV;                     // 16-byte vectors per key row
+  constexpr uint32_t CB = KC * HD * sizeof(TC);   // bytes of one K (or V) chunk
+  constexpr int RH = kA3Threads / KC;             // row groups in the score phase (2)
+  constexpr int DP = HD / 2;                      // dim pairs
+  constexpr int RG = kA3Threads / DP;             // row groups in P.V (4 for HD 64)
+  constexpr int RPT = QT / RG;                    // rows per thread in P.V
+  static_assert(QT % RH == 0 && QT % RG == 0 && RPT >= 1, "tile shape");
+  extern __shared__ __align__(128) unsigned char a3sm[];
+  unsigned char* ring = a3sm;                                        // [stages][K | V]
+  float* qs = reinterpret_cast<float*>(a3sm + kA3Stages * 2 * CB);   // [QT][HD], pre-scaled
+  float* sc = qs + QT * HD;                                          // [QT][KC] scores -> probs
+  float* pacc = sc + QT * KC;                                        // [QT][HD] this split's acc
+  float* s_m = pacc + QT * HD;                                       // [QT]
+  float* s_l = s_m + QT;                                             // [QT]
+  float* s_corr = s_l + QT;                                          // [QT]
+  int* s_kv = reinterpret_cast<int*>(s_corr + QT);                   // [QT]
+  uint64_t* full = reinterpret_cast<uint64_t*>(s_kv + QT);           // [stages]
+
+  TraceScope _trace(TT_ATTN);
+  cgr::cluster_group cl = cgr::this_cluster();
+  const int splits = (int)cl.dim_blocks().z;
+  const int sp = (int)cl.block_rank();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    for (int i = 0; i < kA3Stages; ++i)
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&full[i])) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (stable && tid < 2) {
+    // slots below the committed length do not change during a step: warm this CTA's share of
+    // them in L2 before the dependency wait (a hint only)
+    const int bb = blockIdx.x, hh = blockIdx.z / splits;
+    const int t = stable[(size_t)bb * stable_stride];
+    const int est = ((t + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
+    const int lo = sp * est, hi = min(t, lo + est);
+    if (hi > lo) {
+      const TC* base = reinterpret_cast<const TC*>(tid == 0 ? kv.k : kv.v) + (((size_t)bb * H + hh) * kv.S + lo) * HD;
+      const uint32_t bytes = (uint32_t)((hi - lo) * HD * sizeof(TC));
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"(bytes & ~15u) : "memory");
+    }
+  }
+  pdl_trigger();
+  pdl_wait();
+  _trace.waited();
+  __syncthreads();
+  const int b = blockIdx.x;
+  const int h = blockIdx.z / splits;
+  const int nrows = rows.seq_count[b];
+  const int rbeg = rows.seq_start[b];
+  const int ntiles = (nrows + QT - 1) / QT;
+  const TC* Kc = reinterpret_cast<const TC*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
+  const TC* Vc = reinterpret_cast<const TC*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  const int ld = H * HD;
+  bool failed = false;
+  uint32_t cc = 0;      // chunks consumed by this CTA so far (ring phase)
+  uint32_t issued = 0;  // chunks whose copies were issued (thread 0)
+
+  for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
+    const int r0 = rbeg + qt * QT;
+    const int nq = min(QT, nrows - qt * QT);
+    for (int idx = tid; idx < QT * HD; idx += kA3Threads) {
+      const int i = idx / HD, dd = idx - i * HD;
+      qs[idx] = i < nq ? q[(size_t)(r0 + i) * ld + h * HD + dd] * scale : 0.f;
+    }
+    if (tid < QT) {
+      int kl = tid < nq ? rows.kvlen[r0 + tid] : 0;
+      if (kl > kv.S || kl < 0) {
+        atomicOr(err, kErrIndex);
+        kl = kl < 0 ? 0 : kv.S;
+      }
+      s_kv[tid] = kl;
+      s_m[tid] = -INFINITY;
+      s_l[tid] = 0.f;
+    }
+    __syncthreads();
+    int kv_hi = 0;
+#pragma unroll
+    for (int i = 0; i < QT; ++i) kv_hi = max(kv_hi, s_kv[i]);
+    const int per = ((kv_hi + splits - 1) / splits + KC - 1) / KC * KC;
+    const int lo = sp * per;
+    const int hi = min(kv_hi, lo + per);
+    const int nch = hi > lo ? (hi - lo + KC - 1) / KC : 0;
+    auto issue = [&](int c) {
+      const uint32_t g = cc + c;
+      const int st = g % kA3Stages;
+      const int j0 = lo + c * KC;
+      const int nk = min(KC, hi - j0);
+      const uint32_t bytes = (uint32_t)(nk * HD * sizeof(TC));
+      unsigned char* dst = ring + (size_t)st * 2 * CB;
+      ++issued;
+      a3_expect(&full[st], 2 * bytes);
+      a3_copy(dst, Kc + (size_t)j0 * HD, bytes, &full[st]);
+      a3_copy(dst + CB, Vc + (size_t)j0 * HD, bytes, &full[st]);
+    };
+    if (tid == 0)
+      for (int c = 0; c < nch && c < kA3Stages - 1; ++c) issue(c);
+    float acc[RPT][2];
+#pragma unroll
+    for (int m = 0; m < RPT; ++m) acc[m][0] = acc[m][1] = 0.f;
+    const int dp = tid % DP, rg = tid / DP;
+
+    for (int c = 0; c < nch; ++c) {
+      __syncthreads();  // chunk c-1 fully read: its stage may be refilled
+      if (tid == 0 && c + kA3Stages - 1 < nch) issue(c + kA3Stages - 1);
+      const uint32_t g = cc + c;
+      const int st = g % kA3Stages;
+      if (!failed && !a3_wait(&full[st], (g / kA3Stages) & 1)) failed = true;
+      const TC* Ks = reinterpret_cast<const TC*>(ring + (size_t)st * 2 * CB);
+      const TC* Vs = reinterpret_cast<const TC*>(ring + (size_t)st * 2 * CB + CB);
+      const int j0 = lo + c * KC;
+      const int nk = min(KC, hi - j0);
+      // scores: key j of this chunk, rows rh, rh + RH, ...
+      {
+        const int j = tid % KC, rh = tid / KC;
+        float s[QT / RH];
+#pragma unroll
+        for (int m = 0; m < QT / RH; ++m) s[m] = 0.f;
+        if (j < nk) {
+          const uint4* kr = reinterpret_cast<const uint4*>(Ks + (size_t)j * HD);
+#pragma unroll
+          for (int v = 0; v < NV; ++v) {
+            const int vv = (v + j) % NV;
+            float kf[EV];
+            unpack16(kr[vv], kf, (const TC*)nullptr);
+#pragma unroll
+            for (int m = 0; m < QT / RH; ++m) {
+              if (rh + m * RH < nq) {  // warp-uniform
+                const float* qr = qs + (rh + m * RH) * HD + vv * EV;
+#pragma unroll
+                for (int e = 0; e < EV; ++e) s[m] = fmaf(qr[e], kf[e], s[m]);
+              }
+            }
+          }
+        }
+#pragma unroll
+        for (int m = 0; m < QT / RH; ++m) {
+          const int i = rh + m * RH;
+          const bool ok = j < nk && (j0 + j) < s_kv[i] && i < nq;
+          sc[i * KC + j] = ok ? s[m] : -INFINITY;
+        }
+      }
+      __syncthreads();
+      // online softmax: warp w owns rows w, w + 4
+      for (int i = warp; i < QT; i += kA3Threads / 32) {
+        const float x0 = sc[i * KC + lane], x1 = sc[i * KC + lane + 32];
+        float mx = fmaxf(x0, x1);
+#pragma unroll
+        for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        const float m_old = s_m[i];
+        const float m_new = fmaxf(m_old, mx);
+        float p0 = 0.f, p1 = 0.f, corr = 1.f;
+        if (m_new != -INFINITY) {
+          p0 = x0 == -INFINITY ? 0.f : expf(x0 - m_new);
+          p1 = x1 == -INFINITY ? 0.f : expf(x1 - m_new);
+          corr = m_old == -INFINITY ? 0.f : expf(m_old - m_new);
+        }
+        float ps = p0 + p1;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o);
+        sc[i * KC + lane] = p0;
+        sc[i * KC + lane + 32] = p1;
+        __syncwarp();
+        if (lane == 0) {
+          s_l[i] = s_l[i] * corr + ps;
+          s_m[i] = m_new;
+          s_corr[i] = corr;
+        }
+      }
+      __syncthreads();
+      // P.V: dims (2 dp, 2 dp + 1) of rows rg, rg + RG, ...
+#pragma unroll
+      for (int m = 0; m < RPT; ++m) {
+        const float cr = s_corr[rg + m * RG];
+        acc[m][0] *= cr;
+        acc[m][1] *= cr;
+      }
+      auto pv_key = [&](int j) {
+        float v0, v1;
+        a3_v2(Vs + (size_t)j * HD + 2 * dp, v0, v1);
+#pragma unroll
+        for (int m = 0; m < RPT; ++m) {
+          if (rg + m * RG < nq) {  // warp-uniform: a warp's threads share their rows
+            const float pj = sc[(rg + m * RG) * KC + j];
+            acc[m][0] = fmaf(pj, v0, acc[m][0]);
+            acc[m][1] = fmaf(pj, v1, acc[m][1]);
+          }
+        }
+      };
+      if (nk == KC) {
+        // full chunk: unrolled so that the shared-memory loads of many keys are in flight
+#pragma unroll 16
+        for (int j = 0; j < KC; ++j) pv_key(j);
+      } else {
+        for (int j = 0; j < nk; ++j) pv_key(j);
+      }
+    }
+    cc += nch;
+    // this split's partial accumulators -> shared memory; combine across the cluster
+#pragma unroll
+    for (int m = 0; m < RPT; ++m) {
+      pacc[(rg + m * RG) * HD + 2 * dp] = acc[m][0];
+      pacc[(rg + m * RG) * HD + 2 * dp + 1] = acc[m][1];
+    }
+    cl.sync();
+    {
+      const int dpr = (HD + splits - 1) / splits;
+      const int d0 = sp * dpr;
+      const int nd = min(dpr, HD - d0);
+      for (int idx = tid; idx < nq * nd; idx += kA3Threads) {
+        const int i = idx / nd, dd = d0 + (idx - i * nd);
+        float mr[kMaxClusterSplit], lr[kMaxClusterSplit], ar[kMaxClusterSplit];
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
+          if (k < splits) {
+            mr[k] = *cl.map_shared_rank(&s_m[i], k);
+            lr[k] = *cl.map_shared_rank(&s_l[i], k);
+            ar[k] = *cl.map_shared_rank(&pacc[i * HD + dd], k);
+          }
+        }
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k)
+          if (k < splits) M = fmaxf(M, mr[k]);
+        float L = 0.f, o = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
+          if (k < splits && mr[k] != -INFINITY) {
+            const float w = expf(mr[k] - M);
+            L += w * lr[k];
+            o += w * ar[k];
+          }
+        }
+        out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? o / L : 0.f;
+      }
+    }
+    cl.sync();  // peers are done reading this tile's partials
+  }
+  // after a failed wait, copies may still be in flight: wait (bounded) for the last one issued
+  // into each stage before the CTA's shared memory is released
+  if (__syncthreads_or(failed) && tid == 0) {
+    for (uint32_t st = 0; st < (uint32_t)kA3Stages && st < issued; ++st) {
+      const uint32_t last = issued - 1 - ((issued - 1 - st) % kA3Stages);
+      a3_wait(&full[last % kA3Stages], (last / kA3Stages) & 1);
+    }
+    atomicOr(err, kErrTimeout);
+  }
+}
+
+template <typename TC, int HD>
+size_t attn3_smem() {
+  constexpr int QT = kAttnQT;
+  return (size_t)kA3Stages * 2 * kA3Keys * HD * sizeof(TC) + (size_t)(2 * QT * HD + QT * kA3Keys + 4 * QT) * 4 +
+         kA3Stages * 8 + 16;
+}
+
+template <typename TC, int HD>
+void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
+               int qtiles_grid, int splits, int* err, const int* stable, int stable_stride,
+               int stable_extra, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(B, qtiles_grid, H * splits);
+  cfg.blockDim = dim3(kA3Threads);
+  cfg.dynamicSmemBytes = attn3_smem<TC, HD>();
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = splits;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++g_launches;
+  cudaLaunchKernelEx(&cfg, k_attn3<TC, HD>, q, out, kv, rows, H, scale, err, stable, stable_stride,
+                     stable_extra);
+}
+
 template <typename TC, int HD>
 void launch_cl(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
                int qtiles_grid, int splits, int* err, const int* stable, int stable_stride,
@@ -645,12 +982,33 @@ size_t attention_scratch_floats(int B, int H, int hd) {
 }
 size_t attention_counters(int B, int H) { return (size_t)B * kQTMax * H; }
 
+void kernel_attrs_attn() {
+  cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn3_smem<__nv_bfloat16, 64>());
+  cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn3_smem<__nv_bfloat16, 32>());
+  cudaFuncSetAttribute(k_attn3<float, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn3_smem<float, 64>());
+  cudaFuncSetAttribute(k_attn3<float, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn3_smem<float, 32>());
+}
+
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s, const int* stable, int stable_extra) {
   ProfScope ps(PK_ATTN, 0.0, s);
   if (splits > kMaxClusterSplit) splits = kMaxClusterSplit;
   if (splits < 1) splits = 1;
   const int ss = (int)(sizeof(SeqState) / sizeof(int));
+  if (D.attn_pipe) {
+    if (D.dtype == LCA_BF16) {
+      if (D.hd == 64) launch_a3<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+      else launch_a3<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+    } else {
+      if (D.hd == 64) launch_a3<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+      else launch_a3<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+    }
+    return;
+  }
   if (D.dtype == LCA_BF16) {
     if (D.hd == 64) launch_cl<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
     else launch_cl<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);

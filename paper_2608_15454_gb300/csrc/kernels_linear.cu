@@ -349,8 +349,10 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   __nv_bfloat16* wt = reinterpret_cast<__nv_bfloat16*>(sm);             // [CT][Kr]
   float* gs = reinterpret_cast<float*>(sm + (size_t)CT * Kr * 2);        // [Kr] (NORM)
   float* xs = gs + Kr;                                                   // [MCA][Kr]
-  float* rs = xs + MCA * Kr;                                             // [MCA] sums of squares
-  float* cpart = rs + MCA;                                               // [MCA][CT]
+  float* wss = xs + MCA * Kr;                                            // [NW][MCA] warp sums of squares
+  float* rs = wss + NW * MCA;                                            // [MCA] this CTA's sums of squares
+  float* cpart = reinterpret_cast<float*>(                                // [MCA][CT], 16-byte aligned
+      (reinterpret_cast<uintptr_t>(rs + MCA) + 15) & ~uintptr_t(15));
   uint64_t* bar = reinterpret_cast<uint64_t*>(
       (reinterpret_cast<uintptr_t>(cpart + MCA * CT) + 15) & ~uintptr_t(15));
 
@@ -393,7 +395,6 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
     const bool epi_lane = ksplit == 1 && col0 < ncols && ei < mc && (ec & 1) == 0;
     if (epi_lane) pre = epi_load(a.epi, rbase + r0 + ei, tile * CT + col0 + ec);
     __syncthreads();
-    if (NORM && tid < MCA) rs[tid] = 0.f;
     // raw rows -> registers (loads batched), then x * g -> shared memory with sums of squares
     constexpr int UNR = 8;
     const int nv = MCA * Kr / 4;
@@ -431,13 +432,14 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
         }
       }
     }
-    if (NORM && ksplit == 1) {
+    if (NORM) {
+      // per-warp partial sums of squares over this CTA's K range (no atomics: summed in warp order)
 #pragma unroll
       for (int i = 0; i < MCA; ++i) {
         float t = ss[i];
 #pragma unroll
         for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-        if (lane == 0 && i < mc) atomicAdd(&rs[i], t);
+        if (lane == 0) wss[warp * MCA + i] = t;
       }
     }
     if (!have_w) {
@@ -449,20 +451,12 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
     } else {
       __syncthreads();
     }
-    if (NORM && ksplit > 1) {
-      // a K-split CTA sees part of each row: the full-row sums come from global memory
-      for (int i = warp; i < mc; i += NW) {
-        const float* xr = a.x + (size_t)(rbase + r0 + i) * a.ldx;
-        float t = 0.f;
-        for (int k = lane * 4; k < a.Kd; k += 128) {
-          const float4 q = *reinterpret_cast<const float4*>(xr + k);
-          t += q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
-        }
+    if (NORM && tid < MCA) {
+      // this CTA's share of each row's sum of squares; read after the next barrier
+      float t = 0.f;
 #pragma unroll
-        for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-        if (lane == 0) rs[i] = t;
-      }
-      __syncthreads();
+      for (int w = 0; w < NW; ++w) t += wss[w * MCA + tid];
+      rs[tid] = t;
     }
     if (col0 < ncols) {
       float acc[MCA * kCPW];
@@ -500,7 +494,12 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       for (int j = 0; j < 32; ++j) full[j] = j < MCA * kCPW ? acc[j] : 0.f;
       float v = warp_reduce_scatter32(full, lane);
       if (ksplit == 1) {
-        if (NORM && ei < mc) v *= rsqrtf(rs[ei] / (float)a.Kd + a.eps);
+        if (NORM && ei < mc) {
+          float t = 0.f;
+#pragma unroll
+          for (int w = 0; w < NW; ++w) t += wss[w * MCA + ei];
+          v *= rsqrtf(t / (float)a.Kd + a.eps);
+        }
         const float vn = __shfl_down_sync(0xffffffffu, v, 1);
         if (epi_lane) epi_store<__nv_bfloat16>(a.epi, pre, rbase + r0 + ei, tile * CT + col0 + ec, v, vn);
       } else if (ei < MCA) {
@@ -525,14 +524,20 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
         for (int idx = tid; idx < mc * (CT / 2); idx += NT, ++j) {
           const int i = idx / (CT / 2), c = (idx - i * (CT / 2)) * 2;
           if (c >= ncols) continue;
-          float t0 = 0.f, t1 = 0.f;
-          for (int sp = 0; sp < ksplit; ++sp) {
-            const float* pr = cl.map_shared_rank(cpart + i * CT + c, sp);
-            t0 += pr[0];
-            t1 += pr[1];
+          // every rank's partials (and row sums of squares) in one batch of remote loads, then
+          // added in rank order
+          float t0 = 0.f, t1 = 0.f, sq = 0.f;
+#pragma unroll
+          for (int sp = 0; sp < kMaxKSplit; ++sp) {
+            if (sp < ksplit) {
+              const float2 pv = *reinterpret_cast<const float2*>(cl.map_shared_rank(cpart + i * CT + c, sp));
+              t0 += pv.x;
+              t1 += pv.y;
+              if (NORM) sq += *cl.map_shared_rank(rs + i, sp);
+            }
           }
           if (NORM) {
-            const float sc = rsqrtf(rs[i] / (float)a.Kd + a.eps);
+            const float sc = rsqrtf(sq / (float)a.Kd + a.eps);
             t0 *= sc;
             t1 *= sc;
           }
@@ -669,7 +674,8 @@ template <int MCA, int NW, bool NORM>
 void gemv_bulk_go(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s) {
   constexpr int CT = NW * kCPW;
   const int Kr = a.Kd / ksplit;
-  const size_t smem = (size_t)CT * Kr * 2 + (size_t)Kr * 4 + (size_t)MCA * Kr * 4 + (MCA + MCA * CT) * 4 + 16 + 64;
+  const size_t smem =
+      (size_t)CT * Kr * 2 + (size_t)Kr * 4 + (size_t)MCA * Kr * 4 + (NW * MCA + MCA + MCA * CT) * 4 + 16 + 16 + 64;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((a.N + CT - 1) / CT, ksplit, a.groups);
   cfg.blockDim = dim3(NW * 32);

@@ -1,19 +1,27 @@
 // Tensor-core linear layer for many rows (batched decode, prefill): y = epi(norm?(x) . W^T) with
 // tcgen05 (5th-generation tensor cores) on sm_103a.
 //
-// One CTA computes a 128-row x 64-column tile of y. Per 64-wide K block:
-//   * the weight tile W[n0:n0+64, k:k+64] (bf16, K-major) arrives by a TMA tensor copy with the
-//     128-byte swizzle, completing on an mbarrier;
-//   * each of the 128 threads converts its own activation row x[m0+tid, k:k+64] (fp32, times the
-//     RMSNorm gain) to bf16 and writes it into shared memory in the same swizzled K-major layout,
-//     while accumulating the row's sum of squares;
-//   * one thread issues four tcgen05.mma (M=128, N=64, K=16, bf16 -> fp32) into a TMEM
-//     accumulator and commits them to a second mbarrier that frees the stage.
-// The epilogue reads the accumulator with tcgen05.ld (thread = row), applies the row's inverse
-// RMS and the layer's epilogue. TMEM is allocated only after the grid-dependency wait, so a kernel
-// launched early never holds tensor memory its predecessor needs. Every wait is bounded.
+// The layer is bound by streaming W from HBM up to a few hundred rows, so the grid is laid out
+// for weight bandwidth: CTA (column tile, K slice, group x row pass) owns a BN-column tile of W
+// over one K slice and reads it exactly once for all rows of the pass (up to 512/BN row tiles of
+// 128, each with its own TMEM accumulator). The K slices of one column tile form a thread-block
+// cluster whose partial sums are added through distributed shared memory.
+//
+// Warp roles (192 threads, one CTA per SM):
+//   * warp 0 streams W tiles (TMA tensor copies, 128-byte swizzle) through a ring of stages;
+//     the first ring is issued before the grid-dependency wait, since weights never change;
+//   * warp 1 owns TMEM and issues tcgen05.mma (M=128, N=BN, K=16, bf16 x bf16 -> fp32);
+//   * warps 2-5 turn the fp32 activations into bf16 A tiles (times the RMSNorm gain, with the
+//     row's sum of squares on the side; coalesced: a half-warp reads one row's 64-element block)
+//     and run the epilogue. Each activation is split as
+//     x = hi + lo with hi = bf16(x) and lo = bf16(x - hi), and both halves are multiplied, so the
+//     product keeps about 16 bits of the activation instead of 8 (the weights are exactly bf16).
+// Every wait is bounded; a wait that runs out sets the timeout bit of the device error word and
+// the kernel finishes without further waiting.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+
+#include <cooperative_groups.h>
 
 #include <cstdio>
 
@@ -25,13 +33,9 @@ namespace lca {
 namespace {
 
 constexpr int kUM = 128;     // rows per tile (UMMA M)
-constexpr int kUN = 64;      // columns per tile (UMMA N)
+constexpr int kUN = 64;      // narrowest column tile (UMMA N); layers need N % 64 == 0
 constexpr int kUK = 64;      // K per stage (one 128-byte swizzle row of bf16)
-constexpr int kUStages = 4;
-constexpr int kUThreads = 128;
 constexpr int kUSpins = 1 << 22;
-constexpr uint32_t kATileBytes = kUM * kUK * 2;  // 16 KB
-constexpr uint32_t kBTileBytes = kUN * kUK * 2;  // 8 KB
 
 __device__ __forceinline__ uint32_t su32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -68,17 +72,6 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t saddr) {
   return d;
 }
 
-// Instruction descriptor: D fp32, A and B bf16, both K-major, M = 128, N = kUN.
-constexpr uint32_t kIDesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kUN >> 3) << 17) |
-                            ((uint32_t)(kUM >> 4) << 24);
-
-__device__ __forceinline__ void umma(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
-      "l"(a), "l"(b), "r"(kIDesc), "r"(accumulate)
-      : "memory");
-}
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar))
                : "memory");
@@ -91,45 +84,109 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       : "memory");
 }
 
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<const uint32_t*>(&h);
+constexpr int kU2Threads = 192;
+constexpr int kAStages = 3;
+constexpr uint32_t kAHalf = kUM * kUK * 2;       // 16 KB: one bf16 half of an A tile
+constexpr uint32_t kAStageBytes = 2 * kAHalf;    // hi + lo
+
+template <int BN>
+struct UCfg {
+  static constexpr int kWStages = BN == 128 ? 6 : 8;
+  static constexpr uint32_t kWBytes = BN * kUK * 2;
+  static constexpr int kMaxMT = 512 / BN;  // row tiles held in TMEM at once
+  // D fp32, A and B bf16, both K-major, M = 128, N = BN
+  static constexpr uint32_t kIDesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                                     ((uint32_t)(kUM >> 4) << 24);
+  static constexpr size_t kSmem = (size_t)kWStages * kWBytes + (size_t)kAStages * kAStageBytes +
+                                  (size_t)(kMaxMT + 1) * kUM * 4 + (2 * kWStages + 2 * kAStages + 1) * 8 +
+                                  16 + 1024;
+};
+
+template <int BN>
+__device__ __forceinline__ void umma_n(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
+      "l"(a), "l"(b), "r"(UCfg<BN>::kIDesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void ubar_arrive(uint64_t* b) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
+}
+// bounded wait; once a wait of this thread has failed, later ones return at once
+__device__ __forceinline__ void wait_or_fail(uint64_t* b, uint32_t parity, bool& failed) {
+  if (failed) return;
+  if (!ubar_wait(b, parity)) failed = true;
+}
+__device__ __forceinline__ void split_bf16(float x, uint16_t& hi, uint16_t& lo) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(x);
+  const __nv_bfloat16 l = __float2bfloat16_rn(x - __bfloat162float(h));
+  hi = *reinterpret_cast<const uint16_t*>(&h);
+  lo = *reinterpret_cast<const uint16_t*>(&l);
 }
 
-template <bool NORM>
-__global__ void __launch_bounds__(kUThreads, 1)
-k_umma(LinearArgs a, const __grid_constant__ CUtensorMap tmW, int num_mtiles) {
-  TraceScope _trace(TT_GEMM);
+template <int BN, bool NORM>
+__global__ void __launch_bounds__(kU2Threads, 1)
+k_umma(LinearArgs a, const __grid_constant__ CUtensorMap tmW, int MG, int KS, int tcols) {
+  using C = UCfg<BN>;
+  namespace cgr = cooperative_groups;
+  TraceScope _trace(TT_UMMA);
   extern __shared__ __align__(1024) unsigned char usm_raw[];
-  // 1024-byte aligned stages (128-byte swizzle atoms need it)
-  unsigned char* usm =
+  unsigned char* base =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(usm_raw) + 1023) & ~uintptr_t(1023));
-  unsigned char* As = usm;                                    // [stages][16 KB]
-  unsigned char* Bs = usm + kUStages * kATileBytes;           // [stages][8 KB]
-  uint64_t* full = reinterpret_cast<uint64_t*>(Bs + kUStages * kBTileBytes);  // [stages]
-  uint64_t* done = full + kUStages;                                         // [stages]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + kUStages);
+  unsigned char* Ws = base;                                         // [kWStages][BN x 64 bf16]
+  unsigned char* As = Ws + C::kWStages * C::kWBytes;                // [kAStages][hi | lo]
+  float* ss_s = reinterpret_cast<float*>(As + kAStages * kAStageBytes);  // [kMaxMT][128]
+  float* ssred = ss_s + C::kMaxMT * kUM;                             // [128]
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(ssred + kUM);
+  uint64_t* wempty = wfull + C::kWStages;
+  uint64_t* afull = wempty + C::kWStages;
+  uint64_t* aempty = afull + kAStages;
+  uint64_t* accdone = aempty + kAStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accdone + 1);
+  float* red = reinterpret_cast<float*>(As);  // [128][BN + 1], reuses the A ring after the MMAs
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int n0 = blockIdx.x * kUN;
-  const int grp = blockIdx.z;
+  const int n0 = blockIdx.x * BN;
+  const int ks = blockIdx.y;
+  const int grp = blockIdx.z / MG, mg0 = blockIdx.z % MG;
   const int rbase = grp * a.Mg_stride;
-  const int nkb = a.Kd / kUK;
+  const int nkb = a.Kd / kUK / KS;
+  const int kb0 = ks * nkb;
+  const int wrow = grp * a.N + n0;
 
   if (tid == 0) {
-    for (int s = 0; s < kUStages; ++s) {
-      ubar_init(&full[s], 1);
-      ubar_init(&done[s], 1);
+    for (int i = 0; i < C::kWStages; ++i) {
+      ubar_init(&wfull[i], 1);
+      ubar_init(&wempty[i], 1);
     }
+    for (int i = 0; i < kAStages; ++i) {
+      ubar_init(&afull[i], 128);
+      ubar_init(&aempty[i], 1);
+    }
+    ubar_init(accdone, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
+  }
+  __syncthreads();
+  // weights never change: the first ring of W tiles streams before the grid-dependency wait
+  const int pre = nkb < C::kWStages ? nkb : C::kWStages;
+  uint32_t issued = 0;  // W copies this CTA has issued (thread 0)
+  if (tid == 0) {
+    issued = pre;
+    for (int i = 0; i < pre; ++i) {
+      ubar_expect(&wfull[i], C::kWBytes);
+#pragma unroll
+      for (int h = 0; h < BN / 64; ++h)
+        tma_load_2d(Ws + (size_t)i * C::kWBytes + h * 8192, &tmW, (kb0 + i) * kUK, wrow + h * 64, &wfull[i]);
+    }
   }
   pdl_trigger();
   pdl_wait();
   _trace.waited();
-  if (warp == 0) {
+  if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)),
-                 "r"(kUN)
+                 "r"(tcols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -141,112 +198,251 @@ k_umma(LinearArgs a, const __grid_constant__ CUtensorMap tmW, int num_mtiles) {
   int M = *a.M;
   M = M < a.M_cap ? M : a.M_cap;
   const int ntm = (M + kUM - 1) / kUM;
+  const int npass = (ntm + C::kMaxMT - 1) / C::kMaxMT;
+  int my_passes = (npass - mg0 + MG - 1) / MG;
+  if (my_passes < 1) my_passes = 1;  // the pre-issued W tiles are consumed by a first (possibly empty) pass
   bool failed = false;
-  uint32_t it = 0;  // stage uses so far (mbarrier phases)
+  uint32_t wit = 0, ait = 0;
+  const int r = ((warp & 3) << 5) | lane;  // converter/epilogue row = TMEM lane of this warp quarter
+  const int RPC = kUM / KS;                // rows each cluster rank reduces
 
-  for (int mt = blockIdx.y; mt < ntm && !failed; mt += num_mtiles) {
-    const int m0 = mt * kUM;
-    const int row = m0 + tid;
-    const bool live = row < M;
-    const float* xr = a.x + (size_t)(rbase + (live ? row : 0)) * a.ldx;
-    float ss = 0.f;
-    uint32_t last = 0;
-    for (int kb = 0; kb < nkb; ++kb, ++it) {
-      const int s = it % kUStages;
-      if (it >= (uint32_t)kUStages && !failed) {  // the MMAs that last read this stage must be done
-        if (!ubar_wait(&done[s], ((it / kUStages) - 1) & 1)) failed = true;
-      }
-      // activation row -> bf16, swizzled K-major
-      unsigned char* at = As + (size_t)s * kATileBytes;
-      const int k0 = kb * kUK;
+  for (int ps = 0; ps < my_passes; ++ps) {
+    const int mt_lo = (mg0 + ps * MG) * C::kMaxMT;
+    int nmt = ntm - mt_lo;
+    nmt = nmt < 0 ? 0 : (nmt > C::kMaxMT ? C::kMaxMT : nmt);
+    if (warp == 0) {
+      if (lane == 0) {
+        for (int kb = (ps == 0 ? pre : 0); kb < nkb; ++kb) {
+          const uint32_t it = wit + kb;
+          const int s = it % C::kWStages;
+          if (it >= (uint32_t)C::kWStages) wait_or_fail(&wempty[s], ((it / C::kWStages) - 1) & 1, failed);
+          if (failed) break;
+          ++issued;
+          ubar_expect(&wfull[s], C::kWBytes);
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f), v1 = v0;
-        if (live) {
-          v0 = *reinterpret_cast<const float4*>(xr + k0 + c * 8);
-          v1 = *reinterpret_cast<const float4*>(xr + k0 + c * 8 + 4);
+          for (int h = 0; h < BN / 64; ++h)
+            tma_load_2d(Ws + (size_t)s * C::kWBytes + h * 8192, &tmW, (kb0 + kb) * kUK, wrow + h * 64, &wfull[s]);
         }
-        if (NORM) {
-          ss += v0.x * v0.x + v0.y * v0.y + v0.z * v0.z + v0.w * v0.w;
-          ss += v1.x * v1.x + v1.y * v1.y + v1.z * v1.z + v1.w * v1.w;
-          const float4 g0 = *reinterpret_cast<const float4*>(a.norm + k0 + c * 8);
-          const float4 g1 = *reinterpret_cast<const float4*>(a.norm + k0 + c * 8 + 4);
-          v0.x *= g0.x; v0.y *= g0.y; v0.z *= g0.z; v0.w *= g0.w;
-          v1.x *= g1.x; v1.y *= g1.y; v1.z *= g1.z; v1.w *= g1.w;
-        }
-        uint4 u;
-        u.x = pack_bf16(v0.x, v0.y);
-        u.y = pack_bf16(v0.z, v0.w);
-        u.z = pack_bf16(v1.x, v1.y);
-        u.w = pack_bf16(v1.z, v1.w);
-        const int r = tid;
-        *reinterpret_cast<uint4*>(at + (r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) * 16)) = u;
       }
-      if (tid == 0) {
-        ubar_expect(&full[s], kBTileBytes);
-        tma_load_2d(Bs + (size_t)s * kBTileBytes, &tmW, k0, grp * a.N + n0, &full[s]);
-      }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      __syncthreads();
-      if (tid == 0 && !failed) {
-        if (!ubar_wait(&full[s], (it / kUStages) & 1)) failed = true;
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t abase = su32(As + (size_t)s * kATileBytes);
-        const uint32_t bbase = su32(Bs + (size_t)s * kBTileBytes);
+    } else if (warp == 1) {
+      if (lane == 0) {
+        for (int kb = 0; kb < nkb; ++kb) {
+          const uint32_t it = wit + kb;
+          const int s = it % C::kWStages;
+          wait_or_fail(&wfull[s], (it / C::kWStages) & 1, failed);
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          const uint32_t bbase = su32(Ws + (size_t)s * C::kWBytes);
+          for (int j = 0; j < nmt; ++j) {
+            const uint32_t at = ait + kb * nmt + j;
+            const int sa = at % kAStages;
+            wait_or_fail(&afull[sa], (at / kAStages) & 1, failed);
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t ahi = su32(As + (size_t)sa * kAStageBytes), alo = ahi + kAHalf;
+            const uint32_t d = tmem + (uint32_t)(j * BN);
+            if (!failed) {
 #pragma unroll
-        for (int k = 0; k < kUK / 16; ++k)
-          umma(tmem, sdesc(abase + k * 32), sdesc(bbase + k * 32), (kb > 0 || k > 0) ? 1u : 0u);
-        umma_commit(&done[s]);
+              for (int k = 0; k < kUK / 16; ++k) {
+                umma_n<BN>(d, sdesc(ahi + k * 32), sdesc(bbase + k * 32), (kb > 0 || k > 0) ? 1u : 0u);
+                umma_n<BN>(d, sdesc(alo + k * 32), sdesc(bbase + k * 32), 1u);
+              }
+            }
+            umma_commit(&aempty[sa]);
+          }
+          if (nmt > 0) umma_commit(&wempty[s]);
+          else ubar_arrive(&wempty[s]);
+        }
+        if (nmt > 0) umma_commit(accdone);
+        else ubar_arrive(accdone);
       }
-      last = it;
+    } else {
+      // converters: step st = (kb, j) in the MMA thread's order. A half-warp reads one row's
+      // 64-element block (16 lanes x 16 bytes, coalesced); a warp instruction covers two rows.
+      const int cw = warp - 2, half = lane >> 4, q = lane & 15;
+      if (NORM && q == 0)
+        for (int j = 0; j < nmt; ++j)
+#pragma unroll
+          for (int it = 0; it < 16; ++it) ss_s[j * kUM + 2 * (cw + 4 * it) + half] = 0.f;
+      const int steps = nkb * nmt;
+      float4 cur[16];
+      auto load_step = [&](int st, float4 (&v)[16]) {
+        const int kb = st / nmt, j = st - kb * nmt;
+        const float* xb = a.x + (size_t)(kb0 + kb) * kUK + q * 4;
+#pragma unroll
+        for (int it = 0; it < 16; ++it) {
+          const int row = (mt_lo + j) * kUM + 2 * (cw + 4 * it) + half;
+          v[it] = row < M ? *reinterpret_cast<const float4*>(xb + (size_t)(rbase + row) * a.ldx)
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      };
+      auto convert_step = [&](int st, const float4 (&v)[16]) {
+        const int kb = st / nmt, j = st - kb * nmt;
+        const uint32_t at = ait + st;
+        const int sa = at % kAStages;
+        if (at >= (uint32_t)kAStages) wait_or_fail(&aempty[sa], ((at / kAStages) - 1) & 1, failed);
+        unsigned char* ahi = As + (size_t)sa * kAStageBytes;
+        unsigned char* alo = ahi + kAHalf;
+        const int k0 = (kb0 + kb) * kUK;
+        float4 g = make_float4(1.f, 1.f, 1.f, 1.f);
+        if (NORM) g = *reinterpret_cast<const float4*>(a.norm + k0 + q * 4);
+#pragma unroll
+        for (int it = 0; it < 16; ++it) {
+          const int rr = 2 * (cw + 4 * it) + half;  // row within the tile
+          float e[4] = {v[it].x, v[it].y, v[it].z, v[it].w};
+          if (NORM) {
+            float ss = e[0] * e[0] + e[1] * e[1] + e[2] * e[2] + e[3] * e[3];
+#pragma unroll
+            for (int o = 8; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+            if (q == 0) ss_s[j * kUM + rr] += ss;
+            e[0] *= g.x; e[1] *= g.y; e[2] *= g.z; e[3] *= g.w;
+          }
+          uint16_t h[4], l[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) split_bf16(e[u], h[u], l[u]);
+          const int off = (rr >> 3) * 1024 + (rr & 7) * 128 + (((q >> 1) ^ (rr & 7)) * 16) + (q & 1) * 8;
+          *reinterpret_cast<uint2*>(ahi + off) = make_uint2(h[0] | ((uint32_t)h[1] << 16), h[2] | ((uint32_t)h[3] << 16));
+          *reinterpret_cast<uint2*>(alo + off) = make_uint2(l[0] | ((uint32_t)l[1] << 16), l[2] | ((uint32_t)l[3] << 16));
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        ubar_arrive(&afull[sa]);
+      };
+      // two register buffers in turn: the loads of the next step are in flight while this one
+      // is converted (no register copies that would wait for them)
+      float4 nxt[16];
+      if (steps > 0) load_step(0, cur);
+      for (int st = 0; st < steps; st += 2) {
+        if (st + 1 < steps) load_step(st + 1, nxt);
+        convert_step(st, cur);
+        if (st + 2 < steps) load_step(st + 2, cur);
+        if (st + 1 < steps) convert_step(st + 1, nxt);
+      }
+      // the row sums of squares were written by other converter threads than the epilogue's
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      wait_or_fail(accdone, ps & 1, failed);
     }
-    // accumulator complete when the last commit has arrived
-    if (!failed && !ubar_wait(&done[last % kUStages], (last / kUStages) & 1)) failed = true;
-    if (__syncthreads_or(failed)) {
-      failed = true;
-      break;
-    }
+    __syncwarp();
+    wit += nkb;
+    ait += nkb * nmt;
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const float inv = NORM ? rsqrtf(ss / (float)a.Kd + a.eps) : 1.f;
+    // ---- epilogue of this pass
+    for (int j = 0; j < nmt; ++j) {
+      const int mrow0 = (mt_lo + j) * kUM;
+      if (KS == 1) {
+        if (warp >= 2) {
+          const int row = mrow0 + r;
+          const float inv = NORM ? rsqrtf(ss_s[j * kUM + r] / (float)a.Kd + a.eps) : 1.f;
 #pragma unroll
-    for (int cb = 0; cb < kUN; cb += 32) {
-      uint32_t v[32];
-      const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)cb;
-      asm volatile(
-          "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-          "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-          : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-            "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]),
-            "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]),
-            "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]),
-            "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
-          : "r"(taddr));
-      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-      if (live) {
+          for (int cb = 0; cb < BN; cb += 32) {
+            uint32_t v[32];
+            const uint32_t taddr = tmem + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(j * BN + cb);
+            asm volatile(
+                "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+                "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+                : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+                  "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+                  "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]),
+                  "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]),
+                  "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+                : "r"(taddr));
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+            if (row < M) {
 #pragma unroll
-        for (int j = 0; j < 32; j += 2) {
-          const int col = n0 + cb + j;
-          if (col < a.N) {
-            const EpiPre p = epi_load(a.epi, rbase + row, col);
-            epi_store<__nv_bfloat16>(a.epi, p, rbase + row, col, __uint_as_float(v[j]) * inv,
-                                     __uint_as_float(v[j + 1]) * inv);
+              for (int q = 0; q < 32; q += 2) {
+                const int col = n0 + cb + q;
+                const EpiPre p = epi_load(a.epi, rbase + row, col);
+                epi_store<__nv_bfloat16>(a.epi, p, rbase + row, col, __uint_as_float(v[q]) * inv,
+                                         __uint_as_float(v[q + 1]) * inv);
+              }
+            }
           }
         }
+      } else {
+        cgr::cluster_group cl = cgr::this_cluster();
+        if (warp >= 2) {
+#pragma unroll
+          for (int cb = 0; cb < BN; cb += 32) {
+            uint32_t v[32];
+            const uint32_t taddr = tmem + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(j * BN + cb);
+            asm volatile(
+                "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+                "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+                : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+                  "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+                  "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]),
+                  "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]),
+                  "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+                : "r"(taddr));
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+            for (int q = 0; q < 32; ++q) red[r * (BN + 1) + cb + q] = __uint_as_float(v[q]);
+          }
+          ssred[r] = NORM ? ss_s[j * kUM + r] : 0.f;
+        }
+        cl.sync();
+        // this rank adds up rows [ks * RPC, (ks + 1) * RPC) over the cluster and stores them
+        for (int idx = tid; idx < RPC * (BN / 2); idx += kU2Threads) {
+          const int rl = idx / (BN / 2), c = (idx - rl * (BN / 2)) * 2;
+          const int rt = ks * RPC + rl;
+          // every rank's partials in one batch of remote loads, added in rank order
+          float s0 = 0.f, s1 = 0.f, sq = 0.f;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            if (k < KS) {
+              const float* pr = cl.map_shared_rank(red, k) + rt * (BN + 1) + c;
+              s0 += pr[0];
+              s1 += pr[1];
+              if (NORM) sq += *cl.map_shared_rank(ssred + rt, k);
+            }
+          }
+          const int row = mrow0 + rt;
+          if (row < M) {
+            const float inv = NORM ? rsqrtf(sq / (float)a.Kd + a.eps) : 1.f;
+            const EpiPre p = epi_load(a.epi, rbase + row, n0 + c);
+            epi_store<__nv_bfloat16>(a.epi, p, rbase + row, n0 + c, s0 * inv, s1 * inv);
+          }
+        }
+        cl.sync();
       }
     }
-    // all threads finished reading TMEM before the next tile overwrites it
+    // TMEM reads of this pass are done before the next pass's MMAs overwrite the accumulators
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   }
-  if (failed && tid == 0) atomicOr(a.epi.err, kErrTimeout);
+  // after a failed wait, W copies may still be in flight: wait (bounded) for the last one issued
+  // into each stage before the CTA's shared memory is released
+  const bool any_failed = __syncthreads_or(failed);
+  if (tid == 0 && any_failed) {
+    for (uint32_t s = 0; s < (uint32_t)C::kWStages && s < issued; ++s) {
+      const uint32_t last = issued - 1 - ((issued - 1 - s) % C::kWStages);
+      ubar_wait(&wfull[last % C::kWStages], (last / C::kWStages) & 1);
+    }
+    atomicOr(a.epi.err, kErrTimeout);
+  }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
-  if (warp == 0)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kUN) : "memory");
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tcols) : "memory");
 }
 
-size_t umma_smem_bytes() { return (size_t)kUStages * (kATileBytes + kBTileBytes) + 2 * kUStages * 8 + 16 + 1024; }
+template <int BN, bool NORM>
+void umma_go(const LinearArgs& a, const CUtensorMap& tm, dim3 grid, int MG, int KS, int tcols, cudaStream_t s) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kU2Threads);
+  cfg.dynamicSmemBytes = UCfg<BN>::kSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = KS;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++g_launches;
+  cudaLaunchKernelEx(&cfg, k_umma<BN, NORM>, a, tm, MG, KS, tcols);
+}
 
 }  // namespace
 
@@ -275,27 +471,48 @@ int make_weight_tmap(void* out, const void* W, long long rows, long long K) {
 }
 
 void kernel_attrs_umma() {
-  cudaFuncSetAttribute(k_umma<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)umma_smem_bytes());
-  cudaFuncSetAttribute(k_umma<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)umma_smem_bytes());
+  cudaFuncSetAttribute(k_umma<64, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)UCfg<64>::kSmem);
+  cudaFuncSetAttribute(k_umma<64, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)UCfg<64>::kSmem);
+  cudaFuncSetAttribute(k_umma<128, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)UCfg<128>::kSmem);
+  cudaFuncSetAttribute(k_umma<128, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)UCfg<128>::kSmem);
 }
 
 // Launch on the tensor cores when the layer fits the tile shapes; false otherwise.
+// Shape choice: 128-column tiles when at most four row tiles are typical and the layer is wide
+// enough to fill the GPU with them, else 64; then split K (power of two, at most 8, at least two
+// 64-deep blocks per CTA) while the grid still fits one wave of one CTA per SM.
 bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s) {
   if (!a.tmap || D.dtype != LCA_BF16 || a.N % kUN || a.Kd % kUK) return false;
   const int mt_cap = (a.M_cap + kUM - 1) / kUM;
   const int rows_typ = a.rows_typ > 0 ? a.rows_typ : a.M_cap;
-  int mtiles = (rows_typ + kUM - 1) / kUM;
-  mtiles = mtiles < 1 ? 1 : (mtiles > mt_cap ? mt_cap : mtiles);
-  // keep the grid within a few waves; extra row tiles are walked by the CTAs
-  const int ncol = a.N / kUN;
-  while (mtiles > 1 && (long long)mtiles * ncol * a.groups > 4LL * D.num_sms) mtiles = (mtiles + 1) / 2;
+  int mt_typ = (rows_typ + kUM - 1) / kUM;
+  mt_typ = mt_typ < 1 ? 1 : (mt_typ > mt_cap ? mt_cap : mt_typ);
+  const int sms = D.num_sms > 0 ? D.num_sms : 148;
+  const bool wide = mt_typ <= 4 && a.N % 128 == 0 && (long long)(a.N / 128) * a.groups * 8 >= sms;
+  const int BN = wide ? 128 : 64;
+  const int max_mt = 512 / BN;
+  const int ncol = a.N / BN;
+  const int mt_pass_cap = mt_cap < max_mt ? mt_cap : max_mt;
+  int tcols = 32;
+  while (tcols < mt_pass_cap * BN) tcols <<= 1;
+  int MG = (mt_typ + max_mt - 1) / max_mt;
+  const int MG_cap = (mt_cap + max_mt - 1) / max_mt;
+  MG = MG < 1 ? 1 : (MG > MG_cap ? MG_cap : MG);
+  const int kb = a.Kd / kUK;
+  int KS = 1;
+  while (KS < 8 && kb % (2 * KS) == 0 && kb / (2 * KS) >= 2 &&
+         (long long)ncol * a.groups * MG * (2 * KS) <= sms)
+    KS *= 2;
   CUtensorMap tm;
   memcpy(&tm, a.tmap, sizeof(tm));
-  ++g_launches;
-  if (a.norm)
-    launch_pdl(k_umma<true>, dim3(ncol, mtiles, a.groups), dim3(kUThreads), umma_smem_bytes(), s, a, tm, mtiles);
-  else
-    launch_pdl(k_umma<false>, dim3(ncol, mtiles, a.groups), dim3(kUThreads), umma_smem_bytes(), s, a, tm, mtiles);
+  const dim3 grid(ncol, KS, a.groups * MG);
+  if (BN == 128) {
+    if (a.norm) umma_go<128, true>(a, tm, grid, MG, KS, tcols, s);
+    else umma_go<128, false>(a, tm, grid, MG, KS, tcols, s);
+  } else {
+    if (a.norm) umma_go<64, true>(a, tm, grid, MG, KS, tcols, s);
+    else umma_go<64, false>(a, tm, grid, MG, KS, tcols, s);
+  }
   return true;
 }
 
@@ -306,8 +523,9 @@ LCA_TRACE_SETTER(trace_set_umma)
 using namespace lca;
 
 extern "C" int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N, int32_t K,
-                              const int32_t* M_dev, int32_t* err_dev, void* stream) {
-  if (!x || !W || !y || !M_dev || !err_dev || M < 1 || N < 1 || K < 1) return LCA_E_ARG;
+                              const int32_t* M_dev, int32_t rows_typ, int32_t* err_dev, void* stream) {
+  if (!x || !W || !y || !M_dev || !err_dev || M < 1 || N < 1 || K < 1 || rows_typ < 0 || rows_typ > M)
+    return LCA_E_ARG;
   CUtensorMap tm;
   int st = make_weight_tmap(&tm, W, N, K);
   if (st != LCA_OK) return st;
@@ -329,7 +547,7 @@ extern "C" int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M
   a.groups = 1;
   a.M = M_dev;
   a.M_cap = M;
-  a.rows_typ = M;
+  a.rows_typ = rows_typ > 0 ? rows_typ : M;
   a.tmap = &tm;
   a.epi.mode = EPI_STORE;
   a.epi.y = y;

@@ -251,7 +251,7 @@ int upload_params(lca_ctx* c) {
   return LCA_OK;
 }
 
-bool tiled_for(int rows) { return rows > 64; }
+bool tiled_for(const Dev& D, int rows) { return rows > D.tiled_min_rows; }
 
 const void* tmap_of(lca_ctx* c, const void* W) {
   auto it = c->tmaps.find(W);
@@ -268,7 +268,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
                int M_typ, int qt_grid, int splits, cudaStream_t s, const void* next_w = nullptr,
                size_t next_bytes = 0, const int* stable = nullptr, int stable_extra = 0) {
   Dev& D = c->L.D;
-  const bool tiled = tiled_for(M_typ);
+  const bool tiled = tiled_for(D, M_typ);
   const size_t tb = tw_bytes(D.dtype);
   const size_t b_qkv = 3ull * D.d * D.d * tb, b_o = (size_t)D.d * D.d * tb;
   const size_t b_13 = 2ull * D.F * D.d * tb, b_2 = (size_t)D.d * D.F * tb;
@@ -378,7 +378,7 @@ void run_mlp_heads(lca_ctx* c, int n, cudaStream_t s) {
     a.epi.ldy = a.epi.ldres = D.d;
     a.epi.err = D.err;
     a.tmap = tmap_of(c, a.W);
-    linear(D, a, tiled_for(D.B), s);
+    linear(D, a, tiled_for(D, D.B), s);
   }
 }
 
@@ -747,6 +747,7 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
   kernel_attrs_linear();
   kernel_attrs_step();
   kernel_attrs_umma();
+  kernel_attrs_attn();
   Dev& D = c->L.D;
   {
     int dev = 0, sms = 0;
@@ -759,6 +760,10 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.use_umma = (um && um[0] == '1') ? 0 : 1;
     const char* sc = getenv("LCA_ATTN_SPLIT_CAP");
     D.attn_split_cap = sc ? std::max(1, std::min(8, atoi(sc))) : 4;
+    const char* tr = getenv("LCA_TILED_MIN_ROWS");
+    D.tiled_min_rows = tr ? std::max(0, atoi(tr)) : 64;
+    const char* ap = getenv("LCA_ATTN_PIPE");
+    D.attn_pipe = ap ? (ap[0] == '1') : 1;
   }
   // state and counters start at zero
   if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);

@@ -107,7 +107,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_debug_force_candidates": [P, P, I32],
         "lca_destroy": [P],
         "lca_status_str": [ctypes.c_int],
-        "lca_debug_gemm": [P, P, P, I32, I32, I32, P, P, P],
+        "lca_debug_gemm": [P, P, P, I32, I32, I32, P, I32, P, P],
         "lca_decode_attention_scratch_bytes": [I32, I32, I32, I32, ctypes.POINTER(ctypes.c_size_t)],
         "lca_decode_attention": [P, P, P, P, I32, I32, I32, I32, I32, I32, P, F32, I32, P,
                                  ctypes.c_size_t, P],
@@ -251,7 +251,8 @@ class Context:
 
     TRACE_TAGS = {1: "gemv", 2: "gemv_f32", 3: "gemm", 4: "rowstats", 5: "attn", 6: "head",
                   7: "mb_plan", 8: "mb_fill", 9: "mlp_plan", 10: "verify_plan", 11: "segment",
-                  12: "lm_scatter", 13: "nb_input", 14: "commit", 15: "loop_ctl", 16: "other"}
+                  12: "lm_scatter", 13: "nb_input", 14: "commit", 15: "loop_ctl", 16: "other",
+                  17: "umma"}
 
     def trace(self, n, tau, mode, steps, cap=1 << 18):
         rec = np.zeros(cap, dtype=[("t0", "<u8"), ("t1", "<u8"), ("tw", "<u8"), ("tag", "<i4"),
@@ -307,13 +308,15 @@ def decode_attention(q, out, k_cache, v_cache, kv_len, scale, splits, scratch=No
     return lib.lca_decode_attention(*args, scratch.data_ptr(), scratch.numel(), st.cuda_stream)
 
 
-def debug_gemm(x, W, y, M_dev, err_dev, stream=None):
-    """y[:M] = bf16(x[:M]) . W^T on the tensor cores (tcgen05). x fp32 [M,K], W bf16 [N,K],
-    y fp32 [M,N], M_dev int32 [1] (rows actually used), err_dev int32 [1]. Returns the status."""
+def debug_gemm(x, W, y, M_dev, err_dev, rows_typ=0, stream=None):
+    """y[:M] = x[:M] . W^T on the tensor cores (tcgen05, activations split into two bf16 halves).
+    x fp32 [M,K], W bf16 [N,K], y fp32 [M,N], M_dev int32 [1] (rows actually used), err_dev
+    int32 [1]; rows_typ: row count the launch shape is chosen for (0 = M). Returns the status."""
     import torch
     st = stream if stream is not None else torch.cuda.current_stream(x.device)
     return load_library().lca_debug_gemm(x.data_ptr(), W.data_ptr(), y.data_ptr(), x.shape[0], W.shape[0],
-                                         W.shape[1], M_dev.data_ptr(), err_dev.data_ptr(), st.cuda_stream)
+                                         W.shape[1], M_dev.data_ptr(), rows_typ, err_dev.data_ptr(),
+                                         st.cuda_stream)
 
 
 def decode_attention_scratch_bytes(batch, heads, head_dim, splits):

@@ -4,9 +4,10 @@ full prompts, the bench's context size and its n, tau and unembedding gain).
 The oracle cannot replay a whole batch, so it replays the sampled sequences of each
 workload (``oracle_seqs``) one by one, and the GPU rows of those sequences inside the full
 batch are compared with it: next-byte and drafter logits within the bf16 tolerance (times
-the gain), emitted bytes and t, K equal. A decision may differ only where the oracle's
-margin is inside the tolerance (a near-tie of the top two logits, or a drafter probability
-next to tau); the sequence is then no longer followed. That the sampled rows equal the
+the gain), emitted bytes, t, K and the next c_1 equal. A decision may differ only where the
+oracle's margin for that decision is inside the tolerance (a near-tie of the top two logits
+of the deciding row, or a drafter probability next to tau); the sequence is then no longer
+followed. That the sampled rows equal the
 oracle's single-sequence run also shows that sequences of a batch do not interact.
 """
 import numpy as np
@@ -34,22 +35,32 @@ def lca():
     return mod
 
 
-def _decision_margin(rec, tau):
-    """Smallest distance, in logit units, of any decision of the step from flipping: half
-    the top-two gap of every row, and for each draft half the distance of
-    l_max - LSE from log(tau)."""
+def _gap(row):
+    s = np.sort(row)
+    return 0.5 * (s[-1] - s[-2])
+
+
+def _tau_gap(row, tau):
+    mx = row.max()
+    lse = mx + np.log(np.exp(row - mx).sum())
+    return 0.5 * abs(mx - lse - np.log(tau))
+
+
+def emitted_margin(rec, tau):
+    """Distance, in logit units, of the step's emitted bytes from flipping: the argmax of every
+    emitted draft and the tau test of every draft examined (up to the first rejection)."""
     m = np.inf
-    rows = [rec.nb_logits] + ([rec.mb_logits] if rec.mb_logits is not None and len(rec.mb_logits) else [])
-    for blk in rows:
-        for r in np.atleast_2d(blk):
-            s = np.sort(r)
-            m = min(m, 0.5 * (s[-1] - s[-2]))
-    if rec.mb_logits is not None:
-        for r in np.atleast_2d(rec.mb_logits):
-            mx = r.max()
-            lse = mx + np.log(np.exp(r - mx).sum())
-            m = min(m, 0.5 * abs(mx - lse - np.log(tau)))
+    mb = np.atleast_2d(rec.mb_logits) if rec.mb_logits is not None else np.zeros((0, 256))
+    for i in range(min(rec.a, len(mb))):
+        m = min(m, _gap(mb[i]))
+    for i in range(min(rec.a + 1, len(mb))):
+        m = min(m, _tau_gap(mb[i], tau))
     return m
+
+
+def next_byte_margin(rec):
+    """Distance of the next c_1 (next-byte argmax of the last accepted row) from flipping."""
+    return _gap(np.atleast_2d(rec.nb_logits)[rec.a])
 
 
 @pytest.mark.parametrize("name", ["paper_b32", "paper_long_b8", "mlp_b128"])
@@ -80,12 +91,16 @@ def test_full_size_sampled_sequences(lca, name):
             if n > 1:
                 np.testing.assert_allclose(mb[b], r.mb_logits, atol=tol, rtol=0)
             if out[b] != r.emitted:
-                assert _decision_margin(r, tau) < tol, (b, out[b], r.emitted)
+                assert emitted_margin(r, tau) < tol, (b, out[b], r.emitted)
                 del decs[b]
                 continue
             st = ctx.state(b)
             assert (st["t"], st["K"]) == (r.t, r.K)
             followed[b] += 1
+            # the next c_1 (next-byte argmax at the new last position) is a decision of this step
+            if st["next_byte"] != int(np.argmax(decs[b].nb_last)):
+                assert next_byte_margin(r) < tol, (b, st["next_byte"])
+                del decs[b]
         if not decs:
             break
     assert max(followed.values()) >= 2, followed

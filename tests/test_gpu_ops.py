@@ -69,11 +69,20 @@ def test_decode_attention_rejects_bad_arguments(lca):
     assert lca.decode_attention(q, out, k, v, lens, 0.1, 99, small) == -1
 
 
-@pytest.mark.parametrize("M,Mused,N,K", [(128, 128, 64, 64), (200, 200, 128, 1024), (300, 257, 1024, 1024),
-                                         (64, 17, 192, 4096), (1024, 1000, 3072, 1024)])
-def test_tensor_core_gemm_matches_reference(lca, M, Mused, N, K):
-    """tcgen05 GEMM (TMA weight tiles, 128-byte swizzle, TMEM accumulator) against a PyTorch
-    fp32 product of the same bf16-rounded operands."""
+@pytest.mark.parametrize("M,Mused,N,K,typ", [
+    (128, 128, 64, 64, 0),          # one tile, one K block
+    (200, 200, 128, 1024, 0),       # 128-column tiles, split K in a cluster
+    (300, 257, 1024, 1024, 0),      # ragged rows, cluster split K
+    (64, 17, 192, 4096, 0),         # few rows, deep K
+    (1024, 1000, 3072, 1024, 0),    # eight row tiles in TMEM at once
+    (256, 200, 3072, 1024, 0),      # 128-column tiles, four-way split K
+    (2100, 2050, 512, 1024, 128),   # launch shaped for 128 rows: clustered CTAs walk three row passes
+    (2100, 2100, 256, 320, 0),      # more row tiles than TMEM holds; K blocks not a power of two
+])
+def test_tensor_core_gemm_matches_reference(lca, M, Mused, N, K, typ):
+    """tcgen05 GEMM (TMA weight tiles, 128-byte swizzle, TMEM accumulators, split bf16
+    activations, cluster split-K) against a float64 product of the fp32 activations and the
+    bf16 weights."""
     import torch
     g = torch.Generator(device="cuda").manual_seed(M + N + K)
     x = torch.randn(M, K, device="cuda", generator=g)
@@ -81,11 +90,12 @@ def test_tensor_core_gemm_matches_reference(lca, M, Mused, N, K):
     y = torch.full((M, N), float("nan"), device="cuda")
     Md = torch.tensor([Mused], dtype=torch.int32, device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
-    assert lca.debug_gemm(x, W, y, Md, err) == 0
+    assert lca.debug_gemm(x, W, y, Md, err, rows_typ=typ) == 0
     torch.cuda.synchronize()
     assert int(err.item()) == 0
-    want = x[:Mused].to(torch.bfloat16).float() @ W.float().t()
-    got = y[:Mused]
-    tol = 2e-3 * float(want.abs().max())
-    np.testing.assert_allclose(got.cpu().numpy(), want.cpu().numpy(), atol=tol, rtol=0)
+    want = (x[:Mused].double() @ W.double().t()).cpu().numpy()
+    got = y[:Mused].double().cpu().numpy()
+    # two bf16 halves keep ~2^-17 of each activation; fp32 accumulation over K terms
+    tol = 1e-5 * float(np.abs(want).max())
+    np.testing.assert_allclose(got, want, atol=tol, rtol=0)
     assert torch.isnan(y[Mused:]).all()
