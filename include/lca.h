@@ -172,7 +172,7 @@ int lca_debug_profile(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, i
                       lca_profile* out);
 
 /* Run `steps` step graphs with launch tracing on: thread 0 of every CTA of every kernel records
- * {u64 start_ns, u64 end_ns, u64 wait_done_ns, i32 kernel tag, i32 cta, i32 sm, i32 pad}
+ * {u64 start_ns, u64 end_ns, u64 wait_done_ns, i32 kernel tag, i32 cta, i32 sm, i32 mark_ns}
  * (40 bytes) into `out`
  * (host, room for `cap` records); count = records written. Needs a bf16 context (the trace
  * buffer borrows scratch that the bf16 step does not use). */
@@ -184,9 +184,14 @@ int lca_debug_trace(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int
  * accumulation. x: device fp32 [M][K]; W: device bf16 [N][K]; y: device fp32 [M][N]; M_dev:
  * device int32 rows to compute (<= M); rows_typ: the row count the launch shape is chosen for
  * (0 = M; a smaller value makes CTAs walk several row passes); err_dev: device int32 error word
- * (bit 4: a bounded wait ran out). N and K must be multiples of 64. Asynchronous on `stream`. */
+ * (bit 4: a bounded wait ran out); scratch: device, lca_debug_gemm_scratch_bytes(M, K) bytes, or
+ * NULL. N and K must be multiples of 64. Asynchronous on `stream`. */
 int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N, int32_t K,
-                   const int32_t* M_dev, int32_t rows_typ, int32_t* err_dev, void* stream);
+                   const int32_t* M_dev, int32_t rows_typ, int32_t* err_dev, void* scratch, void* stream);
+/* Bytes of device scratch lca_debug_gemm needs to take the split-rows path (rows split once into
+ * bf16 halves by one kernel, then a GEMM fed entirely by TMA); with scratch == NULL it converts
+ * the activations inside the GEMM instead. */
+size_t lca_debug_gemm_scratch_bytes(int32_t M, int32_t K);
 
 /* Micro-benchmark: one graph of `iters` back-to-back launches of one kernel kind over `rows`
  * rows (0 RMSNorm+QKV, 1 Wo, 2 RMSNorm+W1/W3+SwiGLU, 3 W2, 4 decode attention over the

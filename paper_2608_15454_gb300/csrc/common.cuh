@@ -38,7 +38,7 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 // The pointers are per translation unit (no relocatable device code); trace_set() fills them.
 struct TraceRec {
   unsigned long long t0, t1, tw;  // entry, exit, grid-dependency wait returned
-  int tag, cta, sm, pad;
+  int tag, cta, sm, mark;  // mark: optional mid-kernel time, ns after entry (0: none)
 };
 enum TraceTag : int {
   TT_GEMV = 1, TT_GEMV_F32, TT_GEMM, TT_ROWSTATS, TT_ATTN, TT_HEAD, TT_MB_PLAN, TT_MB_FILL,
@@ -61,8 +61,9 @@ __device__ __forceinline__ unsigned smid() {
 struct TraceScope {
   unsigned long long t0, tw;
   int tag;
+  unsigned mk;  // optional mid-kernel mark: nanoseconds after entry (0: none)
   bool on;
-  __device__ __forceinline__ explicit TraceScope(int t) : t0(0), tw(0), tag(t), on(false) {
+  __device__ __forceinline__ explicit TraceScope(int t) : t0(0), tw(0), tag(t), mk(0), on(false) {
     if (threadIdx.x == 0 && threadIdx.y == 0 && g_trace) {
       on = true;
       t0 = gtimer();
@@ -71,6 +72,9 @@ struct TraceScope {
   }
   __device__ __forceinline__ void waited() {
     if (on) tw = gtimer();
+  }
+  __device__ __forceinline__ void mark() {
+    if (on) mk = (unsigned)(gtimer() - t0);
   }
   __device__ __forceinline__ ~TraceScope() {
     if (on) {
@@ -83,7 +87,7 @@ struct TraceScope {
         r.tag = tag;
         r.cta = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
         r.sm = (int)smid();
-        r.pad = 0;
+        r.mark = (int)mk;
         g_trace[i] = r;
       }
     }
@@ -242,6 +246,12 @@ struct Dev {
   float* o_tab;    // [B][L][d] LM outputs
   float* y_last;   // [B][d] next-byte hidden at t-1 (MLP head input)
   int* kpos;       // [B][S] K(p) of committed positions (prefill scratch)
+  // activations of a tensor-core layer split into two bf16 halves (x * g = hi + lo) and the rows'
+  // inverse RMS, written by k_split_rows and read by TMA in k_tgemm: [as_rows][up to F]
+  __nv_bfloat16* as_hi;
+  __nv_bfloat16* as_lo;
+  float* as_inv;
+  int as_rows;
 
   // rows
   float* x_mb;
@@ -321,10 +331,15 @@ struct LinearArgs {
   size_t pf_bytes[2];
   int rows_typ;  // typical row count (sizes the activation staging); 0: M_cap
   const void* tmap;  // host copy of the weight's TMA tensor map (tensor-core path), or nullptr
+  // host copies of the TMA tensor maps of the split activations (hi, lo) for this Kd, or nullptr:
+  // then the tensor-core path converts the activations inside the GEMM
+  const void* amap;
 };
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s);
 bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s);
 int make_weight_tmap(void* out, const void* W, long long rows, long long K);
+// TMA tensor maps (hi then lo, 128 bytes each) of split activations [rows][K] bf16, 64 x 128 boxes
+int make_split_tmaps(void* out, const void* hi, const void* lo, long long rows, long long K);
 void kernel_attrs_umma();
 void trace_set_umma(TraceRec* buf, unsigned* counter, unsigned cap);
 

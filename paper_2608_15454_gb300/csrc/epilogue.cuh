@@ -107,6 +107,33 @@ static __device__ __forceinline__ EpiPre epi_load(const EpiArgs& e, int r, int c
   return p;
 }
 
+// The same epilogue split for row-wise batching (tensor-core tiles, where a thread owns a row and
+// walks its columns): per-row metadata once, then per pair one float2 operand (the residual
+// pair, or the RoPE cos/sin) that can be loaded a whole chunk of columns ahead of the stores.
+struct EpiRow {
+  int pos, b, slot;
+};
+static __device__ __forceinline__ EpiRow epi_row(const EpiArgs& e, int r) {
+  EpiRow q{0, 0, 0};
+  if (e.mode == EPI_QKV) {
+    q.pos = e.rows.pos[r];
+    q.b = e.rows.b[r];
+    q.slot = e.rows.slot[r];
+  }
+  return q;
+}
+static __device__ __forceinline__ float2 epi_operand(const EpiArgs& e, const EpiRow& q, int r, int c) {
+  if (e.mode == EPI_RESID || e.mode == EPI_RESID_SILU)
+    return *reinterpret_cast<const float2*>(e.res + (size_t)r * e.ldres + c);
+  if (e.mode == EPI_QKV) {
+    const int part = c / e.d;
+    if (part < 2) {
+      const int dd = (c - part * e.d) % e.hd;
+      return e.rope[(size_t)q.pos * (e.hd >> 1) + (dd >> 1)];
+    }
+  }
+  return make_float2(0.f, 0.f);
+}
 template <typename TC>
 static __device__ __forceinline__ void epi_store(const EpiArgs& e, const EpiPre& p, int r, int c, float a0, float a1) {
   switch (e.mode) {
@@ -155,6 +182,19 @@ static __device__ __forceinline__ void epi_store(const EpiArgs& e, const EpiPre&
       break;
     }
   }
+}
+
+
+template <typename TC>
+static __device__ __forceinline__ void epi_out(const EpiArgs& e, const EpiRow& q, float2 op, int r, int c,
+                                               float a0, float a1) {
+  EpiPre p;
+  p.r0 = op.x;
+  p.r1 = op.y;
+  p.cs = op;
+  p.b = q.b;
+  p.slot = q.slot;
+  epi_store<TC>(e, p, r, c, a0, a1);
 }
 
 

@@ -105,6 +105,10 @@ void carve(const lca_config& c, char* base, Layout& L) {
   D.o_tab = cv.take<float>(B * Lt * d);
   D.y_last = cv.take<float>(B * d);
   D.kpos = cv.take<int>(B * S);
+  D.as_rows = (int)(B * NM);
+  D.as_hi = cv.take<__nv_bfloat16>((size_t)D.as_rows * std::max(d, F));
+  D.as_lo = cv.take<__nv_bfloat16>((size_t)D.as_rows * std::max(d, F));
+  D.as_inv = cv.take<float>(D.as_rows);
 
   D.x_mb = cv.take<float>(R * d);
   D.x_enc = cv.take<float>(R * d);
@@ -177,9 +181,13 @@ struct Staging {
 struct alignas(64) TMapBlob {
   unsigned char b[128];
 };
+struct alignas(64) SplitMapBlob {
+  unsigned char b[256];  // hi, lo
+};
 
 struct lca_ctx {
   std::map<const void*, TMapBlob> tmaps;  // TMA tensor maps of the bf16 weights
+  std::map<int, SplitMapBlob> amaps;      // TMA tensor maps of the split activations, by K
   lca_config cfg{};
   Layout L;
   Staging stg{};
@@ -253,6 +261,13 @@ int upload_params(lca_ctx* c) {
 
 bool tiled_for(const Dev& D, int rows) { return rows > D.tiled_min_rows; }
 
+// Split-activation maps for a layer of inner size K whose rows fit the split buffers.
+const void* amap_of(lca_ctx* c, int K, int rows_cap) {
+  if (rows_cap > c->L.D.as_rows) return nullptr;
+  auto it = c->amaps.find(K);
+  return it == c->amaps.end() ? nullptr : it->second.b;
+}
+
 const void* tmap_of(lca_ctx* c, const void* W) {
   auto it = c->tmaps.find(W);
   return it == c->tmaps.end() ? nullptr : it->second.b;
@@ -307,6 +322,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.pf[1] = bk.w13;
     a.pf_bytes[1] = b_13;
     a.tmap = tmap_of(c, a.W);
+    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
     linear(D, a, tiled, s);
     attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra);
     // x += Wo . attn
@@ -323,6 +339,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.pf[1] = nullptr;
     a.pf_bytes[1] = 0;
     a.tmap = tmap_of(c, a.W);
+    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
     linear(D, a, tiled, s);
     // mid = silu(W1 . n(x)) * (W3 . n(x))
     a.x = x;
@@ -335,6 +352,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.pf[0] = nqkv;
     a.pf_bytes[0] = nqkv_b;
     a.tmap = tmap_of(c, a.W);
+    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
     linear(D, a, tiled, s);
     // x += W2 . mid
     a.x = D.mid;
@@ -350,6 +368,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.pf[0] = nx ? nx->wo : nullptr;
     a.pf_bytes[0] = nx ? b_o : 0;
     a.tmap = tmap_of(c, a.W);
+    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
     linear(D, a, tiled, s);
   }
 }
@@ -378,6 +397,7 @@ void run_mlp_heads(lca_ctx* c, int n, cudaStream_t s) {
     a.epi.ldy = a.epi.ldres = D.d;
     a.epi.err = D.err;
     a.tmap = tmap_of(c, a.W);
+    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
     linear(D, a, tiled_for(D, D.B), s);
   }
 }
@@ -784,6 +804,10 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     if (D.mlp_w)
       for (int l = 0; l < D.n_mb; ++l)
         add((char*)D.mlp_w + (size_t)l * D.n_mlp_heads * D.d * D.d * 2, (long long)D.n_mlp_heads * D.d, D.d);
+    for (int K : {D.d, D.F}) {
+      SplitMapBlob blob;
+      if (make_split_tmaps(blob.b, D.as_hi, D.as_lo, D.as_rows, K) == LCA_OK) c->amaps[K] = blob;
+    }
   }
   launch_rope_table(D, cfg->rope_base, c->stream);
   if (check(cudaGetLastError(), "rope") || check(cudaStreamSynchronize(c->stream), "create sync"))

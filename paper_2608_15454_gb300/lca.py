@@ -28,7 +28,7 @@ EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "
            "lca_debug_set_eager", "lca_debug_profile", "lca_debug_bench_kernel", "lca_debug_trace",
            "lca_debug_logits",
            "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str",
-           "lca_debug_gemm",
+           "lca_debug_gemm", "lca_debug_gemm_scratch_bytes",
            "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
            "lca_decode_attention_noalloc_capacity")
 
@@ -107,7 +107,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_debug_force_candidates": [P, P, I32],
         "lca_destroy": [P],
         "lca_status_str": [ctypes.c_int],
-        "lca_debug_gemm": [P, P, P, I32, I32, I32, P, I32, P, P],
+        "lca_debug_gemm": [P, P, P, I32, I32, I32, P, I32, P, P, P],
+        "lca_debug_gemm_scratch_bytes": [I32, I32],
         "lca_decode_attention_scratch_bytes": [I32, I32, I32, I32, ctypes.POINTER(ctypes.c_size_t)],
         "lca_decode_attention": [P, P, P, P, I32, I32, I32, I32, I32, I32, P, F32, I32, P,
                                  ctypes.c_size_t, P],
@@ -118,7 +119,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         f = getattr(lib, name)
         f.argtypes = args
         f.restype = (ctypes.c_char_p if name == "lca_status_str" else
-                     ctypes.c_size_t if name == "lca_decode_attention_noalloc_capacity" else ctypes.c_int)
+                     ctypes.c_size_t if name in ("lca_decode_attention_noalloc_capacity",
+                                                 "lca_debug_gemm_scratch_bytes") else ctypes.c_int)
     _lib = lib
     return lib
 
@@ -256,7 +258,7 @@ class Context:
 
     def trace(self, n, tau, mode, steps, cap=1 << 18):
         rec = np.zeros(cap, dtype=[("t0", "<u8"), ("t1", "<u8"), ("tw", "<u8"), ("tag", "<i4"),
-                                   ("cta", "<i4"), ("sm", "<i4"), ("pad", "<i4")])
+                                   ("cta", "<i4"), ("sm", "<i4"), ("mark", "<i4")])
         cnt = ctypes.c_int32()
         self._check(self.lib.lca_debug_trace(self.h, n, tau, mode, steps, _ptr(rec), cap, ctypes.byref(cnt)),
                     "lca_debug_trace")
@@ -308,15 +310,22 @@ def decode_attention(q, out, k_cache, v_cache, kv_len, scale, splits, scratch=No
     return lib.lca_decode_attention(*args, scratch.data_ptr(), scratch.numel(), st.cuda_stream)
 
 
-def debug_gemm(x, W, y, M_dev, err_dev, rows_typ=0, stream=None):
+def debug_gemm(x, W, y, M_dev, err_dev, rows_typ=0, scratch=None, stream=None):
     """y[:M] = x[:M] . W^T on the tensor cores (tcgen05, activations split into two bf16 halves).
     x fp32 [M,K], W bf16 [N,K], y fp32 [M,N], M_dev int32 [1] (rows actually used), err_dev
-    int32 [1]; rows_typ: row count the launch shape is chosen for (0 = M). Returns the status."""
+    int32 [1]; rows_typ: row count the launch shape is chosen for (0 = M); scratch: a uint8
+    device tensor of debug_gemm_scratch_bytes(M, K) bytes selects the split-rows + TMA path.
+    Returns the status."""
     import torch
     st = stream if stream is not None else torch.cuda.current_stream(x.device)
     return load_library().lca_debug_gemm(x.data_ptr(), W.data_ptr(), y.data_ptr(), x.shape[0], W.shape[0],
                                          W.shape[1], M_dev.data_ptr(), rows_typ, err_dev.data_ptr(),
+                                         scratch.data_ptr() if scratch is not None else None,
                                          st.cuda_stream)
+
+
+def debug_gemm_scratch_bytes(M, K):
+    return load_library().lca_debug_gemm_scratch_bytes(M, K)
 
 
 def decode_attention_scratch_bytes(batch, heads, head_dim, splits):

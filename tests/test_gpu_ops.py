@@ -79,10 +79,11 @@ def test_decode_attention_rejects_bad_arguments(lca):
     (2100, 2050, 512, 1024, 128),   # launch shaped for 128 rows: clustered CTAs walk three row passes
     (2100, 2100, 256, 320, 0),      # more row tiles than TMEM holds; K blocks not a power of two
 ])
-def test_tensor_core_gemm_matches_reference(lca, M, Mused, N, K, typ):
+@pytest.mark.parametrize("split", [False, True])
+def test_tensor_core_gemm_matches_reference(lca, M, Mused, N, K, typ, split):
     """tcgen05 GEMM (TMA weight tiles, 128-byte swizzle, TMEM accumulators, split bf16
     activations, cluster split-K) against a float64 product of the fp32 activations and the
-    bf16 weights."""
+    bf16 weights; both the in-GEMM conversion and the split-rows + TMA path."""
     import torch
     g = torch.Generator(device="cuda").manual_seed(M + N + K)
     x = torch.randn(M, K, device="cuda", generator=g)
@@ -90,7 +91,10 @@ def test_tensor_core_gemm_matches_reference(lca, M, Mused, N, K, typ):
     y = torch.full((M, N), float("nan"), device="cuda")
     Md = torch.tensor([Mused], dtype=torch.int32, device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
-    assert lca.debug_gemm(x, W, y, Md, err, rows_typ=typ) == 0
+    scratch = None
+    if split:
+        scratch = torch.empty(lca.debug_gemm_scratch_bytes(M, K), dtype=torch.uint8, device="cuda")
+    assert lca.debug_gemm(x, W, y, Md, err, rows_typ=typ, scratch=scratch) == 0
     torch.cuda.synchronize()
     assert int(err.item()) == 0
     want = (x[:Mused].double() @ W.double().t()).cpu().numpy()
