@@ -139,6 +139,9 @@ struct KV {
   void* k;
   void* v;
   int S; // slots per (b, h)
+  // host copies of the TMA tensor maps of K and V (bf16, head_dim 64: 64-key x 64-dim boxes with
+  // the 128-byte swizzle), or nullptr; used by the tensor-core decode attention
+  const void* tmaps;
 };
 
 struct EpiArgs {
@@ -227,7 +230,8 @@ struct Dev {
   int use_tma;  // bf16 linear layers use the bulk-copy weight pipeline
   int attn_split_cap;  // largest cluster (key split) of decode attention
   int tiled_min_rows;  // layers with more typical rows than this run on the tensor cores
-  int attn_pipe;       // decode attention: 1 = bulk-copy pipelined kernel, 0 = register-tiled kernel
+  int attn_pipe;       // decode attention: 2 = tensor cores (bf16, head_dim 64), 1 = bulk-copy pipelined
+                       // CUDA-core kernel, 0 = register-tiled kernel
   int use_umma;        // many-row bf16 layers run on the tensor cores (tcgen05)
 
   // weights (storage type; norms and bos fp32)
@@ -340,6 +344,8 @@ bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s);
 int make_weight_tmap(void* out, const void* W, long long rows, long long K);
 // TMA tensor maps (hi then lo, 128 bytes each) of split activations [rows][K] bf16, 64 x 128 boxes
 int make_split_tmaps(void* out, const void* hi, const void* lo, long long rows, long long K);
+// TMA tensor maps (K then V, 128 bytes each) of one bf16 KV-cache layer [rows][64], 64 x 64 boxes
+int make_kv_tmaps(void* out, const void* k, const void* v, long long rows);
 void kernel_attrs_umma();
 void trace_set_umma(TraceRec* buf, unsigned* counter, unsigned cap);
 

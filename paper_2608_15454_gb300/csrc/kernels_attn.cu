@@ -7,6 +7,9 @@
 // With several key splits each CTA writes (max, sum, acc) partials and the last CTA of the
 // (sequence, head) combines them in split order (deterministic).
 #include <cooperative_groups.h>
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cstring>
 #include <mutex>
 
 #include "common.cuh"
@@ -841,6 +844,374 @@ void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B
                      stable_extra);
 }
 
+// ---------------------------------------------------------------- tensor-core decode attention
+// bf16 caches with head_dim 64. One CTA serves (sequence, query tile of up to 16 rows, head, key
+// split): a producer warp streams 64-key chunks of K and V by TMA (128-byte swizzle) through a
+// ring of shared-memory stages, and four compute warps each take every fourth chunk with their
+// own online softmax (no block barrier inside the key loop). Q.K^T and P.V run on the tensor cores
+// (mma.sync m16n8k16, bf16 operands, fp32 accumulation); K and V are exactly bf16, and Q and P
+// are each split into two bf16 halves (x = hi + lo) so that the products keep about 16 bits of
+// them. The warps then combine in shared memory, and the key splits of one (sequence, head)
+// through distributed shared memory in a thread-block cluster.
+constexpr int kA4Warps = 4;
+constexpr int kA4Threads = (kA4Warps + 1) * 32;  // + the producer warp
+constexpr int kA4QT = 16;
+constexpr int kA4Keys = 64;
+constexpr int kA4Stages = 8;
+constexpr uint32_t kA4Chunk = kA4Keys * 64 * 2;  // one K or V chunk: 8 KB
+
+__device__ __forceinline__ void a4_tma(void* dst, const CUtensorMap* m, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+          a3_su32(dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(a3_su32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void ldsm4(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm4t(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// (x0, x1) -> bf16x2 hi and the bf16x2 of the remainders (first element in the low half)
+__device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+  const float2 hf = __bfloat1622float2(h);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+// byte offset of 16-byte chunk c of row j in a [64][128 B] tile with the 128-byte swizzle
+__device__ __forceinline__ uint32_t swz(int j, int c) { return (uint32_t)(j * 128 + ((c ^ (j & 7)) << 4)); }
+
+__global__ void __launch_bounds__(kA4Threads, 1)
+k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
+           const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+           const int* __restrict__ stable, int stable_stride, int stable_extra) {
+  namespace cgr = cooperative_groups;
+  constexpr int HD = 64, QT = kA4QT, KC = kA4Keys, NS = kA4Stages;
+  extern __shared__ __align__(1024) unsigned char a4raw[];
+  unsigned char* ring =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(a4raw) + 1023) & ~uintptr_t(1023));
+  float* qs = reinterpret_cast<float*>(ring + NS * 2 * kA4Chunk);  // [QT][HD], scaled
+  float* pacc = qs + QT * HD;                                       // [QT][HD]
+  float* s_m = pacc + QT * HD;                                      // [QT]
+  float* s_l = s_m + QT;                                            // [QT]
+  int* s_kv = reinterpret_cast<int*>(s_l + QT);                     // [QT]
+  uint64_t* full = reinterpret_cast<uint64_t*>(s_kv + QT);          // [NS]
+  uint64_t* empty = full + NS;                                      // [NS]
+  // after the key loop the ring holds the warps' partial results
+  float* Ow = reinterpret_cast<float*>(ring);                       // [warps][QT][HD]
+  float* mw = Ow + kA4Warps * QT * HD;                              // [warps][QT]
+  float* lw = mw + kA4Warps * QT;                                   // [warps][QT]
+
+  TraceScope _trace(TT_ATTN);
+  cgr::cluster_group cl = cgr::this_cluster();
+  const int splits = (int)cl.dim_blocks().z;
+  const int sp = (int)cl.block_rank();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, t = lane & 3;
+  if (tid == 0) {
+    for (int i = 0; i < NS; ++i) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&full[i])) : "memory");
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&empty[i])) : "memory");
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+  }
+  if (stable && tid < 2) {
+    // committed slots do not change during a step: warm this CTA's share in L2 (a hint)
+    const int bb = blockIdx.x, hh = blockIdx.z / splits;
+    const int tt = stable[(size_t)bb * stable_stride];
+    const int est = ((tt + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
+    const int lo = sp * est, hi = min(tt, lo + est);
+    if (hi > lo) {
+      const __nv_bfloat16* base = reinterpret_cast<const __nv_bfloat16*>(tid == 0 ? kv.k : kv.v) +
+                                  (((size_t)bb * H + hh) * kv.S + lo) * HD;
+      const uint32_t bytes = (uint32_t)((hi - lo) * HD * 2);
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"(bytes & ~15u) : "memory");
+    }
+  }
+  pdl_trigger();
+  pdl_wait();
+  _trace.waited();
+  __syncthreads();
+  const int b = blockIdx.x;
+  const int h = blockIdx.z / splits;
+  const int nrows = rows.seq_count[b];
+  const int rbeg = rows.seq_start[b];
+  const int ntiles = (nrows + QT - 1) / QT;
+  const int ld = H * HD;
+  const int krow0 = (b * H + h) * kv.S;  // first tensor-map row of this (sequence, head)
+  bool failed = false;
+  uint32_t cc = 0, issued = 0;
+
+  for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
+    const int r0 = rbeg + qt * QT;
+    const int nq = min(QT, nrows - qt * QT);
+    for (int idx = tid; idx < QT * HD; idx += kA4Threads) {
+      const int i = idx / HD, dd = idx - i * HD;
+      qs[idx] = i < nq ? q[(size_t)(r0 + i) * ld + h * HD + dd] * scale : 0.f;
+    }
+    if (tid < QT) {
+      int kl = tid < nq ? rows.kvlen[r0 + tid] : 0;
+      if (kl > kv.S || kl < 0) {
+        atomicOr(err, kErrIndex);
+        kl = kl < 0 ? 0 : kv.S;
+      }
+      s_kv[tid] = kl;
+    }
+    __syncthreads();
+    int kv_hi = 0;
+#pragma unroll
+    for (int i = 0; i < QT; ++i) kv_hi = max(kv_hi, s_kv[i]);
+    const int per = ((kv_hi + splits - 1) / splits + KC - 1) / KC * KC;
+    const int lo = sp * per;
+    const int hi = min(kv_hi, lo + per);
+    const int nch = hi > lo ? (hi - lo + KC - 1) / KC : 0;
+
+    // per compute warp: running max, sum and accumulator of rows g and g + 8
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+    float o[8][4];
+#pragma unroll
+    for (int n = 0; n < 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+    if (warp == kA4Warps) {
+      // producer
+      if (lane == 0) {
+        for (int c = 0; c < nch; ++c) {
+          const uint32_t gi = cc + c;
+          const int st = gi % NS;
+          if (gi >= (uint32_t)NS && !failed && !a3_wait(&empty[st], ((gi / NS) - 1) & 1)) failed = true;
+          if (failed) break;
+          ++issued;
+          unsigned char* dst = ring + (size_t)st * 2 * kA4Chunk;
+          a3_expect(&full[st], 2 * kA4Chunk);
+          a4_tma(dst, &tmK, 0, krow0 + lo + c * KC, &full[st]);
+          a4_tma(dst + kA4Chunk, &tmV, 0, krow0 + lo + c * KC, &full[st]);
+        }
+      }
+      __syncwarp();
+    } else {
+      // Q fragments (rows g and g + 8, split into bf16 halves)
+      uint32_t qh[4][4], ql[4][4];
+#pragma unroll
+      for (int ks = 0; ks < 4; ++ks) {
+        const int c0 = 16 * ks + 2 * t;
+        split2(qs[g * HD + c0], qs[g * HD + c0 + 1], qh[ks][0], ql[ks][0]);
+        split2(qs[(g + 8) * HD + c0], qs[(g + 8) * HD + c0 + 1], qh[ks][1], ql[ks][1]);
+        split2(qs[g * HD + c0 + 8], qs[g * HD + c0 + 9], qh[ks][2], ql[ks][2]);
+        split2(qs[(g + 8) * HD + c0 + 8], qs[(g + 8) * HD + c0 + 9], qh[ks][3], ql[ks][3]);
+      }
+      const int kl0 = min(s_kv[g], hi), kl1 = min(s_kv[g + 8], hi);
+      for (int c = warp; c < nch; c += kA4Warps) {
+        const uint32_t gi = cc + c;
+        const int st = gi % NS;
+        if (!failed && !a3_wait(&full[st], (gi / NS) & 1)) failed = true;
+        const uint32_t kb = a3_su32(ring + (size_t)st * 2 * kA4Chunk), vb = kb + kA4Chunk;
+        const int j0 = lo + c * KC;
+        // S = Q K^T over 64 keys: n-tile nt = keys 8 nt .. 8 nt + 7
+        float sacc[8][4];
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+          sacc[nt][0] = sacc[nt][1] = sacc[nt][2] = sacc[nt][3] = 0.f;
+#pragma unroll
+          for (int kp = 0; kp < 2; ++kp) {
+            uint32_t bf[4];
+            // matrices: keys 8 nt + (lane & 7), dims chunks 4 kp + (lane >> 3)
+            ldsm4(kb + swz(8 * nt + (lane & 7), 4 * kp + (lane >> 3)), bf);
+            mma16816(sacc[nt], qh[2 * kp], bf[0], bf[1]);
+            mma16816(sacc[nt], ql[2 * kp], bf[0], bf[1]);
+            mma16816(sacc[nt], qh[2 * kp + 1], bf[2], bf[3]);
+            mma16816(sacc[nt], ql[2 * kp + 1], bf[2], bf[3]);
+          }
+        }
+        // mask, online softmax (rows g, g + 8; the four lanes of a quad share a row)
+        float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+          const int key = j0 + 8 * nt + 2 * t;
+          if (key >= kl0) sacc[nt][0] = -INFINITY;
+          if (key + 1 >= kl0) sacc[nt][1] = -INFINITY;
+          if (key >= kl1) sacc[nt][2] = -INFINITY;
+          if (key + 1 >= kl1) sacc[nt][3] = -INFINITY;
+          mx0 = fmaxf(mx0, fmaxf(sacc[nt][0], sacc[nt][1]));
+          mx1 = fmaxf(mx1, fmaxf(sacc[nt][2], sacc[nt][3]));
+        }
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+        const float n0 = fmaxf(m0, mx0), n1 = fmaxf(m1, mx1);
+        const float cr0 = n0 == -INFINITY ? 1.f : (m0 == -INFINITY ? 0.f : expf(m0 - n0));
+        const float cr1 = n1 == -INFINITY ? 1.f : (m1 == -INFINITY ? 0.f : expf(m1 - n1));
+        m0 = n0;
+        m1 = n1;
+        float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+          sacc[nt][0] = sacc[nt][0] == -INFINITY ? 0.f : expf(sacc[nt][0] - n0);
+          sacc[nt][1] = sacc[nt][1] == -INFINITY ? 0.f : expf(sacc[nt][1] - n0);
+          sacc[nt][2] = sacc[nt][2] == -INFINITY ? 0.f : expf(sacc[nt][2] - n1);
+          sacc[nt][3] = sacc[nt][3] == -INFINITY ? 0.f : expf(sacc[nt][3] - n1);
+          ps0 += sacc[nt][0] + sacc[nt][1];
+          ps1 += sacc[nt][2] + sacc[nt][3];
+          o[nt][0] *= cr0;
+          o[nt][1] *= cr0;
+          o[nt][2] *= cr1;
+          o[nt][3] *= cr1;
+        }
+        l0 = l0 * cr0 + ps0;
+        l1 = l1 * cr1 + ps1;
+        // O += P V: k-step kk = keys 16 kk .. 16 kk + 15; n-tiles of 8 dims
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          uint32_t ph[4], pl[4];
+          split2(sacc[2 * kk][0], sacc[2 * kk][1], ph[0], pl[0]);
+          split2(sacc[2 * kk][2], sacc[2 * kk][3], ph[1], pl[1]);
+          split2(sacc[2 * kk + 1][0], sacc[2 * kk + 1][1], ph[2], pl[2]);
+          split2(sacc[2 * kk + 1][2], sacc[2 * kk + 1][3], ph[3], pl[3]);
+#pragma unroll
+          for (int np = 0; np < 4; ++np) {
+            uint32_t bf[4];
+            // matrices: keys 16 kk + 8 ((lane >> 3) & 1) + (lane & 7), dims chunk 2 np + (lane >> 4)
+            ldsm4t(vb + swz(16 * kk + 8 * ((lane >> 3) & 1) + (lane & 7), 2 * np + (lane >> 4)), bf);
+            mma16816(o[2 * np], ph, bf[0], bf[1]);
+            mma16816(o[2 * np], pl, bf[0], bf[1]);
+            mma16816(o[2 * np + 1], ph, bf[2], bf[3]);
+            mma16816(o[2 * np + 1], pl, bf[2], bf[3]);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a3_su32(&empty[st])) : "memory");
+      }
+      l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+      l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+      l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+      l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+    }
+    __syncthreads();  // every warp is done with the ring: it now holds the warps' partial results
+    if (warp < kA4Warps) {
+      float* ow = Ow + warp * QT * HD;
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) {
+        *reinterpret_cast<float2*>(ow + g * HD + 8 * nt + 2 * t) = make_float2(o[nt][0], o[nt][1]);
+        *reinterpret_cast<float2*>(ow + (g + 8) * HD + 8 * nt + 2 * t) = make_float2(o[nt][2], o[nt][3]);
+      }
+      if (t == 0) {
+        mw[warp * QT + g] = m0;
+        lw[warp * QT + g] = l0;
+        mw[warp * QT + g + 8] = m1;
+        lw[warp * QT + g + 8] = l1;
+      }
+    }
+    __syncthreads();
+    // combine the warps: this split's (max, sum, accumulator) per row
+    for (int idx = tid; idx < QT * HD; idx += kA4Threads) {
+      const int i = idx / HD, dd = idx - i * HD;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kA4Warps; ++w) M = fmaxf(M, mw[w * QT + i]);
+      float L = 0.f, o = 0.f;
+#pragma unroll
+      for (int w = 0; w < kA4Warps; ++w) {
+        const float mv = mw[w * QT + i];
+        const float f = mv == -INFINITY ? 0.f : expf(mv - M);
+        L += f * lw[w * QT + i];
+        o += f * Ow[(w * QT + i) * HD + dd];
+      }
+      pacc[idx] = o;
+      if (dd == 0) {
+        s_m[i] = M;
+        s_l[i] = L;
+      }
+    }
+    cl.sync();
+    {
+      const int dpr = (HD + splits - 1) / splits;
+      const int d0 = sp * dpr;
+      const int nd = min(dpr, HD - d0);
+      for (int idx = tid; idx < nq * nd; idx += kA4Threads) {
+        const int i = idx / nd, dd = d0 + (idx - i * nd);
+        float mr[kMaxClusterSplit], lr[kMaxClusterSplit], ar[kMaxClusterSplit];
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
+          if (k < splits) {
+            mr[k] = *cl.map_shared_rank(&s_m[i], k);
+            lr[k] = *cl.map_shared_rank(&s_l[i], k);
+            ar[k] = *cl.map_shared_rank(&pacc[i * HD + dd], k);
+          }
+        }
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k)
+          if (k < splits) M = fmaxf(M, mr[k]);
+        float L = 0.f, o = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
+          if (k < splits && mr[k] != -INFINITY) {
+            const float w = expf(mr[k] - M);
+            L += w * lr[k];
+            o += w * ar[k];
+          }
+        }
+        out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? o / L : 0.f;
+      }
+    }
+    cl.sync();
+    cc += nch;
+  }
+  // after a failed wait, copies may still be in flight: wait (bounded) for the last one issued
+  // into each stage before the CTA's shared memory is released
+  if (__syncthreads_or(failed) && tid == kA4Warps * 32) {
+    for (uint32_t st = 0; st < (uint32_t)NS && st < issued; ++st) {
+      const uint32_t last = issued - 1 - ((issued - 1 - st) % NS);
+      a3_wait(&full[last % NS], (last / NS) & 1);
+    }
+    atomicOr(err, kErrTimeout);
+  }
+}
+
+size_t attn_mma_smem() {
+  return 1024 + (size_t)kA4Stages * 2 * kA4Chunk + (size_t)(2 * kA4QT * 64 + 3 * kA4QT) * 4 + 2 * kA4Stages * 8 + 16;
+}
+
+void launch_a4(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
+               int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
+               cudaStream_t s) {
+  CUtensorMap tk, tv;
+  memcpy(&tk, kv.tmaps, sizeof(tk));
+  memcpy(&tv, static_cast<const unsigned char*>(kv.tmaps) + 128, sizeof(tv));
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(B, qtiles_grid, H * splits);
+  cfg.blockDim = dim3(kA4Threads);
+  cfg.dynamicSmemBytes = attn_mma_smem();
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = splits;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++g_launches;
+  cudaLaunchKernelEx(&cfg, k_attn_mma, q, out, kv, rows, H, scale, err, tk, tv, stable, stable_stride,
+                     stable_extra);
+}
+
 template <typename TC, int HD>
 void launch_cl(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
                int qtiles_grid, int splits, int* err, const int* stable, int stable_stride,
@@ -982,7 +1353,34 @@ size_t attention_scratch_floats(int B, int H, int hd) {
 }
 size_t attention_counters(int B, int H) { return (size_t)B * kQTMax * H; }
 
+// Tensor maps (K, V) of a bf16 cache layer viewed as [rows][64]: 64-dim x 64-key boxes, 128-byte swizzle.
+int make_kv_tmaps(void* out, const void* k, const void* v, long long rows) {
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  if (!encode) {
+    cudaDriverEntryPointQueryResult qr;
+    void* fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &qr) !=
+            cudaSuccess ||
+        qr != cudaDriverEntryPointSuccess || !fn)
+      return LCA_E_CUDA;
+    encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  const cuuint64_t dims[2] = {64, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {128};
+  const cuuint32_t box[2] = {64, (cuuint32_t)kA4Keys};
+  const cuuint32_t estr[2] = {1, 1};
+  for (int i = 0; i < 2; ++i) {
+    const CUresult r = encode(reinterpret_cast<CUtensorMap*>(static_cast<unsigned char*>(out) + 128 * i),
+                              CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(i ? v : k), dims, strides, box,
+                              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return LCA_E_CUDA;
+  }
+  return LCA_OK;
+}
+
 void kernel_attrs_attn() {
+  cudaFuncSetAttribute(k_attn_mma, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem());
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)attn3_smem<__nv_bfloat16, 64>());
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -999,6 +1397,11 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
   if (splits > kMaxClusterSplit) splits = kMaxClusterSplit;
   if (splits < 1) splits = 1;
   const int ss = (int)(sizeof(SeqState) / sizeof(int));
+  // the tensor-core kernel pays a larger fixed cost per CTA: it needs many (sequence, head) pairs
+  if (D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= 128) {
+    launch_a4(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+    return;
+  }
   if (D.attn_pipe) {
     if (D.dtype == LCA_BF16) {
       if (D.hd == 64) launch_a3<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);

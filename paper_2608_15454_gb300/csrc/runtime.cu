@@ -188,6 +188,7 @@ struct alignas(64) SplitMapBlob {
 struct lca_ctx {
   std::map<const void*, TMapBlob> tmaps;  // TMA tensor maps of the bf16 weights
   std::map<int, SplitMapBlob> amaps;      // TMA tensor maps of the split activations, by K
+  std::map<const void*, SplitMapBlob> kvmaps;  // TMA tensor maps (K, V) of the bf16 cache layers
   lca_config cfg{};
   Layout L;
   Staging stg{};
@@ -779,11 +780,11 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     const char* um = getenv("LCA_NO_UMMA");
     D.use_umma = (um && um[0] == '1') ? 0 : 1;
     const char* sc = getenv("LCA_ATTN_SPLIT_CAP");
-    D.attn_split_cap = sc ? std::max(1, std::min(8, atoi(sc))) : 4;
+    D.attn_split_cap = sc ? std::max(1, std::min(8, atoi(sc))) : 8;
     const char* tr = getenv("LCA_TILED_MIN_ROWS");
     D.tiled_min_rows = tr ? std::max(0, atoi(tr)) : 64;
     const char* ap = getenv("LCA_ATTN_PIPE");
-    D.attn_pipe = ap ? (ap[0] == '1') : 1;
+    D.attn_pipe = ap ? atoi(ap) : 2;
   }
   // state and counters start at zero
   if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);
@@ -808,6 +809,16 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
       SplitMapBlob blob;
       if (make_split_tmaps(blob.b, D.as_hi, D.as_lo, D.as_rows, K) == LCA_OK) c->amaps[K] = blob;
     }
+    if (D.hd == 64)
+      for (auto* v : {&c->L.enc, &c->L.lm, &c->L.nb, &c->L.mb})
+        for (auto& bk : *v) {
+          SplitMapBlob blob;
+          const long long rows = (long long)D.B * D.H * bk.kv.S;
+          if (make_kv_tmaps(blob.b, bk.kv.k, bk.kv.v, rows) == LCA_OK) {
+            c->kvmaps[bk.kv.k] = blob;
+            bk.kv.tmaps = c->kvmaps[bk.kv.k].b;
+          }
+        }
   }
   launch_rope_table(D, cfg->rope_base, c->stream);
   if (check(cudaGetLastError(), "rope") || check(cudaStreamSynchronize(c->stream), "create sync"))
