@@ -179,18 +179,17 @@ int lca_debug_profile(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, i
 int lca_debug_trace(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t steps,
                     void* out, int32_t cap, int32_t* count);
 
-/* The tensor-core linear layer alone: y[0:*M_dev] = x . W^T on tcgen05, with x split into two
- * bf16 halves (x = hi + lo) so that about 16 bits of each activation enter the product, fp32
- * accumulation. x: device fp32 [M][K]; W: device bf16 [N][K]; y: device fp32 [M][N]; M_dev:
- * device int32 rows to compute (<= M); rows_typ: the row count the launch shape is chosen for
- * (0 = M; a smaller value makes CTAs walk several row passes); err_dev: device int32 error word
- * (bit 4: a bounded wait ran out); scratch: device, lca_debug_gemm_scratch_bytes(M, K) bytes, or
- * NULL. N and K must be multiples of 64. Asynchronous on `stream`. */
+/* The tensor-core linear layer alone: y[0:*M_dev] = x . W^T on tcgen05 (two launches: rows split
+ * into bf16 halves x = hi + lo, so that about 16 bits of each activation enter the product, then
+ * a GEMM fed entirely by TMA; fp32 accumulation). x: device fp32 [M][K]; W: device bf16 [N][K];
+ * y: device fp32 [M][N]; M_dev: device int32 rows to compute (<= M); rows_typ: the row count the
+ * launch shape is chosen for (0 = M; a smaller value makes CTAs walk several row tiles); err_dev:
+ * device int32 error word (bit 4: a bounded wait ran out); scratch: device,
+ * lca_debug_gemm_scratch_bytes(M, K) bytes (the split rows). N and K must be multiples of 64.
+ * Asynchronous on `stream`. */
 int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N, int32_t K,
                    const int32_t* M_dev, int32_t rows_typ, int32_t* err_dev, void* scratch, void* stream);
-/* Bytes of device scratch lca_debug_gemm needs to take the split-rows path (rows split once into
- * bf16 halves by one kernel, then a GEMM fed entirely by TMA); with scratch == NULL it converts
- * the activations inside the GEMM instead. */
+/* Bytes of device scratch lca_debug_gemm needs. */
 size_t lca_debug_gemm_scratch_bytes(int32_t M, int32_t K);
 
 /* Micro-benchmark: one graph of `iters` back-to-back launches of one kernel kind over `rows`

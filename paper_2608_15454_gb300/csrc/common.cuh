@@ -335,8 +335,8 @@ struct LinearArgs {
   size_t pf_bytes[2];
   int rows_typ;  // typical row count (sizes the activation staging); 0: M_cap
   const void* tmap;  // host copy of the weight's TMA tensor map (tensor-core path), or nullptr
-  // host copies of the TMA tensor maps of the split activations (hi, lo) for this Kd, or nullptr:
-  // then the tensor-core path converts the activations inside the GEMM
+  // host copies of the TMA tensor maps of the split activations (hi, lo) for this Kd, or nullptr
+  // (then the layer runs on the CUDA cores)
   const void* amap;
 };
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s);

@@ -21,7 +21,7 @@ __device__ __forceinline__ void err_or(int* e, int bits) { atomicOr(e, bits); }
 // steps stay valid while the window start is unchanged: their keys/values are kept in the
 // MB cache (slot = position - window start) and only new committed rows plus the copies are
 // computed. A changed window start (a committed boundary) rebuilds the cache.
-__global__ void k_mb_plan(Dev D) {
+__global__ void k_mb_plan(Dev D, int fill) {
   TraceScope _trace(TT_MB_PLAN);
   pdl_trigger();
   pdl_wait();
@@ -83,6 +83,7 @@ __global__ void k_mb_plan(Dev D) {
       D.head_rows_mb[b * (n - 1) + j] = cnt > 0 ? st0 + cnt - (n - 1) + j : 0;
   }
   __syncthreads();
+  if (!fill) return;  // many sequences: k_mb_fill writes the rows with a full grid
   // window rows: byte p of group k gets o_k + u_k (Algorithm 1, drafting input; residual r_2 added before
   // upsampling); copies beyond t belong to the current group K
   const int M = *D.r_mb.M;
@@ -834,15 +835,22 @@ void kernel_attrs_step() {
 thread_local long long g_launches = 0;
 thread_local ProfHook* g_prof = nullptr;
 
+// One CTA plans the windows; with few sequences it also writes the window rows (one launch less
+// on the latency-bound path), with many the rows are written by k_mb_fill over the whole GPU.
+void launch_mb_fill(const Dev& D, cudaStream_t s);
 void launch_mb_plan(const Dev& D, cudaStream_t s) {
-  ++g_launches;
-  ProfScope ps(PK_GLUE, 0.0, s);
-  launch_pdl(k_mb_plan, dim3(1), dim3(1024), 0, s, D);
+  const int fill = D.B <= 4;
+  {
+    ++g_launches;
+    ProfScope ps(PK_GLUE, 0.0, s);
+    launch_pdl(k_mb_plan, dim3(1), dim3(1024), 0, s, D, fill);
+  }
+  if (!fill) launch_mb_fill(D, s);
 }
 void launch_mb_fill(const Dev& D, cudaStream_t s) {
   ++g_launches;
   ProfScope ps(PK_GLUE, 0.0, s);
-  launch_pdl(k_mb_fill, dim3(152 * 2), dim3(256), 0, s, D);
+  launch_pdl(k_mb_fill, dim3(D.num_sms * 2), dim3(256), 0, s, D);
 }
 void launch_mlp_plan(const Dev& D, cudaStream_t s) {
   ++g_launches;

@@ -105,7 +105,8 @@ void carve(const lca_config& c, char* base, Layout& L) {
   D.o_tab = cv.take<float>(B * Lt * d);
   D.y_last = cv.take<float>(B * d);
   D.kpos = cv.take<int>(B * S);
-  D.as_rows = (int)(B * NM);
+  // split activations of the tensor-core layers: any row set of the step or of prefill (bf16)
+  D.as_rows = c.dtype == LCA_BF16 ? (int)R : 0;
   D.as_hi = cv.take<__nv_bfloat16>((size_t)D.as_rows * std::max(d, F));
   D.as_lo = cv.take<__nv_bfloat16>((size_t)D.as_rows * std::max(d, F));
   D.as_inv = cv.take<float>(D.as_rows);
@@ -782,7 +783,7 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     const char* sc = getenv("LCA_ATTN_SPLIT_CAP");
     D.attn_split_cap = sc ? std::max(1, std::min(8, atoi(sc))) : 8;
     const char* tr = getenv("LCA_TILED_MIN_ROWS");
-    D.tiled_min_rows = tr ? std::max(0, atoi(tr)) : 64;
+    D.tiled_min_rows = tr ? std::max(0, atoi(tr)) : 16;
     const char* ap = getenv("LCA_ATTN_PIPE");
     D.attn_pipe = ap ? atoi(ap) : 2;
   }
@@ -806,6 +807,7 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
       for (int l = 0; l < D.n_mb; ++l)
         add((char*)D.mlp_w + (size_t)l * D.n_mlp_heads * D.d * D.d * 2, (long long)D.n_mlp_heads * D.d, D.d);
     for (int K : {D.d, D.F}) {
+      if (D.as_rows < 1) break;
       SplitMapBlob blob;
       if (make_split_tmaps(blob.b, D.as_hi, D.as_lo, D.as_rows, K) == LCA_OK) c->amaps[K] = blob;
     }

@@ -314,13 +314,16 @@ def debug_gemm(x, W, y, M_dev, err_dev, rows_typ=0, scratch=None, stream=None):
     """y[:M] = x[:M] . W^T on the tensor cores (tcgen05, activations split into two bf16 halves).
     x fp32 [M,K], W bf16 [N,K], y fp32 [M,N], M_dev int32 [1] (rows actually used), err_dev
     int32 [1]; rows_typ: row count the launch shape is chosen for (0 = M); scratch: a uint8
-    device tensor of debug_gemm_scratch_bytes(M, K) bytes selects the split-rows + TMA path.
+    device tensor of debug_gemm_scratch_bytes(M, K) bytes (allocated here when None).
     Returns the status."""
     import torch
     st = stream if stream is not None else torch.cuda.current_stream(x.device)
+    if scratch is None:
+        scratch = torch.empty(debug_gemm_scratch_bytes(x.shape[0], W.shape[1]), dtype=torch.uint8,
+                              device=x.device)
     return load_library().lca_debug_gemm(x.data_ptr(), W.data_ptr(), y.data_ptr(), x.shape[0], W.shape[0],
                                          W.shape[1], M_dev.data_ptr(), rows_typ, err_dev.data_ptr(),
-                                         scratch.data_ptr() if scratch is not None else None,
+                                         scratch.data_ptr(),
                                          st.cuda_stream)
 
 

@@ -100,8 +100,9 @@ _GAINS_PATH = os.path.join(os.path.dirname(__file__), "gains.json")
 
 
 def load_gains() -> dict:
-    """Unembedding gains g (W_u <- g * W_u) chosen on the oracle so that about half
-    of the drafted bytes pass tau = 0.75. Written by ``oracle/calibrate_gain.py``."""
+    """Unembedding gains chosen on the oracle: g (W_u <- g * W_u) so that about half of the
+    drafted bytes pass tau = 0.75, and s (the boundary byte's row of W_u times s) so that
+    generated text holds spaces at the prompts' rate. Written by ``oracle/calibrate_gain.py``."""
     if not os.path.exists(_GAINS_PATH):
         return {}
     with open(_GAINS_PATH) as f:
@@ -109,9 +110,17 @@ def load_gains() -> dict:
 
 
 def gain_for(workload: Workload, calibrated: bool) -> float:
+    return weight_gains(workload, calibrated)["gain"]
+
+
+def weight_gains(workload: Workload, calibrated: bool) -> dict:
+    """Keyword arguments of make_weights for a workload: {"gain": g, "space_gain": s}, both 1
+    for the literal random-init weights."""
     if not calibrated:
-        return 1.0
+        return {"gain": 1.0, "space_gain": 1.0}
     g = load_gains().get(workload.gain_key)
     if g is None:
         raise KeyError(f"no calibrated gain for {workload.gain_key!r}; run oracle/calibrate_gain.py")
-    return float(g["gain"] if isinstance(g, dict) else g)
+    if not isinstance(g, dict):
+        return {"gain": float(g), "space_gain": 1.0}
+    return {"gain": float(g["gain"]), "space_gain": float(g.get("space_gain", 1.0))}

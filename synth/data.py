@@ -139,9 +139,10 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
     return ((u + bias) & np.uint32(0xFFFF0000)).view(np.float32)
 
 
-def make_weights(cfg: ModelConfig, gain: float = 1.0, seed: int = 0) -> dict:
+def make_weights(cfg: ModelConfig, gain: float = 1.0, seed: int = 0, space_gain: float = 1.0) -> dict:
     """name -> float32 array. For dtype "bf16" every value is bf16-representable.
-    ``gain`` multiplies the unembedding before rounding (acceptance calibration)."""
+    ``gain`` multiplies the unembedding before rounding (acceptance calibration);
+    ``space_gain`` multiplies its row of the boundary byte first (boundary-rate calibration)."""
     rng = np.random.default_rng(seed)
     out = {}
     for name, shape in tensor_list(cfg):
@@ -150,6 +151,8 @@ def make_weights(cfg: ModelConfig, gain: float = 1.0, seed: int = 0) -> dict:
         else:
             a = rng.standard_normal(shape, dtype=np.float32)
             a *= np.float32(INIT_STD)
+        if name == "unembed" and space_gain != 1.0:
+            a[cfg.boundary_byte] *= np.float32(space_gain)
         if name == "unembed" and gain != 1.0:
             a = (a * np.float32(gain)).astype(np.float32)
         if cfg.dtype == "bf16" and not is_norm(name):
@@ -159,8 +162,8 @@ def make_weights(cfg: ModelConfig, gain: float = 1.0, seed: int = 0) -> dict:
 
 
 @functools.lru_cache(maxsize=4)
-def cached_weights(cfg: ModelConfig, gain: float = 1.0, seed: int = 0) -> dict:
-    return make_weights(cfg, gain, seed)
+def cached_weights(cfg: ModelConfig, gain: float = 1.0, seed: int = 0, space_gain: float = 1.0) -> dict:
+    return make_weights(cfg, gain, seed, space_gain)
 
 
 def param_count(cfg: ModelConfig) -> int:

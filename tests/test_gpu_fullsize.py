@@ -15,7 +15,7 @@ import pytest
 
 import bench
 from oracle import THRESH, IncrementalDecoder, Model
-from synth import WORKLOADS, cached_weights, gain_for, prompts
+from synth import WORKLOADS, cached_weights, prompts, weight_gains
 from synth.configs import load_gains
 
 pytestmark = pytest.mark.gpu
@@ -67,8 +67,9 @@ def next_byte_margin(rec):
 def test_full_size_sampled_sequences(lca, name):
     w = WORKLOADS[name]
     n, tau = w.n_list[0], w.tau_list[0]
-    gain = gain_for(w, calibrated=w.gain_key in load_gains())
-    W = cached_weights(w.model, gain)
+    wg = weight_gains(w, calibrated=w.gain_key in load_gains())
+    gain = wg["gain"]
+    W = cached_weights(w.model, **wg)
     P = prompts(w, seqs=list(range(w.batch)))
     max_bytes = bench.context_bytes(w, n, bench.DEFAULT_STEPS, bench.DEFAULT_WARMUP,
                                     bench.DEFAULT_PROFILE_STEPS)
