@@ -10,6 +10,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cstring>
+#include <algorithm>
 #include <mutex>
 
 #include "common.cuh"
@@ -516,6 +517,7 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
 // query row for the online softmax (fp32), a pair of head dims per thread for P.V with the
 // probabilities broadcast from shared memory. Key splits of one (sequence, head) form a
 // thread-block cluster and combine (max, sum, accumulator) through distributed shared memory.
+constexpr int kA4MaxSplit = 16;  // largest key split (non-portable cluster size)
 constexpr int kA3Threads = 128;
 constexpr int kA3Keys = 64;     // keys per chunk
 constexpr int kA3Stages = 4;
@@ -776,9 +778,9 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
       const int nd = min(dpr, HD - d0);
       for (int idx = tid; idx < nq * nd; idx += kA3Threads) {
         const int i = idx / nd, dd = d0 + (idx - i * nd);
-        float mr[kMaxClusterSplit], lr[kMaxClusterSplit], ar[kMaxClusterSplit];
+        float mr[kA4MaxSplit], lr[kA4MaxSplit], ar[kA4MaxSplit];
 #pragma unroll
-        for (int k = 0; k < kMaxClusterSplit; ++k) {
+        for (int k = 0; k < kA4MaxSplit; ++k) {
           if (k < splits) {
             mr[k] = *cl.map_shared_rank(&s_m[i], k);
             lr[k] = *cl.map_shared_rank(&s_l[i], k);
@@ -787,11 +789,11 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
         }
         float M = -INFINITY;
 #pragma unroll
-        for (int k = 0; k < kMaxClusterSplit; ++k)
+        for (int k = 0; k < kA4MaxSplit; ++k)
           if (k < splits) M = fmaxf(M, mr[k]);
         float L = 0.f, o = 0.f;
 #pragma unroll
-        for (int k = 0; k < kMaxClusterSplit; ++k) {
+        for (int k = 0; k < kA4MaxSplit; ++k) {
           if (k < splits && mr[k] != -INFINITY) {
             const float w = expf(mr[k] - M);
             L += w * lr[k];
@@ -857,7 +859,6 @@ constexpr int kA4Warps = 4;
 constexpr int kA4Threads = (kA4Warps + 1) * 32;  // + the producer warp
 constexpr int kA4QT = 16;
 constexpr int kA4Keys = 64;
-constexpr int kA4Stages = 8;
 constexpr uint32_t kA4Chunk = kA4Keys * 64 * 2;  // one K or V chunk: 8 KB
 
 __device__ __forceinline__ void a4_tma(void* dst, const CUtensorMap* m, int x, int y, uint64_t* bar) {
@@ -895,12 +896,13 @@ __device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_
 // byte offset of 16-byte chunk c of row j in a [64][128 B] tile with the 128-byte swizzle
 __device__ __forceinline__ uint32_t swz(int j, int c) { return (uint32_t)(j * 128 + ((c ^ (j & 7)) << 4)); }
 
+template <int NS>
 __global__ void __launch_bounds__(kA4Threads, 1)
 k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
            const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
            const int* __restrict__ stable, int stable_stride, int stable_extra) {
   namespace cgr = cooperative_groups;
-  constexpr int HD = 64, QT = kA4QT, KC = kA4Keys, NS = kA4Stages;
+  constexpr int HD = 64, QT = kA4QT, KC = kA4Keys;
   extern __shared__ __align__(1024) unsigned char a4raw[];
   unsigned char* ring =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(a4raw) + 1023) & ~uintptr_t(1023));
@@ -1144,9 +1146,9 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       const int nd = min(dpr, HD - d0);
       for (int idx = tid; idx < nq * nd; idx += kA4Threads) {
         const int i = idx / nd, dd = d0 + (idx - i * nd);
-        float mr[kMaxClusterSplit], lr[kMaxClusterSplit], ar[kMaxClusterSplit];
+        float mr[kA4MaxSplit], lr[kA4MaxSplit], ar[kA4MaxSplit];
 #pragma unroll
-        for (int k = 0; k < kMaxClusterSplit; ++k) {
+        for (int k = 0; k < kA4MaxSplit; ++k) {
           if (k < splits) {
             mr[k] = *cl.map_shared_rank(&s_m[i], k);
             lr[k] = *cl.map_shared_rank(&s_l[i], k);
@@ -1155,11 +1157,11 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
         }
         float M = -INFINITY;
 #pragma unroll
-        for (int k = 0; k < kMaxClusterSplit; ++k)
+        for (int k = 0; k < kA4MaxSplit; ++k)
           if (k < splits) M = fmaxf(M, mr[k]);
         float L = 0.f, o = 0.f;
 #pragma unroll
-        for (int k = 0; k < kMaxClusterSplit; ++k) {
+        for (int k = 0; k < kA4MaxSplit; ++k) {
           if (k < splits && mr[k] != -INFINITY) {
             const float w = expf(mr[k] - M);
             L += w * lr[k];
@@ -1183,8 +1185,9 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   }
 }
 
+template <int NS>
 size_t attn_mma_smem() {
-  return 1024 + (size_t)kA4Stages * 2 * kA4Chunk + (size_t)(2 * kA4QT * 64 + 3 * kA4QT) * 4 + 2 * kA4Stages * 8 + 16;
+  return 1024 + (size_t)NS * 2 * kA4Chunk + (size_t)(2 * kA4QT * 64 + 3 * kA4QT) * 4 + 2 * NS * 8 + 16;
 }
 
 void launch_a4(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
@@ -1196,7 +1199,7 @@ void launch_a4(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA4Threads);
-  cfg.dynamicSmemBytes = attn_mma_smem();
+  cfg.dynamicSmemBytes = attn_mma_smem<8>();
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -1208,7 +1211,7 @@ void launch_a4(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn_mma, q, out, kv, rows, H, scale, err, tk, tv, stable, stable_stride,
+  cudaLaunchKernelEx(&cfg, k_attn_mma<8>, q, out, kv, rows, H, scale, err, tk, tv, stable, stable_stride,
                      stable_extra);
 }
 
@@ -1380,7 +1383,12 @@ int make_kv_tmaps(void* out, const void* k, const void* v, long long rows) {
 }
 
 void kernel_attrs_attn() {
-  cudaFuncSetAttribute(k_attn_mma, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem());
+  cudaFuncSetAttribute(k_attn_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem<8>());
+  cudaFuncSetAttribute(k_attn_mma<8>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(k_attn3<float, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(k_attn3<float, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)attn3_smem<__nv_bfloat16, 64>());
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1394,15 +1402,17 @@ void kernel_attrs_attn() {
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s, const int* stable, int stable_extra) {
   ProfScope ps(PK_ATTN, 0.0, s);
-  if (splits > kMaxClusterSplit) splits = kMaxClusterSplit;
   if (splits < 1) splits = 1;
   const int ss = (int)(sizeof(SeqState) / sizeof(int));
-  // the tensor-core kernel pays a larger fixed cost per CTA: it needs many (sequence, head) pairs
+  // the tensor-core kernel holds one CTA per SM: it pays off with many (sequence, head) pairs;
+  // with few, the CUDA-core pipelined kernel (three CTAs per SM) spreads keys over up to 16 splits
   if (D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= 128) {
-    launch_a4(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+    launch_a4(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, std::min(splits, kA4MaxSplit), D.err, stable, ss,
+              stable_extra, s);
     return;
   }
   if (D.attn_pipe) {
+    splits = std::min(splits, kA4MaxSplit);
     if (D.dtype == LCA_BF16) {
       if (D.hd == 64) launch_a3<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
       else launch_a3<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
@@ -1412,6 +1422,7 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
     }
     return;
   }
+  if (splits > kMaxClusterSplit) splits = kMaxClusterSplit;
   if (D.dtype == LCA_BF16) {
     if (D.hd == 64) launch_cl<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
     else launch_cl<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);

@@ -355,6 +355,9 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       (reinterpret_cast<uintptr_t>(rs + MCA) + 15) & ~uintptr_t(15));
   uint64_t* bar = reinterpret_cast<uint64_t*>(
       (reinterpret_cast<uintptr_t>(cpart + MCA * CT) + 15) & ~uintptr_t(15));
+  uint64_t* rbar = bar + 1;                                              // reduction arrivals (rank 0)
+  float* rbuf = reinterpret_cast<float*>(bar + 2);                       // [kMaxKSplit][MCA][CT] (rank 0)
+  float* rsq = rbuf + kMaxKSplit * MCA * CT;                             // [kMaxKSplit][MCA] (rank 0)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int tile = blockIdx.x;
@@ -376,6 +379,15 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
     if (NORM) bulk_g2s(gs, a.norm + k0, (uint32_t)(Kr * 4), bar);
   }
   prefetch_next(a);
+  if (ksplit > 1) {
+    // rank 0's reduction barrier exists before any peer can arrive on it (before the dependency
+    // wait, so this cluster barrier stays off the critical path)
+    if (tid == 0 && split == 0) {
+      mbar_init(rbar, (uint32_t)(ksplit - 1));
+      fence_mbar_init();
+    }
+    cgr::this_cluster().sync();
+  }
   pdl_trigger();
   pdl_wait();
   _trace.waited();
@@ -506,7 +518,67 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
         cpart[ei * CT + col0 + ec] = v;
       }
     }
-    if (ksplit > 1) {
+    if (ksplit > 1 && M <= MCA) {
+      // a single row chunk: the peers push their partials into rank 0's shared memory and
+      // arrive on its barrier (release, cluster scope), then leave; rank 0 waits, adds the ranks
+      // in order and runs the epilogue. No cluster barrier on the critical path.
+      cgr::cluster_group cl = cgr::this_cluster();
+      __syncthreads();  // this CTA's partials and row sums are complete
+      if (split != 0) {
+        float* dst = cl.map_shared_rank(rbuf, 0) + split * MCA * CT;
+        for (int idx = tid; idx < mc * CT; idx += NT) dst[idx] = cpart[idx];
+        if (NORM && tid < mc) cl.map_shared_rank(rsq, 0)[split * MCA + tid] = rs[tid];
+        __syncthreads();
+        if (tid == 0) {
+          uint32_t remote;
+          asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(rbar)), "r"(0));
+          asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+        }
+      } else {
+        EpiPre pp[2];
+        int np = 0;
+        for (int idx = tid; idx < mc * (CT / 2) && np < 2; idx += NT, ++np) {
+          const int i = idx / (CT / 2), c = (idx - i * (CT / 2)) * 2;
+          if (c < ncols) pp[np] = epi_load(a.epi, rbase + r0 + i, tile * CT + c);
+        }
+        if (tid == 0) {
+          bool ok = false;
+          for (int it = 0; it < kWaitSpins && !ok; ++it) {
+            uint32_t done;
+            asm volatile(
+                "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], 0;\n"
+                " selp.u32 %0, 1, 0, p;\n}"
+                : "=r"(done)
+                : "r"(smem_u32(rbar))
+                : "memory");
+            ok = done != 0;
+          }
+          if (!ok) atomicOr(a.epi.err, kErrTimeout);
+        }
+        __syncthreads();
+        int j = 0;
+        for (int idx = tid; idx < mc * (CT / 2); idx += NT, ++j) {
+          const int i = idx / (CT / 2), c = (idx - i * (CT / 2)) * 2;
+          if (c >= ncols) continue;
+          float t0 = cpart[i * CT + c], t1 = cpart[i * CT + c + 1], sq = NORM ? rs[i] : 0.f;
+#pragma unroll
+          for (int sp = 1; sp < kMaxKSplit; ++sp) {
+            if (sp < ksplit) {
+              t0 += rbuf[(sp * MCA + i) * CT + c];
+              t1 += rbuf[(sp * MCA + i) * CT + c + 1];
+              if (NORM) sq += rsq[sp * MCA + i];
+            }
+          }
+          if (NORM) {
+            const float sc = rsqrtf(sq / (float)a.Kd + a.eps);
+            t0 *= sc;
+            t1 *= sc;
+          }
+          const EpiPre q = j < 2 ? pp[j] : epi_load(a.epi, rbase + r0 + i, tile * CT + c);
+          epi_store<__nv_bfloat16>(a.epi, q, rbase + r0 + i, tile * CT + c, t0, t1);
+        }
+      }
+    } else if (ksplit > 1) {
       // cluster reduction of the K-split partials of this row chunk
       cgr::cluster_group cl = cgr::this_cluster();
       EpiPre pp[2];
@@ -674,8 +746,9 @@ template <int MCA, int NW, bool NORM>
 void gemv_bulk_go(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s) {
   constexpr int CT = NW * kCPW;
   const int Kr = a.Kd / ksplit;
-  const size_t smem =
-      (size_t)CT * Kr * 2 + (size_t)Kr * 4 + (size_t)MCA * Kr * 4 + (NW * MCA + MCA + MCA * CT) * 4 + 16 + 16 + 64;
+  const size_t smem = (size_t)CT * Kr * 2 + (size_t)Kr * 4 + (size_t)MCA * Kr * 4 +
+                      (NW * MCA + MCA + MCA * CT) * 4 + 16 + 16 + 16 +
+                      (size_t)kMaxKSplit * MCA * (CT + 1) * 4 + 64;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((a.N + CT - 1) / CT, ksplit, a.groups);
   cfg.blockDim = dim3(NW * 32);

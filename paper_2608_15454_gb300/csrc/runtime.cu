@@ -276,7 +276,7 @@ const void* tmap_of(lca_ctx* c, const void* W) {
 }
 
 int attn_splits(const Dev& D, int batch_cap, int qtiles) {
-  int s = (2 * 152) / std::max(1, batch_cap * D.H * qtiles);
+  int s = (2 * D.num_sms) / std::max(1, batch_cap * D.H * qtiles);
   return std::max(1, std::min(std::min(s, kMaxAttnSplit), D.attn_split_cap));
 }
 
@@ -781,7 +781,7 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     const char* um = getenv("LCA_NO_UMMA");
     D.use_umma = (um && um[0] == '1') ? 0 : 1;
     const char* sc = getenv("LCA_ATTN_SPLIT_CAP");
-    D.attn_split_cap = sc ? std::max(1, std::min(8, atoi(sc))) : 8;
+    D.attn_split_cap = sc ? std::max(1, std::min(16, atoi(sc))) : 16;
     const char* tr = getenv("LCA_TILED_MIN_ROWS");
     D.tiled_min_rows = tr ? std::max(0, atoi(tr)) : 16;
     const char* ap = getenv("LCA_ATTN_PIPE");
