@@ -189,6 +189,11 @@ int lca_debug_trace(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int
  * Asynchronous on `stream`. */
 int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N, int32_t K,
                    const int32_t* M_dev, int32_t rows_typ, int32_t* err_dev, void* scratch, void* stream);
+/* Where the tensor-core decode attention last gave up a bounded wait (16 int32 to host `out16`;
+ * out16[0] == 0: none since the last call): {set, block x, y, z, warp, which (0: waiting for a
+ * ring slot, 1: waiting for a chunk), chunk, stage, chunks, key lo, key hi, chunks before the
+ * tile, copies issued}. Clears the record. */
+int lca_debug_attn_diag(int32_t* out16);
 /* Bytes of device scratch lca_debug_gemm needs. */
 size_t lca_debug_gemm_scratch_bytes(int32_t M, int32_t K);
 

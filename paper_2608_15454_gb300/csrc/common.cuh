@@ -112,6 +112,9 @@ constexpr int kAttnQT = 8;        // query rows per attention tile (decode)
 constexpr int kErrIndex = 1;   // an index was out of range; the access was skipped
 constexpr int kErrNumeric = 2; // non-finite logits
 constexpr int kErrTimeout = 4; // a bounded wait ran out
+// which kernel family's wait ran out (set together with kErrTimeout; reported on stderr)
+constexpr int kErrWaitAttn3 = 1 << 8, kErrWaitAttnMma = 1 << 9, kErrWaitGemv = 1 << 10, kErrWaitGemm = 1 << 11,
+              kErrWaitGemvReduce = 1 << 12;
 
 // Linear epilogues.
 enum Epi : int {
@@ -232,6 +235,7 @@ struct Dev {
   int tiled_min_rows;  // layers with more typical rows than this run on the tensor cores
   int attn_pipe;       // decode attention: 2 = tensor cores (bf16, head_dim 64), 1 = bulk-copy pipelined
                        // CUDA-core kernel, 0 = register-tiled kernel
+  int attn_ns;         // ring stages of the tensor-core decode attention (4, 6 or 8)
   int use_umma;        // many-row bf16 layers run on the tensor cores (tcgen05)
 
   // weights (storage type; norms and bos fp32)
@@ -359,7 +363,7 @@ void kernel_attrs_attn();
 // change during a step, prefetched into L2 before the dependency wait; stable_extra: rows added.
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s, const int* stable = nullptr,
-               int stable_extra = 0);
+               int stable_extra = 0, bool short_kv = false);
 
 // Step / prefill glue kernels (kernels_step.cu).
 void launch_mb_plan(const Dev& D, cudaStream_t s);

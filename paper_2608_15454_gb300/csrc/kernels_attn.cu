@@ -812,7 +812,7 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
       const uint32_t last = issued - 1 - ((issued - 1 - st) % kA3Stages);
       a3_wait(&full[last % kA3Stages], (last / kA3Stages) & 1);
     }
-    atomicOr(err, kErrTimeout);
+    atomicOr(err, kErrTimeout | kErrWaitAttn3);
   }
 }
 
@@ -850,7 +850,7 @@ void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B
 // bf16 caches with head_dim 64. One CTA serves (sequence, query tile of up to 16 rows, head, key
 // split): a producer warp streams 64-key chunks of K and V by TMA (128-byte swizzle) through a
 // ring of shared-memory stages, and four compute warps each take every fourth chunk with their
-// own online softmax (no block barrier inside the key loop). Q.K^T and P.V run on the tensor cores
+// own online softmax (no block barrier inside the key loop). Two CTAs share an SM. Q.K^T and P.V run on the tensor cores
 // (mma.sync m16n8k16, bf16 operands, fp32 accumulation); K and V are exactly bf16, and Q and P
 // are each split into two bf16 halves (x = hi + lo) so that the products keep about 16 bits of
 // them. The warps then combine in shared memory, and the key splits of one (sequence, head)
@@ -896,18 +896,43 @@ __device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_
 // byte offset of 16-byte chunk c of row j in a [64][128 B] tile with the 128-byte swizzle
 __device__ __forceinline__ uint32_t swz(int j, int c) { return (uint32_t)(j * 128 + ((c ^ (j & 7)) << 4)); }
 
+// The first wait of k_attn_mma that runs out records where it gave up (read by
+// lca_debug_attn_diag): {set, block x, y, z, warp, which (0 ring slot free, 1 chunk landed),
+// chunk, stage, chunks, key lo, key hi, chunks before this tile, copies issued}.
+static __device__ int g_a4_diag[16];
+__device__ __noinline__ void a4_record(int which, uint32_t gi, int st, int nch, int lo, int hi, uint32_t cc,
+                                       uint32_t issued) {
+  if (atomicCAS(&g_a4_diag[0], 0, 1) != 0) return;
+  g_a4_diag[1] = blockIdx.x;
+  g_a4_diag[2] = blockIdx.y;
+  g_a4_diag[3] = blockIdx.z;
+  g_a4_diag[4] = threadIdx.x >> 5;
+  g_a4_diag[5] = which;
+  g_a4_diag[6] = (int)gi;
+  g_a4_diag[7] = st;
+  g_a4_diag[8] = nch;
+  g_a4_diag[9] = lo;
+  g_a4_diag[10] = hi;
+  g_a4_diag[11] = (int)cc;
+  g_a4_diag[12] = (int)issued;
+}
+
 template <int NS>
-__global__ void __launch_bounds__(kA4Threads, 1)
+__global__ void __maxnreg__(200)
 k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
            const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
            const int* __restrict__ stable, int stable_stride, int stable_extra) {
   namespace cgr = cooperative_groups;
   constexpr int HD = 64, QT = kA4QT, KC = kA4Keys;
+  // each stage must have one consumer warp, which takes its phases in order: a warp waiting on a
+  // stage that is still two phases behind would read the parity of the phase before as complete
+  static_assert(NS % kA4Warps == 0, "ring stages must be a multiple of the compute warps");
   extern __shared__ __align__(1024) unsigned char a4raw[];
   unsigned char* ring =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(a4raw) + 1023) & ~uintptr_t(1023));
-  float* qs = reinterpret_cast<float*>(ring + NS * 2 * kA4Chunk);  // [QT][HD], scaled
-  float* pacc = qs + QT * HD;                                       // [QT][HD]
+  unsigned char* qsh = ring + NS * 2 * kA4Chunk;                    // [QT][HD] bf16, swizzled: hi(q * scale)
+  unsigned char* qsl = qsh + QT * HD * 2;                           // the remainders
+  float* pacc = reinterpret_cast<float*>(qsl + QT * HD * 2);        // [QT][HD]
   float* s_m = pacc + QT * HD;                                      // [QT]
   float* s_l = s_m + QT;                                            // [QT]
   int* s_kv = reinterpret_cast<int*>(s_l + QT);                     // [QT]
@@ -963,9 +988,19 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
     const int r0 = rbeg + qt * QT;
     const int nq = min(QT, nrows - qt * QT);
-    for (int idx = tid; idx < QT * HD; idx += kA4Threads) {
-      const int i = idx / HD, dd = idx - i * HD;
-      qs[idx] = i < nq ? q[(size_t)(r0 + i) * ld + h * HD + dd] * scale : 0.f;
+    for (int idx = tid; idx < QT * HD / 2; idx += kA4Threads) {
+      const int i = idx / (HD / 2), dd = (idx - i * (HD / 2)) * 2;
+      float2 v = make_float2(0.f, 0.f);
+      if (i < nq) {
+        v = *reinterpret_cast<const float2*>(q + (size_t)(r0 + i) * ld + h * HD + dd);
+        v.x *= scale;
+        v.y *= scale;
+      }
+      uint32_t hi2, lo2;
+      split2(v.x, v.y, hi2, lo2);
+      const uint32_t off = swz(i, dd >> 3) + (dd & 7) * 2;
+      *reinterpret_cast<uint32_t*>(qsh + off) = hi2;
+      *reinterpret_cast<uint32_t*>(qsl + off) = lo2;
     }
     if (tid < QT) {
       int kl = tid < nq ? rows.kvlen[r0 + tid] : 0;
@@ -995,7 +1030,10 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
         for (int c = 0; c < nch; ++c) {
           const uint32_t gi = cc + c;
           const int st = gi % NS;
-          if (gi >= (uint32_t)NS && !failed && !a3_wait(&empty[st], ((gi / NS) - 1) & 1)) failed = true;
+          if (gi >= (uint32_t)NS && !failed && !a3_wait(&empty[st], ((gi / NS) - 1) & 1)) {
+            failed = true;
+            a4_record(0, gi, st, nch, lo, hi, cc, issued);
+          }
           if (failed) break;
           ++issued;
           unsigned char* dst = ring + (size_t)st * 2 * kA4Chunk;
@@ -1006,37 +1044,38 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       }
       __syncwarp();
     } else {
-      // Q fragments (rows g and g + 8, split into bf16 halves)
-      uint32_t qh[4][4], ql[4][4];
-#pragma unroll
-      for (int ks = 0; ks < 4; ++ks) {
-        const int c0 = 16 * ks + 2 * t;
-        split2(qs[g * HD + c0], qs[g * HD + c0 + 1], qh[ks][0], ql[ks][0]);
-        split2(qs[(g + 8) * HD + c0], qs[(g + 8) * HD + c0 + 1], qh[ks][1], ql[ks][1]);
-        split2(qs[g * HD + c0 + 8], qs[g * HD + c0 + 9], qh[ks][2], ql[ks][2]);
-        split2(qs[(g + 8) * HD + c0 + 8], qs[(g + 8) * HD + c0 + 9], qh[ks][3], ql[ks][3]);
-      }
+      const uint32_t qhb = a3_su32(qsh), qlb = a3_su32(qsl);
       const int kl0 = min(s_kv[g], hi), kl1 = min(s_kv[g + 8], hi);
       for (int c = warp; c < nch; c += kA4Warps) {
         const uint32_t gi = cc + c;
         const int st = gi % NS;
-        if (!failed && !a3_wait(&full[st], (gi / NS) & 1)) failed = true;
+        if (!failed && !a3_wait(&full[st], (gi / NS) & 1)) {
+          failed = true;
+          a4_record(1, gi, st, nch, lo, hi, cc, 0);
+        }
         const uint32_t kb = a3_su32(ring + (size_t)st * 2 * kA4Chunk), vb = kb + kA4Chunk;
         const int j0 = lo + c * KC;
         // S = Q K^T over 64 keys: n-tile nt = keys 8 nt .. 8 nt + 7
         float sacc[8][4];
 #pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-          sacc[nt][0] = sacc[nt][1] = sacc[nt][2] = sacc[nt][3] = 0.f;
+        for (int nt = 0; nt < 8; ++nt) sacc[nt][0] = sacc[nt][1] = sacc[nt][2] = sacc[nt][3] = 0.f;
 #pragma unroll
-          for (int kp = 0; kp < 2; ++kp) {
+        for (int kp = 0; kp < 2; ++kp) {
+          // Q fragments of dims 32 kp .. 32 kp + 31 (rows lane & 15, dims chunk 4 kp + 2 j + (lane >> 4))
+          uint32_t qh0[4], ql0[4], qh1[4], ql1[4];
+          ldsm4(qhb + swz(lane & 15, 4 * kp + (lane >> 4)), qh0);
+          ldsm4(qlb + swz(lane & 15, 4 * kp + (lane >> 4)), ql0);
+          ldsm4(qhb + swz(lane & 15, 4 * kp + 2 + (lane >> 4)), qh1);
+          ldsm4(qlb + swz(lane & 15, 4 * kp + 2 + (lane >> 4)), ql1);
+#pragma unroll
+          for (int nt = 0; nt < 8; ++nt) {
             uint32_t bf[4];
             // matrices: keys 8 nt + (lane & 7), dims chunks 4 kp + (lane >> 3)
             ldsm4(kb + swz(8 * nt + (lane & 7), 4 * kp + (lane >> 3)), bf);
-            mma16816(sacc[nt], qh[2 * kp], bf[0], bf[1]);
-            mma16816(sacc[nt], ql[2 * kp], bf[0], bf[1]);
-            mma16816(sacc[nt], qh[2 * kp + 1], bf[2], bf[3]);
-            mma16816(sacc[nt], ql[2 * kp + 1], bf[2], bf[3]);
+            mma16816(sacc[nt], qh0, bf[0], bf[1]);
+            mma16816(sacc[nt], ql0, bf[0], bf[1]);
+            mma16816(sacc[nt], qh1, bf[2], bf[3]);
+            mma16816(sacc[nt], ql1, bf[2], bf[3]);
           }
         }
         // mask, online softmax (rows g, g + 8; the four lanes of a quad share a row)
@@ -1146,9 +1185,9 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       const int nd = min(dpr, HD - d0);
       for (int idx = tid; idx < nq * nd; idx += kA4Threads) {
         const int i = idx / nd, dd = d0 + (idx - i * nd);
-        float mr[kA4MaxSplit], lr[kA4MaxSplit], ar[kA4MaxSplit];
+        float mr[kMaxClusterSplit], lr[kMaxClusterSplit], ar[kMaxClusterSplit];
 #pragma unroll
-        for (int k = 0; k < kA4MaxSplit; ++k) {
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
           if (k < splits) {
             mr[k] = *cl.map_shared_rank(&s_m[i], k);
             lr[k] = *cl.map_shared_rank(&s_l[i], k);
@@ -1157,11 +1196,11 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
         }
         float M = -INFINITY;
 #pragma unroll
-        for (int k = 0; k < kA4MaxSplit; ++k)
+        for (int k = 0; k < kMaxClusterSplit; ++k)
           if (k < splits) M = fmaxf(M, mr[k]);
         float L = 0.f, o = 0.f;
 #pragma unroll
-        for (int k = 0; k < kA4MaxSplit; ++k) {
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
           if (k < splits && mr[k] != -INFINITY) {
             const float w = expf(mr[k] - M);
             L += w * lr[k];
@@ -1181,25 +1220,27 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       const uint32_t last = issued - 1 - ((issued - 1 - st) % NS);
       a3_wait(&full[last % NS], (last / NS) & 1);
     }
-    atomicOr(err, kErrTimeout);
+    atomicOr(err, kErrTimeout | kErrWaitAttnMma);
   }
 }
 
 template <int NS>
 size_t attn_mma_smem() {
+  // ring, q halves (2 x QT x 64 bf16), pacc (QT x 64 fp32), row stats, barriers
   return 1024 + (size_t)NS * 2 * kA4Chunk + (size_t)(2 * kA4QT * 64 + 3 * kA4QT) * 4 + 2 * NS * 8 + 16;
 }
 
-void launch_a4(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-               int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
-               cudaStream_t s) {
+template <int NS>
+void launch_a4_ns(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
+                  int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
+                  cudaStream_t s) {
   CUtensorMap tk, tv;
   memcpy(&tk, kv.tmaps, sizeof(tk));
   memcpy(&tv, static_cast<const unsigned char*>(kv.tmaps) + 128, sizeof(tv));
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA4Threads);
-  cfg.dynamicSmemBytes = attn_mma_smem<8>();
+  cfg.dynamicSmemBytes = attn_mma_smem<NS>();
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -1211,8 +1252,15 @@ void launch_a4(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn_mma<8>, q, out, kv, rows, H, scale, err, tk, tv, stable, stable_stride,
+  cudaLaunchKernelEx(&cfg, k_attn_mma<NS>, q, out, kv, rows, H, scale, err, tk, tv, stable, stable_stride,
                      stable_extra);
+}
+
+void launch_a4(int ns, const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
+               int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
+               cudaStream_t s) {
+  if (ns == 4) launch_a4_ns<4>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, err, stable, stable_stride, stable_extra, s);
+  else launch_a4_ns<8>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, err, stable, stable_stride, stable_extra, s);
 }
 
 template <typename TC, int HD>
@@ -1383,8 +1431,8 @@ int make_kv_tmaps(void* out, const void* k, const void* v, long long rows) {
 }
 
 void kernel_attrs_attn() {
+  cudaFuncSetAttribute(k_attn_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem<4>());
   cudaFuncSetAttribute(k_attn_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem<8>());
-  cudaFuncSetAttribute(k_attn_mma<8>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<float, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -1400,15 +1448,17 @@ void kernel_attrs_attn() {
 }
 
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
-               int qtiles_grid, int splits, cudaStream_t s, const int* stable, int stable_extra) {
+               int qtiles_grid, int splits, cudaStream_t s, const int* stable, int stable_extra,
+               bool short_kv) {
   ProfScope ps(PK_ATTN, 0.0, s);
   if (splits < 1) splits = 1;
   const int ss = (int)(sizeof(SeqState) / sizeof(int));
-  // the tensor-core kernel holds one CTA per SM: it pays off with many (sequence, head) pairs;
-  // with few, the CUDA-core pipelined kernel (three CTAs per SM) spreads keys over up to 16 splits
-  if (D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= 128) {
-    launch_a4(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, std::min(splits, kA4MaxSplit), D.err, stable, ss,
-              stable_extra, s);
+  // the tensor-core kernel holds two CTAs per SM: it pays off with many (sequence, head) pairs over
+  // long caches; with few pairs, or short caches (the multi-byte window), the CUDA-core pipelined
+  // kernel (three CTAs per SM) runs, spreading keys over up to 16 splits
+  if (D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= 128 && !short_kv) {
+    launch_a4(D.attn_ns, q, out, kv, rows, B, D.H, D.scale, qtiles_grid, std::min(splits, kMaxClusterSplit), D.err,
+              stable, ss, stable_extra, s);
     return;
   }
   if (D.attn_pipe) {
@@ -1437,6 +1487,14 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
 using namespace lca;
 
 extern "C" {
+
+int lca_debug_attn_diag(int32_t* out16) {
+  if (!out16) return LCA_E_ARG;
+  if (cudaMemcpyFromSymbol(out16, g_a4_diag, 16 * sizeof(int)) != cudaSuccess) return LCA_E_CUDA;
+  const int zero[16] = {0};
+  cudaMemcpyToSymbol(g_a4_diag, zero, sizeof(zero));
+  return LCA_OK;
+}
 
 int lca_decode_attention_scratch_bytes(int32_t batch, int32_t heads, int32_t head_dim,
                                        int32_t splits, size_t* out) {

@@ -425,7 +425,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       }
       if (NORM && !have_w) {
         const bool ok = mbar_wait(bar, 0);  // the gain slice travels with the weights
-        if (!ok) atomicOr(a.epi.err, kErrTimeout);
+        if (!ok) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
       }
 #pragma unroll
       for (int u = 0; u < UNR; ++u) {
@@ -458,7 +458,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       // the bounded wait for the weight tile; on a timeout the error is recorded and the
       // kernel runs on (no early exit, so cluster barriers stay matched)
       const bool ok = mbar_wait(bar, 0);
-      if (__syncthreads_or(!ok) && tid == 0) atomicOr(a.epi.err, kErrTimeout);
+      if (__syncthreads_or(!ok) && tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
       have_w = true;
     } else {
       __syncthreads();
@@ -553,7 +553,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
                 : "memory");
             ok = done != 0;
           }
-          if (!ok) atomicOr(a.epi.err, kErrTimeout);
+          if (!ok) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemvReduce);
         }
         __syncthreads();
         int j = 0;
@@ -621,7 +621,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
     }
   }
   if (!have_w) {  // no rows: still wait (bounded) for the copy before leaving
-    if (!mbar_wait(bar, 0) && tid == 0) atomicOr(a.epi.err, kErrTimeout);
+    if (!mbar_wait(bar, 0) && tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
   }
 }
 

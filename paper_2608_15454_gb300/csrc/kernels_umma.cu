@@ -305,9 +305,8 @@ k_split_rows(LinearArgs a, __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __rest
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nw = gridDim.x * (blockDim.x >> 5);
   const int K = a.Kd;
-  for (int rr = blockIdx.x * (blockDim.x >> 5) + warp; rr < a.groups * a.M_cap; rr += nw) {
-    const int grp = rr / a.M_cap, r = rr - grp * a.M_cap;
-    if (r >= M) continue;
+  for (int rr = blockIdx.x * (blockDim.x >> 5) + warp; rr < a.groups * M; rr += nw) {
+    const int grp = rr / M, r = rr - grp * M;
     const size_t row = (size_t)grp * a.Mg_stride + r;
     const float4* xr = reinterpret_cast<const float4*>(a.x + row * a.ldx);
     float ss = 0.f;
@@ -531,7 +530,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
       const uint32_t last = issued - 1 - ((issued - 1 - s) % C::kStages);
       ubar_wait(&full[last % C::kStages], (last / C::kStages) & 1);
     }
-    atomicOr(a.epi.err, kErrTimeout);
+    atomicOr(a.epi.err, kErrTimeout | kErrWaitGemm);
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
@@ -597,7 +596,8 @@ void split_gemm(const Dev& D, const LinearArgs& a, const void* amap, __nv_bfloat
                 float* inv, cudaStream_t s) {
   const int sms = D.num_sms > 0 ? D.num_sms : 148;
   {
-    const int need = a.groups * a.M_cap;
+    // a warp per row; the grid covers the typical rows and its warps walk any further ones
+    const int need = a.groups * (a.rows_typ > 0 ? std::min(a.rows_typ, a.M_cap) : a.M_cap);
     const int blocks = std::max(1, std::min((need + 7) / 8, 4 * sms));
     ++g_launches;
     if (a.norm) launch_pdl(k_split_rows<true>, dim3(blocks), dim3(256), 0, s, a, hi, lo, inv);

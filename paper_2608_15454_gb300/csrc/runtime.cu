@@ -283,7 +283,8 @@ int attn_splits(const Dev& D, int batch_cap, int qtiles) {
 // Run the pre-norm blocks of one module over rows [0, *rows.M) of x (in place).
 void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& rows, int M_cap,
                int M_typ, int qt_grid, int splits, cudaStream_t s, const void* next_w = nullptr,
-               size_t next_bytes = 0, const int* stable = nullptr, int stable_extra = 0) {
+               size_t next_bytes = 0, const int* stable = nullptr, int stable_extra = 0,
+               bool short_kv = false) {
   Dev& D = c->L.D;
   const bool tiled = tiled_for(D, M_typ);
   const size_t tb = tw_bytes(D.dtype);
@@ -326,7 +327,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.tmap = tmap_of(c, a.W);
     a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
     linear(D, a, tiled, s);
-    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra);
+    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra, short_kv);
     // x += Wo . attn
     a.x = D.att;
     a.W = bk.wo;
@@ -413,8 +414,10 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
     if (D.mb_kind == LCA_MB_LCA) {
       launch_mb_plan(D, s);
       const int typ = B * (2 * n - 2);  // typical window rows: new committed bytes + copies
+      // the window holds about two words of keys: a short cache
       run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2), s,
-                c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype));
+                c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype), nullptr, 0,
+                true);
     } else {
       launch_mlp_plan(D, s);
       run_mlp_heads(c, n, s);
@@ -607,6 +610,7 @@ int read_err(lca_ctx* c) {
     CK(cudaMemsetAsync(c->L.D.err, 0, sizeof(int), c->stream));
     CK(cudaStreamSynchronize(c->stream));
   }
+  if (e & ~7) fprintf(stderr, "lca: device error word 0x%x\n", e);
   if (e & kErrTimeout) return LCA_E_TIMEOUT;
   if (e & kErrNumeric) return LCA_E_NUMERIC;
   if (e & kErrIndex) return LCA_E_DEVICE_STATE;
@@ -786,6 +790,8 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.tiled_min_rows = tr ? std::max(0, atoi(tr)) : 16;
     const char* ap = getenv("LCA_ATTN_PIPE");
     D.attn_pipe = ap ? atoi(ap) : 2;
+    const char* an = getenv("LCA_ATTN_NS");
+    D.attn_ns = an ? atoi(an) : 8;
   }
   // state and counters start at zero
   if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);

@@ -28,7 +28,7 @@ EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "
            "lca_debug_set_eager", "lca_debug_profile", "lca_debug_bench_kernel", "lca_debug_trace",
            "lca_debug_logits",
            "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str",
-           "lca_debug_gemm", "lca_debug_gemm_scratch_bytes",
+           "lca_debug_gemm", "lca_debug_gemm_scratch_bytes", "lca_debug_attn_diag",
            "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
            "lca_decode_attention_noalloc_capacity")
 
@@ -109,6 +109,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_status_str": [ctypes.c_int],
         "lca_debug_gemm": [P, P, P, I32, I32, I32, P, I32, P, P, P],
         "lca_debug_gemm_scratch_bytes": [I32, I32],
+        "lca_debug_attn_diag": [P],
         "lca_decode_attention_scratch_bytes": [I32, I32, I32, I32, ctypes.POINTER(ctypes.c_size_t)],
         "lca_decode_attention": [P, P, P, P, I32, I32, I32, I32, I32, I32, P, F32, I32, P,
                                  ctypes.c_size_t, P],
