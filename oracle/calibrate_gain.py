@@ -60,9 +60,15 @@ def run(workload, n, tau, gain, space_gain, steps):
     return acc / (steps * (n - 1)), spaces / max(1, emitted)
 
 
+def _dist(v, target):
+    return abs(math.log(max(v, 1e-6) / target))
+
+
 def bisect(evaluate, lo, hi, target, iters, log):
     """Bisection on log x in [lo, hi] for evaluate(x) ~ target (evaluate increasing in x);
-    returns the x with the value closest to the target and that value."""
+    returns the x whose value is closest to the target in ratio, and that value. The space rate
+    of greedy text jumps between attractors (no spaces at all, or a word-like rhythm), so the
+    distance is |log(value / target)|: a rate of 0 is never the closest."""
     best = None
     a, b = math.log(lo), math.log(hi)
     for _ in range(iters):
@@ -70,7 +76,7 @@ def bisect(evaluate, lo, hi, target, iters, log):
         x = round(math.exp(mid), 4)
         v = evaluate(x)
         log(f"  x={x} -> {v:.3f}")
-        if best is None or abs(v - target) < abs(best[1] - target):
+        if best is None or _dist(v, target) < _dist(best[1], target):
             best = (x, v)
         if v < target:
             a = mid

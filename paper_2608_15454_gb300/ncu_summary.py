@@ -100,7 +100,7 @@ def summarise(launches, workload):
     ns = len(steps)
     lines = [f"Workload `{workload}`: {ns} complete eager decode steps, "
              f"{sum(b - a for a, b in steps) / ns:.1f} launches and {total / ns:.1f} us of summed device "
-             f"time per step (serialised, cold-cache launches under ncu: compare shares, not absolutes).",
+             f"time per step (launches serialised under ncu: compare shares, not absolutes).",
              "", "| kernel | launches/step | us/step | share |", "|---|---|---|---|"]
     for k, (c, t) in sorted(agg.items(), key=lambda x: -x[1][1]):
         lines.append(f"| `{k}` | {c / ns:.1f} | {t / ns:.1f} | {100 * t / total:.1f}% |")
