@@ -159,6 +159,18 @@ struct EpiArgs {
   const float2* rope; // [slots][hd/2] (cos, sin)
   int H, hd, d;
   int* err;
+  // Split on write, for a tensor-core consumer of this output (sp_hi == nullptr: none). Each output
+  // value v (after the residual add or the SwiGLU) is stored once more as bf16 halves of v * sg[c]
+  // (sg: the consumer's RMSNorm gain, nullptr: 1) at sp_hi / sp_lo[row * ldsp + c], and, when ss is
+  // set, the sum of v^2 over each 32-column block c / 32 at ss[row * ss_ld + c / 32] (the consumer's
+  // RMS). sp_only: the fp32 output is not written (the consumer is its only reader).
+  __nv_bfloat16* sp_hi;
+  __nv_bfloat16* sp_lo;
+  int ldsp;
+  const float* sg;
+  float* ss;
+  int ss_ld;
+  int sp_only;
 };
 
 // Per-sequence committed state.
@@ -254,11 +266,16 @@ struct Dev {
   float* o_tab;    // [B][L][d] LM outputs
   float* y_last;   // [B][d] next-byte hidden at t-1 (MLP head input)
   int* kpos;       // [B][S] K(p) of committed positions (prefill scratch)
-  // activations of a tensor-core layer split into two bf16 halves (x * g = hi + lo) and the rows'
-  // inverse RMS, written by k_split_rows and read by TMA in k_tgemm: [as_rows][up to F]
-  __nv_bfloat16* as_hi;
-  __nv_bfloat16* as_lo;
-  float* as_inv;
+  // activations of a tensor-core layer split into two bf16 halves (x * g = hi + lo), in two
+  // buffers that consecutive layers alternate between (a layer reads one while its epilogue
+  // writes the next layer's input into the other): [2][as_rows][up to F]; written by
+  // k_split_rows or by the producing layer's epilogue and read by TMA in k_tgemm. as_ss: sums of
+  // squares of the rows for the RMSNorm, [as_rows][as_ss_ld] (per 32-column block, or the whole
+  // row in slot 0)
+  __nv_bfloat16* as_hi[2];
+  __nv_bfloat16* as_lo[2];
+  float* as_ss;
+  int as_ss_ld;
   int as_rows;
 
   // rows
@@ -339,12 +356,17 @@ struct LinearArgs {
   size_t pf_bytes[2];
   int rows_typ;  // typical row count (sizes the activation staging); 0: M_cap
   const void* tmap;  // host copy of the weight's TMA tensor map (tensor-core path), or nullptr
-  // host copies of the TMA tensor maps of the split activations (hi, lo) for this Kd, or nullptr
-  // (then the layer runs on the CUDA cores)
+  // host copies of the TMA tensor maps of the split activations (hi, lo) of buffer abuf for this
+  // Kd, or nullptr (then the layer runs on the CUDA cores)
   const void* amap;
+  int abuf;      // split buffer (0 or 1) the tensor-core path reads
+  int presplit;  // the producing layer's epilogue already wrote the split input and its sums of
+                 // squares per 32-column block; otherwise k_split_rows runs first
 };
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s);
 bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s);
+// whether linear() runs this layer on the tensor cores when called with tiled = true
+bool umma_ready(const Dev& D, const LinearArgs& a);
 int make_weight_tmap(void* out, const void* W, long long rows, long long K);
 // TMA tensor maps (hi then lo, 128 bytes each) of split activations [rows][K] bf16, 64 x 128 boxes
 int make_split_tmaps(void* out, const void* hi, const void* lo, long long rows, long long K);

@@ -10,6 +10,8 @@
 //  * k_gemm: a persistent tiled FFMA GEMM for many rows (prefill, large batches).
 #include <cooperative_groups.h>
 
+#include <cstdio>
+
 #include "common.cuh"
 #include "epilogue.cuh"
 
@@ -856,6 +858,8 @@ void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s) {
   const bool norm = a.norm != nullptr;
   ProfScope ps(PK_LINEAR, (double)a.N * a.Kd * a.groups * (D.dtype == LCA_BF16 ? 2 : 4), s);
   if (tiled && D.use_umma && linear_umma(D, a, s)) return;
+  // a pre-split input exists only as bf16 halves: callers set presplit only where umma_ready holds
+  if (a.presplit) fprintf(stderr, "lca: pre-split layer input on the CUDA-core path (N %d, K %d)\n", a.N, a.Kd);
   if (D.dtype == LCA_BF16) {
     if (tiled) norm ? launch_gemm<__nv_bfloat16, true>(D, a, s) : launch_gemm<__nv_bfloat16, false>(D, a, s);
     else norm ? launch_gemv<__nv_bfloat16, true>(D, a, s) : launch_gemv<__nv_bfloat16, false>(D, a, s);

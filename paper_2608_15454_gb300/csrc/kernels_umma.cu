@@ -112,6 +112,33 @@ __device__ __forceinline__ uint32_t bf2(float a, float b) {
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
+// Split on write: bf16 halves of NV output values (times the consumer's RMSNorm gain, if any) at
+// columns [c0, c0 + NV) of row r, as 16-byte vectors.
+template <int NV>
+__device__ __forceinline__ void split_store(const EpiArgs& e, int r, int c0, const float (&y)[NV]) {
+  uint32_t h[NV / 2], l[NV / 2];
+#pragma unroll
+  for (int i = 0; i < NV / 4; ++i) {
+    const float4 g = e.sg ? reinterpret_cast<const float4*>(e.sg + c0)[i] : make_float4(1.f, 1.f, 1.f, 1.f);
+    uint16_t h0, h1, h2, h3, l0, l1, l2, l3;
+    split_bf16(y[4 * i] * g.x, h0, l0);
+    split_bf16(y[4 * i + 1] * g.y, h1, l1);
+    split_bf16(y[4 * i + 2] * g.z, h2, l2);
+    split_bf16(y[4 * i + 3] * g.w, h3, l3);
+    h[2 * i] = h0 | ((uint32_t)h1 << 16);
+    h[2 * i + 1] = h2 | ((uint32_t)h3 << 16);
+    l[2 * i] = l0 | ((uint32_t)l1 << 16);
+    l[2 * i + 1] = l2 | ((uint32_t)l3 << 16);
+  }
+  uint4* ph = reinterpret_cast<uint4*>(e.sp_hi + (size_t)r * e.ldsp + c0);
+  uint4* pl = reinterpret_cast<uint4*>(e.sp_lo + (size_t)r * e.ldsp + c0);
+#pragma unroll
+  for (int j = 0; j < NV / 8; ++j) {
+    ph[j] = make_uint4(h[4 * j], h[4 * j + 1], h[4 * j + 2], h[4 * j + 3]);
+    pl[j] = make_uint4(l[4 * j], l[4 * j + 1], l[4 * j + 2], l[4 * j + 3]);
+  }
+}
+
 // ---------------------------------------------------------------- epilogue of 32-column chunks
 // A thread owns one row of the tile and walks its columns in chunks of 32 (a chunk lies inside one
 // head and one of Q/K/V, since d and head_dim are multiples of 32). Operands of a chunk: 32 residual
@@ -145,28 +172,43 @@ __device__ __forceinline__ void chunk_out(const EpiArgs& e, const EpiRow& q, con
       for (int i = 0; i < 8; ++i) y[i] = make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]);
       break;
     }
-    case EPI_RESID: {
-      float4* y = reinterpret_cast<float4*>(e.y + (size_t)r * e.ldy + c0);
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-        y[i] = make_float4(op[i].x + x[4 * i], op[i].y + x[4 * i + 1], op[i].z + x[4 * i + 2], op[i].w + x[4 * i + 3]);
-      break;
-    }
+    case EPI_RESID:
     case EPI_RESID_SILU: {
-      float4* y = reinterpret_cast<float4*>(e.y + (size_t)r * e.ldy + c0);
+      const bool sl = e.mode == EPI_RESID_SILU;
 #pragma unroll
-      for (int i = 0; i < 8; ++i)
-        y[i] = make_float4(op[i].x + silu_f(x[4 * i]), op[i].y + silu_f(x[4 * i + 1]),
-                           op[i].z + silu_f(x[4 * i + 2]), op[i].w + silu_f(x[4 * i + 3]));
+      for (int i = 0; i < 8; ++i) {
+        x[4 * i] = op[i].x + (sl ? silu_f(x[4 * i]) : x[4 * i]);
+        x[4 * i + 1] = op[i].y + (sl ? silu_f(x[4 * i + 1]) : x[4 * i + 1]);
+        x[4 * i + 2] = op[i].z + (sl ? silu_f(x[4 * i + 2]) : x[4 * i + 2]);
+        x[4 * i + 3] = op[i].w + (sl ? silu_f(x[4 * i + 3]) : x[4 * i + 3]);
+      }
+      if (!e.sp_only) {
+        float4* y = reinterpret_cast<float4*>(e.y + (size_t)r * e.ldy + c0);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) y[i] = make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]);
+      }
+      if (e.sp_hi) {
+        split_store<32>(e, r, c0, x);
+        if (e.ss) {
+          float q2 = 0.f;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) q2 += x[i] * x[i];
+          e.ss[(size_t)r * e.ss_ld + (c0 >> 5)] = q2;
+        }
+      }
       break;
     }
     case EPI_SWIGLU: {
       // interleaved (gate, up) columns -> silu(gate) * up at column c / 2
-      float4* y = reinterpret_cast<float4*>(e.y + (size_t)r * e.ldy + (c0 >> 1));
+      float m[16];
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-        y[i] = make_float4(silu_f(x[8 * i]) * x[8 * i + 1], silu_f(x[8 * i + 2]) * x[8 * i + 3],
-                           silu_f(x[8 * i + 4]) * x[8 * i + 5], silu_f(x[8 * i + 6]) * x[8 * i + 7]);
+      for (int i = 0; i < 16; ++i) m[i] = silu_f(x[2 * i]) * x[2 * i + 1];
+      if (!e.sp_only) {
+        float4* y = reinterpret_cast<float4*>(e.y + (size_t)r * e.ldy + (c0 >> 1));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) y[i] = make_float4(m[4 * i], m[4 * i + 1], m[4 * i + 2], m[4 * i + 3]);
+      }
+      if (e.sp_hi) split_store<16>(e, r, c0 >> 1, m);
       break;
     }
     case EPI_QKV: {
@@ -214,18 +256,16 @@ __device__ __forceinline__ void chunk_out(const EpiArgs& e, const EpiRow& q, con
 }
 
 // Epilogue of one 128 x BN accumulator tile for an epilogue warp: thread = TMEM lane = tile row,
-// columns [n0, n0 + BN) of global row `grow`, scaled by *sc_ptr (or 1). The operands of a chunk are
-// loaded before the stores of the chunk before it, those of the first chunk before `wait()` (the
+// columns [n0, n0 + BN) of global row `grow`, scaled by sc. The operands of a chunk are loaded
+// before the stores of the chunk before it, those of the first chunk before `wait()` (the
 // accumulator's completion), so a row costs about one memory latency per two chunks.
 template <int BN, typename Wait>
 __device__ __forceinline__ void tile_epilogue(const EpiArgs& e, uint32_t tbase, int grow, bool ok, int n0,
-                                              const float* sc_ptr, Wait wait) {
+                                              float sc, Wait wait) {
   EpiRow q{0, 0, 0};
   float4 opA[8], opB[8];
-  float sc = 1.f;
   if (ok) {
     q = epi_row(e, grow);
-    if (sc_ptr) sc = *sc_ptr;
     chunk_ops(e, q, grow, n0, opA);
   }
   wait();
@@ -245,16 +285,44 @@ __device__ __forceinline__ void tile_epilogue(const EpiArgs& e, uint32_t tbase, 
   }
 }
 
+// Split on write of one output pair (c even) of the residual and SwiGLU epilogues; returns the
+// pair's contribution to the row's sum of squares (residual add only).
+__device__ __forceinline__ float pair_split(const EpiArgs& e, float2 op, int r, int c, float a0, float a1) {
+  if (e.mode == EPI_SWIGLU) {
+    const float m = silu_f(a0) * a1;
+    const int cm = c >> 1;
+    if (!e.sp_only) e.y[(size_t)r * e.ldy + cm] = m;
+    uint16_t h, l;
+    split_bf16(e.sg ? m * e.sg[cm] : m, h, l);
+    reinterpret_cast<uint16_t*>(e.sp_hi)[(size_t)r * e.ldsp + cm] = h;
+    reinterpret_cast<uint16_t*>(e.sp_lo)[(size_t)r * e.ldsp + cm] = l;
+    return 0.f;
+  }
+  const bool sl = e.mode == EPI_RESID_SILU;
+  const float v0 = op.x + (sl ? silu_f(a0) : a0), v1 = op.y + (sl ? silu_f(a1) : a1);
+  if (!e.sp_only) *reinterpret_cast<float2*>(e.y + (size_t)r * e.ldy + c) = make_float2(v0, v1);
+  const float2 g = e.sg ? *reinterpret_cast<const float2*>(e.sg + c) : make_float2(1.f, 1.f);
+  uint16_t h0, h1, l0, l1;
+  split_bf16(v0 * g.x, h0, l0);
+  split_bf16(v1 * g.y, h1, l1);
+  *reinterpret_cast<uint32_t*>(e.sp_hi + (size_t)r * e.ldsp + c) = h0 | ((uint32_t)h1 << 16);
+  *reinterpret_cast<uint32_t*>(e.sp_lo + (size_t)r * e.ldsp + c) = l0 | ((uint32_t)l1 << 16);
+  return v0 * v0 + v1 * v1;
+}
+
 // Cluster split-K: rank `ks` adds rows [ks * 128 / KS, ...) of the KS partial tiles (each
 // [128][BN + 1] in its CTA's shared memory) and applies the pair epilogue, four items per batch
-// with all loads of a batch before its stores.
+// with all loads of a batch before its stores. inv_s: the tile rows' inverse RMS (nullptr: 1).
+// The 32 lanes of a warp hold 32 consecutive pairs of one row (BN / 2 and the thread count are
+// multiples of 32), so a 32-column block's sum of squares is a reduction over 16 lanes.
 template <int BN, int NT>
 __device__ __forceinline__ void cluster_epilogue(const EpiArgs& e, cooperative_groups::cluster_group& cl,
                                                  float* red, int KS, int ks, int mrow0, int rbase, int M, int n0,
-                                                 const float* inv) {
+                                                 const float* inv_s) {
   const int RPC = kUM / KS;
   const int items = RPC * (BN / 2);
   constexpr int U = 4;
+  const int lane = threadIdx.x & 31;
   for (int base = threadIdx.x; base < items; base += U * NT) {
     float s0[U], s1[U], sc[U];
     float2 op[U];
@@ -280,14 +348,26 @@ __device__ __forceinline__ void cluster_epilogue(const EpiArgs& e, cooperative_g
             s1[u] += pr[1];
           }
         }
-        if (inv) sc[u] = inv[gr[u]];
+        if (inv_s) sc[u] = inv_s[rt];
         q[u] = epi_row(e, gr[u]);
         op[u] = epi_operand(e, q[u], gr[u], col[u]);
       }
     }
+    if (e.sp_hi) {
 #pragma unroll
-    for (int u = 0; u < U; ++u)
-      if (ok[u]) epi_out<__nv_bfloat16>(e, q[u], op[u], gr[u], col[u], s0[u] * sc[u], s1[u] * sc[u]);
+      for (int u = 0; u < U; ++u) {
+        float q2 = ok[u] ? pair_split(e, op[u], gr[u], col[u], s0[u] * sc[u], s1[u] * sc[u]) : 0.f;
+        if (e.ss) {  // ok[u] is the same across the warp
+#pragma unroll
+          for (int o = 8; o; o >>= 1) q2 += __shfl_xor_sync(0xffffffffu, q2, o);
+          if (ok[u] && (lane & 15) == 0) e.ss[(size_t)gr[u] * e.ss_ld + (col[u] >> 5)] = q2;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (ok[u]) epi_out<__nv_bfloat16>(e, q[u], op[u], gr[u], col[u], s0[u] * sc[u], s1[u] * sc[u]);
+    }
   }
 }
 
@@ -295,7 +375,7 @@ __device__ __forceinline__ void cluster_epilogue(const EpiArgs& e, cooperative_g
 template <bool NORM>
 __global__ void __launch_bounds__(256)
 k_split_rows(LinearArgs a, __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo,
-             float* __restrict__ inv) {
+             float* __restrict__ ss, int ss_ld) {
   TraceScope _trace(TT_UMMA);
   pdl_trigger();
   pdl_wait();
@@ -309,28 +389,48 @@ k_split_rows(LinearArgs a, __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __rest
     const int grp = rr / M, r = rr - grp * M;
     const size_t row = (size_t)grp * a.Mg_stride + r;
     const float4* xr = reinterpret_cast<const float4*>(a.x + row * a.ldx);
-    float ss = 0.f;
-    for (int k4 = lane; k4 < K / 4; k4 += 32) {
-      float4 v = xr[k4];
-      if (NORM) {
-        ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-        const float4 g = reinterpret_cast<const float4*>(a.norm)[k4];
-        v.x *= g.x; v.y *= g.y; v.z *= g.z; v.w *= g.w;
+    float sq = 0.f;
+    // four 16-byte loads per lane in flight before the first conversion
+    for (int k0 = 0; k0 < K / 4; k0 += 128) {
+      float4 v[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int k4 = k0 + j * 32 + lane;
+        v[j] = k4 < K / 4 ? xr[k4] : make_float4(0.f, 0.f, 0.f, 0.f);
       }
-      uint16_t h0, h1, h2, h3, l0, l1, l2, l3;
-      split_bf16(v.x, h0, l0);
-      split_bf16(v.y, h1, l1);
-      split_bf16(v.z, h2, l2);
-      split_bf16(v.w, h3, l3);
-      reinterpret_cast<uint2*>(hi + row * K)[k4] = make_uint2(h0 | ((uint32_t)h1 << 16), h2 | ((uint32_t)h3 << 16));
-      reinterpret_cast<uint2*>(lo + row * K)[k4] = make_uint2(l0 | ((uint32_t)l1 << 16), l2 | ((uint32_t)l3 << 16));
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int k4 = k0 + j * 32 + lane;
+        if (k4 >= K / 4) continue;
+        float4 w = v[j];
+        if (NORM) {
+          sq += w.x * w.x + w.y * w.y + w.z * w.z + w.w * w.w;
+          const float4 g = reinterpret_cast<const float4*>(a.norm)[k4];
+          w.x *= g.x; w.y *= g.y; w.z *= g.z; w.w *= g.w;
+        }
+        uint16_t h0, h1, h2, h3, l0, l1, l2, l3;
+        split_bf16(w.x, h0, l0);
+        split_bf16(w.y, h1, l1);
+        split_bf16(w.z, h2, l2);
+        split_bf16(w.w, h3, l3);
+        reinterpret_cast<uint2*>(hi + row * K)[k4] = make_uint2(h0 | ((uint32_t)h1 << 16), h2 | ((uint32_t)h3 << 16));
+        reinterpret_cast<uint2*>(lo + row * K)[k4] = make_uint2(l0 | ((uint32_t)l1 << 16), l2 | ((uint32_t)l3 << 16));
+      }
     }
     if (NORM) {
 #pragma unroll
-      for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-      if (lane == 0) inv[row] = rsqrtf(ss / (float)K + a.eps);
+      for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+      if (lane == 0) ss[row * ss_ld] = sq;
     }
   }
+}
+
+// Inverse RMS of a row from its sums of squares (n slots, summed in order).
+__device__ __forceinline__ float row_inv(const float* ss, int n, int ld, size_t row, int K, float eps) {
+  const float* p = ss + row * ld;
+  float t = 0.f;
+  for (int i = 0; i < n; ++i) t += p[i];
+  return rsqrtf(t / (float)K + eps);
 }
 
 // ---------------------------------------------------------------- TMA-fed tensor-core GEMM
@@ -344,7 +444,8 @@ struct TCfg {
   // D fp32, A and B bf16, both K-major, M = 128, N = BN
   static constexpr uint32_t kIDesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                                      ((uint32_t)(kUM >> 4) << 24);
-  static constexpr size_t kSmem = (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16 + 1024;
+  // ring, barriers, TMEM address, the tile rows' inverse RMS, alignment slack
+  static constexpr size_t kSmem = (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16 + kUM * 4 + 1024;
   static_assert((size_t)kUM * (BN + 1) * 4 <= (size_t)kStages * kStageBytes, "reduction buffer");
 };
 
@@ -360,7 +461,8 @@ __device__ __forceinline__ void tmma(uint32_t tmem_d, uint64_t a, uint64_t b, ui
 template <int BN>
 __global__ void __launch_bounds__(kTThreads, 1)
 k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmAh,
-        const __grid_constant__ CUtensorMap tmAl, const float* __restrict__ inv, int MT, int KS) {
+        const __grid_constant__ CUtensorMap tmAl, const float* __restrict__ ss, int ss_n, int ss_ld, int MT,
+        int KS) {
   using C = TCfg<BN>;
   namespace cgr = cooperative_groups;
   TraceScope _trace(TT_UMMA);
@@ -371,6 +473,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
   uint64_t* empty = full + C::kStages;
   uint64_t* accdone = empty + C::kStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accdone + 1);
+  float* inv_s = reinterpret_cast<float*>(accdone + 1) + 4;  // [128]
   float* red = reinterpret_cast<float*>(ring);  // [128][BN + 1] after the MMAs of a pass
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -490,12 +593,14 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
     __syncwarp();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     if (live) {
+      // the row's inverse RMS, read while the main loop runs
+      float sc = 1.f;
+      if (warp >= 2 && a.norm && mt * kUM + r < M) sc = row_inv(ss, ss_n, ss_ld, rbase + mt * kUM + r, a.Kd, a.eps);
       if (KS == 1) {
         if (warp >= 2) {
           const int row = mt * kUM + r;
           // the accumulator wait sits inside, after the first chunk's operand loads
-          tile_epilogue<BN>(a.epi, tmem + ((uint32_t)((warp & 3) * 32) << 16), rbase + row, row < M, n0,
-                            a.norm ? inv + rbase + row : nullptr, [&] {
+          tile_epilogue<BN>(a.epi, tmem + ((uint32_t)((warp & 3) * 32) << 16), rbase + row, row < M, n0, sc, [&] {
                               wait_or_fail(accdone, ps & 1, failed);
                               asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                             });
@@ -503,6 +608,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
       } else {
         cgr::cluster_group cl = cgr::this_cluster();
         if (warp >= 2) {
+          inv_s[r] = sc;
 #pragma unroll
           for (int cb = 0; cb < BN; cb += 32) {
             uint32_t v[32];
@@ -512,8 +618,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
           }
         }
         cl.sync();
-        cluster_epilogue<BN, kTThreads>(a.epi, cl, red, KS, ks, mt * kUM, rbase, M, n0,
-                                        a.norm ? inv : nullptr);
+        cluster_epilogue<BN, kTThreads>(a.epi, cl, red, KS, ks, mt * kUM, rbase, M, n0, a.norm ? inv_s : nullptr);
         cl.sync();
       }
     }
@@ -540,7 +645,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
 
 template <int BN>
 void tgemm_go(const LinearArgs& a, const CUtensorMap& tw, const CUtensorMap& th, const CUtensorMap& tl,
-              const float* inv, int MT, int KS, cudaStream_t s) {
+              const float* ss, int ss_n, int ss_ld, int MT, int KS, cudaStream_t s) {
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(a.N / BN, KS, a.groups * MT);
   cfg.blockDim = dim3(kTThreads);
@@ -556,7 +661,7 @@ void tgemm_go(const LinearArgs& a, const CUtensorMap& tw, const CUtensorMap& th,
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_tgemm<BN>, a, tw, th, tl, inv, MT, KS);
+  cudaLaunchKernelEx(&cfg, k_tgemm<BN>, a, tw, th, tl, ss, ss_n, ss_ld, MT, KS);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
@@ -588,20 +693,23 @@ int encode_bf16_2d(void* out, const void* base, long long rows, long long K, int
 
 }  // namespace
 
-// Split rows, then the TMA-fed GEMM. The grid covers the typical row count (rows_typ). Tile width
+// Split rows (unless the producing layer's epilogue already did), then the TMA-fed GEMM. The rows'
+// sums of squares (for the RMSNorm) sit in ss[row * ss_ld + i]: one slot from k_split_rows, Kd / 32
+// per-block slots from a producing epilogue. The grid covers the typical row count (rows_typ). Tile width
 // BN (256, 128 or 64, dividing N) and K split KS (power of two, at most 8, at least two 64-deep
 // blocks per CTA, while the grid fits one wave) minimise a simple cost: waves x (BN x K blocks
 // per CTA + a fixed part) + a cluster-reduction term proportional to BN; ties go to the wider tile.
 void split_gemm(const Dev& D, const LinearArgs& a, const void* amap, __nv_bfloat16* hi, __nv_bfloat16* lo,
-                float* inv, cudaStream_t s) {
+                float* ss, int ss_ld, cudaStream_t s) {
   const int sms = D.num_sms > 0 ? D.num_sms : 148;
-  {
+  const int ss_n = a.presplit ? a.Kd / 32 : 1;
+  if (!a.presplit) {
     // a warp per row; the grid covers the typical rows and its warps walk any further ones
     const int need = a.groups * (a.rows_typ > 0 ? std::min(a.rows_typ, a.M_cap) : a.M_cap);
     const int blocks = std::max(1, std::min((need + 7) / 8, 4 * sms));
     ++g_launches;
-    if (a.norm) launch_pdl(k_split_rows<true>, dim3(blocks), dim3(256), 0, s, a, hi, lo, inv);
-    else launch_pdl(k_split_rows<false>, dim3(blocks), dim3(256), 0, s, a, hi, lo, inv);
+    if (a.norm) launch_pdl(k_split_rows<true>, dim3(blocks), dim3(256), 0, s, a, hi, lo, ss, ss_ld);
+    else launch_pdl(k_split_rows<false>, dim3(blocks), dim3(256), 0, s, a, hi, lo, ss, ss_ld);
   }
   const int mt_cap = (a.M_cap + kUM - 1) / kUM;
   const int rows_typ = a.rows_typ > 0 ? a.rows_typ : a.M_cap;
@@ -628,9 +736,9 @@ void split_gemm(const Dev& D, const LinearArgs& a, const void* amap, __nv_bfloat
   memcpy(&tw, a.tmap, sizeof(tw));
   memcpy(&th, amap, sizeof(th));
   memcpy(&tl, static_cast<const unsigned char*>(amap) + 128, sizeof(tl));
-  if (best_bn == 256) tgemm_go<256>(a, tw, th, tl, inv, MT, best_ks, s);
-  else if (best_bn == 128) tgemm_go<128>(a, tw, th, tl, inv, MT, best_ks, s);
-  else tgemm_go<64>(a, tw, th, tl, inv, MT, best_ks, s);
+  if (best_bn == 256) tgemm_go<256>(a, tw, th, tl, ss, ss_n, ss_ld, MT, best_ks, s);
+  else if (best_bn == 128) tgemm_go<128>(a, tw, th, tl, ss, ss_n, ss_ld, MT, best_ks, s);
+  else tgemm_go<64>(a, tw, th, tl, ss, ss_n, ss_ld, MT, best_ks, s);
 }
 
 // Tensor map of a bf16 weight [rows][K] (K innermost) with 64 x 64 boxes and the 128-byte swizzle.
@@ -652,12 +760,18 @@ void kernel_attrs_umma() {
   cudaFuncSetAttribute(k_tgemm<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TCfg<256>::kSmem);
 }
 
-// Launch on the tensor cores when the layer has a weight tensor map and split-activation maps
-// for its K, its rows fit the split buffers and it fits the tile shapes; false otherwise.
+// The tensor cores take a layer that has a weight tensor map and split-activation maps for its K,
+// whose rows fit the split buffers and whose shape fits the tiles.
+bool umma_ready(const Dev& D, const LinearArgs& a) {
+  if (!D.use_umma || !a.tmap || !a.amap || D.dtype != LCA_BF16 || a.N % kUN || a.Kd % kUK) return false;
+  if (a.abuf < 0 || a.abuf > 1 || (a.presplit && a.norm && a.Kd / 32 > D.as_ss_ld)) return false;
+  return (long long)a.groups * a.M_cap <= D.as_rows;
+}
+
+// Launch on the tensor cores if umma_ready; false otherwise.
 bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s) {
-  if (!a.tmap || !a.amap || D.dtype != LCA_BF16 || a.N % kUN || a.Kd % kUK) return false;
-  if ((long long)a.groups * a.M_cap > D.as_rows) return false;
-  split_gemm(D, a, a.amap, D.as_hi, D.as_lo, D.as_inv, s);
+  if (!umma_ready(D, a)) return false;
+  split_gemm(D, a, a.amap, D.as_hi[a.abuf], D.as_lo[a.abuf], D.as_ss, D.as_ss_ld, s);
   return true;
 }
 
@@ -669,7 +783,7 @@ using namespace lca;
 
 extern "C" size_t lca_debug_gemm_scratch_bytes(int32_t M, int32_t K) {
   if (M < 1 || K < 1) return 0;
-  return (size_t)M * K * 2 * 2 + (size_t)M * 4 + 512;
+  return (size_t)M * K * 2 * 2 + (size_t)M * 4 + 512;  // hi, lo, one sum-of-squares slot per row
 }
 
 extern "C" int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N, int32_t K,
@@ -706,10 +820,10 @@ extern "C" int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M
   char* p = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(scratch) + 255) & ~uintptr_t(255));
   __nv_bfloat16* hi = reinterpret_cast<__nv_bfloat16*>(p);
   __nv_bfloat16* lo = hi + (size_t)M * K;
-  float* inv = reinterpret_cast<float*>(lo + (size_t)M * K);
+  float* ss = reinterpret_cast<float*>(lo + (size_t)M * K);
   alignas(64) unsigned char maps[256];
   st = make_split_tmaps(maps, hi, lo, M, K);
   if (st != LCA_OK) return st;
-  split_gemm(D, a, maps, hi, lo, inv, reinterpret_cast<cudaStream_t>(stream));
+  split_gemm(D, a, maps, hi, lo, ss, 1, reinterpret_cast<cudaStream_t>(stream));
   return cudaGetLastError() == cudaSuccess ? LCA_OK : LCA_E_CUDA;
 }

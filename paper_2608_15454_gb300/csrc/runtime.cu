@@ -105,11 +105,15 @@ void carve(const lca_config& c, char* base, Layout& L) {
   D.o_tab = cv.take<float>(B * Lt * d);
   D.y_last = cv.take<float>(B * d);
   D.kpos = cv.take<int>(B * S);
-  // split activations of the tensor-core layers: any row set of the step or of prefill (bf16)
+  // split activations of the tensor-core layers (two alternating buffers) and the rows' sums of
+  // squares: any row set of the step or of prefill (bf16)
   D.as_rows = c.dtype == LCA_BF16 ? (int)R : 0;
-  D.as_hi = cv.take<__nv_bfloat16>((size_t)D.as_rows * std::max(d, F));
-  D.as_lo = cv.take<__nv_bfloat16>((size_t)D.as_rows * std::max(d, F));
-  D.as_inv = cv.take<float>(D.as_rows);
+  for (int i = 0; i < 2; ++i) {
+    D.as_hi[i] = cv.take<__nv_bfloat16>((size_t)D.as_rows * std::max(d, F));
+    D.as_lo[i] = cv.take<__nv_bfloat16>((size_t)D.as_rows * std::max(d, F));
+  }
+  D.as_ss_ld = (int)d / 32;
+  D.as_ss = cv.take<float>((size_t)D.as_rows * D.as_ss_ld);
 
   D.x_mb = cv.take<float>(R * d);
   D.x_enc = cv.take<float>(R * d);
@@ -188,7 +192,7 @@ struct alignas(64) SplitMapBlob {
 
 struct lca_ctx {
   std::map<const void*, TMapBlob> tmaps;  // TMA tensor maps of the bf16 weights
-  std::map<int, SplitMapBlob> amaps;      // TMA tensor maps of the split activations, by K
+  std::map<int, SplitMapBlob> amaps;      // TMA tensor maps of the split activations, by 2 K + buffer
   std::map<const void*, SplitMapBlob> kvmaps;  // TMA tensor maps (K, V) of the bf16 cache layers
   lca_config cfg{};
   Layout L;
@@ -263,10 +267,10 @@ int upload_params(lca_ctx* c) {
 
 bool tiled_for(const Dev& D, int rows) { return rows > D.tiled_min_rows; }
 
-// Split-activation maps for a layer of inner size K whose rows fit the split buffers.
-const void* amap_of(lca_ctx* c, int K, int rows_cap) {
+// Split-activation maps of buffer `buf` for a layer of inner size K whose rows fit the buffers.
+const void* amap_of(lca_ctx* c, int buf, int K, int rows_cap) {
   if (rows_cap > c->L.D.as_rows) return nullptr;
-  auto it = c->amaps.find(K);
+  auto it = c->amaps.find(2 * K + buf);
   return it == c->amaps.end() ? nullptr : it->second.b;
 }
 
@@ -280,7 +284,34 @@ int attn_splits(const Dev& D, int batch_cap, int qtiles) {
   return std::max(1, std::min(std::min(s, kMaxAttnSplit), D.attn_split_cap));
 }
 
-// Run the pre-norm blocks of one module over rows [0, *rows.M) of x (in place).
+// Split on write: the epilogue of `prod` also stores its output as the bf16 halves (times `gain`, the
+// consumer's RMSNorm gain, or 1) that the tensor-core layer `cons` reads from split buffer `buf`,
+// plus per-32-column sums of squares when the consumer normalises. Only when both layers run on
+// the tensor cores; returns whether the link was made.
+bool link_split(const Dev& D, bool tiled, LinearArgs& prod, LinearArgs& cons, int buf, const float* gain,
+                bool drop_fp32) {
+  cons.abuf = buf;
+  cons.presplit = 1;
+  const bool ok = tiled && umma_ready(D, prod) && umma_ready(D, cons) && cons.groups == prod.groups &&
+                  cons.Mg_stride == prod.Mg_stride && prod.abuf != buf && (!gain || cons.Kd == prod.N);
+  if (!ok) {
+    cons.presplit = 0;
+    return false;
+  }
+  prod.epi.sp_hi = D.as_hi[buf];
+  prod.epi.sp_lo = D.as_lo[buf];
+  prod.epi.ldsp = cons.Kd;
+  prod.epi.sg = gain;
+  prod.epi.ss = gain ? D.as_ss : nullptr;
+  prod.epi.ss_ld = D.as_ss_ld;
+  prod.epi.sp_only = drop_fp32 ? 1 : 0;
+  return true;
+}
+
+// Run the pre-norm blocks of one module over rows [0, *rows.M) of x (in place). On the tensor
+// cores, each layer's input is split into bf16 halves by the layer before it (its epilogue writes
+// them into the other of the two split buffers); only a stack's first layer and the attention
+// output go through k_split_rows.
 void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& rows, int M_cap,
                int M_typ, int qt_grid, int splits, cudaStream_t s, const void* next_w = nullptr,
                size_t next_bytes = 0, const int* stable = nullptr, int stable_extra = 0,
@@ -290,26 +321,23 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
   const size_t tb = tw_bytes(D.dtype);
   const size_t b_qkv = 3ull * D.d * D.d * tb, b_o = (size_t)D.d * D.d * tb;
   const size_t b_13 = 2ull * D.F * D.d * tb, b_2 = (size_t)D.d * D.F * tb;
-  for (size_t l = 0; l < blocks.size(); ++l) {
-    Block& bk = blocks[l];
-    const Block* nx = l + 1 < blocks.size() ? &blocks[l + 1] : nullptr;
-    const void* nqkv = nx ? nx->wqkv : next_w;
-    const size_t nqkv_b = nx ? b_qkv : next_bytes;
-    LinearArgs a{};
-    a.groups = 1;
-    a.Mg_stride = 0;
-    a.eps = D.eps;
-    a.M = rows.M;
-    a.M_cap = M_cap;
-    a.rows_typ = M_typ;
-    // RMSNorm -> Q,K,V -> RoPE -> K,V appended to the cache
+  LinearArgs base{};
+  base.groups = 1;
+  base.Mg_stride = 0;
+  base.eps = D.eps;
+  base.M = rows.M;
+  base.M_cap = M_cap;
+  base.rows_typ = M_typ;
+  base.epi.err = D.err;
+  // the QKV layer of block l; split buffer 0
+  auto qkv_args = [&](const Block& bk) {
+    LinearArgs a = base;
     a.x = x;
     a.ldx = D.d;
     a.W = bk.wqkv;
     a.N = 3 * D.d;
     a.Kd = D.d;
     a.norm = bk.attn_norm;
-    a.epi = EpiArgs{};
     a.epi.mode = EPI_QKV;
     a.epi.y = D.qbuf;
     a.epi.ldy = D.d;
@@ -319,60 +347,79 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     a.epi.H = D.H;
     a.epi.hd = D.hd;
     a.epi.d = D.d;
-    a.epi.err = D.err;
     a.pf[0] = bk.wo;
     a.pf_bytes[0] = b_o;
     a.pf[1] = bk.w13;
     a.pf_bytes[1] = b_13;
     a.tmap = tmap_of(c, a.W);
-    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
-    linear(D, a, tiled, s);
+    a.abuf = 0;
+    a.amap = amap_of(c, 0, a.Kd, a.M_cap * a.groups);
+    return a;
+  };
+  LinearArgs aq = blocks.empty() ? base : qkv_args(blocks[0]);
+  for (size_t l = 0; l < blocks.size(); ++l) {
+    Block& bk = blocks[l];
+    const Block* nx = l + 1 < blocks.size() ? &blocks[l + 1] : nullptr;
+    const void* nqkv = nx ? nx->wqkv : next_w;
+    const size_t nqkv_b = nx ? b_qkv : next_bytes;
+    // x += Wo . attn (input split by k_split_rows into buffer 1)
+    LinearArgs ao = base;
+    ao.x = D.att;
+    ao.ldx = D.d;
+    ao.W = bk.wo;
+    ao.N = D.d;
+    ao.Kd = D.d;
+    ao.epi.mode = EPI_RESID;
+    ao.epi.y = x;
+    ao.epi.res = x;
+    ao.epi.ldy = ao.epi.ldres = D.d;
+    ao.pf[0] = bk.w2;
+    ao.pf_bytes[0] = b_2;
+    ao.tmap = tmap_of(c, ao.W);
+    ao.abuf = 1;
+    ao.amap = amap_of(c, 1, ao.Kd, ao.M_cap * ao.groups);
+    // mid = silu(W1 . n(x)) * (W3 . n(x)) (input in buffer 0)
+    LinearArgs a13 = base;
+    a13.x = x;
+    a13.ldx = D.d;
+    a13.W = bk.w13;
+    a13.N = 2 * D.F;
+    a13.Kd = D.d;
+    a13.norm = bk.mlp_norm;
+    a13.epi.mode = EPI_SWIGLU;
+    a13.epi.y = D.mid;
+    a13.epi.ldy = D.F;
+    a13.pf[0] = nqkv;
+    a13.pf_bytes[0] = nqkv_b;
+    a13.tmap = tmap_of(c, a13.W);
+    a13.amap = amap_of(c, 0, a13.Kd, a13.M_cap * a13.groups);
+    // x += W2 . mid (input in buffer 1)
+    LinearArgs a2 = base;
+    a2.x = D.mid;
+    a2.ldx = D.F;
+    a2.W = bk.w2;
+    a2.N = D.d;
+    a2.Kd = D.F;
+    a2.epi.mode = EPI_RESID;
+    a2.epi.y = x;
+    a2.epi.res = x;
+    a2.epi.ldy = a2.epi.ldres = D.d;
+    a2.pf[0] = nx ? nx->wo : nullptr;
+    a2.pf_bytes[0] = nx ? b_o : 0;
+    a2.tmap = tmap_of(c, a2.W);
+    a2.amap = amap_of(c, 1, a2.Kd, a2.M_cap * a2.groups);
+    LinearArgs aq_next = nx ? qkv_args(*nx) : base;
+    link_split(D, tiled, ao, a13, 0, bk.mlp_norm, false);
+    link_split(D, tiled, a13, a2, 1, nullptr, true);
+    if (nx) link_split(D, tiled, a2, aq_next, 0, nx->attn_norm, false);
+
+    // RMSNorm -> Q,K,V -> RoPE -> K,V appended to the cache
+    linear(D, aq, tiled, s);
     attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra, short_kv);
-    // x += Wo . attn
-    a.x = D.att;
-    a.W = bk.wo;
-    a.N = D.d;
-    a.norm = nullptr;
-    a.epi.mode = EPI_RESID;
-    a.epi.y = x;
-    a.epi.res = x;
-    a.epi.ldy = a.epi.ldres = D.d;
-    a.pf[0] = bk.w2;
-    a.pf_bytes[0] = b_2;
-    a.pf[1] = nullptr;
-    a.pf_bytes[1] = 0;
-    a.tmap = tmap_of(c, a.W);
-    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
-    linear(D, a, tiled, s);
-    // mid = silu(W1 . n(x)) * (W3 . n(x))
-    a.x = x;
-    a.W = bk.w13;
-    a.N = 2 * D.F;
-    a.norm = bk.mlp_norm;
-    a.epi.mode = EPI_SWIGLU;
-    a.epi.y = D.mid;
-    a.epi.ldy = D.F;
-    a.pf[0] = nqkv;
-    a.pf_bytes[0] = nqkv_b;
-    a.tmap = tmap_of(c, a.W);
-    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
-    linear(D, a, tiled, s);
-    // x += W2 . mid
-    a.x = D.mid;
-    a.ldx = D.F;
-    a.W = bk.w2;
-    a.N = D.d;
-    a.Kd = D.F;
-    a.norm = nullptr;
-    a.epi.mode = EPI_RESID;
-    a.epi.y = x;
-    a.epi.res = x;
-    a.epi.ldy = a.epi.ldres = D.d;
-    a.pf[0] = nx ? nx->wo : nullptr;
-    a.pf_bytes[0] = nx ? b_o : 0;
-    a.tmap = tmap_of(c, a.W);
-    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
-    linear(D, a, tiled, s);
+    linear(D, ao, tiled, s);
+    linear(D, a13, tiled, s);
+    linear(D, a2, tiled, s);
+    aq = aq_next;
   }
 }
 
@@ -380,7 +427,8 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
 void run_mlp_heads(lca_ctx* c, int n, cudaStream_t s) {
   Dev& D = c->L.D;
   const size_t tb = tw_bytes(D.dtype);
-  for (int l = 0; l < D.n_mb; ++l) {
+  const bool tiled = tiled_for(D, D.B);
+  auto layer = [&](int l) {
     LinearArgs a{};
     a.x = D.x_mb;
     a.ldx = D.d;
@@ -400,8 +448,17 @@ void run_mlp_heads(lca_ctx* c, int n, cudaStream_t s) {
     a.epi.ldy = a.epi.ldres = D.d;
     a.epi.err = D.err;
     a.tmap = tmap_of(c, a.W);
-    a.amap = amap_of(c, a.Kd, a.M_cap * a.groups);
-    linear(D, a, tiled_for(D, D.B), s);
+    a.abuf = l & 1;
+    a.amap = amap_of(c, a.abuf, a.Kd, a.M_cap * a.groups);
+    return a;
+  };
+  // layer l reads split buffer l % 2; its epilogue writes layer l + 1's input into the other one
+  LinearArgs a = layer(0);
+  for (int l = 0; l < D.n_mb; ++l) {
+    LinearArgs an = l + 1 < D.n_mb ? layer(l + 1) : LinearArgs{};
+    if (l + 1 < D.n_mb) link_split(D, tiled, a, an, (l + 1) & 1, nullptr, false);
+    linear(D, a, tiled, s);
+    a = an;
   }
 }
 
@@ -812,11 +869,12 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     if (D.mlp_w)
       for (int l = 0; l < D.n_mb; ++l)
         add((char*)D.mlp_w + (size_t)l * D.n_mlp_heads * D.d * D.d * 2, (long long)D.n_mlp_heads * D.d, D.d);
-    for (int K : {D.d, D.F}) {
-      if (D.as_rows < 1) break;
-      SplitMapBlob blob;
-      if (make_split_tmaps(blob.b, D.as_hi, D.as_lo, D.as_rows, K) == LCA_OK) c->amaps[K] = blob;
-    }
+    for (int K : {D.d, D.F})
+      for (int buf = 0; buf < 2 && D.as_rows > 0; ++buf) {
+        SplitMapBlob blob;
+        if (make_split_tmaps(blob.b, D.as_hi[buf], D.as_lo[buf], D.as_rows, K) == LCA_OK)
+          c->amaps[2 * K + buf] = blob;
+      }
     if (D.hd == 64)
       for (auto* v : {&c->L.enc, &c->L.lm, &c->L.nb, &c->L.mb})
         for (auto& bk : *v) {
