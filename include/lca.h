@@ -172,8 +172,8 @@ int lca_debug_profile(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, i
                       lca_profile* out);
 
 /* Run `steps` step graphs with launch tracing on: thread 0 of every CTA of every kernel records
- * {u64 start_ns, u64 end_ns, u64 wait_done_ns, i32 kernel tag, i32 cta, i32 sm, i32 mark_ns}
- * (40 bytes) into `out`
+ * {u64 start_ns, u64 end_ns, u64 wait_done_ns, i32 kernel tag, i32 cta, i32 sm, i32 mark_ns[3]}
+ * (48 bytes; a mark is a mid-kernel time after entry, 0 if the kernel sets none) into `out`
  * (host, room for `cap` records); count = records written. Needs a bf16 context (the trace
  * buffer borrows scratch that the bf16 step does not use). */
 int lca_debug_trace(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int32_t steps,
@@ -181,7 +181,10 @@ int lca_debug_trace(lca_ctx* ctx, int32_t n, float tau, int32_t accept_mode, int
 
 /* The tensor-core linear layer alone: y[0:*M_dev] = x . W^T on tcgen05 (two launches: rows split
  * into bf16 halves x = hi + lo, so that about 16 bits of each activation enter the product, then
- * a GEMM fed entirely by TMA; fp32 accumulation). x: device fp32 [M][K]; W: device bf16 [N][K];
+ * a GEMM fed entirely by TMA; fp32 accumulation). Up to 64 typical rows (and N a multiple of 128)
+ * the GEMM takes the weights as the MMA's M operand and splits K across a cluster (environment
+ * LCA_SGEMM_MAX_ROWS sets that limit, 0 turns it off); otherwise the activations are the M
+ * operand. x: device fp32 [M][K]; W: device bf16 [N][K];
  * y: device fp32 [M][N]; M_dev: device int32 rows to compute (<= M); rows_typ: the row count the
  * launch shape is chosen for (0 = M; a smaller value makes CTAs walk several row tiles); err_dev:
  * device int32 error word (bit 4: a bounded wait ran out); scratch: device,

@@ -38,12 +38,14 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 // The pointers are per translation unit (no relocatable device code); trace_set() fills them.
 struct TraceRec {
   unsigned long long t0, t1, tw;  // entry, exit, grid-dependency wait returned
-  int tag, cta, sm, mark;  // mark: optional mid-kernel time, ns after entry (0: none)
+  int tag, cta, sm;
+  int mark[3];  // optional mid-kernel times, ns after entry (0: none)
 };
+static_assert(sizeof(TraceRec) == 48, "trace record layout");
 enum TraceTag : int {
   TT_GEMV = 1, TT_GEMV_F32, TT_GEMM, TT_ROWSTATS, TT_ATTN, TT_HEAD, TT_MB_PLAN, TT_MB_FILL,
   TT_MLP_PLAN, TT_VERIFY_PLAN, TT_SEGMENT, TT_LM_SCATTER, TT_NB_INPUT, TT_COMMIT, TT_LOOP_CTL,
-  TT_OTHER, TT_UMMA
+  TT_OTHER, TT_UMMA, TT_SPLIT, TT_SGEMM
 };
 static __device__ TraceRec* g_trace = nullptr;
 static __device__ unsigned int* g_trace_n = nullptr;
@@ -61,9 +63,9 @@ __device__ __forceinline__ unsigned smid() {
 struct TraceScope {
   unsigned long long t0, tw;
   int tag;
-  unsigned mk;  // optional mid-kernel mark: nanoseconds after entry (0: none)
+  unsigned mk[3];  // optional mid-kernel marks: nanoseconds after entry (0: none)
   bool on;
-  __device__ __forceinline__ explicit TraceScope(int t) : t0(0), tw(0), tag(t), mk(0), on(false) {
+  __device__ __forceinline__ explicit TraceScope(int t) : t0(0), tw(0), tag(t), mk{0, 0, 0}, on(false) {
     if (threadIdx.x == 0 && threadIdx.y == 0 && g_trace) {
       on = true;
       t0 = gtimer();
@@ -73,8 +75,12 @@ struct TraceScope {
   __device__ __forceinline__ void waited() {
     if (on) tw = gtimer();
   }
-  __device__ __forceinline__ void mark() {
-    if (on) mk = (unsigned)(gtimer() - t0);
+  __device__ __forceinline__ void mark(int i = 0) {
+    if (on) mk[i] = (unsigned)(gtimer() - t0);
+  }
+  // a mark taken by another thread of the CTA (globaltimer value), handed over through shared memory
+  __device__ __forceinline__ void mark_at(int i, unsigned long long t) {
+    if (on && t > t0) mk[i] = (unsigned)(t - t0);
   }
   __device__ __forceinline__ ~TraceScope() {
     if (on) {
@@ -87,7 +93,9 @@ struct TraceScope {
         r.tag = tag;
         r.cta = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
         r.sm = (int)smid();
-        r.mark = (int)mk;
+        r.mark[0] = (int)mk[0];
+        r.mark[1] = (int)mk[1];
+        r.mark[2] = (int)mk[2];
         g_trace[i] = r;
       }
     }
@@ -248,6 +256,10 @@ struct Dev {
   int attn_pipe;       // decode attention: 2 = tensor cores (bf16, head_dim 64), 1 = bulk-copy pipelined
                        // CUDA-core kernel, 0 = register-tiled kernel
   int attn_ns;         // ring stages of the tensor-core decode attention (4, 6 or 8)
+  int sgemm_max_rows;  // tensor-core layers with at most this many typical rows use the skinny
+                       // (weights-as-M) GEMM; 0: never
+  int sgemm_max_ks;    // largest K split (cluster size) of the skinny GEMM (8, or 16 where the
+                       // GPU schedules 16-CTA clusters of it)
   int use_umma;        // many-row bf16 layers run on the tensor cores (tcgen05)
 
   // weights (storage type; norms and bos fp32)
@@ -368,11 +380,13 @@ bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s);
 // whether linear() runs this layer on the tensor cores when called with tiled = true
 bool umma_ready(const Dev& D, const LinearArgs& a);
 int make_weight_tmap(void* out, const void* W, long long rows, long long K);
-// TMA tensor maps (hi then lo, 128 bytes each) of split activations [rows][K] bf16, 64 x 128 boxes
+// TMA tensor maps of split activations [rows][K] bf16, 128 bytes each, K boxes of 64: (hi, lo) with
+// 128-row boxes, then (hi, lo) with 32-row boxes, then (hi, lo) with 64-row boxes
+constexpr int kSplitMapBytes = 768;
 int make_split_tmaps(void* out, const void* hi, const void* lo, long long rows, long long K);
 // TMA tensor maps (K then V, 128 bytes each) of one bf16 KV-cache layer [rows][64], 64 x 64 boxes
 int make_kv_tmaps(void* out, const void* k, const void* v, long long rows);
-void kernel_attrs_umma();
+void kernel_attrs_umma(Dev* D);
 void trace_set_umma(TraceRec* buf, unsigned* counter, unsigned cap);
 
 size_t attention_scratch_floats(int B, int H, int hd);

@@ -23,6 +23,7 @@
 
 #include <algorithm>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 
 #include "common.cuh"
@@ -376,7 +377,7 @@ template <bool NORM>
 __global__ void __launch_bounds__(256)
 k_split_rows(LinearArgs a, __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __restrict__ lo,
              float* __restrict__ ss, int ss_ld) {
-  TraceScope _trace(TT_UMMA);
+  TraceScope _trace(TT_SPLIT);
   pdl_trigger();
   pdl_wait();
   _trace.waited();
@@ -429,6 +430,7 @@ k_split_rows(LinearArgs a, __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __rest
 __device__ __forceinline__ float row_inv(const float* ss, int n, int ld, size_t row, int K, float eps) {
   const float* p = ss + row * ld;
   float t = 0.f;
+#pragma unroll 8
   for (int i = 0; i < n; ++i) t += p[i];
   return rsqrtf(t / (float)K + eps);
 }
@@ -643,6 +645,476 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN) : "memory");
 }
 
+// ---------------------------------------------------------------- skinny GEMM (few rows)
+// For a few rows the roles swap: the tile computes Y^T [128 output columns][NR rows] =
+// W [128][K] . X [NR][K]^T, with the weights as the MMA's A operand (M = 128) and the split
+// activations as its B operand (N = NR). A stage then moves 16 KB of weights and only NR rows of
+// activations, K is split across a cluster of up to 16 CTAs so that every CTA's weight slice fits
+// its ring (all of it copied before the grid-dependency wait), and the epilogue sees one output
+// column per thread (TMEM lane) and the rows along the TMEM columns: warp-wide stores per row, and
+// the rotary and SwiGLU pairs are adjacent lanes.
+constexpr int kSW = 128;  // output columns per tile (UMMA M)
+
+template <int NR>
+struct SCfg {
+  static constexpr uint32_t kWBytes = kSW * kUK * 2;  // 16 KB
+  static constexpr uint32_t kXBytes = NR * kUK * 2;   // one half (hi or lo) of an activation tile
+  static constexpr uint32_t kStageBytes = kWBytes + 2 * kXBytes;
+  // split-K partials pushed to the rank that finishes them: [KS source ranks][NR / KS rows][128]
+  static constexpr uint32_t kRecvBytes = NR * kSW * 4;
+  // about 104 KB in all, so that a CTA of the next layer's kernel fits beside one of this kernel
+  // on an SM and copies its weights while this one finishes: 3 stages (NR 32), 2 (NR 64)
+  static constexpr int kStages = (104 * 1024 - kRecvBytes) / kStageBytes;
+  // D fp32, A and B bf16, both K-major, M = 128, N = NR
+  static constexpr uint32_t kIDesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(NR >> 3) << 17) |
+                                     ((uint32_t)(kSW >> 4) << 24);
+  static constexpr uint32_t kTmemCols = NR < 32 ? 32 : NR;
+  // ring, receive buffer, barriers (full, empty, accumulator, receive), TMEM address, per-row
+  // inverse RMS / position / sequence / cache slot, two trace times, alignment slack
+  static constexpr size_t kSmem =
+      (size_t)kStages * kStageBytes + kRecvBytes + (2 * kStages + 2) * 8 + 16 + NR * 16 + 16 + 1024;
+  static_assert(NR == 32 || NR == 64, "tile rows");
+  static_assert(kStages >= 2, "ring");
+  static_assert(kStageBytes % 1024 == 0 && kXBytes % 1024 == 0, "swizzle atoms");
+  static_assert(kSmem <= 112 * 1024, "two CTAs per SM");
+};
+
+template <int NR>
+__device__ __forceinline__ void smma(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
+      "l"(a), "l"(b), "r"(SCfg<NR>::kIDesc), "r"(accumulate)
+      : "memory");
+}
+
+// Per-row tile metadata in shared memory.
+struct SRowMeta {
+  float* inv;
+  int* pos;
+  int* b;
+  int* slot;
+};
+
+// Output of value x (accumulator times the row's scale) at global row gr, column c, for one lane
+// of a warp whose 32 lanes hold 32 consecutive columns of the same row; op is the residual value
+// (residual modes), gc the consumer's RMSNorm gain of column c (split on write of a residual
+// output). Every lane of the warp calls it (shuffles).
+__device__ __forceinline__ void scol_out(const EpiArgs& e, size_t gr, int c, int lane, float x, float op,
+                                         float gc, const SRowMeta& m, int rt) {
+  switch (e.mode) {
+    case EPI_STORE:
+      e.y[gr * e.ldy + c] = x;
+      break;
+    case EPI_RESID:
+    case EPI_RESID_SILU: {
+      const float y = op + (e.mode == EPI_RESID_SILU ? silu_f(x) : x);
+      if (!e.sp_only) e.y[gr * e.ldy + c] = y;
+      if (e.sp_hi) {
+        uint16_t h, l;
+        split_bf16(y * gc, h, l);
+        reinterpret_cast<uint16_t*>(e.sp_hi)[gr * e.ldsp + c] = h;
+        reinterpret_cast<uint16_t*>(e.sp_lo)[gr * e.ldsp + c] = l;
+        if (e.ss) {
+          float q2 = y * y;
+#pragma unroll
+          for (int o = 16; o; o >>= 1) q2 += __shfl_xor_sync(0xffffffffu, q2, o);
+          if (lane == 0) e.ss[gr * e.ss_ld + (c >> 5)] = q2;
+        }
+      }
+      break;
+    }
+    case EPI_SWIGLU: {
+      // interleaved (gate, up) columns: the even lane of a pair holds the gate
+      const float u = __shfl_xor_sync(0xffffffffu, x, 1);
+      if (!(lane & 1)) {
+        const float mv = silu_f(x) * u;
+        const int cm = c >> 1;
+        if (!e.sp_only) e.y[gr * e.ldy + cm] = mv;
+        if (e.sp_hi) {
+          uint16_t h, l;
+          split_bf16(e.sg ? mv * e.sg[cm] : mv, h, l);
+          reinterpret_cast<uint16_t*>(e.sp_hi)[gr * e.ldsp + cm] = h;
+          reinterpret_cast<uint16_t*>(e.sp_lo)[gr * e.ldsp + cm] = l;
+        }
+      }
+      break;
+    }
+    case EPI_QKV: {
+      const int part = c / e.d;  // the same across the warp (d is a multiple of 32)
+      const int cc = c - part * e.d;
+      const int h = cc / e.hd;
+      const int dd = cc - h * e.hd;
+      if (part < 2) {
+        // interleaved rotary pairs (2i, 2i + 1) in adjacent lanes
+        const float p = __shfl_xor_sync(0xffffffffu, x, 1);
+        const float2 cs = e.rope[(size_t)m.pos[rt] * (e.hd >> 1) + (dd >> 1)];
+        x = (lane & 1) ? p * cs.y + x * cs.x : x * cs.x - p * cs.y;
+      }
+      if (part == 0) {
+        e.y[gr * e.ldy + cc] = x;
+      } else {
+        const int slot = m.slot[rt];
+        if (slot < 0 || slot >= e.kv.S) {
+          if (lane == 0) atomicOr(e.err, kErrIndex);
+        } else {
+          __nv_bfloat16* base = reinterpret_cast<__nv_bfloat16*>(part == 1 ? e.kv.k : e.kv.v);
+          base[(((size_t)m.b[rt] * e.H + h) * e.kv.S + slot) * e.hd + dd] = __float2bfloat16_rn(x);
+        }
+      }
+      break;
+    }
+  }
+}
+
+// Release-ordered arrive: this thread's earlier accesses, distributed shared memory loads
+// included, are performed before a peer's wait on the phase returns.
+__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait;" ::: "memory"); }
+
+__device__ __forceinline__ uint32_t mapa_u32(uint32_t saddr, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+
+// Cluster split-K of the skinny tile, push side: rank ks owns tile rows [ks * RPC, (ks + 1) * RPC)
+// (RPC = NR / KS). An epilogue thread (one output column) reads its column of the accumulator and
+// stores each row's partial into the owning rank's receive buffer, slot ks (its own rows into its
+// own buffer with plain stores).
+template <int NR, int KS>
+__device__ __forceinline__ void spush(float* recv, int ks, uint32_t tlane, int col) {
+  constexpr int RPC = NR / KS;
+  const uint32_t lbase = su32(recv);
+#pragma unroll 1
+  for (int j0 = 0; j0 < NR; j0 += 32) {
+    uint32_t v[32];
+    tld32(tlane + (uint32_t)j0, v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const int rt = j0 + i, k = rt / RPC, r = rt - k * RPC;
+      const uint32_t off = (uint32_t)(((ks * RPC + r) * kSW + col) * 4);
+      if (k == ks) recv[(ks * RPC + r) * kSW + col] = __uint_as_float(v[i]);
+      else st_cluster_f32(mapa_u32(lbase + off, k), __uint_as_float(v[i]));
+    }
+  }
+}
+
+// Finish side: the rank's rows, each the sum of the KS slots of the receive buffer (in rank
+// order). Once every sum is in registers the thread arrives (relaxed: its reads of the buffer have
+// returned, the sums use them) on the cluster barrier that closes the pass, then writes the rows.
+template <int NR, int KS>
+__device__ __forceinline__ void sfinish(const LinearArgs& a, const float* recv, const SRowMeta& meta, int ks, int mt,
+                                        int rbase, int M, int c, int col, int lane) {
+  constexpr int RPC = NR / KS;
+  const bool resid = a.epi.mode == EPI_RESID || a.epi.mode == EPI_RESID_SILU;
+  const float gc = (resid && a.epi.sp_hi && a.epi.sg) ? a.epi.sg[c] : 1.f;
+  const int nrow = min(RPC, M - (mt * NR + ks * RPC));  // rows of this rank (may be <= 0)
+  float op[RPC], acc[RPC];
+#pragma unroll
+  for (int i = 0; i < RPC; ++i) {
+    const int row = mt * NR + ks * RPC + i;
+    op[i] = resid && i < nrow ? a.epi.res[(size_t)(rbase + row) * a.epi.ldres + c] : 0.f;
+    acc[i] = 0.f;
+#pragma unroll
+    for (int k = 0; k < KS; ++k) acc[i] += recv[(k * RPC + i) * kSW + col];
+  }
+  float dep = 0.f;
+#pragma unroll
+  for (int i = 0; i < RPC; ++i) dep += acc[i];
+  asm volatile("barrier.cluster.arrive.relaxed;" ::"f"(dep) : "memory");
+#pragma unroll
+  for (int i = 0; i < RPC; ++i) {
+    if (i >= nrow) break;  // the same across the warp
+    const int rt = ks * RPC + i;
+    scol_out(a.epi, (size_t)(rbase + mt * NR + rt), c, lane, acc[i] * meta.inv[rt], op[i], gc, meta, rt);
+  }
+}
+
+template <int NR>
+__global__ void __launch_bounds__(kTThreads, 2)
+k_sgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmXh,
+        const __grid_constant__ CUtensorMap tmXl, const float* __restrict__ ss, int ss_n, int ss_ld, int MT,
+        int KS) {
+  using C = SCfg<NR>;
+  namespace cgr = cooperative_groups;
+  TraceScope _trace(TT_SGEMM);
+  extern __shared__ __align__(1024) unsigned char ssm_raw[];
+  unsigned char* ring =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(ssm_raw) + 1023) & ~uintptr_t(1023));
+  float* recv = reinterpret_cast<float*>(ring + C::kStages * C::kStageBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStageBytes + C::kRecvBytes);
+  uint64_t* empty = full + C::kStages;
+  uint64_t* accdone = empty + C::kStages;
+  uint64_t* rbar = accdone + 1;  // the rank's rows: one arrival per peer
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rbar + 1);
+  SRowMeta meta;
+  meta.inv = reinterpret_cast<float*>(rbar + 1) + 4;
+  meta.pos = reinterpret_cast<int*>(meta.inv + NR);
+  meta.b = meta.pos + NR;
+  meta.slot = meta.b + NR;
+  // traced launches: partials pushed, peers' partials received
+  unsigned long long* tmk = reinterpret_cast<unsigned long long*>(meta.slot + NR);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int n0 = blockIdx.x * kSW;
+  const int ks = blockIdx.y;
+  const int grp = blockIdx.z / MT, mt0 = blockIdx.z % MT;
+  const int rbase = grp * a.Mg_stride;
+  const int nkb = a.Kd / kUK / KS;
+  const int kb0 = ks * nkb;
+  const int wrow = grp * a.N + n0;
+
+  if (tid == 0) {
+    for (int i = 0; i < C::kStages; ++i) {
+      ubar_init(&full[i], 1);
+      ubar_init(&empty[i], 1);
+    }
+    ubar_init(accdone, 1);
+    ubar_init(rbar, KS > 1 ? KS - 1 : 1);
+    tmk[0] = tmk[1] = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
+  }
+  __syncthreads();
+  // the peers' receive barriers are initialised before anyone pushes (before the dependency
+  // wait, so this overlaps the previous kernel)
+  if (KS > 1) cooperative_groups::this_cluster().sync();
+  // weights never change: the weight part of the first stages (all of them when the slice fits
+  // the ring) is copied before the dependency wait
+  const int pre = nkb < C::kStages ? nkb : C::kStages;
+  if (tid == 0) {
+    for (int i = 0; i < pre; ++i) {
+      ubar_expect(&full[i], C::kStageBytes);
+      unsigned char* st = ring + (size_t)i * C::kStageBytes;
+      tma_load_2d(st, &tmW, (kb0 + i) * kUK, wrow, &full[i]);
+      tma_load_2d(st + 8192, &tmW, (kb0 + i) * kUK, wrow + 64, &full[i]);
+    }
+  }
+  pdl_trigger();
+  pdl_wait();
+  _trace.waited();
+  int M = *a.M;
+  M = M < a.M_cap ? M : a.M_cap;
+  const int ntm = (M + NR - 1) / NR;
+  int npass = (ntm - mt0 + MT - 1) / MT;
+  if (npass < 1) npass = 1;
+  bool failed = false;
+  uint32_t issued = pre;
+  if (tid == 0) {
+    const int xrow = rbase + mt0 * NR;
+    for (int i = 0; i < pre; ++i) {
+      unsigned char* st = ring + (size_t)i * C::kStageBytes;
+      tma_load_2d(st + C::kWBytes, &tmXh, (kb0 + i) * kUK, xrow, &full[i]);
+      tma_load_2d(st + C::kWBytes + C::kXBytes, &tmXl, (kb0 + i) * kUK, xrow, &full[i]);
+    }
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)),
+                 "r"(C::kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = *tmem_slot;
+  const int eq = warp & 3;                 // TMEM lane quarter of an epilogue warp
+  const int c = n0 + eq * 32 + lane;       // output column of an epilogue thread
+  const uint32_t tlane = tmem + ((uint32_t)(eq * 32) << 16);
+  const int et = (warp - 2) * 32 + lane;   // epilogue thread 0..127
+
+  for (int ps = 0; ps < npass; ++ps) {
+    const int mt = mt0 + ps * MT;
+    const bool live = mt * NR < M;  // the same for every CTA of a cluster
+    const int xrow = rbase + mt * NR;
+    const uint32_t kbase = (uint32_t)ps * nkb;
+    if (warp == 0) {
+      if (lane == 0) {
+        for (int kb = (ps == 0 ? pre : 0); kb < nkb; ++kb) {
+          const uint32_t it = kbase + kb;
+          const int s = it % C::kStages;
+          if (it >= (uint32_t)C::kStages) wait_or_fail(&empty[s], ((it / C::kStages) - 1) & 1, failed);
+          if (failed) break;
+          ++issued;
+          unsigned char* st = ring + (size_t)s * C::kStageBytes;
+          ubar_expect(&full[s], C::kStageBytes);
+          tma_load_2d(st + C::kWBytes, &tmXh, (kb0 + kb) * kUK, xrow, &full[s]);
+          tma_load_2d(st + C::kWBytes + C::kXBytes, &tmXl, (kb0 + kb) * kUK, xrow, &full[s]);
+          tma_load_2d(st, &tmW, (kb0 + kb) * kUK, wrow, &full[s]);
+          tma_load_2d(st + 8192, &tmW, (kb0 + kb) * kUK, wrow + 64, &full[s]);
+        }
+        if (g_trace && ps == 0) {
+          wait_or_fail(accdone, 0, failed);
+          _trace.mark();
+        }
+      }
+    } else if (warp == 1) {
+      if (lane == 0) {
+        for (int kb = 0; kb < nkb; ++kb) {
+          const uint32_t it = kbase + kb;
+          const int s = it % C::kStages;
+          wait_or_fail(&full[s], (it / C::kStages) & 1, failed);
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          const uint32_t wb = su32(ring + (size_t)s * C::kStageBytes);
+          const uint32_t xh = wb + C::kWBytes, xl = xh + C::kXBytes;
+          if (live && !failed) {
+#pragma unroll
+            for (int k = 0; k < kUK / 16; ++k) {
+              smma<NR>(tmem, sdesc(wb + k * 32), sdesc(xh + k * 32), (kb > 0 || k > 0) ? 1u : 0u);
+              smma<NR>(tmem, sdesc(wb + k * 32), sdesc(xl + k * 32), 1u);
+            }
+            umma_commit(&empty[s]);
+          } else {
+            ubar_arrive(&empty[s]);
+          }
+        }
+        if (live) umma_commit(accdone);
+        else ubar_arrive(accdone);
+      }
+    } else {
+      // rows' metadata of this tile: inverse RMS, and for Q/K/V the position, sequence and slot
+      if (et < NR) {
+        const int row = mt * NR + et;
+        float inv = 1.f;
+        if (row < M) {
+          if (a.norm) inv = row_inv(ss, ss_n, ss_ld, rbase + row, a.Kd, a.eps);
+          if (a.epi.mode == EPI_QKV) {
+            meta.pos[et] = a.epi.rows.pos[rbase + row];
+            meta.b[et] = a.epi.rows.b[rbase + row];
+            meta.slot[et] = a.epi.rows.slot[rbase + row];
+          }
+        }
+        meta.inv[et] = inv;
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (live && KS == 1) {
+        const bool resid = a.epi.mode == EPI_RESID || a.epi.mode == EPI_RESID_SILU;
+        const float gc = (resid && a.epi.sp_hi && a.epi.sg) ? a.epi.sg[c] : 1.f;
+        for (int j0 = 0; j0 < NR; j0 += 32) {
+          if (mt * NR + j0 >= M) break;
+          float op[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int row = mt * NR + j0 + i;
+            op[i] = resid && row < M ? a.epi.res[(size_t)(rbase + row) * a.epi.ldres + c] : 0.f;
+          }
+          if (j0 == 0) {
+            wait_or_fail(accdone, ps & 1, failed);
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          }
+          uint32_t v[32];
+          tld32(tlane + (uint32_t)j0, v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int rt = j0 + i;
+            if (mt * NR + rt >= M) break;  // the same across the warp
+            scol_out(a.epi, (size_t)(rbase + mt * NR + rt), c, lane, __uint_as_float(v[i]) * meta.inv[rt], op[i],
+                     gc, meta, rt);
+          }
+        }
+      }
+    }
+    __syncwarp();
+    if (live && KS > 1) {
+      // push the partials to their owners; the owner waits for its KS - 1 peers and finishes its
+      // rows; a cluster barrier closes the pass (no CTA refills a receive buffer, or exits while a
+      // peer may still write to it, before every CTA has read its rows)
+      if (warp >= 2) {
+        wait_or_fail(accdone, ps & 1, failed);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        switch (KS) {
+          case 2: spush<NR, 2>(recv, ks, tlane, eq * 32 + lane); break;
+          case 4: spush<NR, 4>(recv, ks, tlane, eq * 32 + lane); break;
+          case 8: spush<NR, 8>(recv, ks, tlane, eq * 32 + lane); break;
+          default: spush<NR, 16>(recv, ks, tlane, eq * 32 + lane); break;
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (g_trace && et == 0 && ps == 0) tmk[0] = gtimer();
+        if (et == 0) {
+          // one cluster-scope fence orders every epilogue thread's pushes (they precede the barrier)
+          // before the relaxed arrivals on the owners' barriers
+          asm volatile("fence.acq_rel.cluster;" ::: "memory");
+          for (int k = 1; k < KS; ++k) {
+            const int peer = (ks + k) % KS;
+            asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(
+                             mapa_u32(su32(rbar), peer))
+                         : "memory");
+          }
+          bool ok = false;
+          for (int it = 0; it < kUSpins && !ok; ++it) {
+            uint32_t done;
+            asm volatile(
+                "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+                " selp.u32 %0, 1, 0, p;\n}"
+                : "=r"(done)
+                : "r"(su32(rbar)), "r"((uint32_t)(ps & 1))
+                : "memory");
+            ok = done != 0;
+          }
+          if (!ok) failed = true;
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (g_trace && et == 0 && ps == 0) tmk[1] = gtimer();
+        switch (KS) {
+          case 2: sfinish<NR, 2>(a, recv, meta, ks, mt, rbase, M, c, eq * 32 + lane, lane); break;
+          case 4: sfinish<NR, 4>(a, recv, meta, ks, mt, rbase, M, c, eq * 32 + lane, lane); break;
+          case 8: sfinish<NR, 8>(a, recv, meta, ks, mt, rbase, M, c, eq * 32 + lane, lane); break;
+          default: sfinish<NR, 16>(a, recv, meta, ks, mt, rbase, M, c, eq * 32 + lane, lane); break;
+        }
+      } else {
+        asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
+      }
+      cluster_wait();
+    }
+    // this pass's TMEM reads, reduction-buffer and metadata use end before the next pass
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  }
+  if (g_trace) {
+    _trace.mark_at(1, tmk[0]);
+    _trace.mark_at(2, tmk[1]);
+  }
+  const bool any_failed = __syncthreads_or(failed);
+  if (tid == 0 && any_failed) {
+    for (uint32_t s = 0; s < (uint32_t)C::kStages && s < issued; ++s) {
+      const uint32_t last = issued - 1 - ((issued - 1 - s) % C::kStages);
+      ubar_wait(&full[last % C::kStages], (last / C::kStages) & 1);
+    }
+    atomicOr(a.epi.err, kErrTimeout | kErrWaitGemm);
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::kTmemCols)
+                 : "memory");
+}
+
+template <int NR>
+void sgemm_go(const LinearArgs& a, const CUtensorMap& tw, const CUtensorMap& th, const CUtensorMap& tl,
+              const float* ss, int ss_n, int ss_ld, int MT, int KS, cudaStream_t s) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(a.N / kSW, KS, a.groups * MT);
+  cfg.blockDim = dim3(kTThreads);
+  cfg.dynamicSmemBytes = SCfg<NR>::kSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = KS;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++g_launches;
+  cudaLaunchKernelEx(&cfg, k_sgemm<NR>, a, tw, th, tl, ss, ss_n, ss_ld, MT, KS);
+}
+
 template <int BN>
 void tgemm_go(const LinearArgs& a, const CUtensorMap& tw, const CUtensorMap& th, const CUtensorMap& tl,
               const float* ss, int ss_n, int ss_ld, int MT, int KS, cudaStream_t s) {
@@ -711,8 +1183,29 @@ void split_gemm(const Dev& D, const LinearArgs& a, const void* amap, __nv_bfloat
     if (a.norm) launch_pdl(k_split_rows<true>, dim3(blocks), dim3(256), 0, s, a, hi, lo, ss, ss_ld);
     else launch_pdl(k_split_rows<false>, dim3(blocks), dim3(256), 0, s, a, hi, lo, ss, ss_ld);
   }
-  const int mt_cap = (a.M_cap + kUM - 1) / kUM;
   const int rows_typ = a.rows_typ > 0 ? a.rows_typ : a.M_cap;
+  if (rows_typ <= D.sgemm_max_rows && a.N % kSW == 0) {
+    // skinny: NR rows per tile; K split (power of two, at most sgemm_max_ks, dividing the K
+    // blocks and NR) as far as the grid fits one wave of two CTAs per SM
+    const int NR = rows_typ <= 32 ? 32 : 64;
+    const int mtc = (a.M_cap + NR - 1) / NR;
+    const int MT = std::max(1, std::min((rows_typ + NR - 1) / NR, mtc));
+    const int kb = a.Kd / kUK;
+    const long long base = (long long)(a.N / kSW) * a.groups * MT;
+    int KS = 1;
+    // two CTAs fit an SM (about 96 KB of ring each)
+    while (2 * KS <= D.sgemm_max_ks && kb % (2 * KS) == 0 && NR % (2 * KS) == 0 && base * 2 * KS <= 2 * sms)
+      KS *= 2;
+    CUtensorMap tw, th, tl;
+    const int mo = NR == 32 ? 256 : 512;
+    memcpy(&tw, a.tmap, sizeof(tw));
+    memcpy(&th, static_cast<const unsigned char*>(amap) + mo, sizeof(th));
+    memcpy(&tl, static_cast<const unsigned char*>(amap) + mo + 128, sizeof(tl));
+    if (NR == 32) sgemm_go<32>(a, tw, th, tl, ss, ss_n, ss_ld, MT, KS, s);
+    else sgemm_go<64>(a, tw, th, tl, ss, ss_n, ss_ld, MT, KS, s);
+    return;
+  }
+  const int mt_cap = (a.M_cap + kUM - 1) / kUM;
   int MT = (rows_typ + kUM - 1) / kUM;
   MT = MT < 1 ? 1 : (MT > mt_cap ? mt_cap : MT);
   const int kb = a.Kd / kUK;
@@ -747,17 +1240,59 @@ int make_weight_tmap(void* out, const void* W, long long rows, long long K) {
   return encode_bf16_2d(out, W, rows, K, kUN);
 }
 
-// Tensor maps (hi, lo) of the split activations [rows][K] bf16 with 64 x 128 boxes, 128-byte swizzle.
+// Tensor maps (hi, lo) of the split activations [rows][K] bf16 with 128-byte swizzle and K boxes of
+// 64: 128-row boxes (at 0), 32-row boxes (at 256) and 64-row boxes (at 512).
 int make_split_tmaps(void* out, const void* hi, const void* lo, long long rows, long long K) {
   if (K % kUK || rows < 1) return LCA_E_ARG;
-  const int st = encode_bf16_2d(out, hi, rows, K, kUM);
-  return st != LCA_OK ? st : encode_bf16_2d(static_cast<unsigned char*>(out) + 128, lo, rows, K, kUM);
+  unsigned char* o = static_cast<unsigned char*>(out);
+  const int boxes[3] = {kUM, 32, 64};
+  for (int i = 0; i < 3; ++i) {
+    int st = encode_bf16_2d(o + 256 * i, hi, rows, K, boxes[i]);
+    if (st == LCA_OK) st = encode_bf16_2d(o + 256 * i + 128, lo, rows, K, boxes[i]);
+    if (st != LCA_OK) return st;
+  }
+  return LCA_OK;
 }
 
-void kernel_attrs_umma() {
+template <int NR>
+int sgemm_attrs() {
+  cudaFuncSetAttribute(k_sgemm<NR>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SCfg<NR>::kSmem);
+  cudaFuncSetAttribute(k_sgemm<NR>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  // can the GPU hold a 16-CTA cluster of this kernel at all?
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(8, 16, 1);
+  cfg.blockDim = dim3(kTThreads);
+  cfg.dynamicSmemBytes = SCfg<NR>::kSmem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 16;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int nc = 0;
+  if (cudaOccupancyMaxActiveClusters(&nc, k_sgemm<NR>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    nc = 0;
+  }
+  return nc;
+}
+
+// Kernel attributes; with D, the skinny GEMM's largest K split (16 only if 16-CTA clusters of
+// every tile height fit; environment LCA_SGEMM_MAX_KS lowers it) and its row limit (environment
+// LCA_SGEMM_MAX_ROWS, default 64).
+void kernel_attrs_umma(Dev* D) {
   cudaFuncSetAttribute(k_tgemm<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TCfg<64>::kSmem);
   cudaFuncSetAttribute(k_tgemm<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TCfg<128>::kSmem);
   cudaFuncSetAttribute(k_tgemm<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TCfg<256>::kSmem);
+  const int c32 = sgemm_attrs<32>(), c64 = sgemm_attrs<64>();
+  if (D) {
+    D->sgemm_max_ks = (c32 > 0 && c64 > 0) ? 16 : 8;
+    const char* k = getenv("LCA_SGEMM_MAX_KS");
+    if (k) D->sgemm_max_ks = std::max(1, std::min(D->sgemm_max_ks, atoi(k)));
+    const char* e = getenv("LCA_SGEMM_MAX_ROWS");
+    D->sgemm_max_rows = e ? std::max(0, std::min(64, atoi(e))) : 64;
+  }
 }
 
 // The tensor cores take a layer that has a weight tensor map and split-activation maps for its K,
@@ -801,7 +1336,7 @@ extern "C" int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   D.num_sms = sms;
-  kernel_attrs_umma();
+  kernel_attrs_umma(&D);
   LinearArgs a{};
   a.x = x;
   a.ldx = K;
@@ -821,7 +1356,7 @@ extern "C" int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M
   __nv_bfloat16* hi = reinterpret_cast<__nv_bfloat16*>(p);
   __nv_bfloat16* lo = hi + (size_t)M * K;
   float* ss = reinterpret_cast<float*>(lo + (size_t)M * K);
-  alignas(64) unsigned char maps[256];
+  alignas(64) unsigned char maps[kSplitMapBytes];
   st = make_split_tmaps(maps, hi, lo, M, K);
   if (st != LCA_OK) return st;
   split_gemm(D, a, maps, hi, lo, ss, 1, reinterpret_cast<cudaStream_t>(stream));

@@ -187,7 +187,7 @@ struct alignas(64) TMapBlob {
   unsigned char b[128];
 };
 struct alignas(64) SplitMapBlob {
-  unsigned char b[256];  // hi, lo
+  unsigned char b[kSplitMapBytes];  // (hi, lo) maps of split activations, or (K, V) of a cache layer
 };
 
 struct lca_ctx {
@@ -829,7 +829,7 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     return fail(LCA_E_CUDA);
   kernel_attrs_linear();
   kernel_attrs_step();
-  kernel_attrs_umma();
+  kernel_attrs_umma(&c->L.D);
   kernel_attrs_attn();
   Dev& D = c->L.D;
   {

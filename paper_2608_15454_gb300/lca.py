@@ -255,11 +255,12 @@ class Context:
     TRACE_TAGS = {1: "gemv", 2: "gemv_f32", 3: "gemm", 4: "rowstats", 5: "attn", 6: "head",
                   7: "mb_plan", 8: "mb_fill", 9: "mlp_plan", 10: "verify_plan", 11: "segment",
                   12: "lm_scatter", 13: "nb_input", 14: "commit", 15: "loop_ctl", 16: "other",
-                  17: "umma"}
+                  17: "umma", 18: "split", 19: "sgemm"}
 
     def trace(self, n, tau, mode, steps, cap=1 << 18):
         rec = np.zeros(cap, dtype=[("t0", "<u8"), ("t1", "<u8"), ("tw", "<u8"), ("tag", "<i4"),
-                                   ("cta", "<i4"), ("sm", "<i4"), ("mark", "<i4")])
+                                   ("cta", "<i4"), ("sm", "<i4"), ("mark", "<i4"), ("mark2", "<i4"),
+                                   ("mark3", "<i4")])
         cnt = ctypes.c_int32()
         self._check(self.lib.lca_debug_trace(self.h, n, tau, mode, steps, _ptr(rec), cap, ctypes.byref(cnt)),
                     "lca_debug_trace")

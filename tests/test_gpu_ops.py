@@ -79,11 +79,18 @@ def test_decode_attention_rejects_bad_arguments(lca):
     (2100, 2050, 512, 1024, 128),   # launch shaped for 128 rows: clustered CTAs walk 17 row tiles
     (700, 650, 3072, 1024, 256),    # two row tiles per CTA, 256-column tiles
     (2100, 2100, 256, 320, 0),      # more row tiles than TMEM holds; K blocks not a power of two
+    # skinny GEMM (weights as the MMA's M operand) for at most 64 typical rows
+    (32, 32, 1024, 1024, 0),        # 16-way cluster split K, one K block per CTA
+    (32, 19, 8192, 1024, 0),        # ragged rows, two-way split K
+    (64, 50, 3072, 1024, 0),        # 64-row tiles, four-way split K
+    (300, 257, 1024, 4096, 32),     # launch shaped for 32 rows: clusters walk nine row tiles
+    (200, 200, 256, 1088, 64),      # 17 K blocks (no split), ring wraps, ragged last row tile
+    (48, 48, 2048, 2048, 48),       # partial 64-row tile
 ])
 def test_tensor_core_gemm_matches_reference(lca, M, Mused, N, K, typ):
-    """tcgen05 GEMM (TMA weight tiles, 128-byte swizzle, TMEM accumulators, split bf16
-    activations, cluster split-K) against a float64 product of the fp32 activations and the
-    bf16 weights."""
+    """tcgen05 GEMMs (TMA weight tiles, 128-byte swizzle, TMEM accumulators, split bf16
+    activations, cluster split-K; activations as the M operand, or the weights for few rows)
+    against a float64 product of the fp32 activations and the bf16 weights."""
     import torch
     g = torch.Generator(device="cuda").manual_seed(M + N + K)
     x = torch.randn(M, K, device="cuda", generator=g)
