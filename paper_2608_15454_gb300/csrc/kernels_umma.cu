@@ -313,13 +313,14 @@ __device__ __forceinline__ float pair_split(const EpiArgs& e, float2 op, int r, 
 
 // Cluster split-K: rank `ks` adds rows [ks * 128 / KS, ...) of the KS partial tiles (each
 // [128][BN + 1] in its CTA's shared memory) and applies the pair epilogue, four items per batch
-// with all loads of a batch before its stores. inv_s: the tile rows' inverse RMS (nullptr: 1).
+// with all loads of a batch before its stores. inv_s: the tile rows' inverse RMS (nullptr: 1);
+// meta_s: the tile rows' Q/K/V metadata (position, sequence, cache slot), staged in shared memory.
 // The 32 lanes of a warp hold 32 consecutive pairs of one row (BN / 2 and the thread count are
 // multiples of 32), so a 32-column block's sum of squares is a reduction over 16 lanes.
 template <int BN, int NT>
 __device__ __forceinline__ void cluster_epilogue(const EpiArgs& e, cooperative_groups::cluster_group& cl,
                                                  float* red, int KS, int ks, int mrow0, int rbase, int M, int n0,
-                                                 const float* inv_s) {
+                                                 const float* inv_s, const EpiRow* meta_s) {
   const int RPC = kUM / KS;
   const int items = RPC * (BN / 2);
   constexpr int U = 4;
@@ -350,7 +351,7 @@ __device__ __forceinline__ void cluster_epilogue(const EpiArgs& e, cooperative_g
           }
         }
         if (inv_s) sc[u] = inv_s[rt];
-        q[u] = epi_row(e, gr[u]);
+        q[u] = meta_s[rt];
         op[u] = epi_operand(e, q[u], gr[u], col[u]);
       }
     }
@@ -447,7 +448,8 @@ struct TCfg {
   static constexpr uint32_t kIDesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                                      ((uint32_t)(kUM >> 4) << 24);
   // ring, barriers, TMEM address, the tile rows' inverse RMS, alignment slack
-  static constexpr size_t kSmem = (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16 + kUM * 4 + 1024;
+  static constexpr size_t kSmem =
+      (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16 + kUM * 4 + 16 + kUM * sizeof(EpiRow) + 1024;
   static_assert((size_t)kUM * (BN + 1) * 4 <= (size_t)kStages * kStageBytes, "reduction buffer");
 };
 
@@ -476,6 +478,9 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
   uint64_t* accdone = empty + C::kStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accdone + 1);
   float* inv_s = reinterpret_cast<float*>(accdone + 1) + 4;  // [128]
+  // traced launches: epilogue of the first row tile done (one epilogue thread), then pass end
+  unsigned long long* tmk = reinterpret_cast<unsigned long long*>(inv_s + kUM);
+  EpiRow* meta_s = reinterpret_cast<EpiRow*>(tmk + 2);  // [128]
   float* red = reinterpret_cast<float*>(ring);  // [128][BN + 1] after the MMAs of a pass
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -492,6 +497,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
       ubar_init(&full[i], 1);
       ubar_init(&empty[i], 1);
     }
+    tmk[0] = 0;
     ubar_init(accdone, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
@@ -589,7 +595,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
         if (live) umma_commit(accdone);
         else ubar_arrive(accdone);
       }
-    } else if (!live || KS > 1) {
+    } else if (!live) {
       wait_or_fail(accdone, ps & 1, failed);
     }
     __syncwarp();
@@ -606,11 +612,16 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
                               wait_or_fail(accdone, ps & 1, failed);
                               asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                             });
+          if (g_trace && ps == 0 && warp == 2 && lane == 0) tmk[0] = gtimer();
         }
       } else {
         cgr::cluster_group cl = cgr::this_cluster();
         if (warp >= 2) {
+          // the rows' metadata is read while the main loop runs; then the accumulator
           inv_s[r] = sc;
+          meta_s[r] = mt * kUM + r < M ? epi_row(a.epi, rbase + mt * kUM + r) : EpiRow{0, 0, 0};
+          wait_or_fail(accdone, ps & 1, failed);
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
           for (int cb = 0; cb < BN; cb += 32) {
             uint32_t v[32];
@@ -620,10 +631,13 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
           }
         }
         cl.sync();
-        cluster_epilogue<BN, kTThreads>(a.epi, cl, red, KS, ks, mt * kUM, rbase, M, n0, a.norm ? inv_s : nullptr);
+        cluster_epilogue<BN, kTThreads>(a.epi, cl, red, KS, ks, mt * kUM, rbase, M, n0, a.norm ? inv_s : nullptr,
+                                        meta_s);
+        if (g_trace && ps == 0 && warp == 2 && lane == 0) tmk[0] = gtimer();
         cl.sync();
       }
     }
+    if (ps == 0) _trace.mark(2);
     // this pass's TMEM reads and reduction-buffer use end before the next pass's MMAs and copies
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
@@ -631,6 +645,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
   }
   // after a failed wait, copies may still be in flight: wait (bounded) for the last one issued
   // into each stage before the CTA's shared memory is released
+  if (g_trace) _trace.mark_at(1, tmk[0]);
   const bool any_failed = __syncthreads_or(failed);
   if (tid == 0 && any_failed) {
     for (uint32_t s = 0; s < (uint32_t)C::kStages && s < issued; ++s) {
@@ -1291,7 +1306,7 @@ void kernel_attrs_umma(Dev* D) {
     const char* k = getenv("LCA_SGEMM_MAX_KS");
     if (k) D->sgemm_max_ks = std::max(1, std::min(D->sgemm_max_ks, atoi(k)));
     const char* e = getenv("LCA_SGEMM_MAX_ROWS");
-    D->sgemm_max_rows = e ? std::max(0, std::min(64, atoi(e))) : 64;
+    D->sgemm_max_rows = e ? std::max(0, std::min(256, atoi(e))) : 64;
   }
 }
 
