@@ -256,6 +256,7 @@ struct Dev {
   int attn_pipe;       // decode attention: 2 = tensor cores (bf16, head_dim 64), 1 = bulk-copy pipelined
                        // CUDA-core kernel, 0 = register-tiled kernel
   int attn_ns;         // ring stages of the tensor-core decode attention (4, 6 or 8)
+  int attn_min_keys;   // fewest cache keys per key split of a decode attention launch
   int sgemm_max_rows;  // tensor-core layers with at most this many typical rows use the skinny
                        // (weights-as-M) GEMM; 0: never
   int sgemm_max_ks;    // largest K split (cluster size) of the skinny GEMM (8, or 16 where the

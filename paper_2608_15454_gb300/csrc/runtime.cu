@@ -216,6 +216,9 @@ struct lca_ctx {
   int gen_max_new = 0;
   int gen_n = 0;
   bool t_unsynced = false;
+  // typical cache lengths (bytes; latents) that the step graphs' attention key splits are chosen
+  // for: the longest sequence after the last prefill
+  int kv_bytes_typ = 0, kv_lat_typ = 0;
   bool eager = false;
   // kernels per step graph part, by n: [pre-LM + post-LM, LM body]
   std::map<int, std::pair<long long, long long>> launches;
@@ -279,8 +282,16 @@ const void* tmap_of(lca_ctx* c, const void* W) {
   return it == c->tmaps.end() ? nullptr : it->second.b;
 }
 
-int attn_splits(const Dev& D, int batch_cap, int qtiles) {
+constexpr int kMbWindowKeys = 32;  // the multi-byte window's cache: about two words
+
+// Key splits of a decode attention launch: enough CTAs for about two per SM; with
+// D.attn_min_keys > 0, also at least that many keys per split of a cache of about kv_typ keys
+// (measured: more, shorter splits are faster even for caches of a few hundred keys, so the
+// limit is off unless set).
+int attn_splits(const Dev& D, int batch_cap, int qtiles, int kv_typ) {
   int s = (2 * D.num_sms) / std::max(1, batch_cap * D.H * qtiles);
+  if (kv_typ > 0 && D.attn_min_keys > 0)
+    s = std::min(s, std::max(1, (kv_typ + D.attn_min_keys - 1) / D.attn_min_keys));
   return std::max(1, std::min(std::min(s, kMaxAttnSplit), D.attn_split_cap));
 }
 
@@ -472,7 +483,7 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
       launch_mb_plan(D, s);
       const int typ = B * (2 * n - 2);  // typical window rows: new committed bytes + copies
       // the window holds about two words of keys: a short cache
-      run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2), s,
+      run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2, kMbWindowKeys), s,
                 c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype), nullptr, 0,
                 true);
     } else {
@@ -484,7 +495,7 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
   }
   // (1) embed + encoder over the n candidates
   launch_verify_plan(D, s);
-  run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s,
+  run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1, c->kv_bytes_typ + n), s,
             c->L.nb.empty() ? nullptr : c->L.nb[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype),
             &D.seq[0].t, n);
 }
@@ -492,7 +503,7 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
 void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
   Dev& D = c->L.D;
   // about one new latent per sequence every few bytes
-  run_stack(c, c->L.lm, D.x_lm, D.r_lm, D.B * n, D.B, 1, attn_splits(D, D.B, 1), s);
+  run_stack(c, c->L.lm, D.x_lm, D.r_lm, D.B * n, D.B, 1, attn_splits(D, D.B, 1, c->kv_lat_typ + 1), s);
   launch_lm_scatter(D, s);
 }
 
@@ -501,7 +512,7 @@ void enqueue_verify_commit(lca_ctx* c, int n, cudaStream_t s) {
   const int B = D.B;
   // (4) upsample + next-byte decoder over the n candidates, head
   launch_nb_input(D, s);
-  run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1), s, nullptr, 0,
+  run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1, c->kv_bytes_typ + n), s, nullptr, 0,
             &D.seq[0].t, n);
   launch_head(D, D.x_nb, nullptr, D.r_v.M, B * n, D.nb_norm, D.nb_logits, D.nb_arg, D.nb_prob, s);
   // (5) accept + commit
@@ -613,6 +624,17 @@ struct Profiler : ProfHook {
     }
   }
 };
+
+// Destroy every captured step graph (they are captured again on next use).
+void drop_graphs(lca_ctx* c) {
+  cudaStreamSynchronize(c->stream);
+  for (auto& kv : c->step_exec) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : c->gen_exec) cudaGraphExecDestroy(kv.second);
+  c->step_exec.clear();
+  c->gen_exec.clear();
+  for (cudaGraph_t g : c->graphs) cudaGraphDestroy(g);
+  c->graphs.clear();
+}
 
 int get_step_exec(lca_ctx* c, int n, cudaGraphExec_t* ex) {
   auto it = c->step_exec.find(n);
@@ -849,6 +871,8 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.attn_pipe = ap ? atoi(ap) : 2;
     const char* an = getenv("LCA_ATTN_NS");
     D.attn_ns = an ? atoi(an) : 8;
+    const char* mk = getenv("LCA_ATTN_MIN_KEYS");
+    D.attn_min_keys = mk ? std::max(0, atoi(mk)) : 0;
   }
   // state and counters start at zero
   if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);
@@ -992,7 +1016,21 @@ int lca_prefill(lca_ctx* c, int32_t batch, const uint8_t* const* prompts, const 
   c->host_params.batch = batch;
   c->pending_force_accept = c->pending_force_cand = 0;
   int e = read_err(c);
-  return e;
+  if (e != LCA_OK) return e;
+  // cache lengths for the attention key splits; step graphs captured for lengths more than twice
+  // or less than half of these are dropped and captured again
+  std::vector<SeqState> all(batch);
+  CK(cudaMemcpy(all.data(), D.seq, sizeof(SeqState) * batch, cudaMemcpyDeviceToHost));
+  int tb = 1, kl = 1;
+  for (int b = 0; b < batch; ++b) {
+    tb = std::max(tb, all[b].t);
+    kl = std::max(kl, all[b].K);
+  }
+  auto far = [](int x, int y) { return x > 2 * y || y > 2 * x; };
+  if (far(tb, c->kv_bytes_typ) || far(kl, c->kv_lat_typ)) drop_graphs(c);
+  c->kv_bytes_typ = tb;
+  c->kv_lat_typ = kl;
+  return LCA_OK;
 }
 
 static int step_prep(lca_ctx* c, int n, float tau, int mode) {
@@ -1302,7 +1340,7 @@ int lca_debug_bench_kernel(lca_ctx* c, int32_t kind, int32_t rows, int32_t iters
         break;
       case 4: {  // attention over the encoder cache of layer (i % n_enc)
         Block& eb = c->L.enc[i % c->L.enc.size()];
-        attention(D, D.qbuf, D.att, eb.kv, D.r_v, D.B, 1, attn_splits(D, D.B, 1), c->cap);
+        attention(D, D.qbuf, D.att, eb.kv, D.r_v, D.B, 1, attn_splits(D, D.B, 1, kvl[0]), c->cap);
         by = 2.0 * D.H * (double)kvl[0] * D.hd * tb;
         break;
       }
