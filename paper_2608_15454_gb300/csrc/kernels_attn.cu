@@ -1256,6 +1256,370 @@ void launch_a4_ns(const float* q, float* out, const KV& kv, const Rows& rows, in
                      stable_extra);
 }
 
+// ---------------------------------------------------------------- transposed tensor-core attention
+// The same decode attention for query tiles of at most 8 rows (decode steps: n candidates, or one
+// latent, per sequence). The scores are computed transposed, S^T = K Q^T, with the 16 keys of an
+// MMA tile as its M dimension and the query rows as N = 8, so a tile of 8 rows costs half the MMAs
+// of a 16-row one. P^T reaches the P.V product (O^T = V^T P^T, dims as M) through an in-register
+// 8x8 transpose (movmatrix). Q's bf16 halves are loaded into registers once per tile; K and V
+// come by TMA through the ring, as in k_attn_mma.
+constexpr int kA5QT = 8;
+
+__device__ __forceinline__ void ldsm4_(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ uint32_t movt(uint32_t x) {
+  uint32_t y;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+
+template <int NS>
+__global__ void __launch_bounds__(kA4Threads, 1)
+k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
+           const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+           const int* __restrict__ stable, int stable_stride, int stable_extra) {
+  namespace cgr = cooperative_groups;
+  constexpr int HD = 64, QT = kA5QT, KC = kA4Keys;
+  static_assert(NS % kA4Warps == 0, "ring stages must be a multiple of the compute warps");
+  extern __shared__ __align__(1024) unsigned char a5raw[];
+  unsigned char* ring =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(a5raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* qsh = ring + NS * 2 * kA4Chunk;                    // [QT][HD] bf16, swizzled: hi(q * scale)
+  unsigned char* qsl = qsh + QT * HD * 2;                           // the remainders
+  float* pacc = reinterpret_cast<float*>(qsl + QT * HD * 2);        // [QT][HD]
+  float* s_m = pacc + QT * HD;                                      // [QT]
+  float* s_l = s_m + QT;                                            // [QT]
+  int* s_kv = reinterpret_cast<int*>(s_l + QT);                     // [QT]
+  uint64_t* full = reinterpret_cast<uint64_t*>(s_kv + QT);          // [NS]
+  uint64_t* empty = full + NS;                                      // [NS]
+  // after the key loop the ring holds the warps' partial results
+  float* Ow = reinterpret_cast<float*>(ring);                       // [warps][QT][HD]
+  float* mw = Ow + kA4Warps * QT * HD;                              // [warps][QT]
+  float* lw = mw + kA4Warps * QT;                                   // [warps][QT]
+
+  TraceScope _trace(TT_ATTN);
+  cgr::cluster_group cl = cgr::this_cluster();
+  const int splits = (int)cl.dim_blocks().z;
+  const int sp = (int)cl.block_rank();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, t = lane & 3;
+  if (tid == 0) {
+    for (int i = 0; i < NS; ++i) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&full[i])) : "memory");
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&empty[i])) : "memory");
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+  }
+  if (stable && tid < 2) {
+    // committed slots do not change during a step: warm this CTA's share in L2 (a hint)
+    const int bb = blockIdx.x, hh = blockIdx.z / splits;
+    const int tt = stable[(size_t)bb * stable_stride];
+    const int est = ((tt + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
+    const int lo = sp * est, hi = min(tt, lo + est);
+    if (hi > lo) {
+      const __nv_bfloat16* base = reinterpret_cast<const __nv_bfloat16*>(tid == 0 ? kv.k : kv.v) +
+                                  (((size_t)bb * H + hh) * kv.S + lo) * HD;
+      const uint32_t bytes = (uint32_t)((hi - lo) * HD * 2);
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"(bytes & ~15u) : "memory");
+    }
+  }
+  pdl_trigger();
+  pdl_wait();
+  _trace.waited();
+  __syncthreads();
+  const int b = blockIdx.x;
+  const int h = blockIdx.z / splits;
+  const int nrows = rows.seq_count[b];
+  const int rbeg = rows.seq_start[b];
+  const int ntiles = (nrows + QT - 1) / QT;
+  const int ld = H * HD;
+  const int krow0 = (b * H + h) * kv.S;  // first tensor-map row of this (sequence, head)
+  bool failed = false;
+  uint32_t cc = 0, issued = 0;
+
+  for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
+    const int r0 = rbeg + qt * QT;
+    const int nq = min(QT, nrows - qt * QT);
+    for (int idx = tid; idx < QT * HD / 2; idx += kA4Threads) {
+      const int i = idx / (HD / 2), dd = (idx - i * (HD / 2)) * 2;
+      float2 v = make_float2(0.f, 0.f);
+      if (i < nq) {
+        v = *reinterpret_cast<const float2*>(q + (size_t)(r0 + i) * ld + h * HD + dd);
+        v.x *= scale;
+        v.y *= scale;
+      }
+      uint32_t hi2, lo2;
+      split2(v.x, v.y, hi2, lo2);
+      const uint32_t off = swz(i, dd >> 3) + (dd & 7) * 2;
+      *reinterpret_cast<uint32_t*>(qsh + off) = hi2;
+      *reinterpret_cast<uint32_t*>(qsl + off) = lo2;
+    }
+    if (tid < QT) {
+      int kl = tid < nq ? rows.kvlen[r0 + tid] : 0;
+      if (kl > kv.S || kl < 0) {
+        atomicOr(err, kErrIndex);
+        kl = kl < 0 ? 0 : kv.S;
+      }
+      s_kv[tid] = kl;
+    }
+    __syncthreads();
+    int kv_hi = 0;
+#pragma unroll
+    for (int i = 0; i < QT; ++i) kv_hi = max(kv_hi, s_kv[i]);
+    const int per = ((kv_hi + splits - 1) / splits + KC - 1) / KC * KC;
+    const int lo = sp * per;
+    const int hi = min(kv_hi, lo + per);
+    const int nch = hi > lo ? (hi - lo + KC - 1) / KC : 0;
+
+    // per compute warp: running max and (lane-partial) sum of queries 2t, 2t + 1, and O^T for
+    // dims 16 dm + g (+ 8) of those queries
+    float ma = -INFINITY, mb = -INFINITY, la = 0.f, lb = 0.f;
+    float o[4][4];
+#pragma unroll
+    for (int n = 0; n < 4; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+    if (warp == kA4Warps) {
+      // producer
+      if (lane == 0) {
+        for (int c = 0; c < nch; ++c) {
+          const uint32_t gi = cc + c;
+          const int st = gi % NS;
+          if (gi >= (uint32_t)NS && !failed && !a3_wait(&empty[st], ((gi / NS) - 1) & 1)) failed = true;
+          if (failed) break;
+          ++issued;
+          unsigned char* dst = ring + (size_t)st * 2 * kA4Chunk;
+          a3_expect(&full[st], 2 * kA4Chunk);
+          a4_tma(dst, &tmK, 0, krow0 + lo + c * KC, &full[st]);
+          a4_tma(dst + kA4Chunk, &tmV, 0, krow0 + lo + c * KC, &full[st]);
+        }
+      }
+      __syncwarp();
+    } else {
+      // Q^T fragments (B operand): dims 16 ks .. 16 ks + 15 of query rows 0..7
+      uint32_t qh[4][2], ql[4][2];
+      {
+        const uint32_t qhb = a3_su32(qsh), qlb = a3_su32(qsl);
+#pragma unroll
+        for (int kp = 0; kp < 2; ++kp) {
+          uint32_t r[4];
+          // matrices: query rows lane & 7, dims chunk 4 kp + (lane >> 3)
+          ldsm4_(qhb + swz(lane & 7, 4 * kp + (lane >> 3)), r);
+          qh[2 * kp][0] = r[0];
+          qh[2 * kp][1] = r[1];
+          qh[2 * kp + 1][0] = r[2];
+          qh[2 * kp + 1][1] = r[3];
+          ldsm4_(qlb + swz(lane & 7, 4 * kp + (lane >> 3)), r);
+          ql[2 * kp][0] = r[0];
+          ql[2 * kp][1] = r[1];
+          ql[2 * kp + 1][0] = r[2];
+          ql[2 * kp + 1][1] = r[3];
+        }
+      }
+      const int kla = min(s_kv[2 * t], hi), klb = min(s_kv[2 * t + 1], hi);
+      for (int c = warp; c < nch; c += kA4Warps) {
+        const uint32_t gi = cc + c;
+        const int st = gi % NS;
+        if (!failed && !a3_wait(&full[st], (gi / NS) & 1)) failed = true;
+        const uint32_t kb = a3_su32(ring + (size_t)st * 2 * kA4Chunk), vb = kb + kA4Chunk;
+        const int j0 = lo + c * KC;
+        // S^T = K Q^T: m-tile i = keys 16 i .. 16 i + 15 of the chunk
+        float s[4][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.f;
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks) {
+            uint32_t af[4];
+            // matrices: keys 16 i + (lane & 15), dims chunk 2 ks + (lane >> 4)
+            ldsm4_(kb + swz(16 * i + (lane & 15), 2 * ks + (lane >> 4)), af);
+            mma16816(s[i], af, qh[ks][0], qh[ks][1]);
+            mma16816(s[i], af, ql[ks][0], ql[ks][1]);
+          }
+        }
+        // mask; online softmax per query column (the 8 lanes with the same t share a column pair)
+        float xa = -INFINITY, xb = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int key = j0 + 16 * i + g;
+          if (key >= kla) s[i][0] = -INFINITY;
+          if (key >= klb) s[i][1] = -INFINITY;
+          if (key + 8 >= kla) s[i][2] = -INFINITY;
+          if (key + 8 >= klb) s[i][3] = -INFINITY;
+          xa = fmaxf(xa, fmaxf(s[i][0], s[i][2]));
+          xb = fmaxf(xb, fmaxf(s[i][1], s[i][3]));
+        }
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+          xa = fmaxf(xa, __shfl_xor_sync(0xffffffffu, xa, off));
+          xb = fmaxf(xb, __shfl_xor_sync(0xffffffffu, xb, off));
+        }
+        const float na = fmaxf(ma, xa), nb = fmaxf(mb, xb);
+        const float cra = na == -INFINITY ? 1.f : (ma == -INFINITY ? 0.f : expf(ma - na));
+        const float crb = nb == -INFINITY ? 1.f : (mb == -INFINITY ? 0.f : expf(mb - nb));
+        ma = na;
+        mb = nb;
+        float pa = 0.f, pb = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          s[i][0] = s[i][0] == -INFINITY ? 0.f : expf(s[i][0] - na);
+          s[i][1] = s[i][1] == -INFINITY ? 0.f : expf(s[i][1] - nb);
+          s[i][2] = s[i][2] == -INFINITY ? 0.f : expf(s[i][2] - na);
+          s[i][3] = s[i][3] == -INFINITY ? 0.f : expf(s[i][3] - nb);
+          pa += s[i][0] + s[i][2];
+          pb += s[i][1] + s[i][3];
+          o[i][0] *= cra;
+          o[i][1] *= crb;
+          o[i][2] *= cra;
+          o[i][3] *= crb;
+        }
+        la = la * cra + pa;
+        lb = lb * crb + pb;
+        // O^T += V^T P^T: k-step i = keys 16 i .. 16 i + 15; m-tiles of 16 dims
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          // P^T halves as the B operand: transpose the (key, query) 8 x 8 blocks in registers
+          uint32_t h0, l0, h1, l1;
+          split2(s[i][0], s[i][1], h0, l0);
+          split2(s[i][2], s[i][3], h1, l1);
+          const uint32_t bh0 = movt(h0), bh1 = movt(h1), bl0 = movt(l0), bl1 = movt(l1);
+#pragma unroll
+          for (int dm = 0; dm < 4; ++dm) {
+            uint32_t af[4];
+            // matrices (transposed): keys 16 i + 8 (lane >> 4) + (lane & 7), dims chunk 2 dm + ((lane >> 3) & 1)
+            ldsm4t(vb + swz(16 * i + 8 * (lane >> 4) + (lane & 7), 2 * dm + ((lane >> 3) & 1)), af);
+            mma16816(o[dm], af, bh0, bh1);
+            mma16816(o[dm], af, bl0, bl1);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a3_su32(&empty[st])) : "memory");
+      }
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {
+        la += __shfl_xor_sync(0xffffffffu, la, off);
+        lb += __shfl_xor_sync(0xffffffffu, lb, off);
+      }
+    }
+    __syncthreads();  // every warp is done with the ring: it now holds the warps' partial results
+    if (warp < kA4Warps) {
+      float* ow = Ow + warp * QT * HD;
+#pragma unroll
+      for (int dm = 0; dm < 4; ++dm) {
+        ow[(2 * t) * HD + 16 * dm + g] = o[dm][0];
+        ow[(2 * t + 1) * HD + 16 * dm + g] = o[dm][1];
+        ow[(2 * t) * HD + 16 * dm + g + 8] = o[dm][2];
+        ow[(2 * t + 1) * HD + 16 * dm + g + 8] = o[dm][3];
+      }
+      if (g == 0) {
+        mw[warp * QT + 2 * t] = ma;
+        lw[warp * QT + 2 * t] = la;
+        mw[warp * QT + 2 * t + 1] = mb;
+        lw[warp * QT + 2 * t + 1] = lb;
+      }
+    }
+    __syncthreads();
+    // combine the warps: this split's (max, sum, accumulator) per row
+    for (int idx = tid; idx < QT * HD; idx += kA4Threads) {
+      const int i = idx / HD, dd = idx - i * HD;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kA4Warps; ++w) M = fmaxf(M, mw[w * QT + i]);
+      float L = 0.f, ov = 0.f;
+#pragma unroll
+      for (int w = 0; w < kA4Warps; ++w) {
+        const float mv = mw[w * QT + i];
+        const float f = mv == -INFINITY ? 0.f : expf(mv - M);
+        L += f * lw[w * QT + i];
+        ov += f * Ow[(w * QT + i) * HD + dd];
+      }
+      pacc[idx] = ov;
+      if (dd == 0) {
+        s_m[i] = M;
+        s_l[i] = L;
+      }
+    }
+    cl.sync();
+    {
+      const int dpr = (HD + splits - 1) / splits;
+      const int d0 = sp * dpr;
+      const int nd = min(dpr, HD - d0);
+      for (int idx = tid; idx < nq * nd; idx += kA4Threads) {
+        const int i = idx / nd, dd = d0 + (idx - i * nd);
+        float mr[kMaxClusterSplit], lr[kMaxClusterSplit], ar[kMaxClusterSplit];
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
+          if (k < splits) {
+            mr[k] = *cl.map_shared_rank(&s_m[i], k);
+            lr[k] = *cl.map_shared_rank(&s_l[i], k);
+            ar[k] = *cl.map_shared_rank(&pacc[i * HD + dd], k);
+          }
+        }
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k)
+          if (k < splits) M = fmaxf(M, mr[k]);
+        float L = 0.f, ov = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMaxClusterSplit; ++k) {
+          if (k < splits && mr[k] != -INFINITY) {
+            const float w = expf(mr[k] - M);
+            L += w * lr[k];
+            ov += w * ar[k];
+          }
+        }
+        out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? ov / L : 0.f;
+      }
+    }
+    cl.sync();
+    cc += nch;
+  }
+  // after a failed wait, copies may still be in flight: wait (bounded) for the last one issued
+  // into each stage before the CTA's shared memory is released
+  if (__syncthreads_or(failed) && tid == kA4Warps * 32) {
+    for (uint32_t st = 0; st < (uint32_t)NS && st < issued; ++st) {
+      const uint32_t last = issued - 1 - ((issued - 1 - st) % NS);
+      a3_wait(&full[last % NS], (last / NS) & 1);
+    }
+    atomicOr(err, kErrTimeout | kErrWaitAttnMma);
+  }
+}
+
+template <int NS>
+size_t attn_mmt_smem() {
+  // ring, q halves (2 x QT x 64 bf16), pacc (QT x 64 fp32), row stats, barriers
+  return 1024 + (size_t)NS * 2 * kA4Chunk + (size_t)(2 * kA5QT * 64 + 3 * kA5QT) * 4 + 2 * NS * 8 + 16;
+}
+
+template <int NS>
+void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
+                  int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
+                  cudaStream_t s) {
+  CUtensorMap tk, tv;
+  memcpy(&tk, kv.tmaps, sizeof(tk));
+  memcpy(&tv, static_cast<const unsigned char*>(kv.tmaps) + 128, sizeof(tv));
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(B, qtiles_grid, H * splits);
+  cfg.blockDim = dim3(kA4Threads);
+  cfg.dynamicSmemBytes = attn_mmt_smem<NS>();
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = splits;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++g_launches;
+  cudaLaunchKernelEx(&cfg, k_attn_mmt<NS>, q, out, kv, rows, H, scale, err, tk, tv, stable, stable_stride,
+                     stable_extra);
+}
+
 void launch_a4(int ns, const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
                int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
                cudaStream_t s) {
@@ -1433,6 +1797,8 @@ int make_kv_tmaps(void* out, const void* k, const void* v, long long rows) {
 void kernel_attrs_attn() {
   cudaFuncSetAttribute(k_attn_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem<4>());
   cudaFuncSetAttribute(k_attn_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem<8>());
+  cudaFuncSetAttribute(k_attn_mmt<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<4>());
+  cudaFuncSetAttribute(k_attn_mmt<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<8>());
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<float, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -1457,8 +1823,14 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
   // long caches; with few pairs, or short caches (the multi-byte window), the CUDA-core pipelined
   // kernel (three CTAs per SM) runs, spreading keys over up to 16 splits
   if (D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= 128 && !short_kv) {
-    launch_a4(D.attn_ns, q, out, kv, rows, B, D.H, D.scale, qtiles_grid, std::min(splits, kMaxClusterSplit), D.err,
-              stable, ss, stable_extra, s);
+    const int sc = std::min(splits, kMaxClusterSplit);
+    // decode steps (one query tile of a few rows per sequence): the transposed kernel
+    if (qtiles_grid == 1 && D.attn_t) {
+      if (D.attn_ns == 4) launch_a5_ns<4>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, stable, ss, stable_extra, s);
+      else launch_a5_ns<8>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, stable, ss, stable_extra, s);
+    } else {
+      launch_a4(D.attn_ns, q, out, kv, rows, B, D.H, D.scale, qtiles_grid, sc, D.err, stable, ss, stable_extra, s);
+    }
     return;
   }
   if (D.attn_pipe) {

@@ -871,6 +871,8 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.attn_pipe = ap ? atoi(ap) : 2;
     const char* an = getenv("LCA_ATTN_NS");
     D.attn_ns = an ? atoi(an) : 8;
+    const char* at = getenv("LCA_ATTN_T");
+    D.attn_t = (at && at[0] == '0') ? 0 : 1;
     const char* mk = getenv("LCA_ATTN_MIN_KEYS");
     D.attn_min_keys = mk ? std::max(0, atoi(mk)) : 0;
   }
