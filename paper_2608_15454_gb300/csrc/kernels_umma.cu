@@ -262,7 +262,7 @@ __device__ __forceinline__ void chunk_out(const EpiArgs& e, const EpiRow& q, con
 // accumulator's completion), so a row costs about one memory latency per two chunks.
 template <int BN, typename Wait>
 __device__ __forceinline__ void tile_epilogue(const EpiArgs& e, uint32_t tbase, int grow, bool ok, int n0,
-                                              float sc, Wait wait) {
+                                              float sc, Wait wait, unsigned long long* t_first = nullptr) {
   EpiRow q{0, 0, 0};
   float4 opA[8], opB[8];
   if (ok) {
@@ -278,6 +278,7 @@ __device__ __forceinline__ void tile_epilogue(const EpiArgs& e, uint32_t tbase, 
       chunk_ops(e, q, grow, n0 + cb + 32, opB);
       chunk_out<__nv_bfloat16>(e, q, opA, grow, n0 + cb, v, sc);
     }
+    if (t_first && cb == 0) *t_first = gtimer();
     tld32(tbase + (uint32_t)(cb + 32), v);
     if (ok) {
       if (cb + 64 < BN) chunk_ops(e, q, grow, n0 + cb + 64, opA);
@@ -427,12 +428,21 @@ k_split_rows(LinearArgs a, __nv_bfloat16* __restrict__ hi, __nv_bfloat16* __rest
   }
 }
 
-// Inverse RMS of a row from its sums of squares (n slots, summed in order).
+// Inverse RMS of a row from its sums of squares (n slots, summed in order): one slot, or up to 32
+// slots read as 16-byte vectors that are all in flight at once (n a multiple of 4).
 __device__ __forceinline__ float row_inv(const float* ss, int n, int ld, size_t row, int K, float eps) {
   const float* p = ss + row * ld;
   float t = 0.f;
-#pragma unroll 8
-  for (int i = 0; i < n; ++i) t += p[i];
+  if (n == 1) {
+    t = p[0];
+  } else {
+    float4 v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = 4 * i < n ? reinterpret_cast<const float4*>(p)[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) t += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+    for (int i = 32; i < n; ++i) t += p[i];
+  }
   return rsqrtf(t / (float)K + eps);
 }
 
@@ -449,7 +459,7 @@ struct TCfg {
                                      ((uint32_t)(kUM >> 4) << 24);
   // ring, barriers, TMEM address, the tile rows' inverse RMS, alignment slack
   static constexpr size_t kSmem =
-      (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16 + kUM * 4 + 16 + kUM * sizeof(EpiRow) + 1024;
+      (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16 + kUM * 4 + 32 + kUM * sizeof(EpiRow) + 1024;
   static_assert((size_t)kUM * (BN + 1) * 4 <= (size_t)kStages * kStageBytes, "reduction buffer");
 };
 
@@ -478,9 +488,9 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
   uint64_t* accdone = empty + C::kStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accdone + 1);
   float* inv_s = reinterpret_cast<float*>(accdone + 1) + 4;  // [128]
-  // traced launches: epilogue of the first row tile done (one epilogue thread), then pass end
+  // traced launches (one epilogue thread, first row tile): epilogue done, accumulator ready
   unsigned long long* tmk = reinterpret_cast<unsigned long long*>(inv_s + kUM);
-  EpiRow* meta_s = reinterpret_cast<EpiRow*>(tmk + 2);  // [128]
+  EpiRow* meta_s = reinterpret_cast<EpiRow*>(tmk + 4);  // [128]
   float* red = reinterpret_cast<float*>(ring);  // [128][BN + 1] after the MMAs of a pass
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -497,7 +507,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
       ubar_init(&full[i], 1);
       ubar_init(&empty[i], 1);
     }
-    tmk[0] = 0;
+    tmk[0] = tmk[1] = tmk[2] = 0;
     ubar_init(accdone, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
@@ -611,7 +621,9 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
           tile_epilogue<BN>(a.epi, tmem + ((uint32_t)((warp & 3) * 32) << 16), rbase + row, row < M, n0, sc, [&] {
                               wait_or_fail(accdone, ps & 1, failed);
                               asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                            });
+                              if (g_trace && ps == 0 && warp == 2 && lane == 0) tmk[1] = gtimer();
+                            },
+                            (g_trace && ps == 0 && warp == 2 && lane == 0) ? &tmk[2] : nullptr);
           if (g_trace && ps == 0 && warp == 2 && lane == 0) tmk[0] = gtimer();
         }
       } else {
@@ -622,6 +634,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
           meta_s[r] = mt * kUM + r < M ? epi_row(a.epi, rbase + mt * kUM + r) : EpiRow{0, 0, 0};
           wait_or_fail(accdone, ps & 1, failed);
           asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          if (g_trace && ps == 0 && warp == 2 && lane == 0) tmk[1] = gtimer();
 #pragma unroll
           for (int cb = 0; cb < BN; cb += 32) {
             uint32_t v[32];
@@ -637,7 +650,6 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
         cl.sync();
       }
     }
-    if (ps == 0) _trace.mark(2);
     // this pass's TMEM reads and reduction-buffer use end before the next pass's MMAs and copies
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
@@ -645,7 +657,11 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
   }
   // after a failed wait, copies may still be in flight: wait (bounded) for the last one issued
   // into each stage before the CTA's shared memory is released
-  if (g_trace) _trace.mark_at(1, tmk[0]);
+  if (g_trace) {
+    _trace.mark_at(0, tmk[2] ? tmk[2] : tmk[1]);
+    _trace.mark_at(1, tmk[1]);
+    _trace.mark_at(2, tmk[0]);
+  }
   const bool any_failed = __syncthreads_or(failed);
   if (tid == 0 && any_failed) {
     for (uint32_t s = 0; s < (uint32_t)C::kStages && s < issued; ++s) {
@@ -1226,8 +1242,12 @@ void split_gemm(const Dev& D, const LinearArgs& a, const void* amap, __nv_bfloat
   const int kb = a.Kd / kUK;
   int best_bn = 64, best_ks = 1;
   long long best = -1;
+  static const int bn_only = [] {
+    const char* e = getenv("LCA_TGEMM_BN");
+    return e ? atoi(e) : 0;
+  }();
   for (int bn : {256, 128, 64}) {
-    if (a.N % bn) continue;
+    if (a.N % bn || (bn_only && bn != bn_only)) continue;
     const long long base = (long long)(a.N / bn) * a.groups * MT;
     int ks = 1;
     while (ks < 8 && kb % (2 * ks) == 0 && kb / (2 * ks) >= 2 && base * 2 * ks <= sms) ks *= 2;

@@ -303,7 +303,7 @@ bool link_split(const Dev& D, bool tiled, LinearArgs& prod, LinearArgs& cons, in
                 bool drop_fp32) {
   cons.abuf = buf;
   cons.presplit = 1;
-  const bool ok = tiled && umma_ready(D, prod) && umma_ready(D, cons) && cons.groups == prod.groups &&
+  const bool ok = D.split_write && tiled && umma_ready(D, prod) && umma_ready(D, cons) && cons.groups == prod.groups &&
                   cons.Mg_stride == prod.Mg_stride && prod.abuf != buf && (!gain || cons.Kd == prod.N);
   if (!ok) {
     cons.presplit = 0;
@@ -871,6 +871,8 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.attn_pipe = ap ? atoi(ap) : 2;
     const char* an = getenv("LCA_ATTN_NS");
     D.attn_ns = an ? atoi(an) : 8;
+    const char* sw = getenv("LCA_SPLIT_WRITE");
+    D.split_write = (sw && sw[0] == '0') ? 0 : 1;
     const char* at = getenv("LCA_ATTN_T");
     D.attn_t = (at && at[0] == '0') ? 0 : 1;
     const char* mk = getenv("LCA_ATTN_MIN_KEYS");
