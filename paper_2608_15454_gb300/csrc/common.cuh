@@ -258,6 +258,7 @@ struct Dev {
   int attn_ns;         // ring stages of the tensor-core decode attention (4, 6 or 8)
   int attn_min_keys;   // fewest cache keys per key split of a decode attention launch
   int attn_t;          // decode steps use the transposed tensor-core attention (8-row query tiles)
+  int attn_w;          // small-batch decode steps use the warp-walk attention
   int split_write;     // tensor-core layers split their successor's input in their epilogue
   int sgemm_max_rows;  // tensor-core layers with at most this many typical rows use the skinny
                        // (weights-as-M) GEMM; 0: never

@@ -846,6 +846,223 @@ void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B
                      stable_extra);
 }
 
+// ---------------------------------------------------------------- warp-walk decode attention
+// Decode steps of small batches (bf16 caches, head_dim 64, at most 8 query rows per sequence):
+// one CTA per (sequence, head, key split) and no block barrier inside the key loop. Each warp
+// walks its own groups of four consecutive keys; a lane holds two head dims, so a key's K and V
+// rows are single 128-byte warp loads straight from the cache, and the loads of the next group
+// are in flight while the current one is reduced. The scores come from warp reductions, each
+// warp keeps its own online softmax per row, the warps combine in shared memory and the key
+// splits through distributed shared memory.
+constexpr int kAwWarps = 4;
+constexpr int kAwThreads = kAwWarps * 32;
+constexpr int kAwG = 4;  // keys per group
+
+__device__ __forceinline__ float2 aw_bf2(const __nv_bfloat16* p) {
+  const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
+  return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xFFFF0000u));
+}
+
+__global__ void __launch_bounds__(kAwThreads)
+k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err) {
+  namespace cgr = cooperative_groups;
+  constexpr int HD = 64, QT = kAttnQT;
+  __shared__ float Ow[kAwWarps][QT][HD];
+  __shared__ float mw[kAwWarps][QT], lw[kAwWarps][QT];
+  __shared__ float pacc[QT][HD];
+  __shared__ float s_m[QT], s_l[QT];
+
+  TraceScope _trace(TT_ATTN);
+  cgr::cluster_group cl = cgr::this_cluster();
+  const int splits = (int)cl.dim_blocks().z;
+  const int sp = (int)cl.block_rank();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  pdl_trigger();
+  pdl_wait();
+  _trace.waited();
+  const int b = blockIdx.x;
+  const int h = blockIdx.z / splits;
+  const int nrows = rows.seq_count[b];
+  const int rbeg = rows.seq_start[b];
+  const int ntiles = (nrows + QT - 1) / QT;
+  const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
+  const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  const int ld = H * HD;
+
+  for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
+    const int r0 = rbeg + qt * QT;
+    const int nq = min(QT, nrows - qt * QT);
+    // this lane's two dims of every row (pre-scaled), the rows' cache lengths
+    float2 qv[QT];
+    int kl[QT];
+    int kv_hi = 0;
+#pragma unroll
+    for (int i = 0; i < QT; ++i) {
+      qv[i] = make_float2(0.f, 0.f);
+      kl[i] = 0;
+      if (i < nq) {
+        const float2 t = *reinterpret_cast<const float2*>(q + (size_t)(r0 + i) * ld + h * HD + 2 * lane);
+        qv[i] = make_float2(t.x * scale, t.y * scale);
+        int k = rows.kvlen[r0 + i];
+        if (k > kv.S || k < 0) {
+          if (lane == 0 && warp == 0) atomicOr(err, kErrIndex);
+          k = k < 0 ? 0 : kv.S;
+        }
+        kl[i] = k;
+        kv_hi = max(kv_hi, k);
+      }
+    }
+    const int per = ((kv_hi + splits - 1) / splits + kAwG - 1) / kAwG * kAwG;
+    const int lo = sp * per;
+    const int hi = min(kv_hi, lo + per);
+    float m[QT], l[QT];
+    float2 acc[QT];
+#pragma unroll
+    for (int i = 0; i < QT; ++i) {
+      m[i] = -INFINITY;
+      l[i] = 0.f;
+      acc[i] = make_float2(0.f, 0.f);
+    }
+    // groups j0 = lo + kAwG (warp + kAwWarps g); the next group's rows load during this one
+    int j0 = lo + kAwG * warp;
+    float2 kc[kAwG], vc[kAwG];
+#pragma unroll
+    for (int u = 0; u < kAwG; ++u) {
+      const int j = j0 + u;
+      kc[u] = j < hi ? aw_bf2(Kc + (size_t)j * HD + 2 * lane) : make_float2(0.f, 0.f);
+      vc[u] = j < hi ? aw_bf2(Vc + (size_t)j * HD + 2 * lane) : make_float2(0.f, 0.f);
+    }
+    for (; j0 < hi; j0 += kAwG * kAwWarps) {
+      const int jn = j0 + kAwG * kAwWarps;
+      float2 kn[kAwG], vn[kAwG];
+#pragma unroll
+      for (int u = 0; u < kAwG; ++u) {
+        const int j = jn + u;
+        kn[u] = j < hi ? aw_bf2(Kc + (size_t)j * HD + 2 * lane) : make_float2(0.f, 0.f);
+        vn[u] = j < hi ? aw_bf2(Vc + (size_t)j * HD + 2 * lane) : make_float2(0.f, 0.f);
+      }
+#pragma unroll
+      for (int i = 0; i < QT; ++i) {
+        if (i >= nq) break;  // warp-uniform
+        float s[kAwG];
+#pragma unroll
+        for (int u = 0; u < kAwG; ++u) s[u] = qv[i].x * kc[u].x + qv[i].y * kc[u].y;
+#pragma unroll
+        for (int o = 16; o; o >>= 1)
+#pragma unroll
+          for (int u = 0; u < kAwG; ++u) s[u] += __shfl_xor_sync(0xffffffffu, s[u], o);
+        float mx = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < kAwG; ++u) {
+          if (j0 + u >= hi || j0 + u >= kl[i]) s[u] = -INFINITY;
+          mx = fmaxf(mx, s[u]);
+        }
+        if (mx == -INFINITY) continue;
+        const float mn = fmaxf(m[i], mx);
+        const float cr = m[i] == -INFINITY ? 0.f : __expf(m[i] - mn);
+        float ps = 0.f;
+        float2 a = make_float2(acc[i].x * cr, acc[i].y * cr);
+#pragma unroll
+        for (int u = 0; u < kAwG; ++u) {
+          const float p = s[u] == -INFINITY ? 0.f : __expf(s[u] - mn);
+          ps += p;
+          a.x = fmaf(p, vc[u].x, a.x);
+          a.y = fmaf(p, vc[u].y, a.y);
+        }
+        acc[i] = a;
+        l[i] = l[i] * cr + ps;
+        m[i] = mn;
+      }
+#pragma unroll
+      for (int u = 0; u < kAwG; ++u) {
+        kc[u] = kn[u];
+        vc[u] = vn[u];
+      }
+    }
+    // combine the warps: this split's (max, sum, accumulator) per row
+#pragma unroll
+    for (int i = 0; i < QT; ++i) {
+      *reinterpret_cast<float2*>(&Ow[warp][i][2 * lane]) = acc[i];
+      if (lane == 0) {
+        mw[warp][i] = m[i];
+        lw[warp][i] = l[i];
+      }
+    }
+    __syncthreads();
+    for (int idx = tid; idx < QT * HD; idx += kAwThreads) {
+      const int i = idx / HD, dd = idx - i * HD;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kAwWarps; ++w) M = fmaxf(M, mw[w][i]);
+      float L = 0.f, ov = 0.f;
+#pragma unroll
+      for (int w = 0; w < kAwWarps; ++w) {
+        const float f = mw[w][i] == -INFINITY ? 0.f : __expf(mw[w][i] - M);
+        L += f * lw[w][i];
+        ov += f * Ow[w][i][dd];
+      }
+      pacc[i][dd] = ov;
+      if (dd == 0) {
+        s_m[i] = M;
+        s_l[i] = L;
+      }
+    }
+    cl.sync();
+    {
+      const int dpr = (HD + splits - 1) / splits;
+      const int d0 = sp * dpr;
+      const int nd = min(dpr, HD - d0);
+      for (int idx = tid; idx < nq * nd; idx += kAwThreads) {
+        const int i = idx / nd, dd = d0 + (idx - i * nd);
+        float mr[kA4MaxSplit], lr[kA4MaxSplit], ar[kA4MaxSplit];
+#pragma unroll
+        for (int k = 0; k < kA4MaxSplit; ++k) {
+          if (k < splits) {
+            mr[k] = *cl.map_shared_rank(&s_m[i], k);
+            lr[k] = *cl.map_shared_rank(&s_l[i], k);
+            ar[k] = *cl.map_shared_rank(&pacc[i][dd], k);
+          }
+        }
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kA4MaxSplit; ++k)
+          if (k < splits) M = fmaxf(M, mr[k]);
+        float L = 0.f, ov = 0.f;
+#pragma unroll
+        for (int k = 0; k < kA4MaxSplit; ++k) {
+          if (k < splits && mr[k] != -INFINITY) {
+            const float w = __expf(mr[k] - M);
+            L += w * lr[k];
+            ov += w * ar[k];
+          }
+        }
+        out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? ov / L : 0.f;
+      }
+    }
+    cl.sync();  // peers are done reading this tile's partials
+  }
+}
+
+void launch_aw(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale, int splits,
+               int* err, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(B, 1, H * splits);
+  cfg.blockDim = dim3(kAwThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = splits;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  ++g_launches;
+  cudaLaunchKernelEx(&cfg, k_attn_w, q, out, kv, rows, H, scale, err);
+}
+
 // ---------------------------------------------------------------- tensor-core decode attention
 // bf16 caches with head_dim 64. One CTA serves (sequence, query tile of up to 16 rows, head, key
 // split): a producer warp streams 64-key chunks of K and V by TMA (128-byte swizzle) through a
@@ -1800,6 +2017,7 @@ void kernel_attrs_attn() {
   cudaFuncSetAttribute(k_attn_mmt<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<4>());
   cudaFuncSetAttribute(k_attn_mmt<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<8>());
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(k_attn_w, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<float, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<float, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -1835,6 +2053,11 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
   }
   if (D.attn_pipe) {
     splits = std::min(splits, kA4MaxSplit);
+    // decode steps (one query tile per sequence) of bf16 head-dim-64 caches: the warp-walk kernel
+    if (qtiles_grid == 1 && D.attn_w && D.dtype == LCA_BF16 && D.hd == 64) {
+      launch_aw(q, out, kv, rows, B, D.H, D.scale, splits, D.err, s);
+      return;
+    }
     if (D.dtype == LCA_BF16) {
       if (D.hd == 64) launch_a3<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
       else launch_a3<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);

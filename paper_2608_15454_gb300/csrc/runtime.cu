@@ -873,6 +873,8 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.attn_ns = an ? atoi(an) : 8;
     const char* sw = getenv("LCA_SPLIT_WRITE");
     D.split_write = (sw && sw[0] == '0') ? 0 : 1;
+    const char* aw = getenv("LCA_ATTN_W");
+    D.attn_w = (aw && aw[0] == '0') ? 0 : 1;
     const char* at = getenv("LCA_ATTN_T");
     D.attn_t = (at && at[0] == '0') ? 0 : 1;
     const char* mk = getenv("LCA_ATTN_MIN_KEYS");
