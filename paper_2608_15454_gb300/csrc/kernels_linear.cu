@@ -339,8 +339,10 @@ __device__ __forceinline__ void prefetch_next(const LinearArgs& a) {
 // processed in chunks of MCA. With a K-split the `ksplit` CTAs of a column tile form a thread-
 // block cluster: each leaves its partial sums in its own shared memory and rank 0 adds the ranks'
 // partials through distributed shared memory in rank order (no global scratch).
+// (512 threads per SM by registers, four CTAs of four warps, so that a 512-tile launch is resident
+// in one wave)
 template <int MCA, int NW, bool NORM>
-__global__ void __launch_bounds__(NW * 32, 1)
+__global__ void __launch_bounds__(NW * 32, 16 / NW)
 k_gemv_bulk(LinearArgs a, int ksplit) {
   TraceScope _trace(TT_GEMV);
   namespace cgr = cooperative_groups;

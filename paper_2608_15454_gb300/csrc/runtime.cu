@@ -6,7 +6,9 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstdlib>
+#include <thread>
 #include <cstdio>
 #include <cstring>
 #include <map>
@@ -564,19 +566,40 @@ int capture_step(lca_ctx* c, cudaGraph_t g, int n, bool loop, cudaGraphCondition
   return LCA_OK;
 }
 
+// Holds a stream at a host node until release(): the launches (and profiling events) enqueued
+// meanwhile then run back to back, so the event times of a profiled eager step measure the GPU,
+// not the host's enqueue rate. The host-side wait is bounded (about five seconds).
+struct HostGate {
+  std::atomic<int> open{0};
+  static void CUDART_CB wait_fn(void* p) {
+    auto* g = static_cast<HostGate*>(p);
+    for (int i = 0; i < 5000000 && !g->open.load(std::memory_order_acquire); ++i) std::this_thread::yield();
+  }
+  void hold(cudaStream_t s) { cudaLaunchHostFunc(s, wait_fn, this); }
+  void release() { open.store(1, std::memory_order_release); }
+};
+
 // The same step as direct launches on the context stream; the LM decision is read back on
 // the host. Used for per-kernel profiling (profilers cannot see kernels inside graphs with
-// conditional nodes); results are identical to the graph.
+// conditional nodes); results are identical to the graph. When profiling, each of the two
+// segments is enqueued behind a host gate (see HostGate).
 int run_step_eager(lca_ctx* c, int n) {
   Dev& D = c->L.D;
   cudaStream_t s = c->stream;
+  const bool gate = g_prof != nullptr;
+  HostGate g1, g2;
+  if (gate) g1.hold(s);
   enqueue_draft_encode(c, n, s);
   launch_segment(D, 0, 0, s);
+  g1.release();
   int mlm = 0;
   CK(cudaMemcpyAsync(&mlm, D.r_lm.M, sizeof(int), cudaMemcpyDeviceToHost, s));
   CK(cudaStreamSynchronize(s));
+  if (gate) g2.hold(s);
   if (mlm > 0) enqueue_lm(c, n, s);
   enqueue_verify_commit(c, n, s);
+  g2.release();
+  if (gate) CK(cudaStreamSynchronize(s));  // the gate's host node has run before g2 goes away
   CK(cudaGetLastError());
   return LCA_OK;
 }
