@@ -78,6 +78,10 @@ struct TraceScope {
   __device__ __forceinline__ void mark(int i = 0) {
     if (on) mk[i] = (unsigned)(gtimer() - t0);
   }
+  // a plain value (a row count, a chunk count) in a mark slot instead of a time
+  __device__ __forceinline__ void value(int i, unsigned v) {
+    if (on) mk[i] = v;
+  }
   // a mark taken by another thread of the CTA (globaltimer value), handed over through shared memory
   __device__ __forceinline__ void mark_at(int i, unsigned long long t) {
     if (on && t > t0) mk[i] = (unsigned)(t - t0);
@@ -122,6 +126,7 @@ constexpr int kErrNumeric = 2; // non-finite logits
 constexpr int kErrTimeout = 4; // a bounded wait ran out
 // which kernel family's wait ran out (set together with kErrTimeout; reported on stderr)
 constexpr int kErrWaitAttn3 = 1 << 8, kErrWaitAttnMma = 1 << 9, kErrWaitGemv = 1 << 10, kErrWaitGemm = 1 << 11,
+              kErrWaitAttnW = 1 << 13,
               kErrWaitGemvReduce = 1 << 12;
 
 // Linear epilogues.
@@ -399,11 +404,13 @@ void kernel_attrs_linear();
 void kernel_attrs_step();
 void kernel_attrs_attn();
 // Attention of query rows over a KV-cache layer (keys [0, kvlen[r]) of sequence b[r]).
-// stable: optional per-sequence committed length (stride in ints) whose cache prefix does not
-// change during a step, prefetched into L2 before the dependency wait; stable_extra: rows added.
+// stable: optional per-sequence committed length (stride in ints) whose cache prefix (the first
+// stable + stable_add slots) does not change during a step: prefetched into L2, or staged in
+// shared memory, before the dependency wait; stable_extra: rows added; rows_seq: the most query
+// rows a sequence has (a tile-size hint).
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s, const int* stable = nullptr,
-               int stable_extra = 0, bool short_kv = false);
+               int stable_extra = 0, bool short_kv = false, int stable_add = 0, int rows_seq = kAttnQT);
 
 // Step / prefill glue kernels (kernels_step.cu).
 void launch_mb_plan(const Dev& D, cudaStream_t s);

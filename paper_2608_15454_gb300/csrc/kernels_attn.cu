@@ -848,148 +848,232 @@ void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B
 
 // ---------------------------------------------------------------- warp-walk decode attention
 // Decode steps of small batches (bf16 caches, head_dim 64, at most 8 query rows per sequence):
-// one CTA per (sequence, head, key split) and no block barrier inside the key loop. Each warp
-// walks its own groups of four consecutive keys; a lane holds two head dims, so a key's K and V
-// rows are single 128-byte warp loads straight from the cache, and the loads of the next group
-// are in flight while the current one is reduced. The scores come from warp reductions, each
-// warp keeps its own online softmax per row, the warps combine in shared memory and the key
-// splits through distributed shared memory.
+// one CTA per (sequence, head, key split) and no block barrier inside the key loop.
+//
+// Cache slots below the sequence's committed length (`stable`, read from the sequence state, plus
+// `stable_add`) are not written during a decode step, and a step starts only once the step before
+// it has completed (graph launches, and the iterations of the generate loop, run in stream
+// order). So, before the grid-dependency wait, each CTA copies its share of those slots (up to
+// `stage_cap` keys of K and V) into shared memory with two bulk copies on an mbarrier, while its
+// predecessors (the Q/K/V layer that appends this step's rows) are still running. After the wait
+// only the query rows, the cache lengths and the keys appended in this step (or stable keys past
+// the staging capacity) come from global memory.
+//
+// Keys of a CTA: an equal share of the stable slots [0, S) per split, then an equal share of the
+// slots [S, kv_hi) appended in this step. Each warp walks its own groups of four keys; a lane
+// holds two head dims, so a key's K and V rows are single 128-byte warp reads. The scores come from
+// warp reductions, each warp keeps its own online softmax per row, the warps combine in shared
+// memory and the key splits through distributed shared memory. Without `stable` (S = 0) the whole
+// range is split evenly and read from global memory.
 constexpr int kAwWarps = 4;
 constexpr int kAwThreads = kAwWarps * 32;
-constexpr int kAwG = 4;  // keys per group
+constexpr int kAwG = 4;           // keys per group
+constexpr int kAwStageMax = 256;  // keys staged per CTA (64 KB of K and V)
 
 __device__ __forceinline__ float2 aw_bf2(const __nv_bfloat16* p) {
   const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
   return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xFFFF0000u));
 }
 
-__global__ void __launch_bounds__(kAwThreads)
-k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err) {
+// [lo, hi) of split sp when n keys starting at base are shared in groups of kAwG
+__device__ __forceinline__ void aw_share(int base, int n, int splits, int sp, int& lo, int& hi) {
+  const int per = ((n + splits - 1) / splits + kAwG - 1) / kAwG * kAwG;
+  lo = base + min(n, sp * per);
+  hi = base + min(n, sp * per + per);
+}
+
+template <int QT>
+__global__ void __launch_bounds__(kAwThreads, QT <= 4 ? 3 : 2)
+k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
+         const int* __restrict__ stable, int stable_stride, int stable_add, int stage_cap) {
   namespace cgr = cooperative_groups;
-  constexpr int HD = 64, QT = kAttnQT;
+  constexpr int HD = 64;
   __shared__ float Ow[kAwWarps][QT][HD];
   __shared__ float mw[kAwWarps][QT], lw[kAwWarps][QT];
   __shared__ float pacc[QT][HD];
   __shared__ float s_m[QT], s_l[QT];
+  __shared__ __align__(16) float qs[QT][HD];
+  __shared__ int s_kl[QT];
+  __shared__ __align__(8) uint64_t s_bar;   // the staged keys
+  __shared__ __align__(8) uint64_t s_rbar;  // rank 0: the peers' partials have arrived
+  __shared__ int s_stage[3];  // S, first staged slot, staged keys
+  extern __shared__ __align__(128) unsigned char aw_dyn[];
+  __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(aw_dyn);  // [stage_cap][HD]
+  __nv_bfloat16* Vs = Ks + (size_t)stage_cap * HD;                // [stage_cap][HD]
+  float* rbuf = reinterpret_cast<float*>(Vs + (size_t)stage_cap * HD);  // rank 0: [splits][QT][HD]
 
   TraceScope _trace(TT_ATTN);
   cgr::cluster_group cl = cgr::this_cluster();
   const int splits = (int)cl.dim_blocks().z;
   const int sp = (int)cl.block_rank();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  pdl_trigger();
-  pdl_wait();
-  _trace.waited();
+  float* rm = rbuf + (size_t)splits * QT * HD;  // rank 0: [splits][QT] maxima
+  float* rl = rm + splits * QT;                  // rank 0: [splits][QT] sums
   const int b = blockIdx.x;
   const int h = blockIdx.z / splits;
+  const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
+  const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  pdl_trigger();
+  if (tid == 0) {
+    int S = 0, slo = 0, nst = 0;
+    if (stable) {
+      S = stable[(size_t)b * stable_stride] + stable_add;
+      S = S < 0 ? 0 : (S > kv.S ? kv.S : S);
+      int shi;
+      aw_share(0, S, splits, sp, slo, shi);
+      nst = min(shi - slo, stage_cap);
+    }
+    s_stage[0] = S;
+    s_stage[1] = slo;
+    s_stage[2] = nst;
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&s_bar)) : "memory");
+    if (sp == 0 && splits > 1)
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a3_su32(&s_rbar)), "r"(splits - 1) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (nst > 0) {
+      const uint32_t bytes = (uint32_t)(nst * HD * 2);
+      a3_expect(&s_bar, 2 * bytes);
+      a3_copy(Ks, Kc + (size_t)slo * HD, bytes, &s_bar);
+      a3_copy(Vs, Vc + (size_t)slo * HD, bytes, &s_bar);
+    }
+  }
+  // rank 0's arrival barrier exists before any peer can arrive on it (a cluster barrier before
+  // the dependency wait, off the critical path)
+  if (splits > 1) cl.sync();
+  else __syncthreads();
+  const int S = s_stage[0], slo = s_stage[1], nst = s_stage[2];
+  bool staged = nst == 0;  // the staged keys have landed (or there are none)
+  pdl_wait();
+  _trace.waited();
   const int nrows = rows.seq_count[b];
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
-  const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
-  const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
   const int ld = H * HD;
 
+  const int g = lane >> 3, e = lane & 7;  // key slot of this lane in a warp step, its 8 head dims
   for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
     const int r0 = rbeg + qt * QT;
     const int nq = min(QT, nrows - qt * QT);
-    // this lane's two dims of every row (pre-scaled), the rows' cache lengths
-    float2 qv[QT];
+    // the tile's query rows (pre-scaled) and cache lengths in shared memory
+    for (int idx = tid; idx < QT * HD / 4; idx += kAwThreads) {
+      const int i = idx / (HD / 4), c4 = idx - i * (HD / 4);
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (i < nq) {
+        v = *reinterpret_cast<const float4*>(q + (size_t)(r0 + i) * ld + h * HD + 4 * c4);
+        v.x *= scale; v.y *= scale; v.z *= scale; v.w *= scale;
+      }
+      *reinterpret_cast<float4*>(&qs[i][4 * c4]) = v;
+    }
+    if (tid < QT) {
+      int k = 0;
+      if (tid < nq) {
+        k = rows.kvlen[r0 + tid];
+        if (k > kv.S || k < 0) {
+          atomicOr(err, kErrIndex);
+          k = k < 0 ? 0 : kv.S;
+        }
+      }
+      s_kl[tid] = k;
+    }
+    __syncthreads();
     int kl[QT];
     int kv_hi = 0;
 #pragma unroll
     for (int i = 0; i < QT; ++i) {
-      qv[i] = make_float2(0.f, 0.f);
-      kl[i] = 0;
-      if (i < nq) {
-        const float2 t = *reinterpret_cast<const float2*>(q + (size_t)(r0 + i) * ld + h * HD + 2 * lane);
-        qv[i] = make_float2(t.x * scale, t.y * scale);
-        int k = rows.kvlen[r0 + i];
-        if (k > kv.S || k < 0) {
-          if (lane == 0 && warp == 0) atomicOr(err, kErrIndex);
-          k = k < 0 ? 0 : kv.S;
-        }
-        kl[i] = k;
-        kv_hi = max(kv_hi, k);
-      }
+      kl[i] = s_kl[i];
+      kv_hi = max(kv_hi, kl[i]);
     }
-    const int per = ((kv_hi + splits - 1) / splits + kAwG - 1) / kAwG * kAwG;
-    const int lo = sp * per;
-    const int hi = min(kv_hi, lo + per);
-    float m[QT], l[QT];
-    float2 acc[QT];
+    // this split's keys: stable slots [slo2, shi) (the first nst_ok of them staged), then new slots
+    // [nlo, nhi); virtual key v < nsk is slot slo2 + v, else slot nlo + v - nsk
+    int slo2, shi, nlo, nhi;
+    aw_share(0, min(S, kv_hi), splits, sp, slo2, shi);
+    aw_share(S, max(kv_hi - S, 0), splits, sp, nlo, nhi);
+    const int nsk = shi - slo2;
+    const int nv = nsk + (nhi - nlo);
+    const int nst_ok = slo2 == slo ? min(nst, nsk) : 0;  // staged keys usable for this range
+    if (!staged) {
+      if (!a3_wait(&s_bar, 0) && lane == 0 && warp == 0) atomicOr(err, kErrTimeout | kErrWaitAttnW);
+      staged = true;
+    }
+    if (qt == (int)blockIdx.y) _trace.mark(0);  // staged keys landed
+    // each group of 8 lanes walks its own keys (key v0 + g of every warp step) with its own online
+    // softmax per row; a lane holds 8 head dims of the key, so a score is 8 FMAs and 3 shuffles
+    float m[QT], l[QT], acc[QT][8];
 #pragma unroll
     for (int i = 0; i < QT; ++i) {
       m[i] = -INFINITY;
       l[i] = 0.f;
-      acc[i] = make_float2(0.f, 0.f);
-    }
-    // groups j0 = lo + kAwG (warp + kAwWarps g); the next group's rows load during this one
-    int j0 = lo + kAwG * warp;
-    float2 kc[kAwG], vc[kAwG];
 #pragma unroll
-    for (int u = 0; u < kAwG; ++u) {
-      const int j = j0 + u;
-      kc[u] = j < hi ? aw_bf2(Kc + (size_t)j * HD + 2 * lane) : make_float2(0.f, 0.f);
-      vc[u] = j < hi ? aw_bf2(Vc + (size_t)j * HD + 2 * lane) : make_float2(0.f, 0.f);
+      for (int d = 0; d < 8; ++d) acc[i][d] = 0.f;
     }
-    for (; j0 < hi; j0 += kAwG * kAwWarps) {
-      const int jn = j0 + kAwG * kAwWarps;
-      float2 kn[kAwG], vn[kAwG];
-#pragma unroll
-      for (int u = 0; u < kAwG; ++u) {
-        const int j = jn + u;
-        kn[u] = j < hi ? aw_bf2(Kc + (size_t)j * HD + 2 * lane) : make_float2(0.f, 0.f);
-        vn[u] = j < hi ? aw_bf2(Vc + (size_t)j * HD + 2 * lane) : make_float2(0.f, 0.f);
+    for (int v0 = kAwG * warp; v0 < nv; v0 += kAwG * kAwWarps) {
+      const int v = v0 + g;
+      const bool valid = v < nv;
+      const int j = v < nsk ? slo2 + v : nlo + v - nsk;
+      uint4 ku = make_uint4(0u, 0u, 0u, 0u), vu = ku;
+      if (valid) {
+        if (v < nst_ok) {
+          ku = *reinterpret_cast<const uint4*>(Ks + (size_t)v * HD + 8 * e);
+          vu = *reinterpret_cast<const uint4*>(Vs + (size_t)v * HD + 8 * e);
+        } else {
+          ku = *reinterpret_cast<const uint4*>(Kc + (size_t)j * HD + 8 * e);
+          vu = *reinterpret_cast<const uint4*>(Vc + (size_t)j * HD + 8 * e);
+        }
       }
+      float kf[8], vf[8];
+      unpack16(ku, kf, (const __nv_bfloat16*)nullptr);
+      unpack16(vu, vf, (const __nv_bfloat16*)nullptr);
+      // every row of the tile (rows past nq have no keys and stay empty): independent chains
 #pragma unroll
       for (int i = 0; i < QT; ++i) {
-        if (i >= nq) break;  // warp-uniform
-        float s[kAwG];
+        const float4 qa = *reinterpret_cast<const float4*>(&qs[i][8 * e]);
+        const float4 qb = *reinterpret_cast<const float4*>(&qs[i][8 * e + 4]);
+        float sc = qa.x * kf[0];
+        sc = fmaf(qa.y, kf[1], sc); sc = fmaf(qa.z, kf[2], sc); sc = fmaf(qa.w, kf[3], sc);
+        sc = fmaf(qb.x, kf[4], sc); sc = fmaf(qb.y, kf[5], sc); sc = fmaf(qb.z, kf[6], sc);
+        sc = fmaf(qb.w, kf[7], sc);
+        sc += __shfl_xor_sync(0xffffffffu, sc, 1);
+        sc += __shfl_xor_sync(0xffffffffu, sc, 2);
+        sc += __shfl_xor_sync(0xffffffffu, sc, 4);
+        if (!valid || j >= kl[i]) sc = -INFINITY;
+        const float mn = fmaxf(m[i], sc);
+        const float cr = mn == -INFINITY ? 1.f : __expf(m[i] - mn);
+        const float p = sc == -INFINITY ? 0.f : __expf(sc - mn);
 #pragma unroll
-        for (int u = 0; u < kAwG; ++u) s[u] = qv[i].x * kc[u].x + qv[i].y * kc[u].y;
-#pragma unroll
-        for (int o = 16; o; o >>= 1)
-#pragma unroll
-          for (int u = 0; u < kAwG; ++u) s[u] += __shfl_xor_sync(0xffffffffu, s[u], o);
-        float mx = -INFINITY;
-#pragma unroll
-        for (int u = 0; u < kAwG; ++u) {
-          if (j0 + u >= hi || j0 + u >= kl[i]) s[u] = -INFINITY;
-          mx = fmaxf(mx, s[u]);
-        }
-        if (mx == -INFINITY) continue;
-        const float mn = fmaxf(m[i], mx);
-        const float cr = m[i] == -INFINITY ? 0.f : __expf(m[i] - mn);
-        float ps = 0.f;
-        float2 a = make_float2(acc[i].x * cr, acc[i].y * cr);
-#pragma unroll
-        for (int u = 0; u < kAwG; ++u) {
-          const float p = s[u] == -INFINITY ? 0.f : __expf(s[u] - mn);
-          ps += p;
-          a.x = fmaf(p, vc[u].x, a.x);
-          a.y = fmaf(p, vc[u].y, a.y);
-        }
-        acc[i] = a;
-        l[i] = l[i] * cr + ps;
+        for (int d = 0; d < 8; ++d) acc[i][d] = fmaf(p, vf[d], acc[i][d] * cr);
+        l[i] = fmaf(l[i], cr, p);
         m[i] = mn;
       }
-#pragma unroll
-      for (int u = 0; u < kAwG; ++u) {
-        kc[u] = kn[u];
-        vc[u] = vn[u];
-      }
     }
-    // combine the warps: this split's (max, sum, accumulator) per row
+    if (qt == (int)blockIdx.y) _trace.mark(1);  // this warp's keys done
+    // combine the four key slots of the warp (lanes e, e + 8, e + 16, e + 24), then the warps
 #pragma unroll
     for (int i = 0; i < QT; ++i) {
-      *reinterpret_cast<float2*>(&Ow[warp][i][2 * lane]) = acc[i];
-      if (lane == 0) {
-        mw[warp][i] = m[i];
-        lw[warp][i] = l[i];
+      if (i >= nq) break;
+      float M = fmaxf(m[i], __shfl_xor_sync(0xffffffffu, m[i], 8));
+      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 16));
+      const float f = m[i] == -INFINITY ? 0.f : __expf(m[i] - M);
+      float L = l[i] * f;
+      L += __shfl_xor_sync(0xffffffffu, L, 8);
+      L += __shfl_xor_sync(0xffffffffu, L, 16);
+      float o[8];
+#pragma unroll
+      for (int d = 0; d < 8; ++d) {
+        o[d] = acc[i][d] * f;
+        o[d] += __shfl_xor_sync(0xffffffffu, o[d], 8);
+        o[d] += __shfl_xor_sync(0xffffffffu, o[d], 16);
+      }
+      if (g == 0) {
+        *reinterpret_cast<float4*>(&Ow[warp][i][8 * e]) = make_float4(o[0], o[1], o[2], o[3]);
+        *reinterpret_cast<float4*>(&Ow[warp][i][8 * e + 4]) = make_float4(o[4], o[5], o[6], o[7]);
+        if (e == 0) {
+          mw[warp][i] = M;
+          lw[warp][i] = L;
+        }
       }
     }
     __syncthreads();
-    for (int idx = tid; idx < QT * HD; idx += kAwThreads) {
+    for (int idx = tid; idx < nq * HD; idx += kAwThreads) {
       const int i = idx / HD, dd = idx - i * HD;
       float M = -INFINITY;
 #pragma unroll
@@ -1007,7 +1091,67 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
         s_l[i] = L;
       }
     }
+    if (ntiles <= (int)gridDim.y) {
+      // one tile per CTA: the peers push their partials into rank 0's shared memory and arrive on
+      // its barrier (release, cluster scope), then leave; rank 0 waits, combines in split order
+      // and stores the rows. No cluster barrier on the critical path.
+      __syncthreads();  // this CTA's partials are complete
+      if (sp != 0) {
+        float* dst = cl.map_shared_rank(rbuf, 0) + (size_t)sp * QT * HD;
+        for (int idx = tid; idx < nq * HD; idx += kAwThreads) dst[idx] = (&pacc[0][0])[idx];
+        if (tid < nq) {
+          cl.map_shared_rank(rm, 0)[sp * QT + tid] = s_m[tid];
+          cl.map_shared_rank(rl, 0)[sp * QT + tid] = s_l[tid];
+        }
+        __syncthreads();
+        if (tid == 0) {
+          uint32_t remote;
+          asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(a3_su32(&s_rbar)), "r"(0));
+          asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+        }
+        if (qt == (int)blockIdx.y) _trace.mark(2);  // partials pushed
+      } else {
+        if (tid == 0 && splits > 1) {
+          bool ok = false;
+          for (int it = 0; it < kA3Spins && !ok; ++it) {
+            uint32_t done;
+            asm volatile(
+                "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], 0;\n"
+                " selp.u32 %0, 1, 0, p;\n}"
+                : "=r"(done)
+                : "r"(a3_su32(&s_rbar))
+                : "memory");
+            ok = done != 0;
+          }
+          if (!ok) atomicOr(err, kErrTimeout | kErrWaitAttnW);
+        }
+        __syncthreads();
+        if (qt == (int)blockIdx.y) _trace.mark(2);  // every split's partials ready
+        for (int idx = tid; idx < nq * HD; idx += kAwThreads) {
+          const int i = idx / HD, dd = idx - i * HD;
+          float M = s_m[i];
+          for (int k = 1; k < splits; ++k) M = fmaxf(M, rm[k * QT + i]);
+          float L = 0.f, ov = 0.f;
+          if (s_m[i] != -INFINITY) {
+            const float w = __expf(s_m[i] - M);
+            L = w * s_l[i];
+            ov = w * pacc[i][dd];
+          }
+          for (int k = 1; k < splits; ++k) {
+            const float mk = rm[k * QT + i];
+            if (mk != -INFINITY) {
+              const float w = __expf(mk - M);
+              L += w * rl[k * QT + i];
+              ov += w * rbuf[((size_t)k * QT + i) * HD + dd];
+            }
+          }
+          out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? ov / L : 0.f;
+        }
+      }
+      continue;
+    }
     cl.sync();
+    if (qt == (int)blockIdx.y) _trace.mark(2);  // every split's partials ready
     {
       const int dpr = (HD + splits - 1) / splits;
       const int d0 = sp * dpr;
@@ -1041,14 +1185,25 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
     }
     cl.sync();  // peers are done reading this tile's partials
   }
+  // no rows: the staged copies must still land before the CTA leaves (bounded)
+  if (!staged && !a3_wait(&s_bar, 0) && tid == 0) atomicOr(err, kErrTimeout | kErrWaitAttnW);
+}
+
+// Keys staged per CTA of k_attn_w for a cache of S slots in `splits` splits (0: no staging).
+int aw_stage_cap(int S, int splits, bool stable) {
+  if (!stable) return 0;
+  const int per = ((S + splits - 1) / splits + kAwG - 1) / kAwG * kAwG;
+  return std::min(per, kAwStageMax);
 }
 
 void launch_aw(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale, int splits,
-               int* err, cudaStream_t s) {
+               int* err, const int* stable, int stable_stride, int stable_add, int rows_seq, cudaStream_t s) {
+  const int cap = aw_stage_cap(kv.S, splits, stable != nullptr);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, 1, H * splits);
   cfg.blockDim = dim3(kAwThreads);
-  cfg.dynamicSmemBytes = 0;
+  const int qt = rows_seq <= 4 ? 4 : kAttnQT;
+  cfg.dynamicSmemBytes = (size_t)cap * 64 * 2 * 2 + (splits > 1 ? (size_t)splits * qt * (64 + 2) * 4 : 0);
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -1060,7 +1215,12 @@ void launch_aw(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn_w, q, out, kv, rows, H, scale, err);
+  // query tiles of 4 rows when a sequence has at most 4 (fewer registers: three CTAs per SM)
+  if (qt == 4)
+    cudaLaunchKernelEx(&cfg, k_attn_w<4>, q, out, kv, rows, H, scale, err, stable, stable_stride, stable_add, cap);
+  else
+    cudaLaunchKernelEx(&cfg, k_attn_w<kAttnQT>, q, out, kv, rows, H, scale, err, stable, stable_stride, stable_add,
+                       cap);
 }
 
 // ---------------------------------------------------------------- tensor-core decode attention
@@ -2017,7 +2177,12 @@ void kernel_attrs_attn() {
   cudaFuncSetAttribute(k_attn_mmt<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<4>());
   cudaFuncSetAttribute(k_attn_mmt<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<8>());
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  cudaFuncSetAttribute(k_attn_w, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(k_attn_w<4>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(k_attn_w<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       kAwStageMax * 64 * 2 * 2 + kA4MaxSplit * 4 * (64 + 2) * 4);
+  cudaFuncSetAttribute(k_attn_w<kAttnQT>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(k_attn_w<kAttnQT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       kAwStageMax * 64 * 2 * 2 + kA4MaxSplit * kAttnQT * (64 + 2) * 4);
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<float, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<float, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -2033,8 +2198,11 @@ void kernel_attrs_attn() {
 
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s, const int* stable, int stable_extra,
-               bool short_kv) {
+               bool short_kv, int stable_add, int rows_seq) {
   ProfScope ps(PK_ATTN, 0.0, s);
+  const int* stable_aw = stable;
+  // the other kernels take `stable` as the committed byte length of an L2 prefetch hint
+  if (stable_add != 0) stable = nullptr;
   if (splits < 1) splits = 1;
   const int ss = (int)(sizeof(SeqState) / sizeof(int));
   // the tensor-core kernel holds two CTAs per SM: it pays off with many (sequence, head) pairs over
@@ -2055,7 +2223,7 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
     splits = std::min(splits, kA4MaxSplit);
     // decode steps (one query tile per sequence) of bf16 head-dim-64 caches: the warp-walk kernel
     if (qtiles_grid == 1 && D.attn_w && D.dtype == LCA_BF16 && D.hd == 64) {
-      launch_aw(q, out, kv, rows, B, D.H, D.scale, splits, D.err, s);
+      launch_aw(q, out, kv, rows, B, D.H, D.scale, splits, D.err, stable_aw, ss, stable_add, rows_seq, s);
       return;
     }
     if (D.dtype == LCA_BF16) {

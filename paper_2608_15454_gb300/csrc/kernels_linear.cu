@@ -448,6 +448,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
         }
       }
     }
+    if (r0 == 0) _trace.mark(0);  // first row chunk loaded and staged
     if (NORM) {
       // per-warp partial sums of squares over this CTA's K range (no atomics: summed in warp order)
 #pragma unroll
@@ -467,6 +468,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
     } else {
       __syncthreads();
     }
+    if (r0 == 0) _trace.mark(1);  // weights in shared memory
     if (NORM && tid < MCA) {
       // this CTA's share of each row's sum of squares; read after the next barrier
       float t = 0.f;
@@ -509,6 +511,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
 #pragma unroll
       for (int j = 0; j < 32; ++j) full[j] = j < MCA * kCPW ? acc[j] : 0.f;
       float v = warp_reduce_scatter32(full, lane);
+      if (r0 == 0) _trace.mark(2);  // first chunk's dot products reduced in the warps
       if (ksplit == 1) {
         if (NORM && ei < mc) {
           float t = 0.f;

@@ -328,7 +328,7 @@ bool link_split(const Dev& D, bool tiled, LinearArgs& prod, LinearArgs& cons, in
 void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& rows, int M_cap,
                int M_typ, int qt_grid, int splits, cudaStream_t s, const void* next_w = nullptr,
                size_t next_bytes = 0, const int* stable = nullptr, int stable_extra = 0,
-               bool short_kv = false) {
+               bool short_kv = false, int stable_add = 0) {
   Dev& D = c->L.D;
   const bool tiled = tiled_for(D, M_typ);
   const size_t tb = tw_bytes(D.dtype);
@@ -428,7 +428,8 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
 
     // RMSNorm -> Q,K,V -> RoPE -> K,V appended to the cache
     linear(D, aq, tiled, s);
-    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra, short_kv);
+    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra, short_kv, stable_add,
+              std::max(1, M_cap / std::max(1, D.B)));
     linear(D, ao, tiled, s);
     linear(D, a13, tiled, s);
     linear(D, a2, tiled, s);
@@ -505,7 +506,9 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
 void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
   Dev& D = c->L.D;
   // about one new latent per sequence every few bytes
-  run_stack(c, c->L.lm, D.x_lm, D.r_lm, D.B * n, D.B, 1, attn_splits(D, D.B, 1, c->kv_lat_typ + 1), s);
+  // latent slots [0, K] (BOS and the committed latents) do not change during the step
+  run_stack(c, c->L.lm, D.x_lm, D.r_lm, D.B * n, D.B, 1, attn_splits(D, D.B, 1, c->kv_lat_typ + 1), s,
+            nullptr, 0, &D.seq[0].K, 1, false, 1);
   launch_lm_scatter(D, s);
 }
 
@@ -588,7 +591,10 @@ int run_step_eager(lca_ctx* c, int n) {
   cudaStream_t s = c->stream;
   const bool gate = g_prof != nullptr;
   HostGate g1, g2;
+  // the step starts once the previous one has completed (as a graph launch does): kernels read the
+  // committed cache prefix before their grid-dependency wait
   if (gate) g1.hold(s);
+  else CK(cudaStreamSynchronize(s));
   enqueue_draft_encode(c, n, s);
   launch_segment(D, 0, 0, s);
   g1.release();
