@@ -53,6 +53,15 @@ __device__ __forceinline__ void load_w8(const float* p, float (&w)[8]) {
   w[6] = __uint_as_float(b.z); w[7] = __uint_as_float(b.w);
 }
 
+// D += A.B on the tensor cores: m16n8k16, bf16 operands, fp32 accumulation.
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
 // Reduce-scatter of 32 per-lane partial sums: afterwards lane L holds the warp total of
 // value index L (row L / kCPW, column L % kCPW). 31 shuffles.
 __device__ __forceinline__ float warp_reduce_scatter32(float (&v)[32], int lane) {
@@ -332,11 +341,14 @@ __device__ __forceinline__ void prefetch_next(const LinearArgs& a) {
 }
 
 // One tile per CTA: NW*4 output columns x Kr inputs (the CTA's K-split), copied into shared
-// memory by bulk async copies issued before the grid-dependency wait, together with the RMSNorm
-// gain of the K-range. Warps own 4 columns each; lanes stride K by 8, and one activation load
-// from shared memory feeds 4 columns. RMSNorm is folded in: rows are staged as x * g while their
-// sums of squares accumulate, and the per-row inverse RMS scales the dot products. Rows are
-// processed in chunks of MCA. With a K-split the `ksplit` CTAs of a column tile form a thread-
+// memory (one bulk async copy per column, rows padded by 16 bytes) before the grid-dependency
+// wait, together with the RMSNorm gain of the K-range. RMSNorm is folded in: rows are staged as
+// x * g, split into two bf16 halves (x * g = hi + lo, about 16 significant bits), while their sums
+// of squares accumulate, and the per-row inverse RMS scales the dot products. The dot products
+// run on the tensor cores (mma m16n8k16: 16 output columns as M, up to 8 rows as N, hi and lo
+// against the exact bf16 weights, fp32 accumulation), each warp over every NW-th K-step; the
+// warps' partials are summed in shared memory into one (row, column) value per lane, 4 columns
+// per warp. Rows are processed in chunks of MCA. With a K-split the `ksplit` CTAs of a column tile form a thread-
 // block cluster: each leaves its partial sums in its own shared memory and rank 0 adds the ranks'
 // partials through distributed shared memory in rank order (no global scratch).
 // (512 threads per SM by registers, four CTAs of four warps, so that a 512-tile launch is resident
@@ -350,10 +362,13 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   constexpr int NT = NW * 32;
   extern __shared__ __align__(128) unsigned char sm[];
   const int Kr = a.Kd / ksplit;
-  __nv_bfloat16* wt = reinterpret_cast<__nv_bfloat16*>(sm);             // [CT][Kr]
-  float* gs = reinterpret_cast<float*>(sm + (size_t)CT * Kr * 2);        // [Kr] (NORM)
-  float* xs = gs + Kr;                                                   // [MCA][Kr]
-  float* wss = xs + MCA * Kr;                                            // [NW][MCA] warp sums of squares
+  const int KP = Kr + 8;  // padded row (elements): conflict-free fragment loads
+  __nv_bfloat16* wt = reinterpret_cast<__nv_bfloat16*>(sm);             // [CT][KP]
+  float* gs = reinterpret_cast<float*>(sm + (size_t)CT * KP * 2);        // [Kr] (NORM)
+  __nv_bfloat16* xh = reinterpret_cast<__nv_bfloat16*>(gs + Kr);         // [MCA][KP] bf16 high halves
+  __nv_bfloat16* xl = xh + (size_t)MCA * KP;                             // [MCA][KP] bf16 low halves
+  float* red = reinterpret_cast<float*>(xl + (size_t)MCA * KP);          // [NW][CT][8] warp partials
+  float* wss = red + NW * CT * 8;                                        // [NW][MCA] warp sums of squares
   float* rs = wss + NW * MCA;                                            // [MCA] this CTA's sums of squares
   float* cpart = reinterpret_cast<float*>(                                // [MCA][CT], 16-byte aligned
       (reinterpret_cast<uintptr_t>(rs + MCA) + 15) & ~uintptr_t(15));
@@ -375,11 +390,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
     mbar_init(bar, 1);
     fence_mbar_init();
     mbar_expect_tx(bar, (uint32_t)(ncols * Kr * 2 + (NORM ? Kr * 4 : 0)));
-    if (ksplit == 1) {
-      bulk_g2s(wt, W, (uint32_t)(ncols * Kr * 2), bar);
-    } else {
-      for (int c = 0; c < ncols; ++c) bulk_g2s(wt + c * Kr, W + (size_t)c * a.Kd, (uint32_t)(Kr * 2), bar);
-    }
+    for (int c = 0; c < ncols; ++c) bulk_g2s(wt + (size_t)c * KP, W + (size_t)c * a.Kd, (uint32_t)(Kr * 2), bar);
     if (NORM) bulk_g2s(gs, a.norm + k0, (uint32_t)(Kr * 4), bar);
   }
   prefetch_next(a);
@@ -436,15 +447,23 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
         const int idx = base + u * NT;
         if (idx < nv) {
           float4 q = v[u];
+          const int i = (idx * 4) / Kr, kk = idx * 4 - i * Kr;
           if (NORM) {
-            const int i = (idx * 4) / Kr, kk = idx * 4 - i * Kr;
 #pragma unroll
             for (int r = 0; r < MCA; ++r)
               if (r == i) ss[r] += q.x * q.x + q.y * q.y + q.z * q.z + q.w * q.w;
             const float4 g = *reinterpret_cast<const float4*>(gs + kk);
             q.x *= g.x; q.y *= g.y; q.z *= g.z; q.w *= g.w;
           }
-          *reinterpret_cast<float4*>(xs + idx * 4) = q;
+          // x * g = hi + lo in bf16
+          const __nv_bfloat162 h01 = __floats2bfloat162_rn(q.x, q.y), h23 = __floats2bfloat162_rn(q.z, q.w);
+          const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+          const __nv_bfloat162 l01 = __floats2bfloat162_rn(q.x - f01.x, q.y - f01.y);
+          const __nv_bfloat162 l23 = __floats2bfloat162_rn(q.z - f23.x, q.w - f23.y);
+          *reinterpret_cast<uint2*>(xh + (size_t)i * KP + kk) =
+              make_uint2(*reinterpret_cast<const uint32_t*>(&h01), *reinterpret_cast<const uint32_t*>(&h23));
+          *reinterpret_cast<uint2*>(xl + (size_t)i * KP + kk) =
+              make_uint2(*reinterpret_cast<const uint32_t*>(&l01), *reinterpret_cast<const uint32_t*>(&l23));
         }
       }
     }
@@ -476,42 +495,51 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       for (int w = 0; w < NW; ++w) t += wss[w * MCA + tid];
       rs[tid] = t;
     }
-    if (col0 < ncols) {
-      float acc[MCA * kCPW];
+    {
+      // tensor-core dot products: warp w takes K-steps w, w + NW, ...; C[column][row] partials
+      constexpr int MT = CT / 16;
+      const int g = lane >> 2, q4 = lane & 3;
+      float cacc[MT][4];
 #pragma unroll
-      for (int j = 0; j < MCA * kCPW; ++j) acc[j] = 0.f;
-      for (int kk = lane * 8; kk < Kr; kk += 256) {
-        float w[kCPW][8];
-#pragma unroll
-        for (int c = 0; c < kCPW; ++c) {
-          const uint4 u = *reinterpret_cast<const uint4*>(wt + (col0 + c) * Kr + kk);
-          unpack_bf16x2(u.x, w[c][0], w[c][1]);
-          unpack_bf16x2(u.y, w[c][2], w[c][3]);
-          unpack_bf16x2(u.z, w[c][4], w[c][5]);
-          unpack_bf16x2(u.w, w[c][6], w[c][7]);
+      for (int mt = 0; mt < MT; ++mt) cacc[mt][0] = cacc[mt][1] = cacc[mt][2] = cacc[mt][3] = 0.f;
+      const bool brow = g < mc;
+      for (int kb = warp * 16; kb < Kr; kb += NW * 16) {
+        uint32_t bh0 = 0u, bh1 = 0u, bl0 = 0u, bl1 = 0u;
+        if (brow) {
+          const uint32_t* ph = reinterpret_cast<const uint32_t*>(xh + (size_t)g * KP + kb + 2 * q4);
+          const uint32_t* pl = reinterpret_cast<const uint32_t*>(xl + (size_t)g * KP + kb + 2 * q4);
+          bh0 = ph[0];
+          bh1 = ph[4];
+          bl0 = pl[0];
+          bl1 = pl[4];
         }
 #pragma unroll
-        for (int i = 0; i < MCA; ++i) {
-          if (i < mc) {
-            const float4 xa = *reinterpret_cast<const float4*>(xs + i * Kr + kk);
-            const float4 xb = *reinterpret_cast<const float4*>(xs + i * Kr + kk + 4);
-#pragma unroll
-            for (int c = 0; c < kCPW; ++c) {
-              float sacc = acc[i * kCPW + c];
-              sacc = fmaf(w[c][0], xa.x, sacc); sacc = fmaf(w[c][1], xa.y, sacc);
-              sacc = fmaf(w[c][2], xa.z, sacc); sacc = fmaf(w[c][3], xa.w, sacc);
-              sacc = fmaf(w[c][4], xb.x, sacc); sacc = fmaf(w[c][5], xb.y, sacc);
-              sacc = fmaf(w[c][6], xb.z, sacc); sacc = fmaf(w[c][7], xb.w, sacc);
-              acc[i * kCPW + c] = sacc;
-            }
-          }
+        for (int mt = 0; mt < MT; ++mt) {
+          const uint32_t* pa = reinterpret_cast<const uint32_t*>(wt + (size_t)(mt * 16 + g) * KP + kb + 2 * q4);
+          uint32_t af[4];
+          af[0] = pa[0];
+          af[1] = pa[4 * KP];
+          af[2] = pa[4];
+          af[3] = pa[4 * KP + 4];
+          mma_bf16_16816(cacc[mt], af, bh0, bh1);
+          mma_bf16_16816(cacc[mt], af, bl0, bl1);
         }
       }
-      float full[32];
 #pragma unroll
-      for (int j = 0; j < 32; ++j) full[j] = j < MCA * kCPW ? acc[j] : 0.f;
-      float v = warp_reduce_scatter32(full, lane);
-      if (r0 == 0) _trace.mark(2);  // first chunk's dot products reduced in the warps
+      for (int mt = 0; mt < MT; ++mt) {
+        const int f = mt * 16 + g;
+        *reinterpret_cast<float2*>(red + ((size_t)(warp * CT + f) * 8 + 2 * q4)) = make_float2(cacc[mt][0], cacc[mt][1]);
+        *reinterpret_cast<float2*>(red + ((size_t)(warp * CT + f + 8) * 8 + 2 * q4)) =
+            make_float2(cacc[mt][2], cacc[mt][3]);
+      }
+    }
+    __syncthreads();
+    if (col0 < ncols) {
+      // lane (row ei, column col0 + ec): the sum of the warps' partials
+      float v = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) v += red[(w * CT + col0 + ec) * 8 + ei];
+      if (r0 == 0) _trace.mark(2);  // first chunk's dot products summed
       if (ksplit == 1) {
         if (NORM && ei < mc) {
           float t = 0.f;
@@ -753,9 +781,10 @@ template <int MCA, int NW, bool NORM>
 void gemv_bulk_go(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s) {
   constexpr int CT = NW * kCPW;
   const int Kr = a.Kd / ksplit;
-  const size_t smem = (size_t)CT * Kr * 2 + (size_t)Kr * 4 + (size_t)MCA * Kr * 4 +
+  const size_t KP = (size_t)Kr + 8;
+  const size_t smem = (size_t)CT * KP * 2 + (size_t)Kr * 4 + 2 * (size_t)MCA * KP * 2 + (size_t)NW * CT * 8 * 4 +
                       (NW * MCA + MCA + MCA * CT) * 4 + 16 + 16 + 16 +
-                      (size_t)kMaxKSplit * MCA * (CT + 1) * 4 + 64;
+                      (ksplit > 1 ? (size_t)kMaxKSplit * MCA * (CT + 1) * 4 : 0) + 64;  // rank 0's buffers
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((a.N + CT - 1) / CT, ksplit, a.groups);
   cfg.blockDim = dim3(NW * 32);
