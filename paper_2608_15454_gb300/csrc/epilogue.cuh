@@ -82,6 +82,7 @@ struct EpiPre {
   float r0, r1;  // residual pair
   float2 cs;     // RoPE cos/sin
   int b, slot;
+  int pos;       // RoPE position (epi_load_early; the angle follows in epi_load_late)
 };
 
 static __device__ __forceinline__ EpiPre epi_load(const EpiArgs& e, int r, int c) {
@@ -107,6 +108,39 @@ static __device__ __forceinline__ EpiPre epi_load(const EpiArgs& e, int r, int c
     }
   }
   return p;
+}
+
+// epi_load in two halves, so that no load waits on another before the caller's own loads are
+// issued: the first loads everything but the RoPE angle (the row's position instead), the second
+// loads the angle at that position.
+static __device__ __forceinline__ EpiPre epi_load_early(const EpiArgs& e, int r, int c) {
+  EpiPre p;
+  p.r0 = p.r1 = 0.f;
+  p.cs = make_float2(1.f, 0.f);
+  p.b = p.slot = 0;
+  p.pos = 0;
+  if (e.mode == EPI_RESID || e.mode == EPI_RESID_SILU) {
+    const float2 q = *reinterpret_cast<const float2*>(e.res + (size_t)r * e.ldres + c);
+    p.r0 = q.x;
+    p.r1 = q.y;
+  } else if (e.mode == EPI_QKV) {
+    const int part = c / e.d;
+    if (part < 2) p.pos = e.rows.pos[r];
+    if (part > 0) {
+      p.b = e.rows.b[r];
+      p.slot = e.rows.slot[r];
+    }
+  }
+  return p;
+}
+static __device__ __forceinline__ void epi_load_late(const EpiArgs& e, EpiPre& p, int c) {
+  if (e.mode == EPI_QKV) {
+    const int part = c / e.d;
+    if (part < 2) {
+      const int dd = (c - part * e.d) % e.hd;
+      p.cs = e.rope[(size_t)p.pos * (e.hd >> 1) + (dd >> 1)];
+    }
+  }
 }
 
 // The same epilogue split for row-wise batching (tensor-core tiles, where a thread owns a row and
@@ -196,6 +230,7 @@ static __device__ __forceinline__ void epi_out(const EpiArgs& e, const EpiRow& q
   p.cs = op;
   p.b = q.b;
   p.slot = q.slot;
+  p.pos = q.pos;
   epi_store<TC>(e, p, r, c, a0, a1);
 }
 

@@ -342,7 +342,7 @@ __device__ __forceinline__ void prefetch_next(const LinearArgs& a) {
 
 // One tile per CTA: NW*4 output columns x Kr inputs (the CTA's K-split), copied into shared
 // memory (one bulk async copy per column, rows padded by 16 bytes) before the grid-dependency
-// wait, together with the RMSNorm gain of the K-range. RMSNorm is folded in: rows are staged as
+// wait; the RMSNorm gain of the K-range is read into shared memory then too. RMSNorm is folded in: rows are staged as
 // x * g, split into two bf16 halves (x * g = hi + lo, about 16 significant bits), while their sums
 // of squares accumulate, and the per-row inverse RMS scales the dot products. The dot products
 // run on the tensor cores (mma m16n8k16: 16 output columns as M, up to 8 rows as N, hi and lo
@@ -389,9 +389,13 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   if (tid == 0) {
     mbar_init(bar, 1);
     fence_mbar_init();
-    mbar_expect_tx(bar, (uint32_t)(ncols * Kr * 2 + (NORM ? Kr * 4 : 0)));
+    mbar_expect_tx(bar, (uint32_t)(ncols * Kr * 2));
     for (int c = 0; c < ncols; ++c) bulk_g2s(wt + (size_t)c * KP, W + (size_t)c * a.Kd, (uint32_t)(Kr * 2), bar);
-    if (NORM) bulk_g2s(gs, a.norm + k0, (uint32_t)(Kr * 4), bar);
+  }
+  if (NORM) {
+    // the RMSNorm gain of the K-range (a weight: read before the dependency wait)
+    for (int i = tid; i < Kr / 4; i += NT)
+      reinterpret_cast<float4*>(gs)[i] = __ldg(reinterpret_cast<const float4*>(a.norm + k0) + i);
   }
   prefetch_next(a);
   if (ksplit > 1) {
@@ -402,6 +406,8 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       fence_mbar_init();
     }
     cgr::this_cluster().sync();
+  } else if (NORM) {
+    __syncthreads();
   }
   pdl_trigger();
   pdl_wait();
@@ -420,7 +426,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
     // epilogue operands of this lane, loaded while the rows are staged and multiplied
     EpiPre pre{};
     const bool epi_lane = ksplit == 1 && col0 < ncols && ei < mc && (ec & 1) == 0;
-    if (epi_lane) pre = epi_load(a.epi, rbase + r0 + ei, tile * CT + col0 + ec);
+    if (epi_lane) pre = epi_load_early(a.epi, rbase + r0 + ei, tile * CT + col0 + ec);
     __syncthreads();
     // raw rows -> registers (loads batched), then x * g -> shared memory with sums of squares
     constexpr int UNR = 8;
@@ -437,10 +443,6 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
         v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
         if (idx < nv && i < mc)
           v[u] = *reinterpret_cast<const float4*>(a.x + (size_t)(rbase + r0 + i) * a.ldx + k0 + kk);
-      }
-      if (NORM && !have_w) {
-        const bool ok = mbar_wait(bar, 0);  // the gain slice travels with the weights
-        if (!ok) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
       }
 #pragma unroll
       for (int u = 0; u < UNR; ++u) {
@@ -468,6 +470,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       }
     }
     if (r0 == 0) _trace.mark(0);  // first row chunk loaded and staged
+    if (epi_lane) epi_load_late(a.epi, pre, tile * CT + col0 + ec);  // overlaps the dot products
     if (NORM) {
       // per-warp partial sums of squares over this CTA's K range (no atomics: summed in warp order)
 #pragma unroll

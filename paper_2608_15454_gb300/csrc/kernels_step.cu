@@ -26,8 +26,13 @@ __global__ void k_mb_plan(Dev D, int fill) {
   pdl_trigger();
   pdl_wait();
   _trace.waited();
+  // the plan stays in shared memory for the rows and the fill (no global read-back)
   __shared__ int s_cnt[1024];
   __shared__ int s_first[1024];
+  __shared__ int s_start[1024];
+  __shared__ int s_ms[1024];
+  __shared__ int s_K[4], s_gsK[4];  // fill (at most 4 sequences): K and the start of group K
+  __shared__ int s_M;
   const Params P = *D.params;
   const int n = P.n, batch = P.batch;
   const int tid = threadIdx.x;
@@ -35,33 +40,46 @@ __global__ void k_mb_plan(Dev D, int fill) {
     SeqState& st = D.seq[b];
     const int t = st.t, g = st.K;
     const int s = g >= 1 ? D.gstart[(size_t)b * D.L + g - 1] : 0;
+    if (fill && b < 4) {
+      s_K[b] = g;
+      s_gsK[b] = D.gstart[(size_t)b * D.L + g];
+    }
+    int len = st.mb_len;
     if (st.mb_start != s) {
       st.mb_start = s;
-      st.mb_len = 0;
+      len = 0;
     }
-    int first = s + st.mb_len;
+    int first = s + len;
     if (first > t - 1) first = t - 1;
     s_first[b] = first;
     s_cnt[b] = (t - first) + (n - 2);
+    s_ms[b] = s;
     st.mb_len = t - s;
   }
   __syncthreads();
   if (tid == 0) {
     int acc = 0;
     for (int b = 0; b < batch; ++b) {
-      D.r_mb.seq_start[b] = acc;
-      D.r_mb.seq_count[b] = s_cnt[b];
+      s_start[b] = acc;
       acc += s_cnt[b];
+    }
+    if (acc > D.R) {
+      err_or(D.err, kErrIndex);
+      for (int b = 0; b < batch; ++b) {
+        s_start[b] = 0;
+        s_cnt[b] = 0;
+      }
+      acc = 0;
+    }
+    for (int b = 0; b < batch; ++b) {
+      D.r_mb.seq_start[b] = s_start[b];
+      D.r_mb.seq_count[b] = s_cnt[b];
     }
     for (int b = batch; b < D.B; ++b) {
       D.r_mb.seq_start[b] = acc;
       D.r_mb.seq_count[b] = 0;
     }
-    if (acc > D.R) {
-      err_or(D.err, kErrIndex);
-      for (int b = 0; b < batch; ++b) D.r_mb.seq_count[b] = 0;
-      acc = 0;
-    }
+    s_M = acc;
     *D.r_mb.M = acc;
     *D.M_head_mb = batch * (n - 1);
     D.stats->mb_rows += acc;
@@ -69,8 +87,8 @@ __global__ void k_mb_plan(Dev D, int fill) {
   __syncthreads();
   const int warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
   for (int b = warp; b < batch; b += nw) {
-    const int st0 = D.r_mb.seq_start[b], cnt = D.r_mb.seq_count[b];
-    const int s = D.seq[b].mb_start, first = s_first[b];
+    const int st0 = s_start[b], cnt = s_cnt[b];
+    const int s = s_ms[b], first = s_first[b];
     for (int j = lane; j < cnt; j += 32) {
       const int p = first + j;
       const int r = st0 + j;
@@ -82,18 +100,20 @@ __global__ void k_mb_plan(Dev D, int fill) {
     for (int j = lane; j < n - 1; j += 32)
       D.head_rows_mb[b * (n - 1) + j] = cnt > 0 ? st0 + cnt - (n - 1) + j : 0;
   }
-  __syncthreads();
   if (!fill) return;  // many sequences: k_mb_fill writes the rows with a full grid
   // window rows: byte p of group k gets o_k + u_k (Algorithm 1, drafting input; residual r_2 added before
   // upsampling); copies beyond t belong to the current group K
-  const int M = *D.r_mb.M;
+  const int M = s_M;
+  const int nb = batch < 4 ? batch : 4;
   const int d4 = D.d / 4;
   for (int idx = tid; idx < M * d4; idx += blockDim.x) {
     const int r = idx / d4, c4 = idx - r * d4;
-    const int b = D.r_mb.b[r], p = D.r_mb.pos[r];
-    const int g = D.seq[b].K;
-    const int gs = D.gstart[(size_t)b * D.L + g];
-    const int k = (g >= 1 && p < gs) ? g - 1 : g;
+    int b = 0;
+    for (int bb = 1; bb < nb; ++bb)
+      if (r >= s_start[bb] && s_cnt[bb] > 0) b = bb;
+    const int p = s_first[b] + (r - s_start[b]);
+    const int g = s_K[b];
+    const int k = (g >= 1 && p < s_gsK[b]) ? g - 1 : g;
     const float4 o = reinterpret_cast<const float4*>(D.o_tab + ((size_t)b * D.L + k) * D.d)[c4];
     const float4 u = reinterpret_cast<const float4*>(D.u_tab + ((size_t)b * D.L + k) * D.d)[c4];
     reinterpret_cast<float4*>(D.x_mb + (size_t)r * D.d)[c4] = make_float4(o.x + u.x, o.y + u.y, o.z + u.z, o.w + u.w);
