@@ -239,3 +239,30 @@ def test_small_bf16_batch_forced_and_free_steps(lca, mb_kind):
             assert out[b] == r.emitted
             st = ctx.state(b)
             assert (st["t"], st["K"]) == (decs[b].t, decs[b].K)
+
+
+def test_small_bf16_long_context_batch_one(lca):
+    """Batch 1 over a cache longer than the decode attention stages in shared memory (about 8,500
+    bytes in 16 key splits: 256 staged keys per CTA, the rest read from the cache) and a latent
+    cache of about a thousand latents; forced spaces run the LM module on some steps. Logits within
+    the bf16 tolerance, bytes and state equal."""
+    W = make_weights(SMALL_BF16, gain=8.0, seed=6)
+    p = zipf_text(3, 8500)
+    n = 3
+    ctx = new_ctx(lca, SMALL_BF16, W, 1, len(p) + 64, n)
+    ctx.prefill([p])
+    dec = IncrementalDecoder(Model(SMALL_BF16, W))
+    dec.prefill(p)
+    for s in range(6):
+        cand = bytes([32 if s % 2 == 0 else 100, 101 + s, 32 if s % 3 == 0 else 102])
+        a = s % n
+        ctx.force_candidates([cand], n)
+        ctx.force_accept([a])
+        r = dec.step(n, 0.75, THRESH, forced=a, forced_cand=cand)
+        out, cnt = ctx.step(n, 0.75, lca.LCA_THRESH)
+        nb, mb = ctx.logits(n)
+        np.testing.assert_allclose(nb[0], r.nb_logits, atol=BF16_TOL * 8, rtol=0)
+        np.testing.assert_allclose(mb[0], r.mb_logits, atol=BF16_TOL * 8, rtol=0)
+        assert out[0] == r.emitted
+        st = ctx.state(0)
+        assert (st["t"], st["K"]) == (dec.t, dec.K)
