@@ -870,11 +870,6 @@ constexpr int kAwThreads = kAwWarps * 32;
 constexpr int kAwG = 4;           // keys per group
 constexpr int kAwStageMax = 256;  // keys staged per CTA (64 KB of K and V)
 
-__device__ __forceinline__ float2 aw_bf2(const __nv_bfloat16* p) {
-  const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
-  return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xFFFF0000u));
-}
-
 // [lo, hi) of split sp when n keys starting at base are shared in groups of kAwG
 __device__ __forceinline__ void aw_share(int base, int n, int splits, int sp, int& lo, int& hi) {
   const int per = ((n + splits - 1) / splits + kAwG - 1) / kAwG * kAwG;

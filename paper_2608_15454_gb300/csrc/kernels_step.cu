@@ -203,7 +203,6 @@ k_head(Dev D, const float* __restrict__ x, const int* __restrict__ rows, const i
   TraceScope _trace(TT_HEAD);
   constexpr int VEC = sizeof(TW) == 2 ? 1 : 2;
   extern __shared__ float xs[];  // [kHR][d]
-  __shared__ float inv[kHR];
   __shared__ int s_last;
   const int d = D.d;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;

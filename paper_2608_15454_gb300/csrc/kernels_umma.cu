@@ -798,9 +798,6 @@ __device__ __forceinline__ void scol_out(const EpiArgs& e, size_t gr, int c, int
   }
 }
 
-// Release-ordered arrive: this thread's earlier accesses, distributed shared memory loads
-// included, are performed before a peer's wait on the phase returns.
-__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive;" ::: "memory"); }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait;" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t mapa_u32(uint32_t saddr, int rank) {
