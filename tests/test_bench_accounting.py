@@ -1,0 +1,72 @@
+"""The bench's algorithmic-byte accounting (CPU), against the sizes the model's shape fixes:
+one pre-norm Llama block of width d with a 4d SwiGLU MLP holds 16 d^2 weights (Q, K, V, O:
+4 d^2; W1, W3, W2: 12 d^2), 33.55 MB in bf16 at d = 1024, and the paper-size model runs
+2 encoder + 2 next-byte + 2 multi-byte blocks every step and 16 LM blocks when a patch closes."""
+import numpy as np
+
+import bench
+from synth import WORKLOADS
+
+MB = 1e6
+
+
+def _stats(steps, lm_steps, lm_rows):
+    return {"steps": steps, "lm_steps": lm_steps, "lm_rows": lm_rows}
+
+
+def _state(t, K, pgs):
+    return {"t": t, "K": K, "prev_group_start": pgs}
+
+
+def test_weight_bytes_per_step_of_the_paper_model():
+    m = WORKLOADS["paper_b1"].model
+    blk = 16 * 1024 * 1024 * 2
+    assert abs(blk / MB - 33.55) < 0.01
+    unembed = 256 * 1024 * 2
+    s0 = [_state(1000, 130, 990)]
+    # no LM step: 6 blocks and the two heads' unembedding
+    w, _ = bench.algorithmic_bytes(m, 3, 10, _stats(0, 0, 0), _stats(10, 0, 0), s0, s0)
+    assert w == 6 * blk + 2 * unembed
+    assert abs(w / MB - 202.4) < 0.1
+    # every step runs the LM module: 22 blocks, about 738 MB
+    w, _ = bench.algorithmic_bytes(m, 3, 10, _stats(0, 0, 0), _stats(10, 10, 10), s0, s0)
+    assert w == 22 * blk + 2 * unembed
+    assert abs(w / MB - 739.2) < 0.1
+    # n = 1: no drafter, one head
+    w, _ = bench.algorithmic_bytes(m, 1, 10, _stats(0, 0, 0), _stats(10, 0, 0), s0, s0)
+    assert w == 4 * blk + unembed
+
+
+def test_kv_bytes_per_step_of_the_paper_model():
+    """Byte caches: K and V of every encoder and next-byte layer read once at the mid-interval
+    length (16 KB per position over 4 layers: 1024 dims x 2 B x 2 x 4), plus the n appended rows;
+    the window cache of the two multi-byte layers; the LM cache (64 KB per latent over 16 layers)
+    for each new latent row."""
+    m = WORKLOADS["paper_b1"].model
+    n = 3
+    a, b = _state(1000, 130, 990), _state(1030, 134, 1020)
+    _, kv = bench.algorithmic_bytes(m, n, 10, _stats(0, 0, 0), _stats(10, 2, 4), [a], [b])
+    per_pos = 1024 * 2 * 2               # K and V of one layer at one position
+    t_mid, win, k_mid = 1015.0, 10.0, 132.0
+    byte_read = 4 * per_pos * (t_mid + n)
+    byte_append = 4 * per_pos * n
+    window = 2 * per_pos * (win + n)
+    lm = 0.4 * 16 * per_pos * (k_mid + 2)   # 4 LM rows over 10 steps
+    assert np.isclose(kv, byte_read + byte_append + window + lm)
+    assert per_pos * 4 == 16384 and per_pos * 16 == 65536
+
+
+def test_roofline_of_the_dominant_family():
+    prof = {"linear": {"launches": 88, "ms": 0.264, "bytes": 88 * 8.39e6},
+            "attention": {"launches": 22, "ms": 0.110, "bytes": 0.0},
+            "head": {"launches": 2, "ms": 0.02, "bytes": 0.0}}
+    r = bench.roofline(prof, 6670.9, "measured", "nowhere", 1.0e6, 2)
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s" and r["peak"] == 6670.9
+    # 8.39 MB per launch in 3 us: 2,796.7 GB/s
+    assert np.isclose(r["achieved"], 8.39e6 / 3e-6 / 1e9)
+    assert np.isclose(r["frac"], r["achieved"] / 6670.9)
+    assert r["traffic"] is None
+    # attention dominant: its bytes per launch are the step KV bytes times the steps, per launch
+    prof["attention"]["ms"] = 1.0
+    r = bench.roofline(prof, 6670.9, "measured", "nowhere", 1.0e6, 2)
+    assert np.isclose(r["algorithmic_bytes_per_launch"], 2 * 1.0e6 / 22)
