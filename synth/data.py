@@ -10,7 +10,8 @@ Opus-100; Section 4.3), which are not used:
     joined by single spaces;
   * "zipf":  words drawn with probability proportional to rank^-1.1 from a
     lexicon of 5,000 distinct random lowercase words of length 1..12, joined by
-    single spaces (mean patch about 7.5 bytes, space included).
+    single spaces (mean patch about 8.5 bytes, space included: the Zipf-weighted
+    mean word length of this lexicon plus one).
 Weights: standard normal x 0.02 drawn in a fixed tensor order from
 numpy.random.default_rng(0); RMSNorm gains are 1.
 """
