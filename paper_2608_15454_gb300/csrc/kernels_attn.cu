@@ -987,7 +987,10 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
     const int nv = nsk + (nhi - nlo);
     const int nst_ok = slo2 == slo ? min(nst, nsk) : 0;  // staged keys usable for this range
     if (!staged) {
-      if (!a3_wait(&s_bar, 0) && lane == 0 && warp == 0) atomicOr(err, kErrTimeout | kErrWaitAttnW);
+      if (!a3_wait(&s_bar, 0)) {
+        if (lane == 0 && warp == 0) atomicOr(err, kErrTimeout | kErrWaitAttnW);
+        a3_wait(&s_bar, 0);  // once more (bounded) for the copies still in flight
+      }
       staged = true;
     }
     if (qt == (int)blockIdx.y) _trace.mark(0);  // staged keys landed
@@ -1180,8 +1183,11 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
     }
     cl.sync();  // peers are done reading this tile's partials
   }
-  // no rows: the staged copies must still land before the CTA leaves (bounded)
-  if (!staged && !a3_wait(&s_bar, 0) && tid == 0) atomicOr(err, kErrTimeout | kErrWaitAttnW);
+  // no rows: the staged copies must still land before the CTA leaves (bounded, twice)
+  if (!staged && !a3_wait(&s_bar, 0)) {
+    if (tid == 0) atomicOr(err, kErrTimeout | kErrWaitAttnW);
+    a3_wait(&s_bar, 0);
+  }
 }
 
 // Keys staged per CTA of k_attn_w for a cache of S slots in `splits` splits (0: no staging).
