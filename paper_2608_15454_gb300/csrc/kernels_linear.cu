@@ -479,10 +479,12 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       }
     }
     if (!have_w) {
-      // the bounded wait for the weight tile; on a timeout the error is recorded and the
-      // kernel runs on (no early exit, so cluster barriers stay matched)
-      const bool ok = mbar_wait(bar, 0);
-      if (__syncthreads_or(!ok) && tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
+      // the bounded wait for the weight tile; on a timeout the error is recorded, the copies in
+      // flight get one more bounded wait, and the kernel runs on (no early exit, so cluster
+      // barriers stay matched)
+      const bool late = !mbar_wait(bar, 0);
+      if (late) mbar_wait(bar, 0);
+      if (__syncthreads_or(late) && tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
       have_w = true;
     } else {
       __syncthreads();
@@ -655,8 +657,9 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       cl.sync();
     }
   }
-  if (!have_w) {  // no rows: still wait (bounded) for the copy before leaving
-    if (!mbar_wait(bar, 0) && tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
+  if (!have_w && !mbar_wait(bar, 0)) {  // no rows: still wait (bounded, twice) for the copy before leaving
+    if (tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
+    mbar_wait(bar, 0);
   }
 }
 
