@@ -398,3 +398,17 @@ def test_paper_parameter_count():
     n = param_count(PAPER)
     assert abs(n - 373e6) / 373e6 < 0.01
     assert n == 22 * 16 * 1024 ** 2 + 2 * 256 * 1024 + (2 * 22 + 3) * 1024
+
+
+def test_head_decisions_ties_and_probability():
+    """Reading R12 (argmax takes the lowest byte among equal maxima) and R4 (the drafter's
+    probability of its argmax, exp(l_max - logsumexp))."""
+    from oracle.model import greedy, max_prob
+    lg = np.zeros(256)
+    assert greedy(lg) == 0 and abs(max_prob(lg, 0) - 1 / 256) < 1e-15
+    lg[[7, 200]] = 3.0
+    assert greedy(lg) == 7
+    p = max_prob(lg, 7)
+    assert abs(p - np.e ** 3 / (2 * np.e ** 3 + 254)) < 1e-14
+    big = lg + 1e4  # a common offset changes nothing and does not overflow
+    assert greedy(big) == 7 and abs(max_prob(big, 7) - p) < 1e-12
