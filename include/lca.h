@@ -15,7 +15,7 @@
  *   (4) run the next-byte decoder over all n candidates (Algorithm 1, next-byte step);
  *   (5) accept: c_1 always, drafts left to right while their probability is >= tau
  *       (Section 3.1 "Byte Acceptance"; LCA_THRESH), or while they equal the next-byte
- *       argmax (speculative acceptance, Section 5.2 (ii); LCA_SPEC); then keep the
+ *       argmax (speculative acceptance, Section 6.2 (ii); LCA_SPEC); then keep the
  *       accepted prefix of every cache and drop the rest.
  * The meaning of n used here: one next-byte byte plus n-1 drafts, so 1..n bytes are
  * committed per step (the algorithm's "n-2 copies" and "h_2[-(n-1):]").
@@ -63,7 +63,7 @@ extern "C" {
 
 /* acceptance rule */
 #define LCA_THRESH 0 /* draft kept while its drafter probability >= tau (Section 3.1) */
-#define LCA_SPEC 1   /* draft kept while it equals the next-byte argmax (Section 5.2) */
+#define LCA_SPEC 1   /* draft kept while it equals the next-byte argmax (Section 6.2) */
 
 typedef struct lca_ctx lca_ctx; /* opaque, owned by the library */
 
@@ -197,6 +197,13 @@ int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N
  * ring slot, 1: waiting for a chunk), chunk, stage, chunks, key lo, key hi, chunks before the
  * tile, copies issued}. Clears the record. */
 int lca_debug_attn_diag(int32_t* out16);
+/* Test hook for the bounded waits: the first wait of the weight-streaming GEMV for its weight tile
+ * spins at most `spins` times (< 0: the default, 2^22) on the current device. With 0 the wait
+ * reports late at once: the kernel records the timeout bit in the device error word, waits once
+ * more with the full budget for its copies in flight, then completes, and the call returns
+ * LCA_E_TIMEOUT. Outside a test, a call that returns LCA_E_TIMEOUT has undefined results, and if
+ * the second wait ran out as well a copy may have been left in flight: destroy the context. */
+int lca_debug_set_wait_spins(int32_t spins);
 /* Bytes of device scratch lca_debug_gemm needs. */
 size_t lca_debug_gemm_scratch_bytes(int32_t M, int32_t K);
 
@@ -224,13 +231,19 @@ int lca_debug_force_candidates(lca_ctx* ctx, const uint8_t* cand, int32_t n);
  * cache slots [0, kv_len[r]) of its sequence; softmax scale `scale`; fp32 arithmetic.
  *   q, out:   device fp32 [batch * n_rows][heads * head_dim] (RoPE already applied to q).
  *   k_cache, v_cache: device [batch][heads][slots][head_dim] of `dtype` (LCA_F32|LCA_BF16).
- *   kv_len:   device int32 [batch * n_rows], each 1..slots (larger values are clamped).
+ *   kv_len:   device int32 [batch * n_rows], each 1..slots. A larger value is an error: that row
+ *             reads only the slots [0, slots), and the call records LCA_E_DEVICE_STATE in the error
+ *             word, which lca_decode_attention_status returns.
  *   splits:   1..16; the key range of each (sequence, head) is split over `splits` CTAs whose
  *             partial results are combined in a fixed order (deterministic).
  *   scratch:  device memory of >= lca_decode_attention_scratch_bytes(...), 256-byte aligned,
- *             caller-owned; overwritten by the call.
+ *             caller-owned; overwritten by the call. Its first 4 bytes are the call's error word
+ *             (0: no error), cleared at the start of each call and read by
+ *             lca_decode_attention_status.
  * head_dim must be 32 or 64. Asynchronous on `stream` (a cudaStream_t). Returns LCA_E_ARG for
- * bad arguments and LCA_E_CAPACITY for too small a scratch. */
+ * bad arguments and LCA_E_CAPACITY for too small a scratch; what the kernels find while running
+ * (an out-of-range kv_len, a bounded wait that ran out) is read afterwards with
+ * lca_decode_attention_status. */
 int lca_decode_attention_scratch_bytes(int32_t batch, int32_t heads, int32_t head_dim,
                                        int32_t splits, size_t* out);
 int lca_decode_attention(const float* q, float* out, const void* k_cache, const void* v_cache,
@@ -257,6 +270,16 @@ int lca_decode_attention_noalloc(const float* q, float* out, const void* k_cache
                                  int32_t slots, int32_t n_rows, const int32_t* kv_len, float scale,
                                  int32_t splits, void* stream);
 size_t lca_decode_attention_noalloc_capacity(void);
+
+/* Status of the last lca_decode_attention call that used `scratch` (or, for the _noalloc form, of
+ * the last lca_decode_attention_noalloc call on the current device): waits for `stream`, then
+ * returns LCA_OK, LCA_E_DEVICE_STATE (a kv_len beyond slots: that row read only [0, slots)) or
+ * LCA_E_TIMEOUT (a bounded wait ran out). Enqueue nothing between the call and its status read
+ * that reuses the same scratch. The _noalloc form allocates nothing either. The device address of
+ * the library's fixed array is looked up once per device and kept for the life of the process;
+ * after cudaDeviceReset on a device, neither _noalloc call may be used on it again. */
+int lca_decode_attention_status(const void* scratch, void* stream);
+int lca_decode_attention_noalloc_status(void* stream);
 
 int lca_destroy(lca_ctx* ctx);
 const char* lca_status_str(int status);

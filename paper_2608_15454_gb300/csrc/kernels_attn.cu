@@ -2302,6 +2302,35 @@ size_t lca_decode_attention_noalloc_capacity(void) { return kNoAllocScratchBytes
 
 }  // extern "C"
 
+namespace {
+// The status the kernels of the last call recorded in the error word (word 0 of the scratch):
+// waits for the stream, then maps the bits to a status code.
+int op_status(const void* word, cudaStream_t s) {
+  int e = 0;
+  if (cudaMemcpyAsync(&e, word, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess) return LCA_E_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return LCA_E_CUDA;
+  if (e & kErrTimeout) return LCA_E_TIMEOUT;
+  if (e & kErrIndex) return LCA_E_DEVICE_STATE;
+  return LCA_OK;
+}
+}  // namespace
+
+extern "C" {
+
+int lca_decode_attention_status(const void* scratch, void* stream) {
+  if (!scratch || reinterpret_cast<uintptr_t>(scratch) % 256) return LCA_E_ARG;
+  return op_status(scratch, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int lca_decode_attention_noalloc_status(void* stream) {
+  char* base = nullptr;
+  const int st = noalloc_scratch(&base);
+  if (st != LCA_OK) return st;
+  return op_status(base, reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"
+
 namespace lca {
 
 LCA_TRACE_SETTER(trace_set_attn)

@@ -310,11 +310,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 // Bounded wait: false if the phase did not complete within the spin budget.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  for (int i = 0; i < kWaitSpins; ++i)
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int spins = kWaitSpins) {
+  for (int i = 0; i < spins; ++i)
     if (mbar_try_wait(bar, parity)) return true;
   return false;
 }
+
+// Spin budget of the first weight wait of k_gemv_bulk. A test hook (lca_debug_set_wait_spins) can
+// shorten it so that the wait reports late at once; the second wait, which drains the copies in
+// flight before the CTA reads them or leaves, keeps the full budget.
+static __device__ int g_first_wait_spins = kWaitSpins;
 
 // Each CTA prefetches an equal slice of the next layers' weights into L2 (no shared memory or
 // registers are used, so the HBM stream continues across kernel boundaries).
@@ -482,7 +487,7 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       // the bounded wait for the weight tile; on a timeout the error is recorded, the copies in
       // flight get one more bounded wait, and the kernel runs on (no early exit, so cluster
       // barriers stay matched)
-      const bool late = !mbar_wait(bar, 0);
+      const bool late = !mbar_wait(bar, 0, g_first_wait_spins);
       if (late) mbar_wait(bar, 0);
       if (__syncthreads_or(late) && tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
       have_w = true;
@@ -909,3 +914,8 @@ void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s) {
 LCA_TRACE_SETTER(trace_set_linear)
 
 } // namespace lca
+
+extern "C" int lca_debug_set_wait_spins(int32_t spins) {
+  const int v = spins < 0 ? lca::kWaitSpins : spins;
+  return cudaMemcpyToSymbol(lca::g_first_wait_spins, &v, sizeof(v)) == cudaSuccess ? LCA_OK : LCA_E_CUDA;
+}

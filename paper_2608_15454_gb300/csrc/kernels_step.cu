@@ -573,37 +573,49 @@ __global__ void k_commit(Dev D) {
   const int b = blockIdx.x;
   if (b >= batch) return;
   const int tid = threadIdx.x;
-  __shared__ int s_c[64], s_kc[64], s_nb[64], s_ok[64];
+  __shared__ int s_c[64], s_kc[64], s_nb[64];
   __shared__ SeqState s_st;
-  __shared__ int s_e, s_a;
+  __shared__ int s_e, s_a, s_last_sp;
   if (tid < n) {
     s_c[tid] = D.cand[b * D.NMAX + tid];
     s_kc[tid] = D.kc[b * D.NMAX + tid];
     s_nb[tid] = D.nb_arg[b * n + tid];
   }
-  if (tid < n - 1) {
-    s_ok[tid] = P.accept == LCA_SPEC ? D.cand[b * D.NMAX + tid + 1] == D.nb_arg[b * n + tid]
-                                     : D.mb_prob[b * (n - 1) + tid] >= P.tau;
-  }
   if (tid == 0) s_st = D.seq[b];
   __syncthreads();
-  if (tid == 0) {
-    int a = 0, e = 0;
+  if (tid < 32) {
+    // Acceptance scan, one warp per sequence (n <= 16 <= 32 lanes): lane i holds the flag of draft
+    // d_{i+2}: its drafter probability >= tau (threshold acceptance, Section 3.1) or its equality with
+    // the next-byte argmax of the row before it (greedy speculative acceptance, Section 6.2). The
+    // accepted drafts are the leading run of set flags: the index of the first clear bit of the
+    // ballot (lanes >= n-1 vote 0, so a clear bit exists).
+    const int lane = tid;
+    bool ok = false;
+    if (lane < n - 1)
+      ok = P.accept == LCA_SPEC ? s_c[lane + 1] == s_nb[lane] : D.mb_prob[b * (n - 1) + lane] >= P.tau;
+    const unsigned vote = __ballot_sync(0xffffffffu, ok);
+    int a = __ffs(~vote) - 1;
+    int e = 0;
     if (!(P.gen && s_st.done)) {
       if (P.force_accept) {
         a = D.forced_a[b];
         a = a < 0 ? 0 : (a > n - 1 ? n - 1 : a);
-      } else {
-        while (a < n - 1 && s_ok[a]) ++a;
       }
       e = 1 + a;
       if (P.gen) {
         const int rem = s_st.budget - s_st.generated;
         e = e < rem ? e : rem;
       }
+    } else {
+      a = 0;
     }
-    s_e = e;
-    s_a = a;
+    // the last committed boundary byte (it starts the new open segment)
+    const unsigned sp = __ballot_sync(0xffffffffu, lane < e && s_c[lane] == D.boundary);
+    if (lane == 0) {
+      s_e = e;
+      s_a = a;
+      s_last_sp = sp ? 31 - __clz((int)sp) : -1;
+    }
   }
   __syncthreads();
   const int e = s_e, t = s_st.t;
@@ -644,9 +656,7 @@ __global__ void k_commit(Dev D) {
     if (P.gen && i < e && s_st.generated + i < D.S) D.out_gen[(size_t)b * D.S + s_st.generated + i] = (uint8_t)s_c[i];
   }
   if (tid == 0) {
-    int last_sp = -1;
-    for (int i = 0; i < e; ++i)
-      if (s_c[i] == D.boundary) last_sp = i;
+    const int last_sp = s_last_sp;
     SeqState& st = D.seq[b];
     D.out_cnt[b] = e;
     st.t = t + e;

@@ -30,7 +30,8 @@ EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "
            "lca_debug_force_accept", "lca_debug_force_candidates", "lca_destroy", "lca_status_str",
            "lca_debug_gemm", "lca_debug_gemm_scratch_bytes", "lca_debug_attn_diag",
            "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
-           "lca_decode_attention_noalloc_capacity")
+           "lca_decode_attention_noalloc_capacity", "lca_decode_attention_status",
+           "lca_decode_attention_noalloc_status", "lca_debug_set_wait_spins")
 
 
 class LcaConfig(ctypes.Structure):
@@ -115,6 +116,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
                                  ctypes.c_size_t, P],
         "lca_decode_attention_noalloc": [P, P, P, P, I32, I32, I32, I32, I32, I32, P, F32, I32, P],
         "lca_decode_attention_noalloc_capacity": [],
+        "lca_decode_attention_status": [P, P],
+        "lca_decode_attention_noalloc_status": [P],
+        "lca_debug_set_wait_spins": [I32],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
@@ -310,6 +314,17 @@ def decode_attention(q, out, k_cache, v_cache, kv_len, scale, splits, scratch=No
     if noalloc:
         return lib.lca_decode_attention_noalloc(*args, st.cuda_stream)
     return lib.lca_decode_attention(*args, scratch.data_ptr(), scratch.numel(), st.cuda_stream)
+
+
+def decode_attention_status(scratch=None, stream=None, noalloc=False, device=None):
+    """Status the kernels of the last decode_attention call recorded (waits for the stream):
+    0, LCA_E_DEVICE_STATE (-5) for a kv_len beyond the cache, or LCA_E_TIMEOUT (-7)."""
+    import torch
+    lib = load_library()
+    st = stream if stream is not None else torch.cuda.current_stream(device)
+    if noalloc:
+        return lib.lca_decode_attention_noalloc_status(st.cuda_stream)
+    return lib.lca_decode_attention_status(scratch.data_ptr(), st.cuda_stream)
 
 
 def debug_gemm(x, W, y, M_dev, err_dev, rows_typ=0, scratch=None, stream=None):

@@ -58,3 +58,34 @@ def test_non_finite_weight_returns_numeric_error(lca):
         ctx.step(3, 0.75)
     assert e.value.status == -6
     ctx.close()
+
+
+def test_bounded_wait_that_runs_out_returns_timeout(lca):
+    """The first weight wait of the weight-streaming GEMV is cut to zero spins, so it reports late
+    at once (its second wait, with the full budget, still drains the copies): the step returns
+    LCA_E_TIMEOUT without a hang or a fault. With the hook cleared, a new prefill gives the same
+    bytes as a context that never timed out."""
+    from synth import make_weights, zipf_text
+    model = TINY.replace(d_model=256, n_heads=4, head_dim=64, d_ff=1024, n_enc=1, n_lm=2, n_nb=1, n_mb=2,
+                         dtype="bf16")
+    W = make_weights(model, gain=8.0, seed=5)
+    p = zipf_text(0, 300)
+    lib = lca.load_library()
+    ref = lca.Context(model, W, max_batch=1, max_bytes=400, max_n=4)
+    ref.prefill([p])
+    want = [ref.step(3, 0.75) for _ in range(3)]
+    ref.close()
+    ctx = lca.Context(model, W, max_batch=1, max_bytes=400, max_n=4)
+    ctx.prefill([p])
+    assert lib.lca_debug_set_wait_spins(0) == 0
+    try:
+        with pytest.raises(lca.LcaError) as e:
+            ctx.step(3, 0.75)
+        assert e.value.status == -7
+    finally:
+        assert lib.lca_debug_set_wait_spins(-1) == 0
+    ctx.prefill([p])
+    got = [ctx.step(3, 0.75) for _ in range(3)]
+    for (o1, c1), (o2, c2) in zip(got, want):
+        assert o1 == o2 and list(c1) == list(c2)
+    ctx.close()

@@ -307,7 +307,7 @@ def test_n1_is_greedy_next_byte_decoding():
 
 @pytest.mark.parametrize("n", [2, 3, 5])
 def test_spec_acceptance_reproduces_greedy(n):
-    """Section 5.2: speculative acceptance makes the output equal next-byte decoding."""
+    """Section 6.2: speculative acceptance makes the output equal next-byte decoding."""
     M = micro_model(gain=40.0)
     want = greedy_decode(M, PROMPT, 14)
     got, recs = generate_reference(M, PROMPT, n, 0.75, SPEC, 14)
