@@ -155,6 +155,14 @@ int lca_generate_fetch(lca_ctx* ctx, uint8_t* out, int32_t* out_len, int32_t* ac
 int lca_debug_state(lca_ctx* ctx, int32_t b, lca_seq_state* out);
 int lca_debug_stats(lca_ctx* ctx, lca_stats* out);
 
+/* Per-step log: out[i] = 1 if decode step first + i (counted from lca_create, as lca_stats.steps)
+ * ran the LM module, else 0. The last 65,536 steps are kept; older or future steps: LCA_E_ARG. */
+int lca_debug_step_log(lca_ctx* ctx, int64_t first, int32_t count, uint8_t* out);
+/* Accepted-draft histogram of the steps since the last reset: out host [max_n], out[a] = steps
+ * (summed over sequences) that accepted a drafts; reset != 0 zeroes it afterwards. lca_generate
+ * also zeroes it when it starts. */
+int lca_debug_accept_hist(lca_ctx* ctx, int32_t* out, int32_t reset);
+
 /* Run later steps as direct kernel launches instead of one graph (on != 0), so that
  * per-kernel profilers can see them; the LM decision is then read back on the host.
  * Results are identical. */

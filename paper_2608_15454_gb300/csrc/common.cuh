@@ -119,6 +119,7 @@ constexpr int kVocab = 256;
 constexpr int kMaxKSplit = 8;     // split-K ways of the skinny linear kernel
 constexpr int kMaxAttnSplit = 16; // key-range splits of decode attention
 constexpr int kAttnQT = 8;        // query rows per attention tile (decode)
+constexpr int kStepLog = 1 << 16; // steps remembered by the per-step log
 
 // device error word bits
 constexpr int kErrIndex = 1;   // an index was out of range; the access was skipped
@@ -334,6 +335,7 @@ struct Dev {
   Params* params;
   int* err;
   Stats* stats;
+  uint8_t* step_log; // [kStepLog] whether step s ran the LM module, at s % kStepLog
 
   // scratch
   float* lin_part; // split-K partials

@@ -464,6 +464,7 @@ __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handl
     if (b == 0) {
       *D.r_lm.M = total;
       if (use_handle) cudaGraphSetConditional(hcond, total > 0 ? 1u : 0u);
+      D.step_log[D.stats->steps % kStepLog] = total > 0 ? 1 : 0;
       D.stats->steps += 1;
       D.stats->lm_steps += total > 0;
       D.stats->lm_rows += total;

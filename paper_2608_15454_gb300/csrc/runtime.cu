@@ -161,6 +161,7 @@ void carve(const lca_config& c, char* base, Layout& L) {
   D.params = cv.take<Params>(kParamSlots);
   D.err = cv.take<int>(1);
   D.stats = cv.take<Stats>(1);
+  D.step_log = cv.take<uint8_t>(kStepLog);
 
   const size_t gemv_rows = B <= 4 ? R : 64;
   D.lin_part_floats = (size_t)kMaxKSplit * gemv_rows * d;
@@ -1261,6 +1262,28 @@ int lca_debug_stats(lca_ctx* c, lca_stats* out) {
   out->kernels_per_step = it == c->launches.end() ? 0 : it->second.first;
   out->kernels_per_lm_run = it == c->launches.end() ? 0 : it->second.second;
   out->workspace_bytes = (int64_t)c->ws_bytes;
+  return LCA_OK;
+}
+
+int lca_debug_step_log(lca_ctx* c, int64_t first, int32_t count, uint8_t* out) {
+  if (!c || !out || count < 0 || first < 0) return LCA_E_ARG;
+  Stats s;
+  CK(cudaMemcpyAsync(&s, c->L.D.stats, sizeof(s), cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  const long long steps = (long long)s.steps;
+  if (first + count > steps || steps - first > kStepLog) return LCA_E_ARG;
+  std::vector<uint8_t> ring(kStepLog);
+  CK(cudaMemcpy(ring.data(), c->L.D.step_log, kStepLog, cudaMemcpyDeviceToHost));
+  for (int i = 0; i < count; ++i) out[i] = ring[(size_t)((first + i) % kStepLog)];
+  return LCA_OK;
+}
+
+int lca_debug_accept_hist(lca_ctx* c, int32_t* out, int32_t reset) {
+  if (!c) return LCA_E_ARG;
+  Dev& D = c->L.D;
+  if (out) CK(cudaMemcpyAsync(out, D.hist, sizeof(int) * D.NMAX, cudaMemcpyDeviceToHost, c->stream));
+  if (reset) CK(cudaMemsetAsync(D.hist, 0, sizeof(int) * D.NMAX, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
   return LCA_OK;
 }
 

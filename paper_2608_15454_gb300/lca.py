@@ -31,7 +31,8 @@ EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "
            "lca_debug_gemm", "lca_debug_gemm_scratch_bytes", "lca_debug_attn_diag",
            "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
            "lca_decode_attention_noalloc_capacity", "lca_decode_attention_status",
-           "lca_decode_attention_noalloc_status", "lca_debug_set_wait_spins")
+           "lca_decode_attention_noalloc_status", "lca_debug_set_wait_spins",
+           "lca_debug_step_log", "lca_debug_accept_hist")
 
 
 class LcaConfig(ctypes.Structure):
@@ -119,6 +120,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_decode_attention_status": [P, P],
         "lca_decode_attention_noalloc_status": [P],
         "lca_debug_set_wait_spins": [I32],
+        "lca_debug_step_log": [P, ctypes.c_int64, I32, P],
+        "lca_debug_accept_hist": [P, P, I32],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
@@ -245,6 +248,18 @@ class Context:
         s = LcaStats()
         self._check(self.lib.lca_debug_stats(self.h, ctypes.byref(s)), "lca_debug_stats")
         return {f: getattr(s, f) for f, _ in LcaStats._fields_}
+
+    def step_log(self, first, count):
+        """1 per decode step [first, first + count) that ran the LM module, else 0."""
+        out = np.zeros(max(count, 1), dtype=np.uint8)
+        self._check(self.lib.lca_debug_step_log(self.h, first, count, _ptr(out)), "lca_debug_step_log")
+        return out[:count]
+
+    def accept_hist(self, reset=False):
+        """Steps (summed over sequences) by accepted drafts since the last reset, [max_n]."""
+        out = np.zeros(self.max_n, dtype=np.int32)
+        self._check(self.lib.lca_debug_accept_hist(self.h, _ptr(out), 1 if reset else 0), "lca_debug_accept_hist")
+        return out
 
     def set_eager(self, on: bool):
         self._check(self.lib.lca_debug_set_eager(self.h, 1 if on else 0), "lca_debug_set_eager")

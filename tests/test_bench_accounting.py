@@ -57,16 +57,42 @@ def test_kv_bytes_per_step_of_the_paper_model():
 
 
 def test_roofline_of_the_dominant_family():
+    """The family's in-graph time is its share of the eager kernel time times the graph step time,
+    so the families add up to the step; achieved = algorithmic bytes per launch over that time."""
     prof = {"linear": {"launches": 88, "ms": 0.264, "bytes": 88 * 8.39e6},
             "attention": {"launches": 22, "ms": 0.110, "bytes": 0.0},
-            "head": {"launches": 2, "ms": 0.02, "bytes": 0.0}}
-    r = bench.roofline(prof, 6670.9, "measured", "nowhere", 1.0e6, 2)
+            "head": {"launches": 2, "ms": 0.026, "bytes": 0.0}}
+    steps, ms_per_step = 2, 0.1  # graph: 0.1 ms/step against 0.2 ms/step of eager kernel time
+    r = bench.roofline(prof, 6670.9, "measured", "nowhere", 1.0e6, steps, ms_per_step)
     assert r["bound"] == "hbm" and r["unit"] == "GB/s" and r["peak"] == 6670.9
-    # 8.39 MB per launch in 3 us: 2,796.7 GB/s
-    assert np.isclose(r["achieved"], 8.39e6 / 3e-6 / 1e9)
+    share = 0.264 / 0.4
+    assert np.isclose(r["share_of_step"], share)
+    per_launch_s = share * ms_per_step * 1e-3 * steps / 88
+    assert np.isclose(r["achieved"], 8.39e6 / per_launch_s / 1e9)
     assert np.isclose(r["frac"], r["achieved"] / 6670.9)
     assert r["traffic"] is None
+    # the implied kernel time per step never exceeds the step
+    assert r["in_graph_us_per_launch"] * r["launches_per_step"] <= ms_per_step * 1e3 + 1e-9
     # attention dominant: its bytes per launch are the step KV bytes times the steps, per launch
     prof["attention"]["ms"] = 1.0
-    r = bench.roofline(prof, 6670.9, "measured", "nowhere", 1.0e6, 2)
+    r = bench.roofline(prof, 6670.9, "measured", "nowhere", 1.0e6, steps, ms_per_step)
     assert np.isclose(r["algorithmic_bytes_per_launch"], 2 * 1.0e6 / 22)
+
+
+def test_blocks_and_context_size():
+    assert bench.blocks_of(20) == [20]
+    assert bench.blocks_of(130) == [64, 64, 2]
+    assert sum(bench.blocks_of(512)) == 512
+    w = WORKLOADS["paper_b1"]
+    # a block, the warm-up or the profiled steps after one prefill, each at most n bytes a step
+    assert bench.context_bytes(w, 7, 512, 5, 20) == 1024 + (64 + 2) * 7 + 8
+    assert bench.context_bytes(w, 3, 20, 5, 20) == 1024 + (20 + 2) * 3 + 8
+
+
+def test_sweep_covers_the_rest_of_the_metric():
+    class A:
+        sweep, batch, prompt_bytes = "auto", None, None
+    cases = bench.sweep_cases(WORKLOADS["paper_b1"], 3, A)
+    assert cases == [("paper_b1", 4), ("paper_b1", 5), ("paper_b1", 6), ("paper_b1", 7), ("paper_b32", 4)]
+    A.sweep = "none"
+    assert bench.sweep_cases(WORKLOADS["paper_b1"], 3, A) == []
