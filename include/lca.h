@@ -205,11 +205,12 @@ int lca_debug_gemm(const float* x, const void* W, float* y, int32_t M, int32_t N
  * ring slot, 1: waiting for a chunk), chunk, stage, chunks, key lo, key hi, chunks before the
  * tile, copies issued}. Clears the record. */
 int lca_debug_attn_diag(int32_t* out16);
-/* Test hook for the bounded waits: the first wait of the weight-streaming GEMV for its weight tile
- * spins at most `spins` times (< 0: the default, 2^22) on the current device. With 0 the wait
- * reports late at once: the kernel records the timeout bit in the device error word, waits once
- * more with the full budget for its copies in flight, then completes, and the call returns
- * LCA_E_TIMEOUT. Outside a test, a call that returns LCA_E_TIMEOUT has undefined results, and if
+/* Test hook for the bounded waits: the first wait of the weight-streaming GEMV for its weight tile,
+ * and the first wait of each phase of the persistent stack kernel for its weight ring, spin at most
+ * `spins` times (< 0: the default, 2^22) on the current device. With 0 the wait reports late at
+ * once: the kernel records the timeout bit in the device error word, waits once more with the full
+ * budget for its copies in flight, then completes (the stack kernel skips its remaining blocks),
+ * and the call returns LCA_E_TIMEOUT. Outside a test, a call that returns LCA_E_TIMEOUT has undefined results, and if
  * the second wait ran out as well a copy may have been left in flight: destroy the context. */
 int lca_debug_set_wait_spins(int32_t spins);
 /* Bytes of device scratch lca_debug_gemm needs. */

@@ -45,7 +45,7 @@ static_assert(sizeof(TraceRec) == 48, "trace record layout");
 enum TraceTag : int {
   TT_GEMV = 1, TT_GEMV_F32, TT_GEMM, TT_ROWSTATS, TT_ATTN, TT_HEAD, TT_MB_PLAN, TT_MB_FILL,
   TT_MLP_PLAN, TT_VERIFY_PLAN, TT_SEGMENT, TT_LM_SCATTER, TT_NB_INPUT, TT_COMMIT, TT_LOOP_CTL,
-  TT_OTHER, TT_UMMA, TT_SPLIT, TT_SGEMM
+  TT_OTHER, TT_UMMA, TT_SPLIT, TT_SGEMM, TT_STACK
 };
 static __device__ TraceRec* g_trace = nullptr;
 static __device__ unsigned int* g_trace_n = nullptr;
@@ -128,7 +128,7 @@ constexpr int kErrTimeout = 4; // a bounded wait ran out
 // which kernel family's wait ran out (set together with kErrTimeout; reported on stderr)
 constexpr int kErrWaitAttn3 = 1 << 8, kErrWaitAttnMma = 1 << 9, kErrWaitGemv = 1 << 10, kErrWaitGemm = 1 << 11,
               kErrWaitAttnW = 1 << 13,
-              kErrWaitGemvReduce = 1 << 12;
+              kErrWaitGemvReduce = 1 << 12, kErrWaitStack = 1 << 14;
 
 // Linear epilogues.
 enum Epi : int {
@@ -248,6 +248,8 @@ struct ProfScope {
   }
 };
 
+struct StackLayer;
+
 // Workspace layout (device pointers into the caller's workspace).
 struct Dev {
   // shape
@@ -347,7 +349,59 @@ struct Dev {
   float* inv_rms;  // [R]
   float2* rope;    // [max(S,L)][hd/2]
   int rope_slots;
+
+  // persistent stack kernel (bf16, head_dim 64, d <= 1024): layer tables, attention partials and
+  // counters, grid-barrier words; persist = 0 turns it off
+  int persist;
+  int stk_grid;        // CTAs of a launch (one per SM)
+  int stk_splits;      // attention key splits per (sequence, head)
+  StackLayer* stk_enc;
+  StackLayer* stk_lm;
+  StackLayer* stk_nb;
+  StackLayer* stk_mb;
+  float* stk_apart;    // [B][H][splits][rows of a sequence][68]
+  size_t stk_apart_rows;  // rows per (sequence, head, split) the partial buffer holds
+  int* stk_cnt;        // [B * H] last-arriver counters of the attention combine
+  unsigned* stk_bar;   // [4]: grid-barrier arrivals, exits, abort
+  // inputs of the stack kernel's linear phases, written already split by the producing phase:
+  // bf16 halves (v = hi + lo) of the normalised-input rows x * g [R][d], of the attention output
+  // [R][d] and of the SwiGLU output [R][F]; per-row sums of squares of x per 16-column tile [R][d/16]
+  __nv_bfloat16 *stk_ahi, *stk_alo, *stk_thi, *stk_tlo, *stk_mhi, *stk_mlo;
+  float* stk_ss;
+  float* stk_w2part;   // [F / KS][R][d] W2 partial sums per K-slice
+  int* stk_w2cnt;      // [d / 16] last-arriver counters of W2's column tiles
 };
+
+// One block of a stack as the persistent stack kernel reads it (device array, filled at create).
+struct StackLayer {
+  const __nv_bfloat16* wqkv; // [3d][d]
+  const __nv_bfloat16* wo;   // [d][d]
+  const __nv_bfloat16* w13;  // [2F][d], rows interleaved (W1_j, W3_j)
+  const __nv_bfloat16* w2;   // [d][F]
+  const float* attn_norm;
+  const float* mlp_norm;
+  void* k;                   // KV cache layer [B][H][S][64] bf16
+  void* v;
+};
+
+// A stack run by the persistent kernel (kernels_stack.cu).
+struct StackRun {
+  const StackLayer* layers; // device [L]
+  int L;
+  float* x;                 // residual stream rows (in place)
+  Rows rows;
+  int M_cap;
+  int S;                    // cache slots per (sequence, head)
+  const int* stable;        // per-sequence committed cache length (stride in ints), or nullptr
+  int stable_stride;
+  int stable_add;
+};
+bool stack_ready(const Dev& D);
+// Runs the whole stack as one launch; false if the persistent kernel cannot run this stack.
+bool launch_stack(const Dev& D, const StackRun& r, cudaStream_t s);
+void kernel_attrs_stack(Dev* D);
+void stack_set_first_wait(int spins);  // test hook (see lca_debug_set_wait_spins)
+void trace_set_stack(TraceRec* buf, unsigned* counter, unsigned cap);
 
 struct Block {
   const float* attn_norm;

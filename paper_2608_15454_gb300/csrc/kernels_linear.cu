@@ -917,5 +917,6 @@ LCA_TRACE_SETTER(trace_set_linear)
 
 extern "C" int lca_debug_set_wait_spins(int32_t spins) {
   const int v = spins < 0 ? lca::kWaitSpins : spins;
+  lca::stack_set_first_wait(spins);
   return cudaMemcpyToSymbol(lca::g_first_wait_spins, &v, sizeof(v)) == cudaSuccess ? LCA_OK : LCA_E_CUDA;
 }

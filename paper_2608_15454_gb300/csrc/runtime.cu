@@ -173,6 +173,39 @@ void carve(const lca_config& c, char* base, Layout& L) {
   D.inv_rms = cv.take<float>(R);
   D.rope_slots = (int)std::max(S, Lt);
   D.rope = cv.take<float2>((size_t)D.rope_slots * (D.hd / 2));
+  // persistent stack kernel: bf16, head_dim 64, d <= 1024 (one K-slice), up to four sequences
+  const size_t KS = std::min<size_t>(d, 1024);
+  const bool stk = c.dtype == LCA_BF16 && D.hd == 64 && d % 16 == 0 && d <= 1024 && KS % 16 == 0 &&
+                   F % KS == 0 && F / KS <= 4 && B <= 4;
+  if (stk) {
+    D.stk_enc = cv.take<StackLayer>(std::max(c.n_enc, 1));
+    D.stk_lm = cv.take<StackLayer>(std::max(c.n_lm, 1));
+    D.stk_nb = cv.take<StackLayer>(std::max(c.n_nb, 1));
+    D.stk_mb = cv.take<StackLayer>(std::max(c.n_mb, 1));
+    D.stk_apart_rows = (size_t)std::max(S, Lt) + NM;
+    D.stk_apart = cv.take<float>(B * D.H * kMaxAttnSplit * D.stk_apart_rows * 68);
+    D.stk_cnt = cv.take<int>(B * D.H);
+    D.stk_bar = cv.take<unsigned>(64);
+    D.stk_ahi = cv.take<__nv_bfloat16>(R * d);
+    D.stk_alo = cv.take<__nv_bfloat16>(R * d);
+    D.stk_thi = cv.take<__nv_bfloat16>(R * d);
+    D.stk_tlo = cv.take<__nv_bfloat16>(R * d);
+    D.stk_mhi = cv.take<__nv_bfloat16>(R * F);
+    D.stk_mlo = cv.take<__nv_bfloat16>(R * F);
+    D.stk_ss = cv.take<float>(R * (d / 16));
+    D.stk_w2part = cv.take<float>((F / KS) * R * d);
+    D.stk_w2cnt = cv.take<int>(d / 16);
+  } else {
+    D.stk_enc = D.stk_lm = D.stk_nb = D.stk_mb = nullptr;
+    D.stk_apart = nullptr;
+    D.stk_cnt = nullptr;
+    D.stk_bar = nullptr;
+    D.stk_apart_rows = 0;
+    D.stk_ahi = D.stk_alo = D.stk_thi = D.stk_tlo = D.stk_mhi = D.stk_mlo = nullptr;
+    D.stk_ss = nullptr;
+    D.stk_w2part = nullptr;
+    D.stk_w2cnt = nullptr;
+  }
   L.bytes = cv.off + 256;
 }
 
@@ -329,9 +362,23 @@ bool link_split(const Dev& D, bool tiled, LinearArgs& prod, LinearArgs& cons, in
 void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& rows, int M_cap,
                int M_typ, int qt_grid, int splits, cudaStream_t s, const void* next_w = nullptr,
                size_t next_bytes = 0, const int* stable = nullptr, int stable_extra = 0,
-               bool short_kv = false, int stable_add = 0) {
+               bool short_kv = false, int stable_add = 0, const StackLayer* stk = nullptr) {
   Dev& D = c->L.D;
   const bool tiled = tiled_for(D, M_typ);
+  // decode steps with few rows: the whole stack as one persistent launch
+  if (stk && !tiled && !blocks.empty() && stack_ready(D)) {
+    StackRun r{};
+    r.layers = stk;
+    r.L = (int)blocks.size();
+    r.x = x;
+    r.rows = rows;
+    r.M_cap = M_cap;
+    r.S = blocks[0].kv.S;
+    r.stable = stable;
+    r.stable_stride = (int)(sizeof(SeqState) / sizeof(int));
+    r.stable_add = stable_add;
+    if (launch_stack(D, r, s)) return;
+  }
   const size_t tb = tw_bytes(D.dtype);
   const size_t b_qkv = 3ull * D.d * D.d * tb, b_o = (size_t)D.d * D.d * tb;
   const size_t b_13 = 2ull * D.F * D.d * tb, b_2 = (size_t)D.d * D.F * tb;
@@ -489,7 +536,7 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
       // the window holds about two words of keys: a short cache
       run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2, kMbWindowKeys), s,
                 c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype), nullptr, 0,
-                true);
+                true, 0, D.stk_mb);
     } else {
       launch_mlp_plan(D, s);
       run_mlp_heads(c, n, s);
@@ -501,7 +548,7 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
   launch_verify_plan(D, s);
   run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1, c->kv_bytes_typ + n), s,
             c->L.nb.empty() ? nullptr : c->L.nb[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype),
-            &D.seq[0].t, n);
+            &D.seq[0].t, n, false, 0, D.stk_enc);
 }
 
 void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
@@ -509,7 +556,7 @@ void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
   // about one new latent per sequence every few bytes
   // latent slots [0, K] (BOS and the committed latents) do not change during the step
   run_stack(c, c->L.lm, D.x_lm, D.r_lm, D.B * n, D.B, 1, attn_splits(D, D.B, 1, c->kv_lat_typ + 1), s,
-            nullptr, 0, &D.seq[0].K, 1, false, 1);
+            nullptr, 0, &D.seq[0].K, 1, false, 1, D.stk_lm);
   launch_lm_scatter(D, s);
 }
 
@@ -519,7 +566,7 @@ void enqueue_verify_commit(lca_ctx* c, int n, cudaStream_t s) {
   // (4) upsample + next-byte decoder over the n candidates, head
   launch_nb_input(D, s);
   run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1, c->kv_bytes_typ + n), s, nullptr, 0,
-            &D.seq[0].t, n);
+            &D.seq[0].t, n, false, 0, D.stk_nb);
   launch_head(D, D.x_nb, nullptr, D.r_v.M, B * n, D.nb_norm, D.nb_logits, D.nb_arg, D.nb_prob, s);
   // (5) accept + commit
   launch_commit(D, s);
@@ -909,6 +956,12 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.attn_t = (at && at[0] == '0') ? 0 : 1;
     const char* mk = getenv("LCA_ATTN_MIN_KEYS");
     D.attn_min_keys = mk ? std::max(0, atoi(mk)) : 0;
+    const char* pe = getenv("LCA_PERSIST");
+    D.persist = (pe && pe[0] == '1') ? 1 : 0;
+    D.stk_grid = D.num_sms;
+    D.stk_splits = std::max(1, std::min(kMaxAttnSplit, D.num_sms / std::max(1, D.B * D.H)));
+    if (D.stk_enc) kernel_attrs_stack(&D);
+    else D.persist = 0;
   }
   // state and counters start at zero
   if (check(cudaMemsetAsync(c->ws, 0, c->L.bytes, c->stream), "memset")) return fail(LCA_E_CUDA);
@@ -945,6 +998,28 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
             bk.kv.tmaps = c->kvmaps[bk.kv.k].b;
           }
         }
+  }
+  if (D.stk_enc) {
+    // the persistent stack kernel's view of each block
+    auto table = [&](std::vector<Block>& v, StackLayer* dst) -> int {
+      std::vector<StackLayer> h(v.size());
+      for (size_t l = 0; l < v.size(); ++l) {
+        h[l].wqkv = static_cast<const __nv_bfloat16*>(v[l].wqkv);
+        h[l].wo = static_cast<const __nv_bfloat16*>(v[l].wo);
+        h[l].w13 = static_cast<const __nv_bfloat16*>(v[l].w13);
+        h[l].w2 = static_cast<const __nv_bfloat16*>(v[l].w2);
+        h[l].attn_norm = v[l].attn_norm;
+        h[l].mlp_norm = v[l].mlp_norm;
+        h[l].k = v[l].kv.k;
+        h[l].v = v[l].kv.v;
+      }
+      if (h.empty()) return LCA_OK;
+      return check(cudaMemcpyAsync(dst, h.data(), sizeof(StackLayer) * h.size(), cudaMemcpyHostToDevice, c->stream),
+                   "stack tables");
+    };
+    if (table(c->L.enc, D.stk_enc) || table(c->L.lm, D.stk_lm) || table(c->L.nb, D.stk_nb) ||
+        table(c->L.mb, D.stk_mb) || check(cudaStreamSynchronize(c->stream), "stack tables"))
+      return fail(LCA_E_CUDA);
   }
   launch_rope_table(D, cfg->rope_base, c->stream);
   if (check(cudaGetLastError(), "rope") || check(cudaStreamSynchronize(c->stream), "create sync"))
@@ -1459,6 +1534,7 @@ int lca_debug_trace(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t step
   trace_set_attn(buf, counter, capu);
   trace_set_step(buf, counter, capu);
   trace_set_umma(buf, counter, capu);
+  trace_set_stack(buf, counter, capu);
   Params& P = c->host_params;
   P.gen = 0;
   P.force_accept = 0;
@@ -1471,6 +1547,7 @@ int lca_debug_trace(lca_ctx* c, int32_t n, float tau, int32_t mode, int32_t step
   trace_set_attn(nullptr, nullptr, 0);
   trace_set_step(nullptr, nullptr, 0);
   trace_set_umma(nullptr, nullptr, 0);
+  trace_set_stack(nullptr, nullptr, 0);
   unsigned got = 0;
   CK(cudaMemcpy(&got, counter, sizeof(unsigned), cudaMemcpyDeviceToHost));
   got = std::min(got, capu);

@@ -274,7 +274,7 @@ class Context:
     TRACE_TAGS = {1: "gemv", 2: "gemv_f32", 3: "gemm", 4: "rowstats", 5: "attn", 6: "head",
                   7: "mb_plan", 8: "mb_fill", 9: "mlp_plan", 10: "verify_plan", 11: "segment",
                   12: "lm_scatter", 13: "nb_input", 14: "commit", 15: "loop_ctl", 16: "other",
-                  17: "umma", 18: "split", 19: "sgemm"}
+                  17: "umma", 18: "split", 19: "sgemm", 20: "stack"}
 
     def trace(self, n, tau, mode, steps, cap=1 << 18):
         rec = np.zeros(cap, dtype=[("t0", "<u8"), ("t1", "<u8"), ("tw", "<u8"), ("tag", "<i4"),

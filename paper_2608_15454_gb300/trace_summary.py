@@ -31,7 +31,7 @@ if ROOT not in sys.path:
 
 TAGS = {1: "gemv", 2: "gemv_f32", 3: "gemm", 4: "rowstats", 5: "attn", 6: "head", 7: "mb_plan",
         8: "mb_fill", 9: "mlp_plan", 10: "verify_plan", 11: "segment", 12: "lm_scatter",
-        13: "nb_input", 14: "commit", 15: "loop_ctl", 16: "other", 17: "umma", 18: "split", 19: "sgemm"}
+        13: "nb_input", 14: "commit", 15: "loop_ctl", 16: "other", 17: "umma", 18: "split", 19: "sgemm", 20: "stack"}
 PHASES = {"gemv": ("staged", "weights", "dots", "exit"), "attn": ("keys landed", "key loop", "combined", "exit")}
 
 

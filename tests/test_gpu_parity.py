@@ -266,3 +266,32 @@ def test_small_bf16_long_context_batch_one(lca):
         assert out[0] == r.emitted
         st = ctx.state(0)
         assert (st["t"], st["K"]) == (dec.t, dec.K)
+
+
+@pytest.mark.parametrize("mb_kind", ["lca", "mlp"])
+def test_persistent_stack_kernel_matches_oracle(lca, mb_kind, monkeypatch):
+    """The persistent block-stack kernel (LCA_PERSIST=1: every block of a module in one launch, grid
+    barriers between the phases, split-on-write inputs staged by bulk copies) against the oracle at
+    d = 256 with forced boundaries: logits within the bf16 tolerance, bytes and state equal."""
+    monkeypatch.setenv("LCA_PERSIST", "1")
+    model = SMALL_BF16 if mb_kind == "lca" else SMALL_BF16.replace(mb_kind="mlp", n_mb=3, n_mlp_heads=5)
+    W = make_weights(model, gain=8.0, seed=5)
+    prompts = [zipf_text(0, 300)]
+    n = 4
+    ctx = new_ctx(lca, model, W, 1, 600, 6)
+    ctx.prefill(prompts)
+    dec = IncrementalDecoder(Model(model, W))
+    dec.prefill(prompts[0])
+    for s in range(10):
+        cand = bytes([97 + s % 26, 32 if s % 2 == 0 else 98, 99, 32])
+        ctx.force_candidates([cand], n)
+        ctx.force_accept([s % 4])
+        r = dec.step(n, 0.75, THRESH, forced=s % 4, forced_cand=cand)
+        out, cnt = ctx.step(n, 0.75, lca.LCA_THRESH)
+        nb, mb = ctx.logits(n)
+        np.testing.assert_allclose(nb[0], r.nb_logits, atol=BF16_TOL * 8, rtol=0)
+        np.testing.assert_allclose(mb[0], r.mb_logits, atol=BF16_TOL * 8, rtol=0)
+        assert out[0] == r.emitted
+        st = ctx.state(0)
+        assert (st["t"], st["K"]) == (dec.t, dec.K)
+    ctx.close()
