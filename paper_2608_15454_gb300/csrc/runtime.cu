@@ -943,7 +943,7 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     const char* sc = getenv("LCA_ATTN_SPLIT_CAP");
     D.attn_split_cap = sc ? std::max(1, std::min(16, atoi(sc))) : 16;
     const char* tr = getenv("LCA_TILED_MIN_ROWS");
-    D.tiled_min_rows = tr ? std::max(0, atoi(tr)) : 16;
+    D.tiled_min_rows = tr ? std::max(0, atoi(tr)) : 32;
     const char* ap = getenv("LCA_ATTN_PIPE");
     D.attn_pipe = ap ? atoi(ap) : 2;
     const char* an = getenv("LCA_ATTN_NS");

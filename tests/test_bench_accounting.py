@@ -96,3 +96,15 @@ def test_sweep_covers_the_rest_of_the_metric():
     assert cases == [("paper_b1", 4), ("paper_b1", 5), ("paper_b1", 6), ("paper_b1", 7), ("paper_b32", 4)]
     A.sweep = "none"
     assert bench.sweep_cases(WORKLOADS["paper_b1"], 3, A) == []
+
+
+def test_prefill_flops_of_the_paper_model():
+    """Linear FLOPs: 2 x 16 d^2 per row per block (32 d^2 = 33.6 MFLOP at d = 1024); the byte
+    modules see every byte, the LM module every latent plus BOS; causal attention 2 d T (T + 1)
+    per byte layer."""
+    m = WORKLOADS["paper_b1"].model
+    p = b"ab cd"  # 5 bytes, one boundary: 2 latent rows
+    d = 1024
+    lin = 2 * 16 * d * d * (5 * 4 + 2 * 16)
+    att = 2 * d * 5 * 6 * 4 + 2 * d * 2 * 3 * 16
+    assert bench.prefill_flops(m, [p]) == lin + att + 2 * 256 * d
