@@ -77,6 +77,17 @@ typedef struct {
   float rope_base, rms_eps, attn_scale; /* 1e5, 1e-6, 1/sqrt(head_dim) (Section 4.2) */
   int32_t dtype;                   /* LCA_F32 | LCA_BF16 */
   int32_t max_batch, max_bytes, max_n; /* max_bytes bounds prompt + generated + max_n */
+  /* Paged KV caches: every cache layer is a pool of pages of 64 slots, [pages][n_heads][64]
+   * [head_dim], and each sequence maps its slots to pages through a page table (one per module
+   * kind, shared by that module's layers). kv_pages: pages of each encoder and next-byte layer's
+   * pool (byte positions); lm_pages: of each LM-module layer's pool (latents); mb_pages: of each
+   * multi-byte layer's pool (window rows). 0: enough for every sequence at max_bytes positions
+   * (max_bytes + 1 latents). The prefill maps the prompts' pages (LCA_E_CAPACITY if they do not
+   * fit); a decode step maps a page when a sequence's positions, latents or window first reach it,
+   * from a bump counter, and a page stays mapped until the next prefill. A step that finds a pool
+   * exhausted leaves those slots unwritten and returns LCA_E_CAPACITY; its results are then
+   * undefined until the next prefill. max_bytes must stay below 131,072. */
+  int32_t kv_pages, lm_pages, mb_pages;
 } lca_config;
 
 /* One named weight tensor: device pointer, element count, LCA_F32|LCA_BF16.
@@ -162,6 +173,13 @@ int lca_debug_step_log(lca_ctx* ctx, int64_t first, int32_t count, uint8_t* out)
  * (summed over sequences) that accepted a drafts; reset != 0 zeroes it afterwards. lca_generate
  * also zeroes it when it starts. */
 int lca_debug_accept_hist(lca_ctx* ctx, int32_t* out, int32_t reset);
+/* Page table of one cache kind (cache: 0 byte positions of the encoder and next-byte layers, 1 LM
+ * latents, 2 multi-byte windows): out host [max_batch][*row_len], out[b * row_len + j] = the pool
+ * page of slots [64 j, 64 j + 64) of sequence b, or -1 (unmapped); *used = pages mapped from the
+ * pool so far; *pages = the pool's size. cap (entries of out) below max_batch * row_len:
+ * LCA_E_CAPACITY (and *row_len is still set). Synchronises the context's stream. */
+int lca_debug_page_table(lca_ctx* ctx, int32_t cache, int32_t* out, int64_t cap, int32_t* row_len, int32_t* used,
+                         int32_t* pages);
 
 /* Run later steps as direct kernel launches instead of one graph (on != 0), so that
  * per-kernel profilers can see them; the LM decision is then read back on the host.

@@ -125,6 +125,7 @@ constexpr int kStepLog = 1 << 16; // steps remembered by the per-step log
 constexpr int kErrIndex = 1;   // an index was out of range; the access was skipped
 constexpr int kErrNumeric = 2; // non-finite logits
 constexpr int kErrTimeout = 4; // a bounded wait ran out
+constexpr int kErrPages = 8;   // a cache pool had no free page; the slots stayed unmapped
 // which kernel family's wait ran out (set together with kErrTimeout; reported on stderr)
 constexpr int kErrWaitAttn3 = 1 << 8, kErrWaitAttnMma = 1 << 9, kErrWaitGemv = 1 << 10, kErrWaitGemm = 1 << 11,
               kErrWaitAttnW = 1 << 13,
@@ -145,21 +146,103 @@ struct Rows {
   int* b;
   int* pos;
   int* slot;
+  int* page;      // physical page of the row's cache slot (paged caches), written with slot
   int* kvlen;
   int* seq_start; // [B] first row of each sequence (rows of a sequence are contiguous)
   int* seq_count; // [B]
   int* M;         // total rows (device scalar)
 };
 
-// One KV-cache layer: [B][H][S][hd] of the storage type.
+// One KV-cache layer of the storage type. Paged (pt != nullptr): the layer is a pool of pages of
+// kPage slots, [pages][H][kPage][hd]; slot s of sequence b lives in page pt[b * pt_ld + s / kPage]
+// (-1: not mapped). Contiguous (pt == nullptr, the standalone attention op): [B][H][S][hd].
+constexpr int kPage = 64;
 struct KV {
   void* k;
   void* v;
-  int S; // slots per (b, h)
+  int S; // logical slots per (b, h)
   // host copies of the TMA tensor maps of K and V (bf16, head_dim 64: 64-key x 64-dim boxes with
-  // the 128-byte swizzle), or nullptr; used by the tensor-core decode attention
+  // the 128-byte swizzle, over [pages * H * kPage][64] rows when paged), or nullptr; used by the
+  // tensor-core decode attention
   const void* tmaps;
+  const int* pt;  // page table [B][pt_ld], or nullptr
+  int pt_ld;
+  int pages;      // pages of the pool (paged)
 };
+// Element offset of (sequence b, head h, slot s) when slot s lies in physical page pg (paged; the
+// caller checked pg) or in the contiguous layout (pg ignored).
+__device__ __forceinline__ size_t kv_addr(const KV& kv, int H, int hd, int b, int h, int s, int pg) {
+  if (!kv.pt) return (((size_t)b * H + h) * kv.S + s) * hd;
+  return (((size_t)pg * H + h) * kPage + (s & (kPage - 1))) * hd;
+}
+// A cache write of slot s in page pg is in range (the writers take pg from the row's page).
+__device__ __forceinline__ bool kv_write_ok(const KV& kv, int s, int pg) {
+  return s >= 0 && s < kv.S && (!kv.pt || (pg >= 0 && pg < kv.pages));
+}
+// Page of slot s of sequence b from the table, read through L2 (the decode steps' plan kernels
+// map pages while the readers of an earlier launch may still run); an unmapped or out-of-range
+// entry (or a slot past the table) reads page 0, whose keys the callers mask. 0 for the contiguous
+// layout.
+__device__ __forceinline__ int kv_page_cg(const KV& kv, int b, int s) {
+  if (!kv.pt || s < 0 || s / kPage >= kv.pt_ld) return 0;
+  const int pg = __ldcg(kv.pt + (size_t)b * kv.pt_ld + s / kPage);
+  return (pg < 0 || pg >= kv.pages) ? 0 : pg;
+}
+// Element offset of (b, h, s), looking the page up.
+__device__ __forceinline__ size_t kv_off(const KV& kv, int H, int hd, int b, int h, int s) {
+  return kv_addr(kv, H, hd, b, h, s, kv_page_cg(kv, b, s));
+}
+// The page table row of sequence b into shared memory (pt_ld entries, checked as kv_page_cg
+// does); nothing for the contiguous layout. The caller synchronises before the first use.
+__device__ __forceinline__ void kv_stage_pages(const KV& kv, int b, int* s_pt, int tid, int nthreads) {
+  if (!kv.pt) return;
+  for (int i = tid; i < kv.pt_ld; i += nthreads) {
+    const int pg = __ldcg(kv.pt + (size_t)b * kv.pt_ld + i);
+    s_pt[i] = (pg < 0 || pg >= kv.pages) ? 0 : pg;
+  }
+}
+// Shared-memory bytes of a staged page table row (16-byte multiple).
+inline size_t kv_pages_smem(const KV& kv) { return kv.pt ? ((size_t)kv.pt_ld * 4 + 15) / 16 * 16 : 0; }
+// The most page-table entries a reader stages (slots per sequence and cache: kMaxPtRow * kPage).
+constexpr int kMaxPtRow = 2048;
+// L2 prefetch (a hint) of slots [lo, hi) of (b, h) of one cache tensor (base: kv.k or kv.v, elements
+// of es bytes): one bulk prefetch per page, the table entries of up to eight pages loaded before
+// their prefetches are issued.
+__device__ __forceinline__ void kv_prefetch_l2(const KV& kv, const void* base, int es, int H, int hd, int b, int h,
+                                               int lo, int hi) {
+  const char* p = static_cast<const char*>(base);
+  if (!kv.pt) {
+    if (hi > lo) {
+      const uint32_t bytes = (uint32_t)((size_t)(hi - lo) * hd * es) & ~15u;
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p + kv_addr(kv, H, hd, b, h, lo, 0) * es),
+                   "r"(bytes)
+                   : "memory");
+    }
+    return;
+  }
+  for (int s0 = lo & ~(kPage - 1); s0 < hi; s0 += 8 * kPage) {
+    int pg[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) pg[i] = s0 + i * kPage < hi ? kv_page_cg(kv, b, s0 + i * kPage) : 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int a = max(lo, s0 + i * kPage), e = min(hi, s0 + (i + 1) * kPage);
+      if (a < e) {
+        const uint32_t bytes = (uint32_t)((e - a) * hd * es) & ~15u;
+        if (bytes)
+          asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p + kv_addr(kv, H, hd, b, h, a, pg[i]) * es),
+                       "r"(bytes)
+                       : "memory");
+      }
+    }
+  }
+}
+// Slots [s, s + n) that stay inside one page (or all of them, contiguous).
+__device__ __forceinline__ int kv_run(const KV& kv, int s, int n) {
+  if (!kv.pt) return n;
+  const int room = kPage - (s & (kPage - 1));
+  return n < room ? n : room;
+}
 
 struct EpiArgs {
   int mode;
@@ -274,6 +357,16 @@ struct Dev {
                        // GPU schedules 16-CTA clusters of it)
   int use_umma;        // many-row bf16 layers run on the tensor cores (tcgen05)
 
+  // paged KV caches: page tables [B][pt_ld_*] of the byte modules (encoder and next-byte decoder
+  // share positions), the LM module and the multi-byte window; pool sizes in pages; bump
+  // allocators ([0] bytes, [1] LM, [2] window)
+  int* pt_byte;
+  int* pt_lm;
+  int* pt_mb;
+  int pt_ld_byte, pt_ld_lm, pt_ld_mb;
+  int pages_byte, pages_lm, pages_mb;
+  int* pool_next;
+
   // weights (storage type; norms and bos fp32)
   void* embed;   // [256][d]
   void* unembed; // [256][d]
@@ -380,7 +473,7 @@ struct StackLayer {
   const __nv_bfloat16* w2;   // [d][F]
   const float* attn_norm;
   const float* mlp_norm;
-  void* k;                   // KV cache layer [B][H][S][64] bf16
+  void* k;                   // KV cache layer: a pool of pages [pages][H][kPage][64] bf16
   void* v;
 };
 
@@ -392,6 +485,8 @@ struct StackRun {
   Rows rows;
   int M_cap;
   int S;                    // cache slots per (sequence, head)
+  const int* pt;            // the layers' page table [B][pt_ld] (pools of pages [pages][H][kPage][64])
+  int pt_ld, pages;
   const int* stable;        // per-sequence committed cache length (stride in ints), or nullptr
   int stable_stride;
   int stable_add;

@@ -62,12 +62,13 @@ static __device__ __forceinline__ void epi_pair(const EpiArgs& e, int r, int c, 
       } else {
         const int b = e.rows.b[r];
         const int slot = e.rows.slot[r];
-        if (slot < 0 || slot >= e.kv.S) {
+        const int pg = e.kv.pt ? e.rows.page[r] : 0;
+        if (!kv_write_ok(e.kv, slot, pg)) {
           atomicOr(e.err, kErrIndex);
           return;
         }
         TC* base = reinterpret_cast<TC*>(part == 1 ? e.kv.k : e.kv.v);
-        TC* p = base + (((size_t)b * e.H + h) * e.kv.S + slot) * e.hd + dd;
+        TC* p = base + kv_addr(e.kv, e.H, e.hd, b, h, slot, pg) + dd;
         store_cache(p, a0);
         store_cache(p + 1, a1);
       }
@@ -81,7 +82,7 @@ static __device__ __forceinline__ void epi_pair(const EpiArgs& e, int r, int c, 
 struct EpiPre {
   float r0, r1;  // residual pair
   float2 cs;     // RoPE cos/sin
-  int b, slot;
+  int b, slot, pg;  // cache sequence, slot and its page
   int pos;       // RoPE position (epi_load_early; the angle follows in epi_load_late)
 };
 
@@ -89,7 +90,7 @@ static __device__ __forceinline__ EpiPre epi_load(const EpiArgs& e, int r, int c
   EpiPre p;
   p.r0 = p.r1 = 0.f;
   p.cs = make_float2(1.f, 0.f);
-  p.b = p.slot = 0;
+  p.b = p.slot = p.pg = 0;
   if (e.mode == EPI_RESID || e.mode == EPI_RESID_SILU) {
     const float2 q = *reinterpret_cast<const float2*>(e.res + (size_t)r * e.ldres + c);
     p.r0 = q.x;
@@ -105,6 +106,7 @@ static __device__ __forceinline__ EpiPre epi_load(const EpiArgs& e, int r, int c
     if (part > 0) {
       p.b = e.rows.b[r];
       p.slot = e.rows.slot[r];
+      if (e.kv.pt) p.pg = e.rows.page[r];
     }
   }
   return p;
@@ -117,7 +119,7 @@ static __device__ __forceinline__ EpiPre epi_load_early(const EpiArgs& e, int r,
   EpiPre p;
   p.r0 = p.r1 = 0.f;
   p.cs = make_float2(1.f, 0.f);
-  p.b = p.slot = 0;
+  p.b = p.slot = p.pg = 0;
   p.pos = 0;
   if (e.mode == EPI_RESID || e.mode == EPI_RESID_SILU) {
     const float2 q = *reinterpret_cast<const float2*>(e.res + (size_t)r * e.ldres + c);
@@ -129,6 +131,7 @@ static __device__ __forceinline__ EpiPre epi_load_early(const EpiArgs& e, int r,
     if (part > 0) {
       p.b = e.rows.b[r];
       p.slot = e.rows.slot[r];
+      if (e.kv.pt) p.pg = e.rows.page[r];
     }
   }
   return p;
@@ -147,14 +150,15 @@ static __device__ __forceinline__ void epi_load_late(const EpiArgs& e, EpiPre& p
 // walks its columns): per-row metadata once, then per pair one float2 operand (the residual
 // pair, or the RoPE cos/sin) that can be loaded a whole chunk of columns ahead of the stores.
 struct EpiRow {
-  int pos, b, slot;
+  int pos, b, slot, pg;
 };
 static __device__ __forceinline__ EpiRow epi_row(const EpiArgs& e, int r) {
-  EpiRow q{0, 0, 0};
+  EpiRow q{0, 0, 0, 0};
   if (e.mode == EPI_QKV) {
     q.pos = e.rows.pos[r];
     q.b = e.rows.b[r];
     q.slot = e.rows.slot[r];
+    if (e.kv.pt) q.pg = e.rows.page[r];
   }
   return q;
 }
@@ -206,12 +210,12 @@ static __device__ __forceinline__ void epi_store(const EpiArgs& e, const EpiPre&
       if (part == 0) {
         *reinterpret_cast<float2*>(e.y + (size_t)r * e.ldy + cc) = make_float2(a0, a1);
       } else {
-        if (p.slot < 0 || p.slot >= e.kv.S) {
+        if (!kv_write_ok(e.kv, p.slot, p.pg)) {
           atomicOr(e.err, kErrIndex);
           return;
         }
         TC* base = reinterpret_cast<TC*>(part == 1 ? e.kv.k : e.kv.v);
-        TC* q = base + (((size_t)p.b * e.H + h) * e.kv.S + p.slot) * e.hd + dd;
+        TC* q = base + kv_addr(e.kv, e.H, e.hd, p.b, h, p.slot, p.pg) + dd;
         store_cache(q, a0);
         store_cache(q + 1, a1);
       }
@@ -230,6 +234,7 @@ static __device__ __forceinline__ void epi_out(const EpiArgs& e, const EpiRow& q
   p.cs = op;
   p.b = q.b;
   p.slot = q.slot;
+  p.pg = q.pg;
   p.pos = q.pos;
   epi_store<TC>(e, p, r, c, a0, a1);
 }

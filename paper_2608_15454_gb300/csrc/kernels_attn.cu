@@ -60,8 +60,8 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
   const int nrows = rows.seq_count[b];
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
-  const TC* Kc = reinterpret_cast<const TC*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
-  const TC* Vc = reinterpret_cast<const TC*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  const TC* Kc = reinterpret_cast<const TC*>(kv.k);
+  const TC* Vc = reinterpret_cast<const TC*>(kv.v);
   const int ld = H * HD;
 
   // accumulator ownership: row ai, dims ad..ad+DPT-1
@@ -117,8 +117,9 @@ k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, i
           const int e = (tid + u * kThreads) * EV;
           const int kk = e / HD, dd = e - kk * HD;
           if (kk < nk) {
-            uk[u] = *reinterpret_cast<const uint4*>(Kc + (size_t)(j0 + kk) * HD + dd);
-            uv[u] = *reinterpret_cast<const uint4*>(Vc + (size_t)(j0 + kk) * HD + dd);
+            const size_t o = kv_off(kv, H, HD, b, h, j0 + kk) + dd;
+            uk[u] = *reinterpret_cast<const uint4*>(Kc + o);
+            uv[u] = *reinterpret_cast<const uint4*>(Vc + o);
           } else {
             uk[u] = make_uint4(0, 0, 0, 0);
             uv[u] = make_uint4(0, 0, 0, 0);
@@ -310,12 +311,7 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
     const int t = stable[(size_t)bb * stable_stride];
     const int est = ((t + stable_extra + splits - 1) / splits + 15) / 16 * 16;
     const int lo = sp * est, hi = min(t, lo + est);
-    if (hi > lo) {
-      const TC* base = reinterpret_cast<const TC*>(threadIdx.x == 0 ? kv.k : kv.v) +
-                       (((size_t)bb * H + hh) * kv.S + lo) * HD;
-      const uint32_t bytes = (uint32_t)((hi - lo) * HD * sizeof(TC));
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"(bytes & ~15u) : "memory");
-    }
+    kv_prefetch_l2(kv, threadIdx.x == 0 ? kv.k : kv.v, (int)sizeof(TC), H, HD, bb, hh, lo, hi);
   }
   pdl_trigger();
   pdl_wait();
@@ -327,8 +323,8 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
   const int nrows = rows.seq_count[b];
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
-  const TC* Kc = reinterpret_cast<const TC*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
-  const TC* Vc = reinterpret_cast<const TC*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  const TC* Kc = reinterpret_cast<const TC*>(kv.k);
+  const TC* Vc = reinterpret_cast<const TC*>(kv.v);
   const int ld = H * HD;
 
   for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
@@ -372,8 +368,9 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
         for (int r = 0; r < QT; ++r) sc[r] = 0.f;
         if (tid < nk) {
           uint4 kr[NV];
+          const TC* kp = Kc + kv_off(kv, H, HD, b, h, j);
 #pragma unroll
-          for (int v = 0; v < NV; ++v) kr[v] = *reinterpret_cast<const uint4*>(Kc + (size_t)j * HD + v * EV);
+          for (int v = 0; v < NV; ++v) kr[v] = *reinterpret_cast<const uint4*>(kp + v * EV);
 #pragma unroll
           for (int v = 0; v < NV; ++v) {
             float kf[8];
@@ -440,7 +437,7 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
 #pragma unroll
         for (int u = 0; u < KPG; ++u) {
           const int key = kg * KPG + u;
-          if (key < nk) load4(Vc + (size_t)(j0 + key) * HD + dg * 4, vv[u]);
+          if (key < nk) load4(Vc + kv_off(kv, H, HD, b, h, j0 + key) + dg * 4, vv[u]);
           else vv[u][0] = vv[u][1] = vv[u][2] = vv[u][3] = 0.f;
         }
 #pragma unroll
@@ -585,6 +582,7 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
   float* s_corr = s_l + QT;                                          // [QT]
   int* s_kv = reinterpret_cast<int*>(s_corr + QT);                   // [QT]
   uint64_t* full = reinterpret_cast<uint64_t*>(s_kv + QT);           // [stages]
+  int* s_pt = reinterpret_cast<int*>(full + kA3Stages);              // [pt_ld] page table row (paged)
 
   TraceScope _trace(TT_ATTN);
   cgr::cluster_group cl = cgr::this_cluster();
@@ -603,11 +601,7 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
     const int t = stable[(size_t)bb * stable_stride];
     const int est = ((t + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
     const int lo = sp * est, hi = min(t, lo + est);
-    if (hi > lo) {
-      const TC* base = reinterpret_cast<const TC*>(tid == 0 ? kv.k : kv.v) + (((size_t)bb * H + hh) * kv.S + lo) * HD;
-      const uint32_t bytes = (uint32_t)((hi - lo) * HD * sizeof(TC));
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"(bytes & ~15u) : "memory");
-    }
+    kv_prefetch_l2(kv, tid == 0 ? kv.k : kv.v, (int)sizeof(TC), H, HD, bb, hh, lo, hi);
   }
   pdl_trigger();
   pdl_wait();
@@ -618,9 +612,10 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
   const int nrows = rows.seq_count[b];
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
-  const TC* Kc = reinterpret_cast<const TC*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
-  const TC* Vc = reinterpret_cast<const TC*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  const TC* Kc = reinterpret_cast<const TC*>(kv.k);
+  const TC* Vc = reinterpret_cast<const TC*>(kv.v);
   const int ld = H * HD;
+  kv_stage_pages(kv, b, s_pt, tid, kA3Threads);  // published by the tile's first barrier
   bool failed = false;
   uint32_t cc = 0;      // chunks consumed by this CTA so far (ring phase)
   uint32_t issued = 0;  // chunks whose copies were issued (thread 0)
@@ -658,9 +653,11 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
       const uint32_t bytes = (uint32_t)(nk * HD * sizeof(TC));
       unsigned char* dst = ring + (size_t)st * 2 * CB;
       ++issued;
+      // a chunk starts on a page (KC == kPage, lo a multiple of KC) and stays inside it
+      const size_t o = kv_addr(kv, H, HD, b, h, j0, kv.pt ? s_pt[j0 / kPage] : 0);
       a3_expect(&full[st], 2 * bytes);
-      a3_copy(dst, Kc + (size_t)j0 * HD, bytes, &full[st]);
-      a3_copy(dst + CB, Vc + (size_t)j0 * HD, bytes, &full[st]);
+      a3_copy(dst, Kc + o, bytes, &full[st]);
+      a3_copy(dst + CB, Vc + o, bytes, &full[st]);
     };
     if (tid == 0)
       for (int c = 0; c < nch && c < kA3Stages - 1; ++c) issue(c);
@@ -816,11 +813,12 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
   }
 }
 
+// Dynamic shared memory of k_attn3, with pt_bytes of staged page table.
 template <typename TC, int HD>
-size_t attn3_smem() {
+size_t attn3_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
   constexpr int QT = kAttnQT;
   return (size_t)kA3Stages * 2 * kA3Keys * HD * sizeof(TC) + (size_t)(2 * QT * HD + QT * kA3Keys + 4 * QT) * 4 +
-         kA3Stages * 8 + 16;
+         kA3Stages * 8 + 16 + pt_bytes;
 }
 
 template <typename TC, int HD>
@@ -830,7 +828,7 @@ void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA3Threads);
-  cfg.dynamicSmemBytes = attn3_smem<TC, HD>();
+  cfg.dynamicSmemBytes = attn3_smem<TC, HD>(kv_pages_smem(kv));
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -904,10 +902,12 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   float* rm = rbuf + (size_t)splits * QT * HD;  // rank 0: [splits][QT] maxima
   float* rl = rm + splits * QT;                  // rank 0: [splits][QT] sums
+  // the page table row (paged), after the partials' buffer when there is one
+  int* s_pt = reinterpret_cast<int*>(splits > 1 ? rl + splits * QT : rbuf);
   const int b = blockIdx.x;
   const int h = blockIdx.z / splits;
-  const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(kv.k) + ((size_t)b * H + h) * kv.S * HD;
-  const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(kv.v) + ((size_t)b * H + h) * kv.S * HD;
+  const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(kv.k);
+  const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(kv.v);
   pdl_trigger();
   if (tid == 0) {
     int S = 0, slo = 0, nst = 0;
@@ -926,10 +926,18 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
       asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a3_su32(&s_rbar)), "r"(splits - 1) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     if (nst > 0) {
+      // committed slots: their pages were mapped by earlier steps, so the table entries are final
       const uint32_t bytes = (uint32_t)(nst * HD * 2);
       a3_expect(&s_bar, 2 * bytes);
-      a3_copy(Ks, Kc + (size_t)slo * HD, bytes, &s_bar);
-      a3_copy(Vs, Vc + (size_t)slo * HD, bytes, &s_bar);
+      // one copy per page run (at most five pages: 256 keys from a 4-aligned slot)
+      for (int s0 = slo; s0 < slo + nst;) {
+        const int run = kv_run(kv, s0, slo + nst - s0);
+        const size_t o = kv_off(kv, H, HD, b, h, s0);
+        const uint32_t rb = (uint32_t)(run * HD * 2);
+        a3_copy(Ks + (size_t)(s0 - slo) * HD, Kc + o, rb, &s_bar);
+        a3_copy(Vs + (size_t)(s0 - slo) * HD, Vc + o, rb, &s_bar);
+        s0 += run;
+      }
     }
   }
   // rank 0's arrival barrier exists before any peer can arrive on it (a cluster barrier before
@@ -944,6 +952,7 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
   const int ld = H * HD;
+  kv_stage_pages(kv, b, s_pt, tid, kAwThreads);  // published by the tile's first barrier
 
   const int g = lane >> 3, e = lane & 7;  // key slot of this lane in a warp step, its 8 head dims
   for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
@@ -1014,8 +1023,10 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
           ku = *reinterpret_cast<const uint4*>(Ks + (size_t)v * HD + 8 * e);
           vu = *reinterpret_cast<const uint4*>(Vs + (size_t)v * HD + 8 * e);
         } else {
-          ku = *reinterpret_cast<const uint4*>(Kc + (size_t)j * HD + 8 * e);
-          vu = *reinterpret_cast<const uint4*>(Vc + (size_t)j * HD + 8 * e);
+          // paged caches only (the dispatcher checks): page of slot j from the staged table row
+          const size_t o = (((size_t)s_pt[j / kPage] * H + h) * kPage + (j & (kPage - 1))) * HD + 8 * e;
+          ku = *reinterpret_cast<const uint4*>(Kc + o);
+          vu = *reinterpret_cast<const uint4*>(Vc + o);
         }
       }
       float kf[8], vf[8];
@@ -1204,7 +1215,8 @@ void launch_aw(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cfg.gridDim = dim3(B, 1, H * splits);
   cfg.blockDim = dim3(kAwThreads);
   const int qt = rows_seq <= 4 ? 4 : kAttnQT;
-  cfg.dynamicSmemBytes = (size_t)cap * 64 * 2 * 2 + (splits > 1 ? (size_t)splits * qt * (64 + 2) * 4 : 0);
+  cfg.dynamicSmemBytes =
+      (size_t)cap * 64 * 2 * 2 + (splits > 1 ? (size_t)splits * qt * (64 + 2) * 4 : 0) + kv_pages_smem(kv);
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -1316,6 +1328,7 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   int* s_kv = reinterpret_cast<int*>(s_l + QT);                     // [QT]
   uint64_t* full = reinterpret_cast<uint64_t*>(s_kv + QT);          // [NS]
   uint64_t* empty = full + NS;                                      // [NS]
+  int* s_pt = reinterpret_cast<int*>(empty + NS);                   // [pt_ld] page table row (paged)
   // after the key loop the ring holds the warps' partial results
   float* Ow = reinterpret_cast<float*>(ring);                       // [warps][QT][HD]
   float* mw = Ow + kA4Warps * QT * HD;                              // [warps][QT]
@@ -1342,12 +1355,7 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
     const int tt = stable[(size_t)bb * stable_stride];
     const int est = ((tt + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
     const int lo = sp * est, hi = min(tt, lo + est);
-    if (hi > lo) {
-      const __nv_bfloat16* base = reinterpret_cast<const __nv_bfloat16*>(tid == 0 ? kv.k : kv.v) +
-                                  (((size_t)bb * H + hh) * kv.S + lo) * HD;
-      const uint32_t bytes = (uint32_t)((hi - lo) * HD * 2);
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"(bytes & ~15u) : "memory");
-    }
+    kv_prefetch_l2(kv, tid == 0 ? kv.k : kv.v, 2, H, HD, bb, hh, lo, hi);
   }
   pdl_trigger();
   pdl_wait();
@@ -1359,7 +1367,7 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
   const int ld = H * HD;
-  const int krow0 = (b * H + h) * kv.S;  // first tensor-map row of this (sequence, head)
+  kv_stage_pages(kv, b, s_pt, tid, kA4Threads);  // published by the tile's first barrier
   bool failed = false;
   uint32_t cc = 0, issued = 0;
 
@@ -1415,9 +1423,12 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
           if (failed) break;
           ++issued;
           unsigned char* dst = ring + (size_t)st * 2 * kA4Chunk;
+          // tensor-map row of the chunk: 64 slots from a page start (lo is a multiple of KC == kPage)
+          const int j0 = lo + c * KC;
+          const int row = kv.pt ? (s_pt[j0 / kPage] * H + h) * kPage : (b * H + h) * kv.S + j0;
           a3_expect(&full[st], 2 * kA4Chunk);
-          a4_tma(dst, &tmK, 0, krow0 + lo + c * KC, &full[st]);
-          a4_tma(dst + kA4Chunk, &tmV, 0, krow0 + lo + c * KC, &full[st]);
+          a4_tma(dst, &tmK, 0, row, &full[st]);
+          a4_tma(dst + kA4Chunk, &tmV, 0, row, &full[st]);
         }
       }
       __syncwarp();
@@ -1603,9 +1614,9 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
 }
 
 template <int NS>
-size_t attn_mma_smem() {
-  // ring, q halves (2 x QT x 64 bf16), pacc (QT x 64 fp32), row stats, barriers
-  return 1024 + (size_t)NS * 2 * kA4Chunk + (size_t)(2 * kA4QT * 64 + 3 * kA4QT) * 4 + 2 * NS * 8 + 16;
+size_t attn_mma_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
+  // ring, q halves (2 x QT x 64 bf16), pacc (QT x 64 fp32), row stats, barriers, page table row
+  return 1024 + (size_t)NS * 2 * kA4Chunk + (size_t)(2 * kA4QT * 64 + 3 * kA4QT) * 4 + 2 * NS * 8 + 16 + pt_bytes;
 }
 
 template <int NS>
@@ -1618,7 +1629,7 @@ void launch_a4_ns(const float* q, float* out, const KV& kv, const Rows& rows, in
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA4Threads);
-  cfg.dynamicSmemBytes = attn_mma_smem<NS>();
+  cfg.dynamicSmemBytes = attn_mma_smem<NS>(kv_pages_smem(kv));
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -1673,6 +1684,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   int* s_kv = reinterpret_cast<int*>(s_l + QT);                     // [QT]
   uint64_t* full = reinterpret_cast<uint64_t*>(s_kv + QT);          // [NS]
   uint64_t* empty = full + NS;                                      // [NS]
+  int* s_pt = reinterpret_cast<int*>(empty + NS);                   // [pt_ld] page table row (paged)
   // after the key loop the ring holds the warps' partial results
   float* Ow = reinterpret_cast<float*>(ring);                       // [warps][QT][HD]
   float* mw = Ow + kA4Warps * QT * HD;                              // [warps][QT]
@@ -1699,12 +1711,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
     const int tt = stable[(size_t)bb * stable_stride];
     const int est = ((tt + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
     const int lo = sp * est, hi = min(tt, lo + est);
-    if (hi > lo) {
-      const __nv_bfloat16* base = reinterpret_cast<const __nv_bfloat16*>(tid == 0 ? kv.k : kv.v) +
-                                  (((size_t)bb * H + hh) * kv.S + lo) * HD;
-      const uint32_t bytes = (uint32_t)((hi - lo) * HD * 2);
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(base), "r"(bytes & ~15u) : "memory");
-    }
+    kv_prefetch_l2(kv, tid == 0 ? kv.k : kv.v, 2, H, HD, bb, hh, lo, hi);
   }
   pdl_trigger();
   pdl_wait();
@@ -1716,7 +1723,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
   const int ld = H * HD;
-  const int krow0 = (b * H + h) * kv.S;  // first tensor-map row of this (sequence, head)
+  kv_stage_pages(kv, b, s_pt, tid, kA4Threads);  // published by the tile's first barrier
   bool failed = false;
   uint32_t cc = 0, issued = 0;
 
@@ -1770,9 +1777,12 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
           if (failed) break;
           ++issued;
           unsigned char* dst = ring + (size_t)st * 2 * kA4Chunk;
+          // tensor-map row of the chunk: 64 slots from a page start (lo is a multiple of KC == kPage)
+          const int j0 = lo + c * KC;
+          const int row = kv.pt ? (s_pt[j0 / kPage] * H + h) * kPage : (b * H + h) * kv.S + j0;
           a3_expect(&full[st], 2 * kA4Chunk);
-          a4_tma(dst, &tmK, 0, krow0 + lo + c * KC, &full[st]);
-          a4_tma(dst + kA4Chunk, &tmV, 0, krow0 + lo + c * KC, &full[st]);
+          a4_tma(dst, &tmK, 0, row, &full[st]);
+          a4_tma(dst + kA4Chunk, &tmV, 0, row, &full[st]);
         }
       }
       __syncwarp();
@@ -1967,9 +1977,9 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
 }
 
 template <int NS>
-size_t attn_mmt_smem() {
-  // ring, q halves (2 x QT x 64 bf16), pacc (QT x 64 fp32), row stats, barriers
-  return 1024 + (size_t)NS * 2 * kA4Chunk + (size_t)(2 * kA5QT * 64 + 3 * kA5QT) * 4 + 2 * NS * 8 + 16;
+size_t attn_mmt_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
+  // ring, q halves (2 x QT x 64 bf16), pacc (QT x 64 fp32), row stats, barriers, page table row
+  return 1024 + (size_t)NS * 2 * kA4Chunk + (size_t)(2 * kA5QT * 64 + 3 * kA5QT) * 4 + 2 * NS * 8 + 16 + pt_bytes;
 }
 
 template <int NS>
@@ -1982,7 +1992,7 @@ void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, in
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA4Threads);
-  cfg.dynamicSmemBytes = attn_mmt_smem<NS>();
+  cfg.dynamicSmemBytes = attn_mmt_smem<NS>(kv_pages_smem(kv));
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -2180,10 +2190,10 @@ void kernel_attrs_attn() {
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn_w<4>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn_w<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       kAwStageMax * 64 * 2 * 2 + kA4MaxSplit * 4 * (64 + 2) * 4);
+                       kAwStageMax * 64 * 2 * 2 + kA4MaxSplit * 4 * (64 + 2) * 4 + kMaxPtRow * 4);
   cudaFuncSetAttribute(k_attn_w<kAttnQT>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn_w<kAttnQT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       kAwStageMax * 64 * 2 * 2 + kA4MaxSplit * kAttnQT * (64 + 2) * 4);
+                       kAwStageMax * 64 * 2 * 2 + kA4MaxSplit * kAttnQT * (64 + 2) * 4 + kMaxPtRow * 4);
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<float, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn3<float, 32>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -2223,7 +2233,7 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
   if (D.attn_pipe) {
     splits = std::min(splits, kA4MaxSplit);
     // decode steps (one query tile per sequence) of bf16 head-dim-64 caches: the warp-walk kernel
-    if (qtiles_grid == 1 && D.attn_w && D.dtype == LCA_BF16 && D.hd == 64) {
+    if (qtiles_grid == 1 && D.attn_w && D.dtype == LCA_BF16 && D.hd == 64 && kv.pt) {
       launch_aw(q, out, kv, rows, B, D.H, D.scale, splits, D.err, stable_aw, ss, stable_add, rows_seq, s);
       return;
     }

@@ -103,6 +103,19 @@ struct StackArgs {
 
 static __device__ TraceRec* g_trace_s = nullptr;
 
+// The cache layer of a stack layer as the paging helpers see it.
+__device__ __forceinline__ KV cache_view(const StackArgs& a, const StackLayer& Ly) {
+  KV kv;
+  kv.k = Ly.k;
+  kv.v = Ly.v;
+  kv.S = a.r.S;
+  kv.tmaps = nullptr;
+  kv.pt = a.r.pt;
+  kv.pt_ld = a.r.pt_ld;
+  kv.pages = a.r.pages;
+  return kv;
+}
+
 // ---------------------------------------------------------------- primitives
 __device__ __forceinline__ uint32_t su32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
 __device__ __forceinline__ void mb_init(uint64_t* b, uint32_t n) {
@@ -228,7 +241,8 @@ struct Smem {
   uint64_t* empty;      // [slots]
   uint64_t* sbar;       // [2] staging buffers
   float* inv;           // [2][8] inverse RMS of the staged rows
-  int* misc;  // [0] abort, [1] issued, [2] copy warp done, [3] last arriver, [8..15] kl, [16..23] b, [24..31] slot
+  int* misc;  // [0] abort, [1] issued, [2] copy warp done, [3] last arriver, [8..15] kl, [16..23] b, [24..31] slot,
+              // [32..] W2 last arrivers, [40..47] page of the slot
 };
 __device__ __forceinline__ __nv_bfloat16* stage_hi(Smem& S, int b) {
   return reinterpret_cast<__nv_bfloat16*>(S.work + (size_t)b * kStageBufBytes);
@@ -525,15 +539,17 @@ __device__ void linear_phase(const StackArgs& a, const StackLayer& Ly, const Sta
         if (p == PH_QKV) {
           if (ok) {
             const int part = col / a.d, cc = col - part * a.d, h = cc / kSkHD, dd = cc - h * kSkHD;
-            int rb, rslot;
+            int rb, rslot, rpg;
             float2 cs;
             if (r < kSkMC) {
               rb = S.misc[16 + r];
               rslot = S.misc[24 + r];
+              rpg = S.misc[40 + r];
               cs = S.rope[r * (kSkHD / 2) + (dd >> 1)];
             } else {
               rb = a.r.rows.b[r];
               rslot = a.r.rows.slot[r];
+              rpg = a.r.pt ? a.r.rows.page[r] : 0;
               cs = a.rope[(size_t)a.r.rows.pos[r] * (kSkHD / 2) + (dd >> 1)];
             }
             if (part < 2) {
@@ -543,11 +559,11 @@ __device__ void linear_phase(const StackArgs& a, const StackLayer& Ly, const Sta
             }
             if (part == 0) {
               *reinterpret_cast<float2*>(a.q + (size_t)r * a.d + cc) = make_float2(v0, v1);
-            } else if (rslot < 0 || rslot >= a.r.S) {
+            } else if (!kv_write_ok(cache_view(a, Ly), rslot, rpg)) {
               atomicOr(a.err, kErrIndex);
             } else {
               __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(part == 1 ? Ly.k : Ly.v) +
-                                   (((size_t)rb * a.H + h) * a.r.S + rslot) * kSkHD + dd;
+                                   kv_addr(cache_view(a, Ly), a.H, kSkHD, rb, h, rslot, rpg) + dd;
               *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(v0, v1);
             }
           }
@@ -700,8 +716,9 @@ __device__ void attention_phase(const StackArgs& a, const StackLayer& Ly, int c,
       Sb = a.r.stable[(size_t)b * a.r.stable_stride] + a.r.stable_add;
       Sb = Sb < 0 ? 0 : (Sb > a.r.S ? a.r.S : Sb);
     }
-    const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(Ly.k) + ((size_t)b * H + h) * a.r.S * kSkHD;
-    const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(Ly.v) + ((size_t)b * H + h) * a.r.S * kSkHD;
+    const KV kvv = cache_view(a, Ly);
+    const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(Ly.k);
+    const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(Ly.v);
     float* part = a.apart + (((size_t)b * H + h) * splits + sp) * a.apart_rows * kSkPart;
     const int tiles = (nrows + kSkMC - 1) / kSkMC;
     for (int qt = 0; qt < tiles; ++qt) {
@@ -762,7 +779,7 @@ __device__ void attention_phase(const StackArgs& a, const StackLayer& Ly, int c,
           kv[m] = make_uint4(0u, 0u, 0u, 0u);
           if (v < nv) {
             const int slot = v < n1 ? lo1 + v : lo2 + (v - n1);
-            const __nv_bfloat16* base = (m < 4 ? Kc : Vc) + (size_t)slot * kSkHD + e8 * 8;
+            const __nv_bfloat16* base = (m < 4 ? Kc : Vc) + kv_off(kvv, H, kSkHD, b, h, slot) + e8 * 8;
             kv[m] = __ldcg(reinterpret_cast<const uint4*>(base));
           }
         }
@@ -993,6 +1010,7 @@ __global__ void __launch_bounds__(kSkThreads, 1) k_stack(StackArgs a) {
     const bool ok = tid < M;
     S.misc[16 + tid] = ok ? a.r.rows.b[tid] : 0;
     S.misc[24 + tid] = ok ? a.r.rows.slot[tid] : 0;
+    S.misc[40 + tid] = ok && a.r.pt ? a.r.rows.page[tid] : 0;
   }
   if (tid < kSkMC * (kSkHD / 2)) {
     const int r = tid / (kSkHD / 2), j = tid - r * (kSkHD / 2);
@@ -1079,13 +1097,7 @@ __global__ void __launch_bounds__(kSkThreads, 1) k_stack(StackArgs a) {
         Sb = Sb < 0 ? 0 : (Sb > a.r.S ? a.r.S : Sb);
         int lo, hi;
         key_share(0, Sb, a.splits, sp, lo, hi);
-        if (hi > lo) {
-          const char* base = reinterpret_cast<const char*>(lane == 0 ? Ly.k : Ly.v) +
-                             (((size_t)b * a.H + h) * a.r.S + lo) * kSkHD * 2;
-          const size_t bytes = (size_t)(hi - lo) * kSkHD * 2;
-          for (size_t o2 = 0; o2 < bytes; o2 += 65536)
-            prefetch_l2(base + o2, (uint32_t)(bytes - o2 < 65536 ? bytes - o2 : 65536));
-        }
+        kv_prefetch_l2(cache_view(a, Ly), lane == 0 ? Ly.k : Ly.v, 2, a.H, kSkHD, b, h, lo, hi);
       }
     }
     linear_phase(a, Ly, Lnext, z, l, PH_QKV, c, G, M, seq, uses, S);

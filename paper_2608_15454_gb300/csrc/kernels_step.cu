@@ -14,6 +14,27 @@ __device__ __forceinline__ float ld_w(const __nv_bfloat16* p, size_t i) { return
 
 __device__ __forceinline__ void err_or(int* e, int bits) { atomicOr(e, bits); }
 
+// Maps a page to every page of slots [s0, s1] of sequence b that has none, from the pool's bump
+// counter. One thread per sequence row of the table. A page stays mapped until the next prefill
+// (a multi-byte window that restarts reuses its pages); an exhausted pool leaves the entry
+// unmapped and raises kErrPages, and the writers then skip those slots.
+__device__ void map_pages(int* pt, int ld, int pages, int* next, int b, int s0, int s1, int* err) {
+  if (s0 < 0) s0 = 0;
+  for (int j = s0 / kPage; j <= s1 / kPage && j < ld; ++j) {
+    int* e = pt + (size_t)b * ld + j;
+    if (*e < 0) {
+      const int pg = atomicAdd(next, 1);
+      if (pg < pages) *e = pg;
+      else err_or(err, kErrPages);
+    }
+  }
+}
+// Page of slot s of sequence b (after map_pages), -1 if unmapped.
+__device__ __forceinline__ int page_of(const int* pt, int ld, int b, int s) {
+  const int j = s / kPage;
+  return (s < 0 || j >= ld) ? -1 : pt[(size_t)b * ld + j];
+}
+
 // ---------------------------------------------------------------- multi-byte window plan
 // Algorithm 1, drafting: the window of sequence b is the previous and the current latent
 // group, then n-2 copies of the last row. Inside the window the LCA mask is causal, and a
@@ -55,6 +76,8 @@ __global__ void k_mb_plan(Dev D, int fill) {
     s_cnt[b] = (t - first) + (n - 2);
     s_ms[b] = s;
     st.mb_len = t - s;
+    if (s_cnt[b] > 0)
+      map_pages(D.pt_mb, D.pt_ld_mb, D.pages_mb, &D.pool_next[2], b, first - s, first - s + s_cnt[b] - 1, D.err);
   }
   __syncthreads();
   if (tid == 0) {
@@ -95,6 +118,7 @@ __global__ void k_mb_plan(Dev D, int fill) {
       D.r_mb.b[r] = b;
       D.r_mb.pos[r] = p;
       D.r_mb.slot[r] = p - s;
+      D.r_mb.page[r] = page_of(D.pt_mb, D.pt_ld_mb, b, p - s);
       D.r_mb.kvlen[r] = p - s + 1;
     }
     for (int j = lane; j < n - 1; j += 32)
@@ -354,6 +378,12 @@ __global__ void k_verify_plan(Dev D) {
     }
     return;
   }
+  // pages of positions t..t+n-1 (one thread maps; the rows read the table after the barrier)
+  if (tid == 0) {
+    const int t = D.seq[b].t;
+    map_pages(D.pt_byte, D.pt_ld_byte, D.pages_byte, &D.pool_next[0], b, t, min(t + n - 1, D.S - 1), D.err);
+  }
+  __syncthreads();
   if (tid < n) {
     const int i = tid;
     const int t = D.seq[b].t;
@@ -372,6 +402,7 @@ __global__ void k_verify_plan(Dev D) {
     D.r_v.b[r] = b;
     D.r_v.pos[r] = p;
     D.r_v.slot[r] = p;
+    D.r_v.page[r] = page_of(D.pt_byte, D.pt_ld_byte, b, p);
     D.r_v.kvlen[r] = p + 1;
   }
   if (tid == 0) {
@@ -518,9 +549,11 @@ __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handl
     }
     if (tid == 0) {
       D.gstart[(size_t)b * D.L + k] = seg1;
+      map_pages(D.pt_lm, D.pt_ld_lm, D.pages_lm, &D.pool_next[1], b, k, k, D.err);
       D.r_lm.b[row] = b;
       D.r_lm.pos[row] = k;
       D.r_lm.slot[row] = k;
+      D.r_lm.page[row] = page_of(D.pt_lm, D.pt_ld_lm, b, k);
       D.r_lm.kvlen[row] = k + 1;
     }
   }

@@ -233,12 +233,12 @@ __device__ __forceinline__ void chunk_out(const EpiArgs& e, const EpiRow& q, con
 #pragma unroll
         for (int i = 0; i < 8; ++i) y[i] = make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]);
       } else {
-        if (q.slot < 0 || q.slot >= e.kv.S) {
+        if (!kv_write_ok(e.kv, q.slot, q.pg)) {
           atomicOr(e.err, kErrIndex);
           return;
         }
         TC* base = reinterpret_cast<TC*>(part == 1 ? e.kv.k : e.kv.v);
-        TC* p = base + (((size_t)q.b * e.H + h) * e.kv.S + q.slot) * e.hd + dd0;
+        TC* p = base + kv_addr(e.kv, e.H, e.hd, q.b, h, q.slot, q.pg) + dd0;
         if (sizeof(TC) == 2) {
           uint4* d4 = reinterpret_cast<uint4*>(p);
 #pragma unroll
@@ -631,7 +631,7 @@ k_tgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
         if (warp >= 2) {
           // the rows' metadata is read while the main loop runs; then the accumulator
           inv_s[r] = sc;
-          meta_s[r] = mt * kUM + r < M ? epi_row(a.epi, rbase + mt * kUM + r) : EpiRow{0, 0, 0};
+          meta_s[r] = mt * kUM + r < M ? epi_row(a.epi, rbase + mt * kUM + r) : EpiRow{0, 0, 0, 0};
           wait_or_fail(accdone, ps & 1, failed);
           asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
           if (g_trace && ps == 0 && warp == 2 && lane == 0) tmk[1] = gtimer();
@@ -701,9 +701,9 @@ struct SCfg {
                                      ((uint32_t)(kSW >> 4) << 24);
   static constexpr uint32_t kTmemCols = NR < 32 ? 32 : NR;
   // ring, receive buffer, barriers (full, empty, accumulator, receive), TMEM address, per-row
-  // inverse RMS / position / sequence / cache slot, two trace times, alignment slack
+  // inverse RMS / position / sequence / cache slot / its page, two trace times, alignment slack
   static constexpr size_t kSmem =
-      (size_t)kStages * kStageBytes + kRecvBytes + (2 * kStages + 2) * 8 + 16 + NR * 16 + 16 + 1024;
+      (size_t)kStages * kStageBytes + kRecvBytes + (2 * kStages + 2) * 8 + 16 + NR * 20 + 16 + 1024;
   static_assert(NR == 32 || NR == 64, "tile rows");
   static_assert(kStages >= 2, "ring");
   static_assert(kStageBytes % 1024 == 0 && kXBytes % 1024 == 0, "swizzle atoms");
@@ -725,6 +725,7 @@ struct SRowMeta {
   int* pos;
   int* b;
   int* slot;
+  int* pg;
 };
 
 // Output of value x (accumulator times the row's scale) at global row gr, column c, for one lane
@@ -785,12 +786,12 @@ __device__ __forceinline__ void scol_out(const EpiArgs& e, size_t gr, int c, int
       if (part == 0) {
         e.y[gr * e.ldy + cc] = x;
       } else {
-        const int slot = m.slot[rt];
-        if (slot < 0 || slot >= e.kv.S) {
+        const int slot = m.slot[rt], pg = m.pg[rt];
+        if (!kv_write_ok(e.kv, slot, pg)) {
           if (lane == 0) atomicOr(e.err, kErrIndex);
         } else {
           __nv_bfloat16* base = reinterpret_cast<__nv_bfloat16*>(part == 1 ? e.kv.k : e.kv.v);
-          base[(((size_t)m.b[rt] * e.H + h) * e.kv.S + slot) * e.hd + dd] = __float2bfloat16_rn(x);
+          base[kv_addr(e.kv, e.H, e.hd, m.b[rt], h, slot, pg) + dd] = __float2bfloat16_rn(x);
         }
       }
       break;
@@ -884,8 +885,9 @@ k_sgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
   meta.pos = reinterpret_cast<int*>(meta.inv + NR);
   meta.b = meta.pos + NR;
   meta.slot = meta.b + NR;
+  meta.pg = meta.slot + NR;
   // traced launches: partials pushed, peers' partials received
-  unsigned long long* tmk = reinterpret_cast<unsigned long long*>(meta.slot + NR);
+  unsigned long long* tmk = reinterpret_cast<unsigned long long*>(meta.pg + NR);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n0 = blockIdx.x * kSW;
@@ -1014,6 +1016,7 @@ k_sgemm(LinearArgs a, const __grid_constant__ CUtensorMap tmW, const __grid_cons
             meta.pos[et] = a.epi.rows.pos[rbase + row];
             meta.b[et] = a.epi.rows.b[rbase + row];
             meta.slot[et] = a.epi.rows.slot[rbase + row];
+            meta.pg[et] = a.epi.kv.pt ? a.epi.rows.page[rbase + row] : 0;
           }
         }
         meta.inv[et] = inv;

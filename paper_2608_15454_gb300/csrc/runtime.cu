@@ -70,12 +70,25 @@ void carve(const lca_config& c, char* base, Layout& L) {
   const size_t d = D.d, F = D.F, tb = tw_bytes(c.dtype);
   const size_t B = D.B, S = D.S, Lt = D.L, R = D.R, NM = D.NMAX;
 
+  // paged caches: page tables and pool sizes (pages of kPage positions)
+  D.pt_ld_byte = (int)((S + kPage - 1) / kPage);
+  D.pt_ld_lm = (int)((Lt + kPage - 1) / kPage);
+  D.pt_ld_mb = D.pt_ld_byte;
+  D.pages_byte = c.kv_pages > 0 ? c.kv_pages : (int)B * D.pt_ld_byte;
+  D.pages_lm = c.lm_pages > 0 ? c.lm_pages : (int)B * D.pt_ld_lm;
+  D.pages_mb = c.mb_pages > 0 ? c.mb_pages : (int)B * D.pt_ld_mb;
+  D.pt_byte = cv.take<int>(B * D.pt_ld_byte);
+  D.pt_lm = cv.take<int>(B * D.pt_ld_lm);
+  D.pt_mb = cv.take<int>(B * D.pt_ld_mb);
+  D.pool_next = cv.take<int>(4);
+
   D.embed = cv.take<char>(256 * d * tb);
   D.unembed = cv.take<char>(256 * d * tb);
   D.bos = cv.take<float>(d);
   D.nb_norm = cv.take<float>(d);
   D.mb_norm = cv.take<float>(d);
-  auto blocks = [&](std::vector<Block>& v, int n, size_t slots) {
+  // every cache layer: a pool of pages [pages][H][kPage][hd] behind its module's page table
+  auto blocks = [&](std::vector<Block>& v, int n, size_t slots, const int* pt, int pt_ld, int pages) {
     v.resize(n);
     for (auto& b : v) {
       b.attn_norm = cv.take<float>(d);
@@ -85,15 +98,18 @@ void carve(const lca_config& c, char* base, Layout& L) {
       b.w13 = cv.take<char>(2 * F * d * tb);
       b.w2 = cv.take<char>(d * F * tb);
       b.kv.S = (int)slots;
-      b.kv.k = cv.take<char>(B * D.H * slots * D.hd * tb);
-      b.kv.v = cv.take<char>(B * D.H * slots * D.hd * tb);
+      b.kv.pt = pt;
+      b.kv.pt_ld = pt_ld;
+      b.kv.pages = pages;
+      b.kv.k = cv.take<char>((size_t)pages * D.H * kPage * D.hd * tb);
+      b.kv.v = cv.take<char>((size_t)pages * D.H * kPage * D.hd * tb);
     }
   };
-  blocks(L.enc, c.n_enc, S);
-  blocks(L.lm, c.n_lm, Lt);
-  blocks(L.nb, c.n_nb, S);
+  blocks(L.enc, c.n_enc, S, D.pt_byte, D.pt_ld_byte, D.pages_byte);
+  blocks(L.lm, c.n_lm, Lt, D.pt_lm, D.pt_ld_lm, D.pages_lm);
+  blocks(L.nb, c.n_nb, S, D.pt_byte, D.pt_ld_byte, D.pages_byte);
   if (c.mb_kind == LCA_MB_LCA) {
-    blocks(L.mb, c.n_mb, S);
+    blocks(L.mb, c.n_mb, S, D.pt_mb, D.pt_ld_mb, D.pages_mb);
     D.mlp_w = nullptr;
   } else {
     L.mb.clear();
@@ -129,6 +145,7 @@ void carve(const lca_config& c, char* base, Layout& L) {
     r.b = cv.take<int>(R);
     r.pos = cv.take<int>(R);
     r.slot = cv.take<int>(R);
+    r.page = cv.take<int>(R);
     r.kvlen = cv.take<int>(R);
     r.seq_start = cv.take<int>(B);
     r.seq_count = cv.take<int>(B);
@@ -288,6 +305,9 @@ int validate(const lca_config* c) {
   if (c->mb_kind == LCA_MB_MLP && c->n_mlp_heads < c->max_n - 1) return LCA_E_ARG;
   if (c->n_enc < 0 || c->n_lm < 0 || c->n_nb < 0 || c->n_mb < 0) return LCA_E_ARG;
   if (c->boundary_byte < 0 || c->boundary_byte > 255) return LCA_E_ARG;
+  if (c->kv_pages < 0 || c->lm_pages < 0 || c->mb_pages < 0) return LCA_E_ARG;
+  // the attention kernels stage a sequence's page table row in shared memory
+  if ((c->max_bytes + kPage) / kPage > kMaxPtRow) return LCA_E_ARG;
   return LCA_OK;
 }
 
@@ -374,6 +394,9 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     r.rows = rows;
     r.M_cap = M_cap;
     r.S = blocks[0].kv.S;
+    r.pt = blocks[0].kv.pt;
+    r.pt_ld = blocks[0].kv.pt_ld;
+    r.pages = blocks[0].kv.pages;
     r.stable = stable;
     r.stable_stride = (int)(sizeof(SeqState) / sizeof(int));
     r.stable_add = stable_add;
@@ -766,9 +789,10 @@ int read_err(lca_ctx* c) {
     CK(cudaMemsetAsync(c->L.D.err, 0, sizeof(int), c->stream));
     CK(cudaStreamSynchronize(c->stream));
   }
-  if (e & ~7) fprintf(stderr, "lca: device error word 0x%x\n", e);
+  if (e & ~15) fprintf(stderr, "lca: device error word 0x%x\n", e);
   if (e & kErrTimeout) return LCA_E_TIMEOUT;
   if (e & kErrNumeric) return LCA_E_NUMERIC;
+  if (e & kErrPages) return LCA_E_CAPACITY;
   if (e & kErrIndex) return LCA_E_DEVICE_STATE;
   return LCA_OK;
 }
@@ -992,8 +1016,9 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
       for (auto* v : {&c->L.enc, &c->L.lm, &c->L.nb, &c->L.mb})
         for (auto& bk : *v) {
           SplitMapBlob blob;
-          const long long rows = (long long)D.B * D.H * bk.kv.S;
-          if (make_kv_tmaps(blob.b, bk.kv.k, bk.kv.v, rows) == LCA_OK) {
+          const long long rows = (long long)bk.kv.pages * D.H * kPage;
+          // the kernels address rows with 32-bit coordinates
+          if (rows <= 0x7fffffffLL && make_kv_tmaps(blob.b, bk.kv.k, bk.kv.v, rows) == LCA_OK) {
             c->kvmaps[bk.kv.k] = blob;
             bk.kv.tmaps = c->kvmaps[bk.kv.k].b;
           }
@@ -1085,6 +1110,20 @@ int lca_prefill(lca_ctx* c, int32_t batch, const uint8_t* const* prompts, const 
   std::vector<int> kv1(M), lkv1(Mlm);
   for (int r = 0; r < M; ++r) kv1[r] = rp[r] + 1;
   for (int r = 0; r < Mlm; ++r) lkv1[r] = lp[r] + 1;
+  // pages of the prompts' positions and latents, in sequence order; those of later positions and
+  // of the multi-byte windows are mapped by the decode steps
+  std::vector<int> ptb((size_t)D.B * D.pt_ld_byte, -1), ptl((size_t)D.B * D.pt_ld_lm, -1),
+      ptm((size_t)D.B * D.pt_ld_mb, -1);
+  int npb = 0, npl = 0;
+  for (int b = 0; b < batch; ++b) {
+    for (int j = 0; j * kPage < lens[b]; ++j) ptb[(size_t)b * D.pt_ld_byte + j] = npb++;
+    for (int j = 0; j * kPage < K[b] + 1; ++j) ptl[(size_t)b * D.pt_ld_lm + j] = npl++;
+  }
+  if (npb > D.pages_byte || npl > D.pages_lm) return LCA_E_CAPACITY;
+  std::vector<int> rpg(M), lpg(Mlm);
+  for (int r = 0; r < M; ++r) rpg[r] = ptb[(size_t)rb[r] * D.pt_ld_byte + rp[r] / kPage];
+  for (int r = 0; r < Mlm; ++r) lpg[r] = ptl[(size_t)lb[r] * D.pt_ld_lm + lp[r] / kPage];
+  const int pool_next[4] = {npb, npl, 0, 0};
   std::vector<int> last(batch);
   for (int b = 0; b < batch; ++b) last[b] = row0[b] + lens[b] - 1;
   auto up = [&](void* dst, const void* src, size_t n) {
@@ -1093,10 +1132,13 @@ int lca_prefill(lca_ctx* c, int32_t batch, const uint8_t* const* prompts, const 
   if (up(c->stg.bytes, bytes.data(), M) || up(c->stg.row0, row0.data(), batch * 4) ||
       up(c->stg.lens, lens, batch * 4) || up(c->stg.lm_row0, lm_row0.data(), batch * 4) ||
       up(D.r_v.b, rb.data(), M * 4) || up(D.r_v.pos, rp.data(), M * 4) ||
-      up(D.r_v.slot, rp.data(), M * 4) || up(D.r_v.kvlen, kv1.data(), M * 4) ||
+      up(D.r_v.slot, rp.data(), M * 4) || up(D.r_v.page, rpg.data(), M * 4) || up(D.r_v.kvlen, kv1.data(), M * 4) ||
       up(D.r_v.seq_start, ss.data(), D.B * 4) || up(D.r_v.seq_count, sc.data(), D.B * 4) ||
       up(D.r_v.M, &M, 4) || up(D.r_lm.b, lb.data(), Mlm * 4) || up(D.r_lm.pos, lp.data(), Mlm * 4) ||
-      up(D.r_lm.slot, lp.data(), Mlm * 4) || up(D.r_lm.kvlen, lkv1.data(), Mlm * 4) ||
+      up(D.r_lm.slot, lp.data(), Mlm * 4) || up(D.r_lm.page, lpg.data(), Mlm * 4) ||
+      up(D.r_lm.kvlen, lkv1.data(), Mlm * 4) || up(D.pt_byte, ptb.data(), ptb.size() * 4) ||
+      up(D.pt_lm, ptl.data(), ptl.size() * 4) || up(D.pt_mb, ptm.data(), ptm.size() * 4) ||
+      up(D.pool_next, pool_next, sizeof(pool_next)) ||
       up(D.r_lm.seq_start, ls.data(), D.B * 4) || up(D.r_lm.seq_count, lc.data(), D.B * 4) ||
       up(D.r_lm.M, &Mlm, 4) || up(D.head_rows_v, last.data(), batch * 4) || up(D.M_head_v, &batch, 4))
     return LCA_E_CUDA;
@@ -1362,6 +1404,25 @@ int lca_debug_accept_hist(lca_ctx* c, int32_t* out, int32_t reset) {
   return LCA_OK;
 }
 
+int lca_debug_page_table(lca_ctx* c, int32_t cache, int32_t* out, int64_t cap, int32_t* row_len, int32_t* used,
+                         int32_t* pages) {
+  if (!c || !row_len || !used || !pages || cache < 0 || cache > 2) return LCA_E_ARG;
+  Dev& D = c->L.D;
+  const int* pt = cache == 0 ? D.pt_byte : cache == 1 ? D.pt_lm : D.pt_mb;
+  const int ld = cache == 0 ? D.pt_ld_byte : cache == 1 ? D.pt_ld_lm : D.pt_ld_mb;
+  const int np = cache == 0 ? D.pages_byte : cache == 1 ? D.pages_lm : D.pages_mb;
+  *row_len = ld;
+  *pages = np;
+  const size_t n = (size_t)D.B * ld;
+  if (!out || cap < (int64_t)n) return LCA_E_CAPACITY;
+  int next[4];
+  CK(cudaMemcpyAsync(out, pt, n * 4, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaMemcpyAsync(next, D.pool_next, sizeof(next), cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  *used = std::min(next[cache], np);
+  return LCA_OK;
+}
+
 int lca_debug_set_eager(lca_ctx* c, int32_t on) {
   if (!c) return LCA_E_ARG;
   c->eager = on != 0;
@@ -1427,6 +1488,12 @@ int lca_debug_bench_kernel(lca_ctx* c, int32_t kind, int32_t rows, int32_t iters
   CK(cudaMemcpyAsync(D.r_v.b, z.data(), rows * 4, cudaMemcpyHostToDevice, s));
   CK(cudaMemcpyAsync(D.r_v.pos, pos.data(), rows * 4, cudaMemcpyHostToDevice, s));
   CK(cudaMemcpyAsync(D.r_v.slot, pos.data(), rows * 4, cudaMemcpyHostToDevice, s));
+  // slots [0, rows) of sequence 0 lie in its first page (rows <= 64), mapped by the prefill
+  std::vector<int> pg0(rows);
+  CK(cudaMemcpyAsync(pg0.data(), D.pt_byte, 4, cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  for (int i = 1; i < rows; ++i) pg0[i] = pg0[0];
+  CK(cudaMemcpyAsync(D.r_v.page, pg0.data(), rows * 4, cudaMemcpyHostToDevice, s));
   CK(cudaMemcpyAsync(D.r_v.kvlen, kvl.data(), rows * 4, cudaMemcpyHostToDevice, s));
   CK(cudaMemcpyAsync(D.r_v.seq_start, ss.data(), D.B * 4, cudaMemcpyHostToDevice, s));
   CK(cudaMemcpyAsync(D.r_v.seq_count, sc.data(), D.B * 4, cudaMemcpyHostToDevice, s));

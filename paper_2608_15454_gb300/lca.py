@@ -18,6 +18,7 @@ LCA_OK = 0
 LCA_F32, LCA_BF16 = 0, 1
 LCA_MB_LCA, LCA_MB_MLP = 0, 1
 LCA_THRESH, LCA_SPEC = 0, 1
+LCA_E_ARG, LCA_E_CAPACITY, LCA_E_DEVICE_STATE, LCA_E_TIMEOUT = -1, -2, -5, -7
 
 STATUS = {0: "LCA_OK", -1: "LCA_E_ARG", -2: "LCA_E_CAPACITY", -3: "LCA_E_WEIGHTS", -4: "LCA_E_CUDA",
           -5: "LCA_E_DEVICE_STATE", -6: "LCA_E_NUMERIC", -7: "LCA_E_TIMEOUT", -8: "LCA_E_STATE"}
@@ -32,7 +33,7 @@ EXPORTS = ("lca_workspace_bytes", "lca_create", "lca_prefill", "lca_mbp_step", "
            "lca_decode_attention_scratch_bytes", "lca_decode_attention", "lca_decode_attention_noalloc",
            "lca_decode_attention_noalloc_capacity", "lca_decode_attention_status",
            "lca_decode_attention_noalloc_status", "lca_debug_set_wait_spins",
-           "lca_debug_step_log", "lca_debug_accept_hist")
+           "lca_debug_step_log", "lca_debug_accept_hist", "lca_debug_page_table")
 
 
 class LcaConfig(ctypes.Structure):
@@ -42,7 +43,8 @@ class LcaConfig(ctypes.Structure):
                 ("n_mb", ctypes.c_int32), ("mb_kind", ctypes.c_int32), ("n_mlp_heads", ctypes.c_int32),
                 ("boundary_byte", ctypes.c_int32), ("rope_base", ctypes.c_float),
                 ("rms_eps", ctypes.c_float), ("attn_scale", ctypes.c_float), ("dtype", ctypes.c_int32),
-                ("max_batch", ctypes.c_int32), ("max_bytes", ctypes.c_int32), ("max_n", ctypes.c_int32)]
+                ("max_batch", ctypes.c_int32), ("max_bytes", ctypes.c_int32), ("max_n", ctypes.c_int32),
+                ("kv_pages", ctypes.c_int32), ("lm_pages", ctypes.c_int32), ("mb_pages", ctypes.c_int32)]
 
 
 class LcaTensor(ctypes.Structure):
@@ -122,6 +124,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "lca_debug_set_wait_spins": [I32],
         "lca_debug_step_log": [P, ctypes.c_int64, I32, P],
         "lca_debug_accept_hist": [P, P, I32],
+        "lca_debug_page_table": [P, I32, P, ctypes.c_int64, P, P, P],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
@@ -133,13 +136,17 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     return lib
 
 
-def make_config(model, max_batch: int, max_bytes: int, max_n: int) -> LcaConfig:
-    """lca_config from a synth.ModelConfig."""
+def make_config(model, max_batch: int, max_bytes: int, max_n: int, kv_pages: int = 0,
+                lm_pages: int = 0, mb_pages: int = 0) -> LcaConfig:
+    """lca_config from a synth.ModelConfig (kv_pages, lm_pages, mb_pages: pages of 64 slots in
+    each byte-cache, LM-cache and window-cache layer's pool, 0 = enough for every sequence at
+    max_bytes)."""
     return LcaConfig(model.d_model, model.n_heads, model.head_dim, model.d_ff, model.vocab,
                      model.n_enc, model.n_lm, model.n_nb, model.n_mb,
                      LCA_MB_MLP if model.mb_kind == "mlp" else LCA_MB_LCA, model.n_mlp_heads,
                      model.boundary_byte, model.rope_base, model.rms_eps, model.attn_scale,
-                     LCA_BF16 if model.dtype == "bf16" else LCA_F32, max_batch, max_bytes, max_n)
+                     LCA_BF16 if model.dtype == "bf16" else LCA_F32, max_batch, max_bytes, max_n,
+                     kv_pages, lm_pages, mb_pages)
 
 
 def _ptr(a: np.ndarray):
@@ -150,14 +157,15 @@ class Context:
     """One lca_ctx: weights and workspace on a CUDA device, prompts and outputs on the host."""
 
     def __init__(self, model, weights: dict, max_batch: int, max_bytes: int, max_n: int,
-                 device: str = "cuda", stream=None):
+                 device: str = "cuda", stream=None, kv_pages: int = 0, lm_pages: int = 0,
+                 mb_pages: int = 0):
         import torch
         self.torch = torch
         self.lib = load_library()
         self.model = model
         self.device = torch.device(device)
         self.max_n = max_n
-        self.cfg = make_config(model, max_batch, max_bytes, max_n)
+        self.cfg = make_config(model, max_batch, max_bytes, max_n, kv_pages, lm_pages, mb_pages)
         wdt = torch.bfloat16 if model.dtype == "bf16" else torch.float32
         self._weights = {}
         tensors = []
@@ -260,6 +268,18 @@ class Context:
         out = np.zeros(self.max_n, dtype=np.int32)
         self._check(self.lib.lca_debug_accept_hist(self.h, _ptr(out), 1 if reset else 0), "lca_debug_accept_hist")
         return out
+
+    def page_table(self, cache):
+        """(table [max_batch][row_len] of pool pages or -1, pages mapped, pool pages) of cache kind
+        0 (byte positions), 1 (LM latents) or 2 (multi-byte windows)."""
+        ld, used, pages = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+        self.lib.lca_debug_page_table(self.h, cache, None, 0, ctypes.byref(ld), ctypes.byref(used),
+                                      ctypes.byref(pages))
+        out = np.zeros(self.cfg.max_batch * ld.value, dtype=np.int32)
+        self._check(self.lib.lca_debug_page_table(self.h, cache, _ptr(out), out.size, ctypes.byref(ld),
+                                                  ctypes.byref(used), ctypes.byref(pages)),
+                    "lca_debug_page_table")
+        return out.reshape(self.cfg.max_batch, ld.value), used.value, pages.value
 
     def set_eager(self, on: bool):
         self._check(self.lib.lca_debug_set_eager(self.h, 1 if on else 0), "lca_debug_set_eager")
