@@ -192,11 +192,18 @@ __device__ __forceinline__ int kv_page_cg(const KV& kv, int b, int s) {
 __device__ __forceinline__ size_t kv_off(const KV& kv, int H, int hd, int b, int h, int s) {
   return kv_addr(kv, H, hd, b, h, s, kv_page_cg(kv, b, s));
 }
-// The page table row of sequence b into shared memory (pt_ld entries, checked as kv_page_cg
-// does); nothing for the contiguous layout. The caller synchronises before the first use.
-__device__ __forceinline__ void kv_stage_pages(const KV& kv, int b, int* s_pt, int tid, int nthreads) {
+// The page table row of sequence b into shared memory, in two halves so that the loads overlap the
+// caller's other loads: kv_pages_load issues this thread's first entry (tid < pt_ld), the caller
+// issues its own loads, then kv_pages_store writes that entry and loads and writes the rest of the
+// row (pt_ld entries, checked as kv_page_cg does). Nothing for the contiguous layout. The caller
+// synchronises before the first use.
+__device__ __forceinline__ int kv_pages_load(const KV& kv, int b, int tid) {
+  return (kv.pt && tid < kv.pt_ld) ? __ldcg(kv.pt + (size_t)b * kv.pt_ld + tid) : 0;
+}
+__device__ __forceinline__ void kv_pages_store(const KV& kv, int b, int* s_pt, int tid, int nthreads, int first) {
   if (!kv.pt) return;
-  for (int i = tid; i < kv.pt_ld; i += nthreads) {
+  if (tid < kv.pt_ld) s_pt[tid] = (first < 0 || first >= kv.pages) ? 0 : first;
+  for (int i = tid + nthreads; i < kv.pt_ld; i += nthreads) {
     const int pg = __ldcg(kv.pt + (size_t)b * kv.pt_ld + i);
     s_pt[i] = (pg < 0 || pg >= kv.pages) ? 0 : pg;
   }
@@ -234,6 +241,27 @@ __device__ __forceinline__ void kv_prefetch_l2(const KV& kv, const void* base, i
                        "r"(bytes)
                        : "memory");
       }
+    }
+  }
+}
+// The same hint for K and V by a whole warp: lane i takes pages i, i + 32, ... of the range, so
+// that the table lookups of up to 32 pages are in flight together.
+__device__ __forceinline__ void kv_prefetch_l2_warp(const KV& kv, int es, int H, int hd, int b, int h, int lo,
+                                                    int hi, int lane) {
+  if (!kv.pt) {
+    if (lane < 2) kv_prefetch_l2(kv, lane ? kv.v : kv.k, es, H, hd, b, h, lo, hi);
+    return;
+  }
+  for (int s0 = (lo & ~(kPage - 1)) + lane * kPage; s0 < hi; s0 += 32 * kPage) {
+    const int a = max(lo, s0), e = min(hi, s0 + kPage);
+    const int pg = kv_page_cg(kv, b, a);
+    const uint32_t bytes = (uint32_t)((e - a) * hd * es) & ~15u;
+    const size_t o = kv_addr(kv, H, hd, b, h, a, pg) * es;
+    if (bytes) {
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const char*>(kv.k) + o), "r"(bytes)
+                   : "memory");
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const char*>(kv.v) + o), "r"(bytes)
+                   : "memory");
     }
   }
 }
@@ -346,7 +374,9 @@ struct Dev {
   int tiled_min_rows;  // layers with more typical rows than this run on the tensor cores
   int attn_pipe;       // decode attention: 2 = tensor cores (bf16, head_dim 64), 1 = bulk-copy pipelined
                        // CUDA-core kernel, 0 = register-tiled kernel
-  int attn_ns;         // ring stages of the tensor-core decode attention (4, 6 or 8)
+  int attn_ns;         // ring stages of the tensor-core prefill attention (4 or 8)
+  int attn_ns_t;       // ring stages of the tensor-core decode attention (4, 8 or 12)
+  int attn_tc_min;     // fewest (sequence, head) pairs for the tensor-core attention kernels
   int attn_min_keys;   // fewest cache keys per key split of a decode attention launch
   int attn_t;          // decode steps use the transposed tensor-core attention (8-row query tiles)
   int attn_w;          // small-batch decode steps use the warp-walk attention
@@ -556,12 +586,12 @@ void kernel_attrs_step();
 void kernel_attrs_attn();
 // Attention of query rows over a KV-cache layer (keys [0, kvlen[r]) of sequence b[r]).
 // stable: optional per-sequence committed length (stride in ints) whose cache prefix (the first
-// stable + stable_add slots) does not change during a step: prefetched into L2, or staged in
-// shared memory, before the dependency wait; stable_extra: rows added; rows_seq: the most query
-// rows a sequence has (a tile-size hint).
+// stable + stable_add slots) does not change during a step: the warp-walk decode kernel stages it
+// in shared memory before the dependency wait; rows_seq: the most query rows a sequence has (a
+// tile-size hint).
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s, const int* stable = nullptr,
-               int stable_extra = 0, bool short_kv = false, int stable_add = 0, int rows_seq = kAttnQT);
+               bool short_kv = false, int stable_add = 0, int rows_seq = kAttnQT);
 
 // Step / prefill glue kernels (kernels_step.cu).
 void launch_mb_plan(const Dev& D, cudaStream_t s);

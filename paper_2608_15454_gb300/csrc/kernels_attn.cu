@@ -285,7 +285,7 @@ __device__ __forceinline__ void load4(const float* p, float (&v)[4]) {
 template <typename TC, int HD>
 __global__ void __launch_bounds__(kA2Threads)
 k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
-        int* err, const int* __restrict__ stable, int stable_stride, int stable_extra) {
+        int* err) {
   namespace cgr = cooperative_groups;
   constexpr int QT = kAttnQT;
   constexpr int EV = 16 / (int)sizeof(TC);
@@ -304,15 +304,6 @@ k_attn2(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
   cgr::cluster_group cl = cgr::this_cluster();
   const int splits = (int)cl.dim_blocks().z;
   const int sp = (int)cl.block_rank();
-  if (stable && threadIdx.x < 2) {
-    // Cache slots below the committed length do not change during a step: prefetch this CTA's
-    // approximate K (thread 0) and V (thread 1) range into L2 before the dependency wait.
-    const int bb = blockIdx.x, hh = blockIdx.z / splits;
-    const int t = stable[(size_t)bb * stable_stride];
-    const int est = ((t + stable_extra + splits - 1) / splits + 15) / 16 * 16;
-    const int lo = sp * est, hi = min(t, lo + est);
-    kv_prefetch_l2(kv, threadIdx.x == 0 ? kv.k : kv.v, (int)sizeof(TC), H, HD, bb, hh, lo, hi);
-  }
   pdl_trigger();
   pdl_wait();
   _trace.waited();
@@ -560,7 +551,7 @@ __device__ __forceinline__ void a3_v2(const __nv_bfloat16* p, float& a, float& b
 template <typename TC, int HD>
 __global__ void __launch_bounds__(kA3Threads, 3)
 k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
-        int* err, const int* __restrict__ stable, int stable_stride, int stable_extra) {
+        int* err) {
   namespace cgr = cooperative_groups;
   constexpr int QT = kAttnQT;                     // query rows per tile (8)
   constexpr int KC = kA3Keys;
@@ -594,28 +585,19 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&full[i])) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (stable && tid < 2) {
-    // slots below the committed length do not change during a step: warm this CTA's share of
-    // them in L2 before the dependency wait (a hint only)
-    const int bb = blockIdx.x, hh = blockIdx.z / splits;
-    const int t = stable[(size_t)bb * stable_stride];
-    const int est = ((t + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
-    const int lo = sp * est, hi = min(t, lo + est);
-    kv_prefetch_l2(kv, tid == 0 ? kv.k : kv.v, (int)sizeof(TC), H, HD, bb, hh, lo, hi);
-  }
   pdl_trigger();
   pdl_wait();
   _trace.waited();
   __syncthreads();
   const int b = blockIdx.x;
   const int h = blockIdx.z / splits;
+  const int pt0 = kv_pages_load(kv, b, tid);  // stored with the first tile's loads
   const int nrows = rows.seq_count[b];
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
   const TC* Kc = reinterpret_cast<const TC*>(kv.k);
   const TC* Vc = reinterpret_cast<const TC*>(kv.v);
   const int ld = H * HD;
-  kv_stage_pages(kv, b, s_pt, tid, kA3Threads);  // published by the tile's first barrier
   bool failed = false;
   uint32_t cc = 0;      // chunks consumed by this CTA so far (ring phase)
   uint32_t issued = 0;  // chunks whose copies were issued (thread 0)
@@ -637,6 +619,7 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
       s_m[tid] = -INFINITY;
       s_l[tid] = 0.f;
     }
+    if (qt == (int)blockIdx.y) kv_pages_store(kv, b, s_pt, tid, kA3Threads, pt0);
     __syncthreads();
     int kv_hi = 0;
 #pragma unroll
@@ -823,8 +806,7 @@ size_t attn3_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
 
 template <typename TC, int HD>
 void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-               int qtiles_grid, int splits, int* err, const int* stable, int stable_stride,
-               int stable_extra, cudaStream_t s) {
+               int qtiles_grid, int splits, int* err, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA3Threads);
@@ -840,8 +822,7 @@ void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn3<TC, HD>, q, out, kv, rows, H, scale, err, stable, stable_stride,
-                     stable_extra);
+  cudaLaunchKernelEx(&cfg, k_attn3<TC, HD>, q, out, kv, rows, H, scale, err);
 }
 
 // ---------------------------------------------------------------- warp-walk decode attention
@@ -909,7 +890,7 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
   const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(kv.k);
   const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(kv.v);
   pdl_trigger();
-  if (tid == 0) {
+  if (warp == 0) {
     int S = 0, slo = 0, nst = 0;
     if (stable) {
       S = stable[(size_t)b * stable_stride] + stable_add;
@@ -918,26 +899,30 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
       aw_share(0, S, splits, sp, slo, shi);
       nst = min(shi - slo, stage_cap);
     }
-    s_stage[0] = S;
-    s_stage[1] = slo;
-    s_stage[2] = nst;
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&s_bar)) : "memory");
-    if (sp == 0 && splits > 1)
-      asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a3_su32(&s_rbar)), "r"(splits - 1) : "memory");
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    if (nst > 0) {
-      // committed slots: their pages were mapped by earlier steps, so the table entries are final
-      const uint32_t bytes = (uint32_t)(nst * HD * 2);
-      a3_expect(&s_bar, 2 * bytes);
-      // one copy per page run (at most five pages: 256 keys from a 4-aligned slot)
-      for (int s0 = slo; s0 < slo + nst;) {
-        const int run = kv_run(kv, s0, slo + nst - s0);
-        const size_t o = kv_off(kv, H, HD, b, h, s0);
-        const uint32_t rb = (uint32_t)(run * HD * 2);
-        a3_copy(Ks + (size_t)(s0 - slo) * HD, Kc + o, rb, &s_bar);
-        a3_copy(Vs + (size_t)(s0 - slo) * HD, Vc + o, rb, &s_bar);
-        s0 += run;
-      }
+    // committed slots (their pages were mapped by earlier steps, so the table entries are final):
+    // lane i copies the run of the staged range in the i-th page (at most five: 256 keys from a
+    // 4-aligned slot), all lanes' page lookups in flight together; contiguous: lane 0, one run
+    const int p0 = slo & ~(kPage - 1);
+    const int a = kv.pt ? max(slo, p0 + lane * kPage) : slo;
+    const int e = kv.pt ? min(slo + nst, p0 + (lane + 1) * kPage) : slo + nst;
+    const bool mine = a < e && (kv.pt || lane == 0);
+    const int pg = mine ? kv_page_cg(kv, b, a) : 0;
+    if (lane == 0) {
+      s_stage[0] = S;
+      s_stage[1] = slo;
+      s_stage[2] = nst;
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&s_bar)) : "memory");
+      if (sp == 0 && splits > 1)
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a3_su32(&s_rbar)), "r"(splits - 1) : "memory");
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+      if (nst > 0) a3_expect(&s_bar, 2u * (uint32_t)(nst * HD * 2));
+    }
+    __syncwarp();
+    if (mine) {
+      const size_t o = kv_addr(kv, H, HD, b, h, a, pg);
+      const uint32_t rb = (uint32_t)((e - a) * HD * 2);
+      a3_copy(Ks + (size_t)(a - slo) * HD, Kc + o, rb, &s_bar);
+      a3_copy(Vs + (size_t)(a - slo) * HD, Vc + o, rb, &s_bar);
     }
   }
   // rank 0's arrival barrier exists before any peer can arrive on it (a cluster barrier before
@@ -948,22 +933,37 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
   bool staged = nst == 0;  // the staged keys have landed (or there are none)
   pdl_wait();
   _trace.waited();
-  const int nrows = rows.seq_count[b];
-  const int rbeg = rows.seq_start[b];
-  const int ntiles = (nrows + QT - 1) / QT;
+  const int pt0 = kv_pages_load(kv, b, tid);  // stored with the first tile's loads
   const int ld = H * HD;
-  kv_stage_pages(kv, b, s_pt, tid, kAwThreads);  // published by the tile's first barrier
+  // One sequence (a grid of one sequence): its rows start at 0, so the first tile's query rows and
+  // cache lengths are loaded together with the row count (rows past the count are dropped after).
+  static_assert(QT * 64 / 4 <= kAwThreads, "one query vector per thread");
+  const bool one_seq = gridDim.x == 1;
+  float4 q_pre = make_float4(0.f, 0.f, 0.f, 0.f);
+  int kl_pre = 0;
+  if (one_seq) {
+    const int r0 = (int)blockIdx.y * QT;
+    if (tid < QT * HD / 4) {
+      const int i = tid / (HD / 4), c4 = tid - i * (HD / 4);
+      q_pre = *reinterpret_cast<const float4*>(q + (size_t)(r0 + i) * ld + h * HD + 4 * c4);
+    }
+    if (tid < QT) kl_pre = rows.kvlen[r0 + tid];
+  }
+  const int nrows = rows.seq_count[b];
+  const int rbeg = one_seq ? 0 : rows.seq_start[b];
+  const int ntiles = (nrows + QT - 1) / QT;
 
   const int g = lane >> 3, e = lane & 7;  // key slot of this lane in a warp step, its 8 head dims
   for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
     const int r0 = rbeg + qt * QT;
     const int nq = min(QT, nrows - qt * QT);
+    const bool pre = one_seq && qt == (int)blockIdx.y;
     // the tile's query rows (pre-scaled) and cache lengths in shared memory
     for (int idx = tid; idx < QT * HD / 4; idx += kAwThreads) {
       const int i = idx / (HD / 4), c4 = idx - i * (HD / 4);
       float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
       if (i < nq) {
-        v = *reinterpret_cast<const float4*>(q + (size_t)(r0 + i) * ld + h * HD + 4 * c4);
+        v = pre ? q_pre : *reinterpret_cast<const float4*>(q + (size_t)(r0 + i) * ld + h * HD + 4 * c4);
         v.x *= scale; v.y *= scale; v.z *= scale; v.w *= scale;
       }
       *reinterpret_cast<float4*>(&qs[i][4 * c4]) = v;
@@ -971,7 +971,7 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
     if (tid < QT) {
       int k = 0;
       if (tid < nq) {
-        k = rows.kvlen[r0 + tid];
+        k = pre ? kl_pre : rows.kvlen[r0 + tid];
         if (k > kv.S || k < 0) {
           atomicOr(err, kErrIndex);
           k = k < 0 ? 0 : kv.S;
@@ -979,6 +979,7 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
       }
       s_kl[tid] = k;
     }
+    if (qt == (int)blockIdx.y) kv_pages_store(kv, b, s_pt, tid, kAwThreads, pt0);
     __syncthreads();
     int kl[QT];
     int kv_hi = 0;
@@ -1310,8 +1311,7 @@ __device__ __noinline__ void a4_record(int which, uint32_t gi, int st, int nch, 
 template <int NS>
 __global__ void __maxnreg__(200)
 k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
-           const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-           const int* __restrict__ stable, int stable_stride, int stable_extra) {
+           const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
   namespace cgr = cooperative_groups;
   constexpr int HD = 64, QT = kA4QT, KC = kA4Keys;
   // each stage must have one consumer warp, which takes its phases in order: a warp waiting on a
@@ -1349,14 +1349,6 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
   }
-  if (stable && tid < 2) {
-    // committed slots do not change during a step: warm this CTA's share in L2 (a hint)
-    const int bb = blockIdx.x, hh = blockIdx.z / splits;
-    const int tt = stable[(size_t)bb * stable_stride];
-    const int est = ((tt + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
-    const int lo = sp * est, hi = min(tt, lo + est);
-    kv_prefetch_l2(kv, tid == 0 ? kv.k : kv.v, 2, H, HD, bb, hh, lo, hi);
-  }
   pdl_trigger();
   pdl_wait();
   _trace.waited();
@@ -1367,7 +1359,6 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
   const int ld = H * HD;
-  kv_stage_pages(kv, b, s_pt, tid, kA4Threads);  // published by the tile's first barrier
   bool failed = false;
   uint32_t cc = 0, issued = 0;
 
@@ -1396,6 +1387,9 @@ k_attn_mma(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       }
       s_kv[tid] = kl;
     }
+    // prefill tiles are long: the table row is loaded here (a register held across the query
+    // staging would spill)
+    if (qt == (int)blockIdx.y) kv_pages_store(kv, b, s_pt, tid, kA4Threads, kv_pages_load(kv, b, tid));
     __syncthreads();
     int kv_hi = 0;
 #pragma unroll
@@ -1621,8 +1615,7 @@ size_t attn_mma_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
 
 template <int NS>
 void launch_a4_ns(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-                  int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
-                  cudaStream_t s) {
+                  int qtiles_grid, int splits, int* err, cudaStream_t s) {
   CUtensorMap tk, tv;
   memcpy(&tk, kv.tmaps, sizeof(tk));
   memcpy(&tv, static_cast<const unsigned char*>(kv.tmaps) + 128, sizeof(tv));
@@ -1641,8 +1634,7 @@ void launch_a4_ns(const float* q, float* out, const KV& kv, const Rows& rows, in
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn_mma<NS>, q, out, kv, rows, H, scale, err, tk, tv, stable, stable_stride,
-                     stable_extra);
+  cudaLaunchKernelEx(&cfg, k_attn_mma<NS>, q, out, kv, rows, H, scale, err, tk, tv);
 }
 
 // ---------------------------------------------------------------- transposed tensor-core attention
@@ -1668,8 +1660,7 @@ __device__ __forceinline__ uint32_t movt(uint32_t x) {
 template <int NS>
 __global__ void __launch_bounds__(kA4Threads, 1)
 k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
-           const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-           const int* __restrict__ stable, int stable_stride, int stable_extra) {
+           const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
   namespace cgr = cooperative_groups;
   constexpr int HD = 64, QT = kA5QT, KC = kA4Keys;
   static_assert(NS % kA4Warps == 0, "ring stages must be a multiple of the compute warps");
@@ -1705,25 +1696,17 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
   }
-  if (stable && tid < 2) {
-    // committed slots do not change during a step: warm this CTA's share in L2 (a hint)
-    const int bb = blockIdx.x, hh = blockIdx.z / splits;
-    const int tt = stable[(size_t)bb * stable_stride];
-    const int est = ((tt + stable_extra + splits - 1) / splits + KC - 1) / KC * KC;
-    const int lo = sp * est, hi = min(tt, lo + est);
-    kv_prefetch_l2(kv, tid == 0 ? kv.k : kv.v, 2, H, HD, bb, hh, lo, hi);
-  }
   pdl_trigger();
   pdl_wait();
   _trace.waited();
   __syncthreads();
   const int b = blockIdx.x;
   const int h = blockIdx.z / splits;
+  const int pt0 = kv_pages_load(kv, b, tid);  // stored with the first tile's loads
   const int nrows = rows.seq_count[b];
   const int rbeg = rows.seq_start[b];
   const int ntiles = (nrows + QT - 1) / QT;
   const int ld = H * HD;
-  kv_stage_pages(kv, b, s_pt, tid, kA4Threads);  // published by the tile's first barrier
   bool failed = false;
   uint32_t cc = 0, issued = 0;
 
@@ -1752,6 +1735,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       }
       s_kv[tid] = kl;
     }
+    if (qt == (int)blockIdx.y) kv_pages_store(kv, b, s_pt, tid, kA4Threads, pt0);
     __syncthreads();
     int kv_hi = 0;
 #pragma unroll
@@ -1984,8 +1968,7 @@ size_t attn_mmt_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
 
 template <int NS>
 void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-                  int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
-                  cudaStream_t s) {
+                  int qtiles_grid, int splits, int* err, cudaStream_t s) {
   CUtensorMap tk, tv;
   memcpy(&tk, kv.tmaps, sizeof(tk));
   memcpy(&tv, static_cast<const unsigned char*>(kv.tmaps) + 128, sizeof(tv));
@@ -2004,21 +1987,18 @@ void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, in
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn_mmt<NS>, q, out, kv, rows, H, scale, err, tk, tv, stable, stable_stride,
-                     stable_extra);
+  cudaLaunchKernelEx(&cfg, k_attn_mmt<NS>, q, out, kv, rows, H, scale, err, tk, tv);
 }
 
 void launch_a4(int ns, const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-               int qtiles_grid, int splits, int* err, const int* stable, int stable_stride, int stable_extra,
-               cudaStream_t s) {
-  if (ns == 4) launch_a4_ns<4>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, err, stable, stable_stride, stable_extra, s);
-  else launch_a4_ns<8>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, err, stable, stable_stride, stable_extra, s);
+               int qtiles_grid, int splits, int* err, cudaStream_t s) {
+  if (ns == 4) launch_a4_ns<4>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, err, s);
+  else launch_a4_ns<8>(q, out, kv, rows, B, H, scale, qtiles_grid, splits, err, s);
 }
 
 template <typename TC, int HD>
 void launch_cl(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-               int qtiles_grid, int splits, int* err, const int* stable, int stable_stride,
-               int stable_extra, cudaStream_t s) {
+               int qtiles_grid, int splits, int* err, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA2Threads);
@@ -2033,8 +2013,7 @@ void launch_cl(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn2<TC, HD>, q, out, kv, rows, H, scale, err, stable, stable_stride,
-                     stable_extra);
+  cudaLaunchKernelEx(&cfg, k_attn2<TC, HD>, q, out, kv, rows, H, scale, err);
 }
 
 template <typename TC, int HD>
@@ -2187,6 +2166,7 @@ void kernel_attrs_attn() {
   cudaFuncSetAttribute(k_attn_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem<8>());
   cudaFuncSetAttribute(k_attn_mmt<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<4>());
   cudaFuncSetAttribute(k_attn_mmt<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<8>());
+  cudaFuncSetAttribute(k_attn_mmt<12>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<12>());
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn_w<4>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn_w<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -2208,25 +2188,24 @@ void kernel_attrs_attn() {
 }
 
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
-               int qtiles_grid, int splits, cudaStream_t s, const int* stable, int stable_extra,
-               bool short_kv, int stable_add, int rows_seq) {
+               int qtiles_grid, int splits, cudaStream_t s, const int* stable, bool short_kv, int stable_add,
+               int rows_seq) {
   ProfScope ps(PK_ATTN, 0.0, s);
-  const int* stable_aw = stable;
-  // the other kernels take `stable` as the committed byte length of an L2 prefetch hint
-  if (stable_add != 0) stable = nullptr;
   if (splits < 1) splits = 1;
   const int ss = (int)(sizeof(SeqState) / sizeof(int));
   // the tensor-core kernel holds two CTAs per SM: it pays off with many (sequence, head) pairs over
   // long caches; with few pairs, or short caches (the multi-byte window), the CUDA-core pipelined
   // kernel (three CTAs per SM) runs, spreading keys over up to 16 splits
-  if (D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= 128 && !short_kv) {
+  if (D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= D.attn_tc_min && !short_kv) {
     const int sc = std::min(splits, kMaxClusterSplit);
     // decode steps (one query tile of a few rows per sequence): the transposed kernel
     if (qtiles_grid == 1 && D.attn_t) {
-      if (D.attn_ns == 4) launch_a5_ns<4>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, stable, ss, stable_extra, s);
-      else launch_a5_ns<8>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, stable, ss, stable_extra, s);
+      if (D.attn_ns_t == 4) launch_a5_ns<4>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, s);
+      else if (D.attn_ns_t == 12)
+        launch_a5_ns<12>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, s);
+      else launch_a5_ns<8>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, s);
     } else {
-      launch_a4(D.attn_ns, q, out, kv, rows, B, D.H, D.scale, qtiles_grid, sc, D.err, stable, ss, stable_extra, s);
+      launch_a4(D.attn_ns, q, out, kv, rows, B, D.H, D.scale, qtiles_grid, sc, D.err, s);
     }
     return;
   }
@@ -2234,25 +2213,25 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
     splits = std::min(splits, kA4MaxSplit);
     // decode steps (one query tile per sequence) of bf16 head-dim-64 caches: the warp-walk kernel
     if (qtiles_grid == 1 && D.attn_w && D.dtype == LCA_BF16 && D.hd == 64 && kv.pt) {
-      launch_aw(q, out, kv, rows, B, D.H, D.scale, splits, D.err, stable_aw, ss, stable_add, rows_seq, s);
+      launch_aw(q, out, kv, rows, B, D.H, D.scale, splits, D.err, stable, ss, stable_add, rows_seq, s);
       return;
     }
     if (D.dtype == LCA_BF16) {
-      if (D.hd == 64) launch_a3<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
-      else launch_a3<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+      if (D.hd == 64) launch_a3<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+      else launch_a3<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
     } else {
-      if (D.hd == 64) launch_a3<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
-      else launch_a3<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+      if (D.hd == 64) launch_a3<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+      else launch_a3<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
     }
     return;
   }
   if (splits > kMaxClusterSplit) splits = kMaxClusterSplit;
   if (D.dtype == LCA_BF16) {
-    if (D.hd == 64) launch_cl<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
-    else launch_cl<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+    if (D.hd == 64) launch_cl<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+    else launch_cl<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
   } else {
-    if (D.hd == 64) launch_cl<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
-    else launch_cl<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, stable, ss, stable_extra, s);
+    if (D.hd == 64) launch_cl<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+    else launch_cl<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
   }
 }
 

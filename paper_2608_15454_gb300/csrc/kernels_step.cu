@@ -17,17 +17,29 @@ __device__ __forceinline__ void err_or(int* e, int bits) { atomicOr(e, bits); }
 // Maps a page to every page of slots [s0, s1] of sequence b that has none, from the pool's bump
 // counter. One thread per sequence row of the table. A page stays mapped until the next prefill
 // (a multi-byte window that restarts reuses its pages); an exhausted pool leaves the entry
-// unmapped and raises kErrPages, and the writers then skip those slots.
-__device__ void map_pages(int* pt, int ld, int pages, int* next, int b, int s0, int s1, int* err) {
+// unmapped (-1) and raises kErrPages, and the writers then skip those slots. Returns the pages of
+// slots s0 and s1 in *pg0 and *pg1.
+__device__ void map_pages(int* pt, int ld, int pages, int* next, int b, int s0, int s1, int* err, int* pg0,
+                          int* pg1) {
   if (s0 < 0) s0 = 0;
+  int first = -1, last = -1;
   for (int j = s0 / kPage; j <= s1 / kPage && j < ld; ++j) {
     int* e = pt + (size_t)b * ld + j;
-    if (*e < 0) {
-      const int pg = atomicAdd(next, 1);
-      if (pg < pages) *e = pg;
-      else err_or(err, kErrPages);
+    int pg = *e;
+    if (pg < 0) {
+      pg = atomicAdd(next, 1);
+      if (pg < pages) {
+        *e = pg;
+      } else {
+        err_or(err, kErrPages);
+        pg = -1;
+      }
     }
+    if (j == s0 / kPage) first = pg;
+    last = pg;
   }
+  *pg0 = first;
+  *pg1 = last;
 }
 // Page of slot s of sequence b (after map_pages), -1 if unmapped.
 __device__ __forceinline__ int page_of(const int* pt, int ld, int b, int s) {
@@ -52,6 +64,7 @@ __global__ void k_mb_plan(Dev D, int fill) {
   __shared__ int s_first[1024];
   __shared__ int s_start[1024];
   __shared__ int s_ms[1024];
+  __shared__ int s_pg0[1024], s_pg1[1024];  // pages of the first and last window row of each sequence
   __shared__ int s_K[4], s_gsK[4];  // fill (at most 4 sequences): K and the start of group K
   __shared__ int s_M;
   const Params P = *D.params;
@@ -76,8 +89,12 @@ __global__ void k_mb_plan(Dev D, int fill) {
     s_cnt[b] = (t - first) + (n - 2);
     s_ms[b] = s;
     st.mb_len = t - s;
+    int pg0 = -1, pg1 = -1;
     if (s_cnt[b] > 0)
-      map_pages(D.pt_mb, D.pt_ld_mb, D.pages_mb, &D.pool_next[2], b, first - s, first - s + s_cnt[b] - 1, D.err);
+      map_pages(D.pt_mb, D.pt_ld_mb, D.pages_mb, &D.pool_next[2], b, first - s, first - s + s_cnt[b] - 1, D.err,
+                &pg0, &pg1);
+    s_pg0[b] = pg0;
+    s_pg1[b] = pg1;
   }
   __syncthreads();
   if (tid == 0) {
@@ -118,7 +135,8 @@ __global__ void k_mb_plan(Dev D, int fill) {
       D.r_mb.b[r] = b;
       D.r_mb.pos[r] = p;
       D.r_mb.slot[r] = p - s;
-      D.r_mb.page[r] = page_of(D.pt_mb, D.pt_ld_mb, b, p - s);
+      const int sl = p - s, f0 = (first - s) / kPage, l0 = (first - s + cnt - 1) / kPage;
+      D.r_mb.page[r] = sl / kPage == f0 ? s_pg0[b] : sl / kPage == l0 ? s_pg1[b] : page_of(D.pt_mb, D.pt_ld_mb, b, sl);
       D.r_mb.kvlen[r] = p - s + 1;
     }
     for (int j = lane; j < n - 1; j += 32)
@@ -378,10 +396,12 @@ __global__ void k_verify_plan(Dev D) {
     }
     return;
   }
-  // pages of positions t..t+n-1 (one thread maps; the rows read the table after the barrier)
+  // pages of positions t..t+n-1 (one thread maps them: at most two pages for n <= 64)
+  __shared__ int s_pg[2];
   if (tid == 0) {
     const int t = D.seq[b].t;
-    map_pages(D.pt_byte, D.pt_ld_byte, D.pages_byte, &D.pool_next[0], b, t, min(t + n - 1, D.S - 1), D.err);
+    map_pages(D.pt_byte, D.pt_ld_byte, D.pages_byte, &D.pool_next[0], b, t, min(t + n - 1, D.S - 1), D.err,
+              &s_pg[0], &s_pg[1]);
   }
   __syncthreads();
   if (tid < n) {
@@ -402,7 +422,7 @@ __global__ void k_verify_plan(Dev D) {
     D.r_v.b[r] = b;
     D.r_v.pos[r] = p;
     D.r_v.slot[r] = p;
-    D.r_v.page[r] = page_of(D.pt_byte, D.pt_ld_byte, b, p);
+    D.r_v.page[r] = p / kPage == t / kPage ? s_pg[0] : s_pg[1];
     D.r_v.kvlen[r] = p + 1;
   }
   if (tid == 0) {
@@ -549,11 +569,12 @@ __global__ void k_segment(Dev D, cudaGraphConditionalHandle hcond, int use_handl
     }
     if (tid == 0) {
       D.gstart[(size_t)b * D.L + k] = seg1;
-      map_pages(D.pt_lm, D.pt_ld_lm, D.pages_lm, &D.pool_next[1], b, k, k, D.err);
+      int pg, pg1;
+      map_pages(D.pt_lm, D.pt_ld_lm, D.pages_lm, &D.pool_next[1], b, k, k, D.err, &pg, &pg1);
       D.r_lm.b[row] = b;
       D.r_lm.pos[row] = k;
       D.r_lm.slot[row] = k;
-      D.r_lm.page[row] = page_of(D.pt_lm, D.pt_ld_lm, b, k);
+      D.r_lm.page[row] = pg;
       D.r_lm.kvlen[row] = k + 1;
     }
   }

@@ -381,8 +381,8 @@ bool link_split(const Dev& D, bool tiled, LinearArgs& prod, LinearArgs& cons, in
 // output go through k_split_rows.
 void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& rows, int M_cap,
                int M_typ, int qt_grid, int splits, cudaStream_t s, const void* next_w = nullptr,
-               size_t next_bytes = 0, const int* stable = nullptr, int stable_extra = 0,
-               bool short_kv = false, int stable_add = 0, const StackLayer* stk = nullptr) {
+               size_t next_bytes = 0, const int* stable = nullptr, bool short_kv = false, int stable_add = 0,
+               const StackLayer* stk = nullptr) {
   Dev& D = c->L.D;
   const bool tiled = tiled_for(D, M_typ);
   // decode steps with few rows: the whole stack as one persistent launch
@@ -499,7 +499,7 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
 
     // RMSNorm -> Q,K,V -> RoPE -> K,V appended to the cache
     linear(D, aq, tiled, s);
-    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, stable_extra, short_kv, stable_add,
+    attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, short_kv, stable_add,
               std::max(1, M_cap / std::max(1, D.B)));
     linear(D, ao, tiled, s);
     linear(D, a13, tiled, s);
@@ -558,7 +558,7 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
       const int typ = B * (2 * n - 2);  // typical window rows: new committed bytes + copies
       // the window holds about two words of keys: a short cache
       run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2, kMbWindowKeys), s,
-                c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype), nullptr, 0,
+                c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype), nullptr,
                 true, 0, D.stk_mb);
     } else {
       launch_mlp_plan(D, s);
@@ -571,7 +571,7 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
   launch_verify_plan(D, s);
   run_stack(c, c->L.enc, D.x_enc, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1, c->kv_bytes_typ + n), s,
             c->L.nb.empty() ? nullptr : c->L.nb[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype),
-            &D.seq[0].t, n, false, 0, D.stk_enc);
+            &D.seq[0].t, false, 0, D.stk_enc);
 }
 
 void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
@@ -579,7 +579,7 @@ void enqueue_lm(lca_ctx* c, int n, cudaStream_t s) {
   // about one new latent per sequence every few bytes
   // latent slots [0, K] (BOS and the committed latents) do not change during the step
   run_stack(c, c->L.lm, D.x_lm, D.r_lm, D.B * n, D.B, 1, attn_splits(D, D.B, 1, c->kv_lat_typ + 1), s,
-            nullptr, 0, &D.seq[0].K, 1, false, 1, D.stk_lm);
+            nullptr, 0, &D.seq[0].K, false, 1, D.stk_lm);
   launch_lm_scatter(D, s);
 }
 
@@ -589,7 +589,7 @@ void enqueue_verify_commit(lca_ctx* c, int n, cudaStream_t s) {
   // (4) upsample + next-byte decoder over the n candidates, head
   launch_nb_input(D, s);
   run_stack(c, c->L.nb, D.x_nb, D.r_v, B * n, B * n, 1, attn_splits(D, B, 1, c->kv_bytes_typ + n), s, nullptr, 0,
-            &D.seq[0].t, n, false, 0, D.stk_nb);
+            &D.seq[0].t, false, 0, D.stk_nb);
   launch_head(D, D.x_nb, nullptr, D.r_v.M, B * n, D.nb_norm, D.nb_logits, D.nb_arg, D.nb_prob, s);
   // (5) accept + commit
   launch_commit(D, s);
@@ -972,6 +972,10 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.attn_pipe = ap ? atoi(ap) : 2;
     const char* an = getenv("LCA_ATTN_NS");
     D.attn_ns = an ? atoi(an) : 8;
+    const char* ant = getenv("LCA_ATTN_NS_T");
+    D.attn_ns_t = ant ? atoi(ant) : 8;
+    const char* atm = getenv("LCA_ATTN_TC_MIN");
+    D.attn_tc_min = atm ? std::max(0, atoi(atm)) : 128;
     const char* sw = getenv("LCA_SPLIT_WRITE");
     D.split_write = (sw && sw[0] == '0') ? 0 : 1;
     const char* aw = getenv("LCA_ATTN_W");
