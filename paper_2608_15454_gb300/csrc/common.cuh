@@ -377,6 +377,7 @@ struct Dev {
   int attn_ns;         // ring stages of the tensor-core prefill attention (4 or 8)
   int attn_ns_t;       // ring stages of the tensor-core decode attention (4, 8 or 12)
   int attn_tc_min;     // fewest (sequence, head) pairs for the tensor-core attention kernels
+  int gemv_ks_big, gemv_ks_small;  // K-split of the weight-streaming GEMV (K >= 2048, K < 2048)
   int attn_min_keys;   // fewest cache keys per key split of a decode attention launch
   int attn_t;          // decode steps use the transposed tensor-core attention (8-row query tiles)
   int attn_w;          // small-batch decode steps use the warp-walk attention

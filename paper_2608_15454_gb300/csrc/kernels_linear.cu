@@ -823,7 +823,7 @@ bool launch_gemv_tma(const Dev& D, const LinearArgs& a, int rows_typ, cudaStream
   if (a.N % 8 || a.Kd % 256) return false;
   int ksplit = 1;
   if (a.groups == 1 && a.N <= 2048) {
-    ksplit = a.Kd >= 2048 ? 8 : 4;
+    ksplit = a.Kd >= 2048 ? D.gemv_ks_big : D.gemv_ks_small;
     while (ksplit > 1 && ((a.Kd % ksplit) || ((a.Kd / ksplit) % 256))) ksplit >>= 1;
   }
   if (a.Kd / ksplit > 4096) return false;

@@ -976,6 +976,13 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.attn_ns_t = ant ? atoi(ant) : 8;
     const char* atm = getenv("LCA_ATTN_TC_MIN");
     D.attn_tc_min = atm ? std::max(0, atoi(atm)) : 128;
+    const char* kb = getenv("LCA_GEMV_KS_BIG");
+    const char* ks = getenv("LCA_GEMV_KS_SMALL");
+    auto pow2 = [](int v) { int p = 1; while (p * 2 <= v && p < kMaxKSplit) p *= 2; return p; };
+    // measured at batch 1 and 32 (paper-size layers): a cluster reduction costs more than the
+    // bandwidth of more CTAs buys for K = 1024 (Wo), and four ways are best for K = 4096 (W2)
+    D.gemv_ks_big = kb ? pow2(std::max(2, atoi(kb))) : 4;
+    D.gemv_ks_small = ks ? pow2(std::max(1, atoi(ks))) : 1;
     const char* sw = getenv("LCA_SPLIT_WRITE");
     D.split_write = (sw && sw[0] == '0') ? 0 : 1;
     const char* aw = getenv("LCA_ATTN_W");
