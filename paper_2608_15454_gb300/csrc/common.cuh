@@ -288,7 +288,8 @@ struct EpiArgs {
   // value v (after the residual add or the SwiGLU) is stored once more as bf16 halves of v * sg[c]
   // (sg: the consumer's RMSNorm gain, nullptr: 1) at sp_hi / sp_lo[row * ldsp + c], and, when ss is
   // set, the sum of v^2 over each 32-column block c / 32 at ss[row * ss_ld + c / 32] (the consumer's
-  // RMS). sp_only: the fp32 output is not written (the consumer is its only reader).
+  // RMS; a weight-streaming GEMV producer writes per 16-column block instead, for a GEMV
+  // consumer). sp_only: the fp32 output is not written (the consumer is its only reader).
   __nv_bfloat16* sp_hi;
   __nv_bfloat16* sp_lo;
   int ldsp;
@@ -424,6 +425,10 @@ struct Dev {
   __nv_bfloat16* as_lo[2];
   float* as_ss;
   int as_ss_ld;
+  // sums of squares per 16-column block of split rows written by GEMV epilogues, [as_rows][d / 16]
+  float* gv_ss;
+  int gv_ss_ld;
+  int gemv_split;  // GEMV layers take pre-split inputs from GEMV producers (1) or stage fp32 rows (0)
   int as_rows;
 
   // rows
@@ -565,7 +570,18 @@ struct LinearArgs {
   int abuf;      // split buffer (0 or 1) the tensor-core path reads
   int presplit;  // the producing layer's epilogue already wrote the split input and its sums of
                  // squares per 32-column block; otherwise k_split_rows runs first
+  // Weight-streaming GEMV only: the producing layer's epilogue wrote this layer's input as bf16
+  // halves of x * g (g: this layer's RMSNorm gain, or 1) into split buffer abuf, [rows][Kd], and,
+  // with a norm, the sums of x^2 per 16-column block into Dev::gv_ss; the rows are then staged by
+  // bulk copies. The launcher fills ghi, glo, gss, gss_ld from the workspace.
+  int gsplit;
+  const __nv_bfloat16* ghi;
+  const __nv_bfloat16* glo;
+  const float* gss;
+  int gss_ld;
 };
+// Whether a bf16 layer without tiling runs on the bulk-copy GEMV (k_gemv_bulk).
+bool gemv_bulk_ok(const Dev& D, const LinearArgs& a);
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s);
 bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s);
 // whether linear() runs this layer on the tensor cores when called with tiled = true
@@ -590,9 +606,13 @@ void kernel_attrs_attn();
 // stable + stable_add slots) does not change during a step: the warp-walk decode kernel stages it
 // in shared memory before the dependency wait; rows_seq: the most query rows a sequence has (a
 // tile-size hint).
+// osh/osl: also store the output as bf16 halves there (same [rows][H * hd] layout), the pre-split
+// input of a weight-streaming GEMV; only where attention_split_out holds for these arguments.
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s, const int* stable = nullptr,
-               bool short_kv = false, int stable_add = 0, int rows_seq = kAttnQT);
+               bool short_kv = false, int stable_add = 0, int rows_seq = kAttnQT, __nv_bfloat16* osh = nullptr,
+               __nv_bfloat16* osl = nullptr);
+bool attention_split_out(const Dev& D, const KV& kv, int B, int qtiles_grid, bool short_kv);
 
 // Step / prefill glue kernels (kernels_step.cu).
 void launch_mb_plan(const Dev& D, cudaStream_t s);

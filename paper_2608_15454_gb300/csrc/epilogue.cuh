@@ -225,6 +225,38 @@ static __device__ __forceinline__ void epi_store(const EpiArgs& e, const EpiPre&
 }
 
 
+// Split on write by the weight-streaming GEMV: the final values of the column pair (c, c + 1) of row
+// r (after the residual add, or the SwiGLU, which gives one value at column c / 2) as bf16 halves of
+// v * g (g0, g1: the consumer's RMSNorm gain at those columns, or 1) at sp_hi / sp_lo[r * ldsp + c];
+// returns the sum of the values' squares (before the gain).
+static __device__ __forceinline__ float epi_split_pair(const EpiArgs& e, const EpiPre& p, int r, int c, float a0,
+                                                       float a1, float g0, float g1) {
+  float v0 = a0, v1 = a1;
+  if (e.mode == EPI_RESID) {
+    v0 = p.r0 + a0;
+    v1 = p.r1 + a1;
+  } else if (e.mode == EPI_RESID_SILU) {
+    v0 = p.r0 + silu_f(a0);
+    v1 = p.r1 + silu_f(a1);
+  } else if (e.mode == EPI_SWIGLU) {
+    const float m = silu_f(a0) * a1;
+    const __nv_bfloat16 h = __float2bfloat16_rn(m * g0);
+    const __nv_bfloat16 l = __float2bfloat16_rn(m * g0 - __bfloat162float(h));
+    const size_t o = (size_t)r * e.ldsp + (c >> 1);
+    e.sp_hi[o] = h;
+    e.sp_lo[o] = l;
+    return m * m;
+  }
+  const float x0 = v0 * g0, x1 = v1 * g1;
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+  const float2 hf = __bfloat1622float2(h);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
+  const size_t o = (size_t)r * e.ldsp + c;
+  *reinterpret_cast<__nv_bfloat162*>(e.sp_hi + o) = h;
+  *reinterpret_cast<__nv_bfloat162*>(e.sp_lo + o) = l;
+  return v0 * v0 + v1 * v1;
+}
+
 template <typename TC>
 static __device__ __forceinline__ void epi_out(const EpiArgs& e, const EpiRow& q, float2 op, int r, int c,
                                                float a0, float a1) {

@@ -35,6 +35,17 @@ __device__ __forceinline__ void unpack16(const uint4& u, float* f, const __nv_bf
   f[6] = __uint_as_float(u.w << 16); f[7] = __uint_as_float(u.w & 0xFFFF0000u);
 }
 
+// An attention output value v at element o of [rows][H * HD]; with osh set, also as bf16 halves
+// (v = hi + lo) at the same place of osh / osl, the staged input of a weight-streaming GEMV.
+__device__ __forceinline__ void out_store(float* out, __nv_bfloat16* osh, __nv_bfloat16* osl, size_t o, float v) {
+  out[o] = v;
+  if (osh) {
+    const __nv_bfloat16 hv = __float2bfloat16_rn(v);
+    osh[o] = hv;
+    osl[o] = __float2bfloat16_rn(v - __bfloat162float(hv));
+  }
+}
+
 template <typename TC, int HD>
 __global__ void __launch_bounds__(kThreads)
 k_attn(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
@@ -551,7 +562,7 @@ __device__ __forceinline__ void a3_v2(const __nv_bfloat16* p, float& a, float& b
 template <typename TC, int HD>
 __global__ void __launch_bounds__(kA3Threads, 3)
 k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale,
-        int* err) {
+        int* err, __nv_bfloat16* osh, __nv_bfloat16* osl) {
   namespace cgr = cooperative_groups;
   constexpr int QT = kAttnQT;                     // query rows per tile (8)
   constexpr int KC = kA3Keys;
@@ -780,7 +791,7 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
             o += w * ar[k];
           }
         }
-        out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? o / L : 0.f;
+        out_store(out, osh, osl, (size_t)(r0 + i) * ld + h * HD + dd, L > 0.f ? o / L : 0.f);
       }
     }
     cl.sync();  // peers are done reading this tile's partials
@@ -806,7 +817,7 @@ size_t attn3_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
 
 template <typename TC, int HD>
 void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-               int qtiles_grid, int splits, int* err, cudaStream_t s) {
+               int qtiles_grid, int splits, int* err, __nv_bfloat16* osh, __nv_bfloat16* osl, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
   cfg.blockDim = dim3(kA3Threads);
@@ -822,7 +833,7 @@ void launch_a3(const float* q, float* out, const KV& kv, const Rows& rows, int B
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn3<TC, HD>, q, out, kv, rows, H, scale, err);
+  cudaLaunchKernelEx(&cfg, k_attn3<TC, HD>, q, out, kv, rows, H, scale, err, osh, osl);
 }
 
 // ---------------------------------------------------------------- warp-walk decode attention
@@ -859,7 +870,8 @@ __device__ __forceinline__ void aw_share(int base, int n, int splits, int sp, in
 template <int QT>
 __global__ void __launch_bounds__(kAwThreads, QT <= 4 ? 3 : 2)
 k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
-         const int* __restrict__ stable, int stable_stride, int stable_add, int stage_cap) {
+         const int* __restrict__ stable, int stable_stride, int stable_add, int stage_cap, __nv_bfloat16* osh,
+         __nv_bfloat16* osl) {
   namespace cgr = cooperative_groups;
   constexpr int HD = 64;
   __shared__ float Ow[kAwWarps][QT][HD];
@@ -1155,7 +1167,7 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
               ov += w * rbuf[((size_t)k * QT + i) * HD + dd];
             }
           }
-          out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? ov / L : 0.f;
+          out_store(out, osh, osl, (size_t)(r0 + i) * ld + h * HD + dd, L > 0.f ? ov / L : 0.f);
         }
       }
       continue;
@@ -1190,7 +1202,7 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
             ov += w * ar[k];
           }
         }
-        out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? ov / L : 0.f;
+        out_store(out, osh, osl, (size_t)(r0 + i) * ld + h * HD + dd, L > 0.f ? ov / L : 0.f);
       }
     }
     cl.sync();  // peers are done reading this tile's partials
@@ -1210,7 +1222,8 @@ int aw_stage_cap(int S, int splits, bool stable) {
 }
 
 void launch_aw(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale, int splits,
-               int* err, const int* stable, int stable_stride, int stable_add, int rows_seq, cudaStream_t s) {
+               int* err, const int* stable, int stable_stride, int stable_add, int rows_seq, __nv_bfloat16* osh,
+               __nv_bfloat16* osl, cudaStream_t s) {
   const int cap = aw_stage_cap(kv.S, splits, stable != nullptr);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, 1, H * splits);
@@ -1231,10 +1244,11 @@ void launch_aw(const float* q, float* out, const KV& kv, const Rows& rows, int B
   ++g_launches;
   // query tiles of 4 rows when a sequence has at most 4 (fewer registers: three CTAs per SM)
   if (qt == 4)
-    cudaLaunchKernelEx(&cfg, k_attn_w<4>, q, out, kv, rows, H, scale, err, stable, stable_stride, stable_add, cap);
+    cudaLaunchKernelEx(&cfg, k_attn_w<4>, q, out, kv, rows, H, scale, err, stable, stable_stride, stable_add, cap, osh,
+                       osl);
   else
     cudaLaunchKernelEx(&cfg, k_attn_w<kAttnQT>, q, out, kv, rows, H, scale, err, stable, stable_stride, stable_add,
-                       cap);
+                       cap, osh, osl);
 }
 
 // ---------------------------------------------------------------- tensor-core decode attention
@@ -1660,7 +1674,8 @@ __device__ __forceinline__ uint32_t movt(uint32_t x) {
 template <int NS>
 __global__ void __launch_bounds__(kA4Threads, 1)
 k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
-           const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
+           const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, __nv_bfloat16* osh,
+           __nv_bfloat16* osl) {
   namespace cgr = cooperative_groups;
   constexpr int HD = 64, QT = kA5QT, KC = kA4Keys;
   static_assert(NS % kA4Warps == 0, "ring stages must be a multiple of the compute warps");
@@ -1943,7 +1958,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
             ov += w * ar[k];
           }
         }
-        out[(size_t)(r0 + i) * ld + h * HD + dd] = L > 0.f ? ov / L : 0.f;
+        out_store(out, osh, osl, (size_t)(r0 + i) * ld + h * HD + dd, L > 0.f ? ov / L : 0.f);
       }
     }
     cl.sync();
@@ -1968,7 +1983,7 @@ size_t attn_mmt_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
 
 template <int NS>
 void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
-                  int qtiles_grid, int splits, int* err, cudaStream_t s) {
+                  int qtiles_grid, int splits, int* err, __nv_bfloat16* osh, __nv_bfloat16* osl, cudaStream_t s) {
   CUtensorMap tk, tv;
   memcpy(&tk, kv.tmaps, sizeof(tk));
   memcpy(&tv, static_cast<const unsigned char*>(kv.tmaps) + 128, sizeof(tv));
@@ -1987,7 +2002,7 @@ void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, in
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn_mmt<NS>, q, out, kv, rows, H, scale, err, tk, tv);
+  cudaLaunchKernelEx(&cfg, k_attn_mmt<NS>, q, out, kv, rows, H, scale, err, tk, tv, osh, osl);
 }
 
 void launch_a4(int ns, const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
@@ -2187,23 +2202,37 @@ void kernel_attrs_attn() {
                        (int)attn3_smem<float, 32>());
 }
 
+// The attention kernel family a launch of these arguments uses: tensor cores (prefill or decode).
+static bool attn_tensor_cores(const Dev& D, const KV& kv, int B, bool short_kv) {
+  return D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= D.attn_tc_min && !short_kv;
+}
+
+bool attention_split_out(const Dev& D, const KV& kv, int B, int qtiles_grid, bool short_kv) {
+  if (attn_tensor_cores(D, kv, B, short_kv)) return qtiles_grid == 1 && D.attn_t;
+  return D.attn_pipe != 0;
+}
+
 void attention(const Dev& D, const float* q, float* out, const KV& kv, const Rows& rows, int B,
                int qtiles_grid, int splits, cudaStream_t s, const int* stable, bool short_kv, int stable_add,
-               int rows_seq) {
+               int rows_seq, __nv_bfloat16* osh, __nv_bfloat16* osl) {
   ProfScope ps(PK_ATTN, 0.0, s);
   if (splits < 1) splits = 1;
+  if (osh && !attention_split_out(D, kv, B, qtiles_grid, short_kv)) {
+    fprintf(stderr, "lca: split attention output requested from a kernel without it\n");
+    osh = osl = nullptr;
+  }
   const int ss = (int)(sizeof(SeqState) / sizeof(int));
   // the tensor-core kernel holds two CTAs per SM: it pays off with many (sequence, head) pairs over
   // long caches; with few pairs, or short caches (the multi-byte window), the CUDA-core pipelined
   // kernel (three CTAs per SM) runs, spreading keys over up to 16 splits
-  if (D.attn_pipe == 2 && D.dtype == LCA_BF16 && D.hd == 64 && kv.tmaps && B * D.H >= D.attn_tc_min && !short_kv) {
+  if (attn_tensor_cores(D, kv, B, short_kv)) {
     const int sc = std::min(splits, kMaxClusterSplit);
     // decode steps (one query tile of a few rows per sequence): the transposed kernel
     if (qtiles_grid == 1 && D.attn_t) {
-      if (D.attn_ns_t == 4) launch_a5_ns<4>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, s);
+      if (D.attn_ns_t == 4) launch_a5_ns<4>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, osh, osl, s);
       else if (D.attn_ns_t == 12)
-        launch_a5_ns<12>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, s);
-      else launch_a5_ns<8>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, s);
+        launch_a5_ns<12>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, osh, osl, s);
+      else launch_a5_ns<8>(q, out, kv, rows, B, D.H, D.scale, 1, sc, D.err, osh, osl, s);
     } else {
       launch_a4(D.attn_ns, q, out, kv, rows, B, D.H, D.scale, qtiles_grid, sc, D.err, s);
     }
@@ -2213,15 +2242,17 @@ void attention(const Dev& D, const float* q, float* out, const KV& kv, const Row
     splits = std::min(splits, kA4MaxSplit);
     // decode steps (one query tile per sequence) of bf16 head-dim-64 caches: the warp-walk kernel
     if (qtiles_grid == 1 && D.attn_w && D.dtype == LCA_BF16 && D.hd == 64 && kv.pt) {
-      launch_aw(q, out, kv, rows, B, D.H, D.scale, splits, D.err, stable, ss, stable_add, rows_seq, s);
+      launch_aw(q, out, kv, rows, B, D.H, D.scale, splits, D.err, stable, ss, stable_add, rows_seq, osh, osl, s);
       return;
     }
     if (D.dtype == LCA_BF16) {
-      if (D.hd == 64) launch_a3<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
-      else launch_a3<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+      if (D.hd == 64)
+        launch_a3<__nv_bfloat16, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, osh, osl, s);
+      else
+        launch_a3<__nv_bfloat16, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, osh, osl, s);
     } else {
-      if (D.hd == 64) launch_a3<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
-      else launch_a3<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, s);
+      if (D.hd == 64) launch_a3<float, 64>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, osh, osl, s);
+      else launch_a3<float, 32>(q, out, kv, rows, B, D.H, D.scale, qtiles_grid, splits, D.err, osh, osl, s);
     }
     return;
   }

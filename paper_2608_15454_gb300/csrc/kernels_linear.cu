@@ -355,7 +355,10 @@ __device__ __forceinline__ void prefetch_next(const LinearArgs& a) {
 // partials through distributed shared memory in rank order (no global scratch).
 // (512 threads per SM by registers, four CTAs of four warps, so that a 512-tile launch is resident
 // in one wave)
-template <int MCA, int NW, bool NORM>
+// GS: the rows come pre-split from the producing layer (LinearArgs::gsplit); SP: this layer's
+// epilogue also writes its output split for the next layer (EpiArgs::sp_hi). Both are template
+// flags so that a launch carries only the code of its own staging and epilogue.
+template <int MCA, int NW, bool NORM, bool GS, bool SP>
 __global__ void __launch_bounds__(NW * 32, 16 / NW)
 k_gemv_bulk(LinearArgs a, int ksplit) {
   TraceScope _trace(TT_GEMV);
@@ -372,12 +375,15 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   float* red = reinterpret_cast<float*>(xl + (size_t)MCA * KP);          // [NW][CT][8] warp partials
   float* wss = red + NW * CT * 8;                                        // [NW][MCA] warp sums of squares
   float* rs = wss + NW * MCA;                                            // [MCA] this CTA's sums of squares
+  float* tq = rs + MCA;                 // [MCA][CT / 2] split on write: squares per column pair
+  float* sgs = tq + MCA * CT / 2;       // [CT] split on write: the consumer's RMSNorm gain
   float* cpart = reinterpret_cast<float*>(                                // [MCA][CT], 16-byte aligned
-      (reinterpret_cast<uintptr_t>(rs + MCA) + 15) & ~uintptr_t(15));
+      (reinterpret_cast<uintptr_t>(sgs + CT) + 15) & ~uintptr_t(15));
   uint64_t* bar = reinterpret_cast<uint64_t*>(
       (reinterpret_cast<uintptr_t>(cpart + MCA * CT) + 15) & ~uintptr_t(15));
   uint64_t* rbar = bar + 1;                                              // reduction arrivals (rank 0)
-  float* rbuf = reinterpret_cast<float*>(bar + 2);                       // [kMaxKSplit][MCA][CT] (rank 0)
+  uint64_t* xbar = bar + 2;                                              // pre-split rows landed
+  float* rbuf = reinterpret_cast<float*>(bar + 3);                       // [kMaxKSplit][MCA][CT] (rank 0)
   float* rsq = rbuf + kMaxKSplit * MCA * CT;                             // [kMaxKSplit][MCA] (rank 0)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -390,15 +396,18 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
                            (size_t)tile * CT * a.Kd + k0;
   if (tid == 0) {
     mbar_init(bar, 1);
+    mbar_init(xbar, 1);
     fence_mbar_init();
     mbar_expect_tx(bar, (uint32_t)(ncols * Kr * 2));
     for (int c = 0; c < ncols; ++c) bulk_g2s(wt + (size_t)c * KP, W + (size_t)c * a.Kd, (uint32_t)(Kr * 2), bar);
   }
-  if (NORM) {
+  if (NORM && !GS) {
     // the RMSNorm gain of the K-range (a weight: read before the dependency wait)
     for (int i = tid; i < Kr / 4; i += NT)
       reinterpret_cast<float4*>(gs)[i] = __ldg(reinterpret_cast<const float4*>(a.norm + k0) + i);
   }
+  // split on write: the next layer's RMSNorm gain at this tile's columns (a weight)
+  if (SP && tid < CT) sgs[tid] = (a.epi.sg && tile * CT + tid < a.N) ? __ldg(a.epi.sg + tile * CT + tid) : 1.f;
   prefetch_next(a);
   if (ksplit > 1) {
     // rank 0's reduction barrier exists before any peer can arrive on it (before the dependency
@@ -416,6 +425,20 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   _trace.waited();
 
   const int rbase = grp * a.Mg_stride;
+  // pre-split rows, bf16 halves [rows][Kd]: one bulk copy per row and half into the staging rows;
+  // the first chunk's copies go out before the row count is read (rows up to M_cap exist)
+  auto gsplit_issue = [&](int r0, int nr) {
+    mbar_expect_tx(xbar, (uint32_t)(nr * Kr * 4));
+    for (int i = 0; i < nr; ++i) {
+      const size_t o = (size_t)(rbase + r0 + i) * a.Kd + k0;
+      bulk_g2s(xh + (size_t)i * KP, a.ghi + o, (uint32_t)(Kr * 2), xbar);
+      bulk_g2s(xl + (size_t)i * KP, a.glo + o, (uint32_t)(Kr * 2), xbar);
+    }
+  };
+  const int nr0 = min(MCA, a.M_cap);
+  if (GS && tid == 0 && nr0 > 0) gsplit_issue(0, nr0);
+  uint32_t xphase = 0;      // chunks whose pre-split copies were waited for
+  bool x_pending = GS && nr0 > 0;
   int M = *a.M;
   M = M < a.M_cap ? M : a.M_cap;
   if (M < 0) M = 0;
@@ -430,6 +453,34 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
     const bool epi_lane = ksplit == 1 && col0 < ncols && ei < mc && (ec & 1) == 0;
     if (epi_lane) pre = epi_load_early(a.epi, rbase + r0 + ei, tile * CT + col0 + ec);
     __syncthreads();
+    if (tid < MCA * CT / 2) tq[tid] = 0.f;
+    if constexpr (GS) {
+      // rows split by the producing layer's epilogue: bulk copies (the first chunk's are in flight)
+      if (r0 > 0 && tid == 0) gsplit_issue(r0, mc);
+      const int nr = r0 == 0 ? nr0 : mc;
+      if (NORM) {
+        // each row's sum of squares from the producer's 16-column partial sums (warp i % NW);
+        // the cluster's rank 0 alone contributes it to the K-split sum
+        const int nb = a.Kd / 16;
+        for (int i = 0; i < MCA; ++i) {
+          float t = 0.f;
+          if (i % NW == warp) {
+            if (i < nr)
+              for (int j = lane; j < nb; j += 32) t += __ldcg(a.gss + (size_t)(rbase + r0 + i) * a.gss_ld + j);
+#pragma unroll
+            for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+          }
+          if (lane == 0) wss[warp * MCA + i] = (i % NW == warp && split == 0) ? t : 0.f;
+        }
+      }
+      // the bounded wait for the rows; on a timeout the error is recorded and the copies get one
+      // more bounded wait
+      const bool late = !mbar_wait(xbar, xphase & 1);
+      if (late) mbar_wait(xbar, xphase & 1);
+      if (late && tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
+      ++xphase;
+      x_pending = false;
+    } else {
     // raw rows -> registers (loads batched), then x * g -> shared memory with sums of squares
     constexpr int UNR = 8;
     const int nv = MCA * Kr / 4;
@@ -471,8 +522,6 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
         }
       }
     }
-    if (r0 == 0) _trace.mark(0);  // first row chunk loaded and staged
-    if (epi_lane) epi_load_late(a.epi, pre, tile * CT + col0 + ec);  // overlaps the dot products
     if (NORM) {
       // per-warp partial sums of squares over this CTA's K range (no atomics: summed in warp order)
 #pragma unroll
@@ -483,6 +532,9 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
         if (lane == 0) wss[warp * MCA + i] = t;
       }
     }
+    }
+    if (r0 == 0) _trace.mark(0);  // first row chunk loaded and staged
+    if (epi_lane) epi_load_late(a.epi, pre, tile * CT + col0 + ec);  // overlaps the dot products
     if (!have_w) {
       // the bounded wait for the weight tile; on a timeout the error is recorded, the copies in
       // flight get one more bounded wait, and the kernel runs on (no early exit, so cluster
@@ -555,11 +607,31 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
           v *= rsqrtf(t / (float)a.Kd + a.eps);
         }
         const float vn = __shfl_down_sync(0xffffffffu, v, 1);
-        if (epi_lane) epi_store<__nv_bfloat16>(a.epi, pre, rbase + r0 + ei, tile * CT + col0 + ec, v, vn);
+        if (epi_lane) {
+          const int cl = col0 + ec;
+          if (!SP || !a.epi.sp_only) epi_store<__nv_bfloat16>(a.epi, pre, rbase + r0 + ei, tile * CT + cl, v, vn);
+          if constexpr (SP) {
+            tq[ei * (CT / 2) + (cl >> 1)] =
+                epi_split_pair(a.epi, pre, rbase + r0 + ei, tile * CT + cl, v, vn, sgs[cl], sgs[cl + 1]);
+          }
+        }
       } else if (ei < MCA) {
         cpart[ei * CT + col0 + ec] = v;
       }
     }
+    // split on write with a norm: this tile's sums of squares per 16-column block and row, added
+    // in column order (the same sums on every run)
+    auto write_tss = [&]() {
+      __syncthreads();
+      if (tid < mc * (CT / 16)) {
+        const int i = tid / (CT / 16), sl = tid - i * (CT / 16);
+        float t = 0.f;
+#pragma unroll
+        for (int p = 0; p < 8; ++p) t += tq[i * (CT / 2) + sl * 8 + p];
+        a.epi.ss[(size_t)(rbase + r0 + i) * a.epi.ss_ld + tile * (CT / 16) + sl] = t;
+      }
+    };
+    if (SP && ksplit == 1 && a.epi.ss) write_tss();
     if (ksplit > 1 && M <= MCA) {
       // a single row chunk: the peers push their partials into rank 0's shared memory and
       // arrive on its barrier (release, cluster scope), then leave; rank 0 waits, adds the ranks
@@ -617,8 +689,13 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
             t1 *= sc;
           }
           const EpiPre q = j < 2 ? pp[j] : epi_load(a.epi, rbase + r0 + i, tile * CT + c);
-          epi_store<__nv_bfloat16>(a.epi, q, rbase + r0 + i, tile * CT + c, t0, t1);
+          if (!SP || !a.epi.sp_only) epi_store<__nv_bfloat16>(a.epi, q, rbase + r0 + i, tile * CT + c, t0, t1);
+          if constexpr (SP) {
+            tq[i * (CT / 2) + (c >> 1)] =
+                epi_split_pair(a.epi, q, rbase + r0 + i, tile * CT + c, t0, t1, sgs[c], sgs[c + 1]);
+          }
         }
+        if (SP && a.epi.ss) write_tss();
       }
     } else if (ksplit > 1) {
       // cluster reduction of the K-split partials of this row chunk
@@ -656,8 +733,13 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
             t1 *= sc;
           }
           const EpiPre q = j < 2 ? pp[j] : epi_load(a.epi, rbase + r0 + i, tile * CT + c);
-          epi_store<__nv_bfloat16>(a.epi, q, rbase + r0 + i, tile * CT + c, t0, t1);
+          if (!SP || !a.epi.sp_only) epi_store<__nv_bfloat16>(a.epi, q, rbase + r0 + i, tile * CT + c, t0, t1);
+          if constexpr (SP) {
+            tq[i * (CT / 2) + (c >> 1)] =
+                epi_split_pair(a.epi, q, rbase + r0 + i, tile * CT + c, t0, t1, sgs[c], sgs[c + 1]);
+          }
         }
+        if (SP && a.epi.ss) write_tss();
       }
       cl.sync();
     }
@@ -665,6 +747,10 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   if (!have_w && !mbar_wait(bar, 0)) {  // no rows: still wait (bounded, twice) for the copy before leaving
     if (tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
     mbar_wait(bar, 0);
+  }
+  if (GS && x_pending && !mbar_wait(xbar, 0)) {  // no rows: the first chunk's row copies too
+    if (tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
+    mbar_wait(xbar, 0);
   }
 }
 
@@ -791,8 +877,15 @@ void gemv_bulk_go(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s)
   const int Kr = a.Kd / ksplit;
   const size_t KP = (size_t)Kr + 8;
   const size_t smem = (size_t)CT * KP * 2 + (size_t)Kr * 4 + 2 * (size_t)MCA * KP * 2 + (size_t)NW * CT * 8 * 4 +
-                      (NW * MCA + MCA + MCA * CT) * 4 + 16 + 16 + 16 +
+                      (NW * MCA + MCA + MCA * CT / 2 + CT + MCA * CT) * 4 + 16 + 16 + 24 +
                       (ksplit > 1 ? (size_t)kMaxKSplit * MCA * (CT + 1) * 4 : 0) + 64;  // rank 0's buffers
+  LinearArgs b = a;
+  if (b.gsplit) {
+    b.ghi = D.as_hi[b.abuf];
+    b.glo = D.as_lo[b.abuf];
+    b.gss = D.gv_ss;
+    b.gss_ld = D.gv_ss_ld;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((a.N + CT - 1) / CT, ksplit, a.groups);
   cfg.blockDim = dim3(NW * 32);
@@ -808,25 +901,43 @@ void gemv_bulk_go(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s)
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_gemv_bulk<MCA, NW, NORM>, a, ksplit);
+  const bool sp = b.epi.sp_hi != nullptr;
+  if (b.gsplit) {
+    if (sp) cudaLaunchKernelEx(&cfg, k_gemv_bulk<MCA, NW, NORM, true, true>, b, ksplit);
+    else cudaLaunchKernelEx(&cfg, k_gemv_bulk<MCA, NW, NORM, true, false>, b, ksplit);
+  } else {
+    if (sp) cudaLaunchKernelEx(&cfg, k_gemv_bulk<MCA, NW, NORM, false, true>, b, ksplit);
+    else cudaLaunchKernelEx(&cfg, k_gemv_bulk<MCA, NW, NORM, false, false>, b, ksplit);
+  }
 }
 
 template <int MCA, bool NORM>
 void gemv_bulk_width(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t s) {
   // wide layers with many rows: 32-column CTAs keep the grid within one wave
-  if (MCA >= 8 && ksplit == 1 && a.N >= 4096) gemv_bulk_go<MCA, 8, NORM>(D, a, ksplit, s);
-  else gemv_bulk_go<MCA, 4, NORM>(D, a, ksplit, s);
+  if constexpr (MCA >= 8) {
+    if (ksplit == 1 && a.N >= 4096) {
+      gemv_bulk_go<MCA, 8, NORM>(D, a, ksplit, s);
+      return;
+    }
+  }
+  gemv_bulk_go<MCA, 4, NORM>(D, a, ksplit, s);
 }
 
-template <bool NORM>
-bool launch_gemv_tma(const Dev& D, const LinearArgs& a, int rows_typ, cudaStream_t s) {
-  if (a.N % 8 || a.Kd % 256) return false;
+// K-split of the bulk-copy GEMV for this layer, or 0 when the layer does not fit it.
+int gemv_bulk_ksplit(const Dev& D, const LinearArgs& a) {
+  if (a.N % 8 || a.Kd % 256) return 0;
   int ksplit = 1;
   if (a.groups == 1 && a.N <= 2048) {
     ksplit = a.Kd >= 2048 ? D.gemv_ks_big : D.gemv_ks_small;
     while (ksplit > 1 && ((a.Kd % ksplit) || ((a.Kd / ksplit) % 256))) ksplit >>= 1;
   }
-  if (a.Kd / ksplit > 4096) return false;
+  return a.Kd / ksplit > 4096 ? 0 : ksplit;
+}
+
+template <bool NORM>
+bool launch_gemv_tma(const Dev& D, const LinearArgs& a, int rows_typ, cudaStream_t s) {
+  const int ksplit = gemv_bulk_ksplit(D, a);
+  if (!ksplit) return false;
   // activations staged per chunk of the typical row count (shared memory sets CTAs per SM)
   const int mt = rows_typ < a.M_cap ? rows_typ : a.M_cap;
   if (mt <= 1) gemv_bulk_width<1, NORM>(D, a, ksplit, s);
@@ -882,18 +993,25 @@ void attrs_one() {
 
 void kernel_attrs_linear() {
   const int mx = 200 * 1024;
+#define LCA_ATTR_BULK1(M, W, N, G, P)                                                                        \
+  cudaFuncSetAttribute(k_gemv_bulk<M, W, N, G, P>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);       \
+  cudaFuncSetAttribute(k_gemv_bulk<M, W, N, G, P>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 #define LCA_ATTR_BULK(M, W)                                                                                   \
-  cudaFuncSetAttribute(k_gemv_bulk<M, W, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);           \
-  cudaFuncSetAttribute(k_gemv_bulk<M, W, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);          \
-  cudaFuncSetAttribute(k_gemv_bulk<M, W, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);         \
-  cudaFuncSetAttribute(k_gemv_bulk<M, W, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  LCA_ATTR_BULK(1, 4) LCA_ATTR_BULK(2, 4) LCA_ATTR_BULK(4, 4) LCA_ATTR_BULK(8, 4)
-  LCA_ATTR_BULK(1, 8) LCA_ATTR_BULK(2, 8) LCA_ATTR_BULK(4, 8) LCA_ATTR_BULK(8, 8)
+  LCA_ATTR_BULK1(M, W, true, false, false) LCA_ATTR_BULK1(M, W, true, false, true)                          \
+  LCA_ATTR_BULK1(M, W, true, true, false) LCA_ATTR_BULK1(M, W, true, true, true)                            \
+  LCA_ATTR_BULK1(M, W, false, false, false) LCA_ATTR_BULK1(M, W, false, false, true)                        \
+  LCA_ATTR_BULK1(M, W, false, true, false) LCA_ATTR_BULK1(M, W, false, true, true)
+  LCA_ATTR_BULK(1, 4) LCA_ATTR_BULK(2, 4) LCA_ATTR_BULK(4, 4) LCA_ATTR_BULK(8, 4) LCA_ATTR_BULK(8, 8)
 #undef LCA_ATTR_BULK
+#undef LCA_ATTR_BULK1
   attrs_one<__nv_bfloat16, true>();
   attrs_one<__nv_bfloat16, false>();
   attrs_one<float, true>();
   attrs_one<float, false>();
+}
+
+bool gemv_bulk_ok(const Dev& D, const LinearArgs& a) {
+  return D.dtype == LCA_BF16 && D.use_tma && gemv_bulk_ksplit(D, a) > 0;
 }
 
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s) {
@@ -902,6 +1020,8 @@ void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s) {
   if (tiled && D.use_umma && linear_umma(D, a, s)) return;
   // a pre-split input exists only as bf16 halves: callers set presplit only where umma_ready holds
   if (a.presplit) fprintf(stderr, "lca: pre-split layer input on the CUDA-core path (N %d, K %d)\n", a.N, a.Kd);
+  if (a.gsplit && (tiled || !gemv_bulk_ok(D, a)))
+    fprintf(stderr, "lca: pre-split GEMV input off the bulk-copy GEMV (N %d, K %d)\n", a.N, a.Kd);
   if (D.dtype == LCA_BF16) {
     if (tiled) norm ? launch_gemm<__nv_bfloat16, true>(D, a, s) : launch_gemm<__nv_bfloat16, false>(D, a, s);
     else norm ? launch_gemv<__nv_bfloat16, true>(D, a, s) : launch_gemv<__nv_bfloat16, false>(D, a, s);

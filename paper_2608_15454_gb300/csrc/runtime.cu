@@ -132,6 +132,8 @@ void carve(const lca_config& c, char* base, Layout& L) {
   }
   D.as_ss_ld = (int)d / 32;
   D.as_ss = cv.take<float>((size_t)D.as_rows * D.as_ss_ld);
+  D.gv_ss_ld = (int)d / 16;
+  D.gv_ss = cv.take<float>((size_t)D.as_rows * D.gv_ss_ld);
 
   D.x_mb = cv.take<float>(R * d);
   D.x_enc = cv.take<float>(R * d);
@@ -375,6 +377,30 @@ bool link_split(const Dev& D, bool tiled, LinearArgs& prod, LinearArgs& cons, in
   return true;
 }
 
+// Split on write between two weight-streaming GEMV layers (few rows): the producer's epilogue also
+// stores its output as bf16 halves of v * gain (gain: the consumer's RMSNorm gain, or 1) into
+// split buffer `buf`, with the sums of v^2 per 16-column block when the consumer normalises, and
+// the consumer stages its rows by bulk copies instead of loading and splitting fp32 rows. Only
+// when both layers run on the bulk-copy GEMV; returns whether the link was made.
+bool link_split_gemv(const Dev& D, bool tiled, LinearArgs& prod, LinearArgs& cons, int buf, const float* gain,
+                     bool drop_fp32) {
+  const bool resid = prod.epi.mode == EPI_RESID, swiglu = prod.epi.mode == EPI_SWIGLU;
+  const bool ok = D.gemv_split && !tiled && D.as_rows > 0 && cons.M_cap <= D.as_rows && prod.groups == 1 &&
+                  cons.groups == 1 && !prod.epi.sp_hi && gemv_bulk_ok(D, prod) && gemv_bulk_ok(D, cons) &&
+                  ((resid && cons.Kd == prod.N) || (swiglu && !gain && cons.Kd == prod.N / 2));
+  if (!ok) return false;
+  cons.gsplit = 1;
+  cons.abuf = buf;
+  prod.epi.sp_hi = D.as_hi[buf];
+  prod.epi.sp_lo = D.as_lo[buf];
+  prod.epi.ldsp = cons.Kd;
+  prod.epi.sg = gain;
+  prod.epi.ss = gain ? D.gv_ss : nullptr;
+  prod.epi.ss_ld = D.gv_ss_ld;
+  prod.epi.sp_only = drop_fp32 ? 1 : 0;
+  return true;
+}
+
 // Run the pre-norm blocks of one module over rows [0, *rows.M) of x (in place). On the tensor
 // cores, each layer's input is split into bf16 halves by the layer before it (its epilogue writes
 // them into the other of the two split buffers); only a stack's first layer and the attention
@@ -496,11 +522,22 @@ void run_stack(lca_ctx* c, std::vector<Block>& blocks, float* x, const Rows& row
     link_split(D, tiled, ao, a13, 0, bk.mlp_norm, false);
     link_split(D, tiled, a13, a2, 1, nullptr, true);
     if (nx) link_split(D, tiled, a2, aq_next, 0, nx->attn_norm, false);
+    link_split_gemv(D, tiled, ao, a13, 0, bk.mlp_norm, false);
+    link_split_gemv(D, tiled, a13, a2, 1, nullptr, true);
+    if (nx) link_split_gemv(D, tiled, a2, aq_next, 0, nx->attn_norm, false);
+    // the attention output as Wo's pre-split input (split buffer 1: a2 of the block before has read it)
+    const bool att_split = D.gemv_split && !tiled && D.as_rows > 0 && M_cap <= D.as_rows && gemv_bulk_ok(D, ao) &&
+                           attention_split_out(D, bk.kv, D.B, qt_grid, short_kv);
+    if (att_split) {
+      ao.gsplit = 1;
+      ao.abuf = 1;
+    }
 
     // RMSNorm -> Q,K,V -> RoPE -> K,V appended to the cache
     linear(D, aq, tiled, s);
     attention(D, D.qbuf, D.att, bk.kv, rows, D.B, qt_grid, splits, s, stable, short_kv, stable_add,
-              std::max(1, M_cap / std::max(1, D.B)));
+              std::max(1, M_cap / std::max(1, D.B)), att_split ? D.as_hi[1] : nullptr,
+              att_split ? D.as_lo[1] : nullptr);
     linear(D, ao, tiled, s);
     linear(D, a13, tiled, s);
     linear(D, a2, tiled, s);
@@ -976,6 +1013,8 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     D.attn_ns_t = ant ? atoi(ant) : 8;
     const char* atm = getenv("LCA_ATTN_TC_MIN");
     D.attn_tc_min = atm ? std::max(0, atoi(atm)) : 128;
+    const char* gsw = getenv("LCA_GEMV_SPLIT");
+    D.gemv_split = (gsw && gsw[0] == '0') ? 0 : 1;
     const char* kb = getenv("LCA_GEMV_KS_BIG");
     const char* ks = getenv("LCA_GEMV_KS_SMALL");
     auto pow2 = [](int v) { int p = 1; while (p * 2 <= v && p < kMaxKSplit) p *= 2; return p; };
