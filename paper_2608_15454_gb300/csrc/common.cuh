@@ -580,8 +580,9 @@ struct LinearArgs {
   const float* gss;
   int gss_ld;
 };
-// Whether a bf16 layer without tiling runs on the bulk-copy GEMV (k_gemv_bulk).
+// Whether a bf16 layer without tiling runs on the bulk-copy GEMV (k_gemv_bulk), and its K-split.
 bool gemv_bulk_ok(const Dev& D, const LinearArgs& a);
+int gemv_bulk_ksplit(const Dev& D, const LinearArgs& a);
 void linear(const Dev& D, const LinearArgs& a, bool tiled, cudaStream_t s);
 bool linear_umma(const Dev& D, const LinearArgs& a, cudaStream_t s);
 // whether linear() runs this layer on the tensor cores when called with tiled = true

@@ -427,12 +427,16 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
   const int rbase = grp * a.Mg_stride;
   // pre-split rows, bf16 halves [rows][Kd]: one bulk copy per row and half into the staging rows;
   // the first chunk's copies go out before the row count is read (rows up to M_cap exist)
+  // with a norm, each row's 16-column partial sums of squares (Kd / 16 floats) come along into the
+  // gain's staging area, which a pre-split layer does not use (the producer applied the gain)
+  const int nb = a.Kd / 16;
   auto gsplit_issue = [&](int r0, int nr) {
-    mbar_expect_tx(xbar, (uint32_t)(nr * Kr * 4));
+    mbar_expect_tx(xbar, (uint32_t)(nr * Kr * 4 + (NORM ? nr * nb * 4 : 0)));
     for (int i = 0; i < nr; ++i) {
       const size_t o = (size_t)(rbase + r0 + i) * a.Kd + k0;
       bulk_g2s(xh + (size_t)i * KP, a.ghi + o, (uint32_t)(Kr * 2), xbar);
       bulk_g2s(xl + (size_t)i * KP, a.glo + o, (uint32_t)(Kr * 2), xbar);
+      if (NORM) bulk_g2s(gs + (size_t)i * nb, a.gss + (size_t)(rbase + r0 + i) * a.gss_ld, (uint32_t)(nb * 4), xbar);
     }
   };
   const int nr0 = min(MCA, a.M_cap);
@@ -458,21 +462,6 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       // rows split by the producing layer's epilogue: bulk copies (the first chunk's are in flight)
       if (r0 > 0 && tid == 0) gsplit_issue(r0, mc);
       const int nr = r0 == 0 ? nr0 : mc;
-      if (NORM) {
-        // each row's sum of squares from the producer's 16-column partial sums (warp i % NW);
-        // the cluster's rank 0 alone contributes it to the K-split sum
-        const int nb = a.Kd / 16;
-        for (int i = 0; i < MCA; ++i) {
-          float t = 0.f;
-          if (i % NW == warp) {
-            if (i < nr)
-              for (int j = lane; j < nb; j += 32) t += __ldcg(a.gss + (size_t)(rbase + r0 + i) * a.gss_ld + j);
-#pragma unroll
-            for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-          }
-          if (lane == 0) wss[warp * MCA + i] = (i % NW == warp && split == 0) ? t : 0.f;
-        }
-      }
       // the bounded wait for the rows; on a timeout the error is recorded and the copies get one
       // more bounded wait
       const bool late = !mbar_wait(xbar, xphase & 1);
@@ -480,6 +469,20 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       if (late && tid == 0) atomicOr(a.epi.err, kErrTimeout | kErrWaitGemv);
       ++xphase;
       x_pending = false;
+      if (NORM) {
+        // each row's sum of squares from the staged partial sums (warp i % NW); the cluster's rank 0
+        // alone contributes it to the K-split sum
+        for (int i = 0; i < MCA; ++i) {
+          float t = 0.f;
+          if (i % NW == warp) {
+            if (i < nr)
+              for (int j = lane; j < nb; j += 32) t += gs[(size_t)i * nb + j];
+#pragma unroll
+            for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+          }
+          if (lane == 0) wss[warp * MCA + i] = (i % NW == warp && split == 0) ? t : 0.f;
+        }
+      }
     } else {
     // raw rows -> registers (loads batched), then x * g -> shared memory with sums of squares
     constexpr int UNR = 8;
@@ -558,9 +561,13 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
       // tensor-core dot products: warp w takes K-steps w, w + NW, ...; C[column][row] partials
       constexpr int MT = CT / 16;
       const int g = lane >> 2, q4 = lane & 3;
-      float cacc[MT][4];
+      // the high and low halves' products accumulate separately (two independent MMA chains)
+      float cacc[MT][4], cacl[MT][4];
 #pragma unroll
-      for (int mt = 0; mt < MT; ++mt) cacc[mt][0] = cacc[mt][1] = cacc[mt][2] = cacc[mt][3] = 0.f;
+      for (int mt = 0; mt < MT; ++mt) {
+        cacc[mt][0] = cacc[mt][1] = cacc[mt][2] = cacc[mt][3] = 0.f;
+        cacl[mt][0] = cacl[mt][1] = cacl[mt][2] = cacl[mt][3] = 0.f;
+      }
       const bool brow = g < mc;
       for (int kb = warp * 16; kb < Kr; kb += NW * 16) {
         uint32_t bh0 = 0u, bh1 = 0u, bl0 = 0u, bl1 = 0u;
@@ -581,11 +588,13 @@ k_gemv_bulk(LinearArgs a, int ksplit) {
           af[2] = pa[4];
           af[3] = pa[4 * KP + 4];
           mma_bf16_16816(cacc[mt], af, bh0, bh1);
-          mma_bf16_16816(cacc[mt], af, bl0, bl1);
+          mma_bf16_16816(cacl[mt], af, bl0, bl1);
         }
       }
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) cacc[mt][e] += cacl[mt][e];
         const int f = mt * 16 + g;
         *reinterpret_cast<float2*>(red + ((size_t)(warp * CT + f) * 8 + 2 * q4)) = make_float2(cacc[mt][0], cacc[mt][1]);
         *reinterpret_cast<float2*>(red + ((size_t)(warp * CT + f + 8) * 8 + 2 * q4)) =
@@ -923,16 +932,6 @@ void gemv_bulk_width(const Dev& D, const LinearArgs& a, int ksplit, cudaStream_t
   gemv_bulk_go<MCA, 4, NORM>(D, a, ksplit, s);
 }
 
-// K-split of the bulk-copy GEMV for this layer, or 0 when the layer does not fit it.
-int gemv_bulk_ksplit(const Dev& D, const LinearArgs& a) {
-  if (a.N % 8 || a.Kd % 256) return 0;
-  int ksplit = 1;
-  if (a.groups == 1 && a.N <= 2048) {
-    ksplit = a.Kd >= 2048 ? D.gemv_ks_big : D.gemv_ks_small;
-    while (ksplit > 1 && ((a.Kd % ksplit) || ((a.Kd / ksplit) % 256))) ksplit >>= 1;
-  }
-  return a.Kd / ksplit > 4096 ? 0 : ksplit;
-}
 
 template <bool NORM>
 bool launch_gemv_tma(const Dev& D, const LinearArgs& a, int rows_typ, cudaStream_t s) {
@@ -1008,6 +1007,17 @@ void kernel_attrs_linear() {
   attrs_one<__nv_bfloat16, false>();
   attrs_one<float, true>();
   attrs_one<float, false>();
+}
+
+// K-split of the bulk-copy GEMV for this layer, or 0 when the layer does not fit it.
+int gemv_bulk_ksplit(const Dev& D, const LinearArgs& a) {
+  if (a.N % 8 || a.Kd % 256) return 0;
+  int ksplit = 1;
+  if (a.groups == 1 && a.N <= 2048) {
+    ksplit = a.Kd >= 2048 ? D.gemv_ks_big : D.gemv_ks_small;
+    while (ksplit > 1 && ((a.Kd % ksplit) || ((a.Kd / ksplit) % 256))) ksplit >>= 1;
+  }
+  return a.Kd / ksplit > 4096 ? 0 : ksplit;
 }
 
 bool gemv_bulk_ok(const Dev& D, const LinearArgs& a) {

@@ -387,7 +387,10 @@ bool link_split_gemv(const Dev& D, bool tiled, LinearArgs& prod, LinearArgs& con
   const bool resid = prod.epi.mode == EPI_RESID, swiglu = prod.epi.mode == EPI_SWIGLU;
   const bool ok = D.gemv_split && !tiled && D.as_rows > 0 && cons.M_cap <= D.as_rows && prod.groups == 1 &&
                   cons.groups == 1 && !prod.epi.sp_hi && gemv_bulk_ok(D, prod) && gemv_bulk_ok(D, cons) &&
-                  ((resid && cons.Kd == prod.N) || (swiglu && !gain && cons.Kd == prod.N / 2));
+                  ((resid && cons.Kd == prod.N) || (swiglu && !gain && cons.Kd == prod.N / 2)) &&
+                  // a normalising consumer stages the rows' partial squares (8 rows x Kd / 16) in the
+                  // gain's area of Kd / ksplit floats
+                  (!gain || gemv_bulk_ksplit(D, cons) <= 2);
   if (!ok) return false;
   cons.gsplit = 1;
   cons.abuf = buf;
