@@ -376,7 +376,7 @@ struct Dev {
   int attn_pipe;       // decode attention: 2 = tensor cores (bf16, head_dim 64), 1 = bulk-copy pipelined
                        // CUDA-core kernel, 0 = register-tiled kernel
   int attn_ns;         // ring stages of the tensor-core prefill attention (4 or 8)
-  int attn_ns_t;       // ring stages of the tensor-core decode attention (4, 8 or 12)
+  int attn_ns_t;       // ring stages of the tensor-core decode attention (4, 8 or 12; half as many compute warps)
   int attn_tc_min;     // fewest (sequence, head) pairs for the tensor-core attention kernels
   int gemv_ks_big, gemv_ks_small;  // K-split of the weight-streaming GEMV (K >= 2048, K < 2048)
   int attn_min_keys;   // fewest cache keys per key split of a decode attention launch

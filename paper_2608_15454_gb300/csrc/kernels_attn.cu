@@ -1671,14 +1671,14 @@ __device__ __forceinline__ uint32_t movt(uint32_t x) {
   return y;
 }
 
-template <int NS>
-__global__ void __launch_bounds__(kA4Threads, 1)
+template <int NS, int NWC>
+__global__ void __launch_bounds__((NWC + 1) * 32, 1)
 k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, int H, float scale, int* err,
            const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, __nv_bfloat16* osh,
            __nv_bfloat16* osl) {
   namespace cgr = cooperative_groups;
   constexpr int HD = 64, QT = kA5QT, KC = kA4Keys;
-  static_assert(NS % kA4Warps == 0, "ring stages must be a multiple of the compute warps");
+  static_assert(NS % NWC == 0, "ring stages must be a multiple of the compute warps");
   extern __shared__ __align__(1024) unsigned char a5raw[];
   unsigned char* ring =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(a5raw) + 1023) & ~uintptr_t(1023));
@@ -1693,8 +1693,8 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   int* s_pt = reinterpret_cast<int*>(empty + NS);                   // [pt_ld] page table row (paged)
   // after the key loop the ring holds the warps' partial results
   float* Ow = reinterpret_cast<float*>(ring);                       // [warps][QT][HD]
-  float* mw = Ow + kA4Warps * QT * HD;                              // [warps][QT]
-  float* lw = mw + kA4Warps * QT;                                   // [warps][QT]
+  float* mw = Ow + NWC * QT * HD;                              // [warps][QT]
+  float* lw = mw + NWC * QT;                                   // [warps][QT]
 
   TraceScope _trace(TT_ATTN);
   cgr::cluster_group cl = cgr::this_cluster();
@@ -1728,7 +1728,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   for (int qt = blockIdx.y; qt < ntiles; qt += gridDim.y) {
     const int r0 = rbeg + qt * QT;
     const int nq = min(QT, nrows - qt * QT);
-    for (int idx = tid; idx < QT * HD / 2; idx += kA4Threads) {
+    for (int idx = tid; idx < QT * HD / 2; idx += ((NWC + 1) * 32)) {
       const int i = idx / (HD / 2), dd = (idx - i * (HD / 2)) * 2;
       float2 v = make_float2(0.f, 0.f);
       if (i < nq) {
@@ -1750,7 +1750,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       }
       s_kv[tid] = kl;
     }
-    if (qt == (int)blockIdx.y) kv_pages_store(kv, b, s_pt, tid, kA4Threads, pt0);
+    if (qt == (int)blockIdx.y) kv_pages_store(kv, b, s_pt, tid, ((NWC + 1) * 32), pt0);
     __syncthreads();
     int kv_hi = 0;
 #pragma unroll
@@ -1766,7 +1766,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
     float o[4][4];
 #pragma unroll
     for (int n = 0; n < 4; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
-    if (warp == kA4Warps) {
+    if (warp == NWC) {
       // producer
       if (lane == 0) {
         for (int c = 0; c < nch; ++c) {
@@ -1807,7 +1807,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
         }
       }
       const int kla = min(s_kv[2 * t], hi), klb = min(s_kv[2 * t + 1], hi);
-      for (int c = warp; c < nch; c += kA4Warps) {
+      for (int c = warp; c < nch; c += NWC) {
         const uint32_t gi = cc + c;
         const int st = gi % NS;
         if (!failed && !a3_wait(&full[st], (gi / NS) & 1)) failed = true;
@@ -1892,7 +1892,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       }
     }
     __syncthreads();  // every warp is done with the ring: it now holds the warps' partial results
-    if (warp < kA4Warps) {
+    if (warp < NWC) {
       float* ow = Ow + warp * QT * HD;
 #pragma unroll
       for (int dm = 0; dm < 4; ++dm) {
@@ -1910,14 +1910,14 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
     }
     __syncthreads();
     // combine the warps: this split's (max, sum, accumulator) per row
-    for (int idx = tid; idx < QT * HD; idx += kA4Threads) {
+    for (int idx = tid; idx < QT * HD; idx += ((NWC + 1) * 32)) {
       const int i = idx / HD, dd = idx - i * HD;
       float M = -INFINITY;
 #pragma unroll
-      for (int w = 0; w < kA4Warps; ++w) M = fmaxf(M, mw[w * QT + i]);
+      for (int w = 0; w < NWC; ++w) M = fmaxf(M, mw[w * QT + i]);
       float L = 0.f, ov = 0.f;
 #pragma unroll
-      for (int w = 0; w < kA4Warps; ++w) {
+      for (int w = 0; w < NWC; ++w) {
         const float mv = mw[w * QT + i];
         const float f = mv == -INFINITY ? 0.f : expf(mv - M);
         L += f * lw[w * QT + i];
@@ -1934,7 +1934,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
       const int dpr = (HD + splits - 1) / splits;
       const int d0 = sp * dpr;
       const int nd = min(dpr, HD - d0);
-      for (int idx = tid; idx < nq * nd; idx += kA4Threads) {
+      for (int idx = tid; idx < nq * nd; idx += ((NWC + 1) * 32)) {
         const int i = idx / nd, dd = d0 + (idx - i * nd);
         float mr[kMaxClusterSplit], lr[kMaxClusterSplit], ar[kMaxClusterSplit];
 #pragma unroll
@@ -1966,7 +1966,7 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
   }
   // after a failed wait, copies may still be in flight: wait (bounded) for the last one issued
   // into each stage before the CTA's shared memory is released
-  if (__syncthreads_or(failed) && tid == kA4Warps * 32) {
+  if (__syncthreads_or(failed) && tid == NWC * 32) {
     for (uint32_t st = 0; st < (uint32_t)NS && st < issued; ++st) {
       const uint32_t last = issued - 1 - ((issued - 1 - st) % NS);
       a3_wait(&full[last % NS], (last / NS) & 1);
@@ -1980,6 +1980,10 @@ size_t attn_mmt_smem(size_t pt_bytes = (size_t)kMaxPtRow * 4) {
   // ring, q halves (2 x QT x 64 bf16), pacc (QT x 64 fp32), row stats, barriers, page table row
   return 1024 + (size_t)NS * 2 * kA4Chunk + (size_t)(2 * kA5QT * 64 + 3 * kA5QT) * 4 + 2 * NS * 8 + 16 + pt_bytes;
 }
+// Compute warps of k_attn_mmt with NS ring stages: two stages per warp (one being read, one in
+// flight).
+template <int NS>
+constexpr int mmt_warps() { return NS / 2 < 4 ? 4 : NS / 2; }
 
 template <int NS>
 void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
@@ -1989,7 +1993,8 @@ void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, in
   memcpy(&tv, static_cast<const unsigned char*>(kv.tmaps) + 128, sizeof(tv));
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(B, qtiles_grid, H * splits);
-  cfg.blockDim = dim3(kA4Threads);
+  constexpr int NWC = mmt_warps<NS>();
+  cfg.blockDim = dim3((NWC + 1) * 32);
   cfg.dynamicSmemBytes = attn_mmt_smem<NS>(kv_pages_smem(kv));
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
@@ -2002,7 +2007,7 @@ void launch_a5_ns(const float* q, float* out, const KV& kv, const Rows& rows, in
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   ++g_launches;
-  cudaLaunchKernelEx(&cfg, k_attn_mmt<NS>, q, out, kv, rows, H, scale, err, tk, tv, osh, osl);
+  cudaLaunchKernelEx(&cfg, k_attn_mmt<NS, NWC>, q, out, kv, rows, H, scale, err, tk, tv, osh, osl);
 }
 
 void launch_a4(int ns, const float* q, float* out, const KV& kv, const Rows& rows, int B, int H, float scale,
@@ -2179,9 +2184,12 @@ int make_kv_tmaps(void* out, const void* k, const void* v, long long rows) {
 void kernel_attrs_attn() {
   cudaFuncSetAttribute(k_attn_mma<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem<4>());
   cudaFuncSetAttribute(k_attn_mma<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mma_smem<8>());
-  cudaFuncSetAttribute(k_attn_mmt<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<4>());
-  cudaFuncSetAttribute(k_attn_mmt<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<8>());
-  cudaFuncSetAttribute(k_attn_mmt<12>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_mmt_smem<12>());
+  cudaFuncSetAttribute(k_attn_mmt<4, mmt_warps<4>()>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn_mmt_smem<4>());
+  cudaFuncSetAttribute(k_attn_mmt<8, mmt_warps<8>()>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn_mmt_smem<8>());
+  cudaFuncSetAttribute(k_attn_mmt<12, mmt_warps<12>()>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn_mmt_smem<12>());
   cudaFuncSetAttribute(k_attn3<__nv_bfloat16, 64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn_w<4>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaFuncSetAttribute(k_attn_w<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,

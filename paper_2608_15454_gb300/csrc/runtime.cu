@@ -1013,7 +1013,7 @@ int lca_create(const lca_config* cfg, const lca_tensor* weights, int n_weights, 
     const char* an = getenv("LCA_ATTN_NS");
     D.attn_ns = an ? atoi(an) : 8;
     const char* ant = getenv("LCA_ATTN_NS_T");
-    D.attn_ns_t = ant ? atoi(ant) : 8;
+    D.attn_ns_t = ant ? atoi(ant) : 12;  // 12 stages: six compute warps (measured at batch 8-128)
     const char* atm = getenv("LCA_ATTN_TC_MIN");
     D.attn_tc_min = atm ? std::max(0, atoi(atm)) : 128;
     const char* gsw = getenv("LCA_GEMV_SPLIT");
