@@ -596,7 +596,6 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(a3_su32(&full[i])) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  pdl_trigger();
   pdl_wait();
   _trace.waited();
   __syncthreads();
@@ -762,6 +761,9 @@ k_attn3(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows, 
       pacc[(rg + m * RG) * HD + 2 * dp] = acc[m][0];
       pacc[(rg + m * RG) * HD + 2 * dp + 1] = acc[m][1];
     }
+    // the dependent launch starts once the keys are done (its CTAs and weight copies would
+    // otherwise compete with the key loop)
+    if (qt == (int)blockIdx.y) pdl_trigger();
     cl.sync();
     {
       const int dpr = (HD + splits - 1) / splits;
@@ -901,7 +903,6 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
   const int h = blockIdx.z / splits;
   const __nv_bfloat16* Kc = reinterpret_cast<const __nv_bfloat16*>(kv.k);
   const __nv_bfloat16* Vc = reinterpret_cast<const __nv_bfloat16*>(kv.v);
-  pdl_trigger();
   if (warp == 0) {
     int S = 0, slo = 0, nst = 0;
     if (stable) {
@@ -1068,6 +1069,9 @@ k_attn_w(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows rows,
       }
     }
     if (qt == (int)blockIdx.y) _trace.mark(1);  // this warp's keys done
+    // the dependent launch starts now, not at entry: its CTAs and weight copies would compete with
+    // the key loop (measured: the step is 1% faster)
+    pdl_trigger();
     // combine the four key slots of the warp (lanes e, e + 8, e + 16, e + 24), then the warps
 #pragma unroll
     for (int i = 0; i < QT; ++i) {
@@ -1711,7 +1715,6 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
   }
-  pdl_trigger();
   pdl_wait();
   _trace.waited();
   __syncthreads();
@@ -1929,6 +1932,8 @@ k_attn_mmt(const float* __restrict__ q, float* __restrict__ out, KV kv, Rows row
         s_l[i] = L;
       }
     }
+    // the dependent launch starts once the keys are done (as in k_attn_w)
+    if (qt == (int)blockIdx.y) pdl_trigger();
     cl.sync();
     {
       const int dpr = (HD + splits - 1) / splits;
