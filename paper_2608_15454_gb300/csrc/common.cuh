@@ -244,33 +244,6 @@ __device__ __forceinline__ void kv_prefetch_l2(const KV& kv, const void* base, i
     }
   }
 }
-// The same hint for K and V by a whole warp: lane i takes pages i, i + 32, ... of the range, so
-// that the table lookups of up to 32 pages are in flight together.
-__device__ __forceinline__ void kv_prefetch_l2_warp(const KV& kv, int es, int H, int hd, int b, int h, int lo,
-                                                    int hi, int lane) {
-  if (!kv.pt) {
-    if (lane < 2) kv_prefetch_l2(kv, lane ? kv.v : kv.k, es, H, hd, b, h, lo, hi);
-    return;
-  }
-  for (int s0 = (lo & ~(kPage - 1)) + lane * kPage; s0 < hi; s0 += 32 * kPage) {
-    const int a = max(lo, s0), e = min(hi, s0 + kPage);
-    const int pg = kv_page_cg(kv, b, a);
-    const uint32_t bytes = (uint32_t)((e - a) * hd * es) & ~15u;
-    const size_t o = kv_addr(kv, H, hd, b, h, a, pg) * es;
-    if (bytes) {
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const char*>(kv.k) + o), "r"(bytes)
-                   : "memory");
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const char*>(kv.v) + o), "r"(bytes)
-                   : "memory");
-    }
-  }
-}
-// Slots [s, s + n) that stay inside one page (or all of them, contiguous).
-__device__ __forceinline__ int kv_run(const KV& kv, int s, int n) {
-  if (!kv.pt) return n;
-  const int room = kPage - (s & (kPage - 1));
-  return n < room ? n : room;
-}
 
 struct EpiArgs {
   int mode;

@@ -152,9 +152,6 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
                "l"(src), "r"(bytes), "r"(su32(bar))
                : "memory");
 }
-__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
 // order this thread's generic-proxy view before its later bulk copies (async proxy)
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 // barrier of the compute warps (named barrier 1; the copy warp does not take part)
@@ -306,17 +303,6 @@ struct PhaseIn {
   int ss_ld;
 };
 __device__ __forceinline__ int chunk_rows(int M, int chunk) { return min(kSkMC, M - chunk * kSkMC); }
-// first block after the group that starts at block k0
-__device__ __forceinline__ int group_end(int M, int nsl, int nblk, int k0) {
-  int rows = 0, k = k0;
-  while (k < nblk) {
-    const int mc = chunk_rows(M, k / nsl);
-    if (rows + mc > kSkMC) break;
-    rows += mc;
-    ++k;
-  }
-  return k;
-}
 
 // Thread 0: bulk copies of the blocks [k0, k1) into staging buffer b (rows packed from slot 0).
 __device__ void issue_group(const PhaseIn& in, int KS, int M, int nsl, int k0, int k1, int b, Smem& S,
