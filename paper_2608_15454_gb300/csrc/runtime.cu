@@ -595,7 +595,10 @@ void enqueue_draft_encode(lca_ctx* c, int n, cudaStream_t s) {
   if (n >= 2) {
     if (D.mb_kind == LCA_MB_LCA) {
       launch_mb_plan(D, s);
-      const int typ = B * (2 * n - 2);  // typical window rows: new committed bytes + copies
+      // typical window rows. A single sequence rebuilds its window after most committed boundaries:
+      // about a word of bytes, the n new bytes and the n - 2 copies. In a batch the sequences that
+      // only append their n new bytes and n - 2 copies set the count.
+      const int typ = B == 1 ? 2 * n + 6 : B * (2 * n - 2);
       // the window holds about two words of keys: a short cache
       run_stack(c, c->L.mb, D.x_mb, D.r_mb, D.R, typ, 2, attn_splits(D, B, 2, kMbWindowKeys), s,
                 c->L.enc.empty() ? nullptr : c->L.enc[0].wqkv, 3ull * D.d * D.d * tw_bytes(D.dtype), nullptr,
