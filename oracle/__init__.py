@@ -7,6 +7,7 @@ path, with which it shares no code.
 from .decode import (SPEC, THRESH, IncrementalDecoder, StepRecord, generate_incremental,
                      generate_reference, greedy_decode)
 from .model import Model, forward_full
+from .sampling import Sampling
 
 __all__ = ["SPEC", "THRESH", "IncrementalDecoder", "StepRecord", "generate_incremental",
-           "generate_reference", "greedy_decode", "Model", "forward_full"]
+           "generate_reference", "greedy_decode", "Model", "forward_full", "Sampling"]

@@ -17,6 +17,10 @@ Speculative-decoding acceptance (Section 6.2, acceptance method (ii)) is the gre
 d_i is kept while it equals the next-byte argmax at the position before it, so the
 output equals plain next-byte decoding. Meaning of n (a reading): one next-byte
 byte plus n-1 drafts per step, so 1..n bytes are emitted per step.
+
+With a ``Sampling`` (``oracle/sampling.py``) both decoders draw c_1 and the drafts instead of
+taking argmaxes, and speculative acceptance becomes the rejection rule of speculative sampling;
+the first byte of the step after a rejection is drawn from the residual distribution.
 """
 from __future__ import annotations
 
@@ -26,6 +30,8 @@ import numpy as np
 
 from .model import (Model, causal_mask, forward_full, greedy, max_prob, mb_draft_logits,
                     closed_segments, latent_index)
+from .sampling import (ACCEPT, DRAFT, NEXT, Sampling, draw, residual_dist, sample_index,
+                       sampling_dist, spec_keep)
 
 THRESH = 0
 SPEC = 1
@@ -63,6 +69,49 @@ def accept_count(mode, drafts, probs, nb_logits, tau, forced=None):
     return a
 
 
+def sampled_drafts(mbl, samp: Sampling, t, b):
+    """Drafts d_2..d_n drawn from the MB head's sampling distributions (stream DRAFT at t), with
+    the drafter's model probabilities softmax(l)[d] that threshold acceptance compares with tau."""
+    drafts, probs = [], []
+    for i, r in enumerate(mbl):
+        q = sampling_dist(r, samp.temperature, samp.top_p)
+        d = sample_index(q, draw(samp.seed, t, b, DRAFT, i))
+        drafts.append(d)
+        probs.append(max_prob(r, d))
+    return drafts, probs
+
+
+def sampled_accept(mode, drafts, probs, mbl, nbl, tau, samp: Sampling, t, b, forced=None):
+    """(a, rejected): accepted drafts, a prefix, and whether the step ended on a draft that
+    speculative acceptance rejected (threshold acceptance drops the rest without a correction)."""
+    if forced is not None:
+        return int(forced), False
+    a = 0
+    for i, d in enumerate(drafts):
+        if mode == THRESH:
+            ok = probs[i] >= tau
+        elif mode == SPEC:
+            P = sampling_dist(nbl[i], samp.temperature, samp.top_p)
+            Q = sampling_dist(mbl[i], samp.temperature, samp.top_p)
+            ok = spec_keep(P, Q, d, draw(samp.seed, t, b, ACCEPT, i))
+        else:
+            raise ValueError(mode)
+        if not ok:
+            return a, mode == SPEC
+        a += 1
+    return a, False
+
+
+def carried_dist(rejected, a, e, mbl, nbl, samp: Sampling):
+    """Distribution of the next step's c_1 when it is not the plain next-byte distribution of the
+    last committed row: the residual norm(max(0, P_a - Q_a)) after a rejection at row a that the
+    budget did not cut. None otherwise."""
+    if not rejected or e - 1 != a:
+        return None
+    return residual_dist(sampling_dist(nbl[a], samp.temperature, samp.top_p),
+                         sampling_dist(mbl[a], samp.temperature, samp.top_p))
+
+
 def _force(force, step):
     if force is None:
         return None
@@ -70,21 +119,29 @@ def _force(force, step):
 
 
 def generate_reference(model: Model, prompt, n, tau, mode, G, force=None, record_nb=False,
-                       force_cand=None):
+                       force_cand=None, samp: Sampling | None = None, b=0):
     """Algorithm 1 with a full recompute per step. Returns (generated bytes, [StepRecord]).
     force: accepted-draft counts per step (test hook); force_cand(step) -> n candidate bytes
-    that replace c_1, d_2..d_n (test hook for driving boundaries through a step)."""
+    that replace c_1, d_2..d_n (test hook for driving boundaries through a step).
+    samp: sample instead of taking argmaxes, with the draws of sequence index b."""
     x = bytearray(prompt)
     out = bytearray()
     recs = []
     step = 0
+    carried = None
     while len(out) < G:
         F = forward_full(model, x)
         t = len(x)
-        c1 = greedy(F.nb_logits[t - 1])
         mbl = mb_draft_logits(model, F.Kp, F.o, F.u, t, n, x, y_last=F.y[t - 1])
-        drafts = [greedy(r) for r in mbl]
-        probs = [max_prob(r, d) for r, d in zip(mbl, drafts)]
+        if samp is None:
+            c1 = greedy(F.nb_logits[t - 1])
+            drafts = [greedy(r) for r in mbl]
+            probs = [max_prob(r, d) for r, d in zip(mbl, drafts)]
+        else:
+            p1 = carried if carried is not None else sampling_dist(
+                F.nb_logits[t - 1], samp.temperature, samp.top_p)
+            c1 = sample_index(p1, draw(samp.seed, t, b, NEXT, 0))
+            drafts, probs = sampled_drafts(mbl, samp, t, b)
         cand = bytes([c1] + drafts)
         fc = force_cand(step) if force_cand is not None else None
         if fc is not None:
@@ -92,8 +149,14 @@ def generate_reference(model: Model, prompt, n, tau, mode, G, force=None, record
         nbl = None
         if mode == SPEC or record_nb:
             nbl = forward_full(model, bytes(x) + cand).nb_logits[t:t + n]
-        a = accept_count(mode, list(cand[1:]), probs, nbl, tau, _force(force, step))
+        if samp is None:
+            a = accept_count(mode, list(cand[1:]), probs, nbl, tau, _force(force, step))
+        else:
+            a, rejected = sampled_accept(mode, list(cand[1:]), probs, mbl, nbl, tau, samp, t, b,
+                                         _force(force, step))
         e = min(1 + a, G - len(out))
+        if samp is not None:
+            carried = carried_dist(rejected, a, e, mbl, nbl, samp)
         em = cand[:e]
         x += em
         out += em
@@ -131,6 +194,7 @@ class IncrementalDecoder:
         self.kv = {s: [[k, v] for k, v in F.caches[s]] for s in ("enc", "lm", "nb")}
         self.nb_last = F.nb_logits[-1]
         self.y_last = F.y[-1]
+        self.carried = None  # c_1 distribution carried from a rejection (sampled decoding)
         return F
 
     @property
@@ -160,16 +224,24 @@ class IncrementalDecoder:
         T = x.shape[0]
         return self.m.run_stack(prefix, x, pos, lambda n_prev: causal_mask(n_prev, T), caches)
 
-    def step(self, n, tau, mode, forced=None, budget=None, forced_cand=None):
+    def step(self, n, tau, mode, forced=None, budget=None, forced_cand=None,
+             samp: Sampling | None = None, b=0):
         """One decode step. forced: accepted-draft count (test hook); forced_cand: n bytes
-        replacing c_1, d_2..d_n (test hook); budget: cap on the committed bytes."""
+        replacing c_1, d_2..d_n (test hook); budget: cap on the committed bytes; samp: sample
+        with the draws of sequence index b instead of taking argmaxes."""
         m, cfg = self.m, self.cfg
         t, K = self.t, self.K
         # draft (Algorithm 1, drafting step)
-        c1 = greedy(self.nb_last)
         mbl = mb_draft_logits(m, self.Kp, self.o, self.u, t, n, self.x, y_last=self.y_last)
-        drafts = [greedy(r) for r in mbl]
-        probs = [max_prob(r, d) for r, d in zip(mbl, drafts)]
+        if samp is None:
+            c1 = greedy(self.nb_last)
+            drafts = [greedy(r) for r in mbl]
+            probs = [max_prob(r, d) for r, d in zip(mbl, drafts)]
+        else:
+            p1 = self.carried if self.carried is not None else sampling_dist(
+                self.nb_last, samp.temperature, samp.top_p)
+            c1 = sample_index(p1, draw(samp.seed, t, b, NEXT, 0))
+            drafts, probs = sampled_drafts(mbl, samp, t, b)
         cand = bytes([c1] + drafts) if forced_cand is None else bytes(forced_cand)
         pos = np.arange(t, t + n)
         # encoder over the n candidates, appended after the cached keys
@@ -195,8 +267,13 @@ class IncrementalDecoder:
         y_c, nb_new = self._stack_cached("nb", o_ext[Kc] + h_c, pos)
         nbl = m.head(y_c, "nb.norm")
         # accept (Algorithm 1, acceptance step) and commit the accepted prefix
-        a = accept_count(mode, list(cand[1:]), probs, nbl, tau, forced)
+        if samp is None:
+            a = accept_count(mode, list(cand[1:]), probs, nbl, tau, forced)
+        else:
+            a, rejected = sampled_accept(mode, list(cand[1:]), probs, mbl, nbl, tau, samp, t, b,
+                                         forced)
         e = 1 + a if budget is None else min(1 + a, budget)
+        self.carried = None if samp is None else carried_dist(rejected, a, e, mbl, nbl, samp)
         self.x += cand[:e]
         self.h_e = h_all[:t + e]
         self.Kp += Kc[:e]
@@ -217,7 +294,8 @@ class IncrementalDecoder:
         return StepRecord(c1, drafts, probs, a, cand[:e], mbl, nbl, t=self.t, K=K_new)
 
 
-def generate_incremental(model: Model, prompt, n, tau, mode, G, force=None, force_cand=None):
+def generate_incremental(model: Model, prompt, n, tau, mode, G, force=None, force_cand=None,
+                         samp: Sampling | None = None, b=0):
     """Cached decode loop with the same stopping rule as ``generate_reference``."""
     dec = IncrementalDecoder(model)
     dec.prefill(prompt)
@@ -226,7 +304,8 @@ def generate_incremental(model: Model, prompt, n, tau, mode, G, force=None, forc
     step = 0
     while len(out) < G:
         fc = force_cand(step) if force_cand is not None else None
-        r = dec.step(n, tau, mode, _force(force, step), budget=G - len(out), forced_cand=fc)
+        r = dec.step(n, tau, mode, _force(force, step), budget=G - len(out), forced_cand=fc,
+                     samp=samp, b=b)
         out += r.emitted
         recs.append(r)
         step += 1
