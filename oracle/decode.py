@@ -28,8 +28,8 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
-from .model import (Model, causal_mask, forward_full, greedy, max_prob, mb_draft_logits,
-                    closed_segments, latent_index)
+from .model import (Model, boundary_flags, causal_mask, forward_full, greedy, latent_index,
+                    max_prob, mb_draft_logits, segments_of)
 from .sampling import (ACCEPT, DRAFT, NEXT, Sampling, draw, residual_dist, sample_index,
                        sampling_dist, spec_keep)
 
@@ -160,11 +160,17 @@ def generate_reference(model: Model, prompt, n, tau, mode, G, force=None, record
         em = cand[:e]
         x += em
         out += em
-        rec = StepRecord(c1, drafts, probs, a, em, mbl, nbl, t=len(x),
-                         K=int(latent_index(model.cfg, x)[-1]))
+        rec = StepRecord(c1, drafts, probs, a, em, mbl, nbl, t=len(x), K=_latents(model, x))
         recs.append(rec)
         step += 1
     return bytes(out), recs
+
+
+def _latents(model: Model, x):
+    """K(t-1) of bytes x: the closed segments (a forward for the learned predictor)."""
+    if model.cfg.boundary == "learned":
+        return int(forward_full(model, x).Kp[-1])
+    return int(latent_index(model.cfg, x)[-1])
 
 
 def greedy_decode(model: Model, prompt, G):
@@ -187,6 +193,7 @@ class IncrementalDecoder:
     def prefill(self, prompt):
         F = forward_full(self.m, prompt, keep_caches=True)
         self.x = bytearray(prompt)
+        self.b = [bool(f) for f in F.b]  # boundary flags of the committed bytes
         self.h_e = F.h_e
         self.Kp = list(int(k) for k in F.Kp)
         self.u = F.u
@@ -206,12 +213,12 @@ class IncrementalDecoder:
         return self.Kp[-1] if self.Kp else 0
 
     def open_start(self):
-        segs = closed_segments(self.cfg, self.x)
+        segs = segments_of(self.b)
         return segs[-1][1] + 1 if segs else 0
 
     def group_starts(self):
         """(start of group K(t-1)-1 or -1, start of group K(t-1))."""
-        segs = closed_segments(self.cfg, self.x)
+        segs = segments_of(self.b)
         g = self.K
 
         def st(j):
@@ -229,7 +236,7 @@ class IncrementalDecoder:
         """One decode step. forced: accepted-draft count (test hook); forced_cand: n bytes
         replacing c_1, d_2..d_n (test hook); budget: cap on the committed bytes; samp: sample
         with the draws of sequence index b instead of taking argmaxes."""
-        m, cfg = self.m, self.cfg
+        m = self.m
         t, K = self.t, self.K
         # draft (Algorithm 1, drafting step)
         mbl = mb_draft_logits(m, self.Kp, self.o, self.u, t, n, self.x, y_last=self.y_last)
@@ -246,12 +253,14 @@ class IncrementalDecoder:
         pos = np.arange(t, t + n)
         # encoder over the n candidates, appended after the cached keys
         h_c, enc_new = self._stack_cached("enc", m.embed(cand), pos)
-        # segments closed by candidate boundaries; z over committed + candidate bytes
+        # segments closed by candidate boundaries (by the byte, or predicted from h_e of the
+        # candidate); z over committed + candidate bytes
+        cb = boundary_flags(m, cand, h_c)
         h_all = np.concatenate([self.h_e, h_c], axis=0)
         Kc, z_new, k_run = [], [], K
         seg_start = self.open_start()
-        for i, c in enumerate(cand):
-            if c == cfg.boundary_byte:
+        for i in range(n):
+            if cb[i]:
                 k_run += 1
                 z_new.append(h_all[seg_start:t + i + 1].mean(axis=0))
                 seg_start = t + i + 1
@@ -275,6 +284,7 @@ class IncrementalDecoder:
         e = 1 + a if budget is None else min(1 + a, budget)
         self.carried = None if samp is None else carried_dist(rejected, a, e, mbl, nbl, samp)
         self.x += cand[:e]
+        self.b += [bool(f) for f in cb[:e]]
         self.h_e = h_all[:t + e]
         self.Kp += Kc[:e]
         K_new = self.Kp[-1]

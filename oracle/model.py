@@ -6,8 +6,9 @@ this package. The CUDA product path never calls it and shares no code with it;
 both sides receive their inputs from ``synth`` alone.
 
 Plain numpy float64, written for reading, not for speed. The model is the one of
-Section 2.2 (encoder module, space-rule boundaries, mean-pool downsampling, LM
-module with a [BOS] latent, upsampling by duplication, next-byte decoder) plus
+Section 2.2 (encoder module, boundaries by the space rule or by a learned predictor
+on the encoder states, mean-pool downsampling, LM module with a [BOS] latent,
+upsampling by duplication, next-byte decoder) plus
 the multi-byte head of Section 3 (LCA mask, residual r_2 added before
 upsampling, shared unembedding). Blocks follow Llama 3 (Section 4.2): pre-norm
 RMSNorm (eps 1e-6), rotary embeddings (base 1e5), SwiGLU MLP, no biases.
@@ -23,6 +24,8 @@ Readings taken where the paper is silent (each is also listed with the design no
   * no final norm on h_e or on the LM output; separate final RMSNorms for the
     next-byte and multi-byte heads; unembedding untied from the embedding.
   * argmax breaks ties toward the lowest byte value.
+  * the learned boundary predictor is w_2 . SiLU(W_1 h_e[p]) + c, a boundary where its
+    probability sigmoid(.) exceeds 0.5 (where the logit is positive).
 """
 from __future__ import annotations
 
@@ -148,23 +151,49 @@ class Model:
 
 def boundaries(cfg: ModelConfig, x):
     """Space rule: b_p = [x_p == 0x20]; the boundary byte is the last byte of its
-    segment (the learned predictor of Section 2.2 is replaced by this rule)."""
+    segment (used in place of the learned predictor of Section 2.2)."""
     return np.frombuffer(bytes(x), dtype=np.uint8) == cfg.boundary_byte
 
 
-def latent_index(cfg: ModelConfig, x):
-    """K(p) = number of boundaries at positions <= p."""
-    return np.cumsum(boundaries(cfg, x)).astype(np.int64)
+def boundary_logits(model: "Model", h):
+    """Learned boundary predictor of Section 2.2 on encoder states h [T, d]: the logit of the
+    boundary probability, w_2 . SiLU(W_1 h_p) + c."""
+    w = model.w
+    return silu(h @ w["bp.w1"].T) @ w["bp.w2"] + w["bp.bias"][0]
 
 
-def closed_segments(cfg: ModelConfig, x):
-    """[(start, end)] inclusive byte ranges of closed segments S_1..S_K (Section 2.2)."""
+def boundary_flags(model: "Model", x, h_e):
+    """b_p for bytes x with encoder states h_e (Algorithm 1, boundary step): the space rule on
+    the bytes, or the learned predictor, b_p = [sigmoid(logit_p) > 0.5] = [logit_p > 0]."""
+    if model.cfg.boundary == "learned":
+        return boundary_logits(model, h_e) > 0.0
+    return boundaries(model.cfg, x)
+
+
+def latent_index_of(b):
+    """K(p) = number of boundaries at positions <= p, from the flags b."""
+    return np.cumsum(np.asarray(b, dtype=bool)).astype(np.int64)
+
+
+def segments_of(b):
+    """[(start, end)] inclusive byte ranges of the closed segments S_1..S_K (Section 2.2): each
+    ends at a boundary and starts after the previous one."""
     segs, start = [], 0
-    for p, b in enumerate(boundaries(cfg, x)):
-        if b:
+    for p, f in enumerate(b):
+        if f:
             segs.append((start, p))
             start = p + 1
     return segs
+
+
+def latent_index(cfg: ModelConfig, x):
+    """K(p) under the space rule."""
+    return latent_index_of(boundaries(cfg, x))
+
+
+def closed_segments(cfg: ModelConfig, x):
+    """Closed segments under the space rule."""
+    return segments_of(boundaries(cfg, x))
 
 
 def group_start(cfg: ModelConfig, x, g):
@@ -185,9 +214,11 @@ def window_draft_inputs(cfg: ModelConfig, Kp, o, u, t, n, x):
     """Rows of the MB window of Algorithm 1 (drafting step) at committed length t:
     the previous and the current group (from the first byte of group K(t-1)-1, or
     of group 0) then n-2 copies of the last row at positions t..t+n-3.
+    The groups come from K(p) (x, the committed bytes, is not needed: group g >= 1 starts at
+    its boundary byte, the first p with K(p) = g).
     Returns (inputs [W,d], positions [W], groups [W])."""
     g = int(Kp[t - 1])
-    s = group_start(cfg, x, g - 1) if g >= 1 else 0
+    s = next(p for p in range(t) if Kp[p] >= g - 1) if g >= 1 else 0
     pos = list(range(s, t)) + list(range(t, t + n - 2))
     grp = [int(Kp[p]) for p in range(s, t)] + [g] * (n - 2)
     m = np.stack([o[k] + u[k] for k in grp])
@@ -231,13 +262,13 @@ def full_sequence_lca_logits(model: Model, Kp, o, u, extra=0):
 
 class Forward:
     """All intermediate values of one full forward over committed bytes x_0..x_{T-1}."""
-    __slots__ = ("x", "h_e", "Kp", "segs", "z", "u", "o", "y", "nb_logits", "caches")
+    __slots__ = ("x", "h_e", "b", "Kp", "segs", "z", "u", "o", "y", "nb_logits", "caches")
 
 
 def forward_full(model: Model, x, keep_caches=False):
     """Definition of the forward over bytes x (Section 2.2 and the forward part of Algorithm 1):
-    embed, encoder (causal, RoPE at byte position) -> h_e; space boundaries; mean-pool
-    closed segments -> z_1..z_K; LM module over [BOS, z_1..z_K] (causal, RoPE at latent
+    embed, encoder (causal, RoPE at byte position) -> h_e; boundaries (space rule, or the
+    learned predictor on h_e); mean-pool closed segments -> z_1..z_K; LM module over [BOS, z_1..z_K] (causal, RoPE at latent
     index) -> o_0..o_K; next-byte decoder over o_{K(p)} + h_e[p] (causal) -> y; final
     norm and unembedding -> next-byte logits (row p predicts x_{p+1})."""
     cfg = model.cfg
@@ -247,8 +278,9 @@ def forward_full(model: Model, x, keep_caches=False):
     pos = np.arange(T)
     causal = lambda n_prev: causal_mask(n_prev, T)
     F.h_e, enc_kv = model.run_stack("enc", model.embed(x), pos, causal)
-    F.Kp = latent_index(cfg, x)
-    F.segs = closed_segments(cfg, x)
+    F.b = boundary_flags(model, x, F.h_e)
+    F.Kp = latent_index_of(F.b)
+    F.segs = segments_of(F.b)
     F.z = pool(F.h_e, F.segs)
     F.u = np.concatenate([model.w["lm.bos"][None, :], F.z], axis=0)
     K1 = F.u.shape[0]

@@ -35,6 +35,8 @@ class ModelConfig:
     mb_kind: str = "lca"  # "lca" | "mlp"
     n_mlp_heads: int = 0  # MLP head only: independent heads (drafts per step = heads)
     dtype: str = "f32"    # "f32" | "bf16": storage type of weights and KV caches
+    boundary: str = "space"  # "space": byte rule | "learned": predictor on the encoder states
+    d_bp: int = 0         # learned predictor only: hidden width of its MLP
     boundary_byte: int = BOUNDARY_BYTE
     rope_base: float = 1.0e5
     rms_eps: float = 1.0e-6

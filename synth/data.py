@@ -126,6 +126,8 @@ def tensor_list(cfg: ModelConfig) -> list:
         raise ValueError(cfg.mb_kind)
     out.append(("mb.norm", (d,)))
     out.append(("unembed", (v, d)))
+    if cfg.boundary == "learned":  # drawn last, so the other tensors do not change
+        out += [("bp.w1", (cfg.d_bp, d)), ("bp.w2", (cfg.d_bp,)), ("bp.bias", (1,))]
     return out
 
 
@@ -140,15 +142,19 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
     return ((u + bias) & np.uint32(0xFFFF0000)).view(np.float32)
 
 
-def make_weights(cfg: ModelConfig, gain: float = 1.0, seed: int = 0, space_gain: float = 1.0) -> dict:
+def make_weights(cfg: ModelConfig, gain: float = 1.0, seed: int = 0, space_gain: float = 1.0,
+                 bp_bias: float = 0.0) -> dict:
     """name -> float32 array. For dtype "bf16" every value is bf16-representable.
     ``gain`` multiplies the unembedding before rounding (acceptance calibration);
-    ``space_gain`` multiplies its row of the boundary byte first (boundary-rate calibration)."""
+    ``space_gain`` multiplies its row of the boundary byte first (boundary-rate calibration);
+    ``bp_bias`` is the learned boundary predictor's output bias (its boundary rate)."""
     rng = np.random.default_rng(seed)
     out = {}
     for name, shape in tensor_list(cfg):
         if is_norm(name):
             a = np.ones(shape, dtype=np.float32)
+        elif name == "bp.bias":
+            a = np.full(shape, bp_bias, dtype=np.float32)
         else:
             a = rng.standard_normal(shape, dtype=np.float32)
             a *= np.float32(INIT_STD)

@@ -7,8 +7,9 @@ and ``IncrementalDecoder`` must agree with it:
 
   e_p    = E[x_p]
   h_e    = encoder blocks over e (causal, RoPE at byte position p)
-  b_p    = [x_p == 0x20]; K(p) = #{q <= p : b_q}; closed segment k = bytes after the (k-1)-th
-           boundary up to and including the k-th
+  b_p    = [x_p == 0x20], or with the learned predictor [sum_j w2_j SiLU(sum_c W1_jc h_e[p]_c) + c0 > 0];
+           K(p) = #{q <= p : b_q}; closed segment k = bytes after the (k-1)-th boundary up to and
+           including the k-th
   z_k    = mean of h_e over segment k;  u_0 = BOS, u_k = z_k
   o      = LM blocks over u_0..u_K (causal, RoPE at latent index)
   y_p    = next-byte blocks over o_{K(p)} + h_e[p] (causal, RoPE p); logits_p = W_u RMSNorm_nb(y_p)
@@ -36,6 +37,7 @@ from synth.configs import ModelConfig
 
 CFG = ModelConfig(d_model=8, n_heads=2, head_dim=4, d_ff=12, n_enc=1, n_lm=2, n_nb=1, n_mb=2, dtype="f32")
 CFG_MLP = CFG.replace(mb_kind="mlp", n_mb=3, n_mlp_heads=3)
+CFG_BP = CFG.replace(boundary="learned", d_bp=6)
 SP = 0x20
 
 
@@ -71,6 +73,10 @@ def make_weights(cfg, seed, unembed_scale=1.5):
         for j in range(cfg.n_mlp_heads):
             for l in range(cfg.n_mb):
                 W[f"mlp.{j}.{l}.w"] = _mat(rng, d, d, 0.5)
+    if cfg.boundary == "learned":
+        W["bp.w1"] = _mat(rng, cfg.d_bp, d, 0.5)
+        W["bp.w2"] = [_g(rng, 1.0) for _ in range(cfg.d_bp)]
+        W["bp.bias"] = [0.0]
     return W
 
 
@@ -154,19 +160,28 @@ def _prob(row, i):
     return math.exp(row[i] - mx) / sum(math.exp(z - mx) for z in row)
 
 
+def _bp_logit(W, h):
+    hid = [_silu(sum(W["bp.w1"][j][c] * h[c] for c in range(len(h)))) for j in range(len(W["bp.w2"]))]
+    return sum(W["bp.w2"][j] * hid[j] for j in range(len(hid))) + W["bp.bias"][0]
+
+
 def brute_forward(cfg, W, x):
     """Every intermediate of the definition over bytes x."""
     T = len(x)
     causal = lambda t, s: s <= t  # noqa: E731
     h_e = _stack(cfg, W, "enc", cfg.n_enc, [list(W["embed"][c]) for c in x], list(range(T)), causal)
+    if cfg.boundary == "learned":
+        bnd = [_bp_logit(W, h_e[p]) > 0.0 for p in range(T)]
+    else:
+        bnd = [c == SP for c in x]
     Kp, k = [], 0
-    for c in x:
-        k += c == SP
+    for p in range(T):
+        k += bnd[p]
         Kp.append(k)
     # closed segment k (1-based): after the (k-1)-th boundary up to and including the k-th
     z, start = [], 0
     for p in range(T):
-        if x[p] == SP:
+        if bnd[p]:
             seg = range(start, p + 1)
             z.append([sum(h_e[q][c] for q in seg) / len(seg) for c in range(cfg.d_model)])
             start = p + 1
@@ -175,7 +190,7 @@ def brute_forward(cfg, W, x):
     y = _stack(cfg, W, "nb", cfg.n_nb, [[o[Kp[p]][c] + h_e[p][c] for c in range(cfg.d_model)] for p in range(T)],
                list(range(T)), causal)
     logits = [_head(cfg, W, "nb.norm", y[p]) for p in range(T)]
-    return {"h_e": h_e, "Kp": Kp, "z": z, "u": u, "o": o, "y": y, "nb": logits}
+    return {"h_e": h_e, "b": bnd, "Kp": Kp, "z": z, "u": u, "o": o, "y": y, "nb": logits}
 
 
 def brute_draft(cfg, W, x, n, F=None):
@@ -340,3 +355,59 @@ def test_loop_through_boundaries_equals_scalar_loop(lca, mode):
     assert want.count(SP) >= 3
     if mode == THRESH:
         assert 0 < sum(acc) < (n - 1) * len(acc)
+
+
+# ----------------------------------------------------------------------------- learned boundaries
+@pytest.fixture(scope="module")
+def learned():
+    """The learned predictor with its bias set so that about a third of the positions of the text
+    end a segment (the scalar logits' upper tercile)."""
+    W = make_weights(CFG_BP, 9)
+    h = brute_forward(CFG, W, TEXT)["h_e"]
+    lg = sorted(_bp_logit(W, r) for r in h)
+    W["bp.bias"] = [-0.5 * (lg[2 * len(lg) // 3] + lg[2 * len(lg) // 3 - 1])]
+    return W, as_model(CFG_BP, W)
+
+
+def test_learned_boundaries_forward_equals_scalar_chain(learned):
+    W, M = learned
+    B = brute_forward(CFG_BP, W, TEXT)
+    F = forward_full(M, TEXT)
+    assert 4 <= sum(B["b"]) <= 12 and B["b"] != [c == SP for c in TEXT]
+    np.testing.assert_array_equal(F.b, B["b"])
+    np.testing.assert_array_equal(F.Kp, B["Kp"])
+    np.testing.assert_allclose(F.z, B["z"], rtol=1e-10, atol=1e-10)
+    np.testing.assert_allclose(F.o, B["o"], rtol=1e-10, atol=1e-10)
+    np.testing.assert_allclose(F.nb_logits, B["nb"], rtol=1e-9, atol=1e-9)
+
+
+@pytest.mark.parametrize("t", [1, 5, 9, 14, 23])
+def test_learned_boundaries_window_equals_scalar_definition(learned, t):
+    W, M = learned
+    x = TEXT[:t]
+    F = forward_full(M, x)
+    got = mb_draft_logits(M, F.Kp, F.o, F.u, t, 4, x)
+    np.testing.assert_allclose(got, brute_draft(CFG_BP, W, x, 4), rtol=1e-9, atol=1e-9)
+
+
+@pytest.mark.parametrize("mode", [THRESH, SPEC])
+def test_learned_boundaries_generation_equals_scalar_loop(learned, mode):
+    """Segments close wherever the predictor fires on the encoder state of a candidate, accepted or
+    rejected, so the LM module runs on speculative latents and the cached decoder rolls them back."""
+    from oracle import generate_incremental
+    W, M = learned
+    prompt = TEXT[:8]
+    n, G = 4, 16
+    tau = 0.0
+    if mode == THRESH:
+        probs = sorted(_prob(r, _argmax(r)) for r in brute_draft(CFG_BP, W, list(prompt), n))
+        tau = 0.5 * (probs[0] + probs[-1])
+    want, acc = brute_generate(CFG_BP, W, prompt, n, tau, mode, G)
+    got, recs = generate_reference(M, prompt, n, tau, mode, G)
+    assert got == want
+    assert [r.a for r in recs] == acc
+    inc, irecs = generate_incremental(M, prompt, n, tau, mode, G)
+    assert inc == want
+    assert [r.a for r in irecs] == acc
+    assert [(r.t, r.K) for r in irecs] == [(r.t, r.K) for r in recs]
+    assert recs[-1].K > forward_full(M, prompt).Kp[-1]  # segments closed during generation

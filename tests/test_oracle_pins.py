@@ -412,3 +412,33 @@ def test_head_decisions_ties_and_probability():
     assert abs(p - np.e ** 3 / (2 * np.e ** 3 + 254)) < 1e-14
     big = lg + 1e4  # a common offset changes nothing and does not overflow
     assert greedy(big) == 7 and abs(max_prob(big, 7) - p) < 1e-12
+
+
+def test_learned_predictor_that_fires_on_spaces_is_the_space_rule():
+    """A predictor that reads a space marker of the embedding, behind an encoder whose output
+    projections are zero (so h_e = embedding), must segment, pool, draft and decode exactly as the
+    space rule does, through the cached decoder's rollbacks as well."""
+    cfg_l = MICRO.replace(boundary="learned", d_bp=1)
+    W = make_weights(cfg_l, gain=40.0, seed=3)
+    W["embed"][:, 0] = 0.0
+    W["embed"][0x20, 0] = 4.0
+    W["enc.0.wo"][:] = 0.0
+    W["enc.0.w2"][:] = 0.0
+    W["bp.w1"][:] = 0.0
+    W["bp.w1"][0, 0] = 1.0
+    W["bp.w2"][:] = 1.0
+    W["bp.bias"][:] = -1.0  # SiLU(4) - 1 > 0 on a space, SiLU(0) - 1 < 0 elsewhere
+    ML, MS = om.Model(cfg_l, W), om.Model(MICRO, W)
+    x = b"ab cd  efg h"
+    FL, FS = om.forward_full(ML, x), om.forward_full(MS, x)
+    assert list(FL.b) == [c == 0x20 for c in x]
+    np.testing.assert_array_equal(FL.nb_logits, FS.nb_logits)
+    pats = [b"ab c", b" abc", b"a  b", b"abcd", b"x y "]
+    fc = lambda s: pats[s % len(pats)]  # noqa: E731
+    for mode in (THRESH, SPEC):
+        want, rw = generate_incremental(MS, PROMPT, 4, 0.6, mode, 24, force_cand=fc)
+        got, rg = generate_incremental(ML, PROMPT, 4, 0.6, mode, 24, force_cand=fc)
+        assert got == want
+        assert [(r.a, r.t, r.K) for r in rg] == [(r.a, r.t, r.K) for r in rw]
+        ref, rr = generate_reference(ML, PROMPT, 4, 0.6, mode, 24, force_cand=fc)
+        assert ref == want and [r.K for r in rr] == [r.K for r in rw]
