@@ -25,6 +25,7 @@ the first byte of the step after a rejection is drawn from the residual distribu
 from __future__ import annotations
 
 from dataclasses import dataclass, field
+from types import SimpleNamespace
 
 import numpy as np
 
@@ -231,27 +232,15 @@ class IncrementalDecoder:
         T = x.shape[0]
         return self.m.run_stack(prefix, x, pos, lambda n_prev: causal_mask(n_prev, T), caches)
 
-    def step(self, n, tau, mode, forced=None, budget=None, forced_cand=None,
-             samp: Sampling | None = None, b=0):
-        """One decode step. forced: accepted-draft count (test hook); forced_cand: n bytes
-        replacing c_1, d_2..d_n (test hook); budget: cap on the committed bytes; samp: sample
-        with the draws of sequence index b instead of taking argmaxes."""
-        m = self.m
-        t, K = self.t, self.K
-        # draft (Algorithm 1, drafting step)
-        mbl = mb_draft_logits(m, self.Kp, self.o, self.u, t, n, self.x, y_last=self.y_last)
-        if samp is None:
-            c1 = greedy(self.nb_last)
-            drafts = [greedy(r) for r in mbl]
-            probs = [max_prob(r, d) for r, d in zip(mbl, drafts)]
-        else:
-            p1 = self.carried if self.carried is not None else sampling_dist(
-                self.nb_last, samp.temperature, samp.top_p)
-            c1 = sample_index(p1, draw(samp.seed, t, b, NEXT, 0))
-            drafts, probs = sampled_drafts(mbl, samp, t, b)
-        cand = bytes([c1] + drafts) if forced_cand is None else bytes(forced_cand)
+    def run_candidates(self, cand):
+        """The forward part of a step over candidate bytes at positions t..t+len(cand)-1: encoder
+        rows after the cached keys, the boundaries and the segments they close (mean pools over
+        committed and candidate states), the LM module on those latents, the next-byte decoder
+        over o_{K(p)} + h_e[p]. Nothing is kept until ``commit``; ``nbl`` of the result holds the
+        next-byte logits of the candidate rows."""
+        m, t, K, n = self.m, self.t, self.K, len(cand)
         pos = np.arange(t, t + n)
-        # encoder over the n candidates, appended after the cached keys
+        # encoder over the candidates, appended after the cached keys
         h_c, enc_new = self._stack_cached("enc", m.embed(cand), pos)
         # segments closed by candidate boundaries (by the byte, or predicted from h_e of the
         # candidate); z over committed + candidate bytes
@@ -274,7 +263,52 @@ class IncrementalDecoder:
             o_ext = np.concatenate([self.o, o_new], axis=0)
         # next-byte decoder over o_{K(p)} + h_e[p]
         y_c, nb_new = self._stack_cached("nb", o_ext[Kc] + h_c, pos)
-        nbl = m.head(y_c, "nb.norm")
+        return SimpleNamespace(cand=bytes(cand), cb=cb, h_all=h_all, Kc=Kc, u=u_ext, o=o_ext,
+                               enc=enc_new, lm=lm_new, nb=nb_new, y=y_c, nbl=m.head(y_c, "nb.norm"))
+
+    def commit(self, P, e):
+        """Keep the first e candidate rows of ``run_candidates``' result in every cache (and the
+        latents their segments closed); drop the rest."""
+        t, K = self.t, self.K
+        self.x += P.cand[:e]
+        self.b += [bool(f) for f in P.cb[:e]]
+        self.h_e = P.h_all[:t + e]
+        self.Kp += P.Kc[:e]
+        K_new = self.Kp[-1]
+        for s, new in (("enc", P.enc), ("nb", P.nb)):
+            for l, (k, v) in enumerate(new):
+                self.kv[s][l][0] = np.concatenate([self.kv[s][l][0], k[:e]], axis=0)
+                self.kv[s][l][1] = np.concatenate([self.kv[s][l][1], v[:e]], axis=0)
+        keep = K_new - K
+        if keep > 0:
+            for l, (k, v) in enumerate(P.lm):
+                self.kv["lm"][l][0] = np.concatenate([self.kv["lm"][l][0], k[:keep]], axis=0)
+                self.kv["lm"][l][1] = np.concatenate([self.kv["lm"][l][1], v[:keep]], axis=0)
+        self.u = P.u[:K_new + 1]
+        self.o = P.o[:K_new + 1]
+        self.nb_last = P.nbl[e - 1]
+        self.y_last = P.y[e - 1]
+
+    def step(self, n, tau, mode, forced=None, budget=None, forced_cand=None,
+             samp: Sampling | None = None, b=0):
+        """One decode step. forced: accepted-draft count (test hook); forced_cand: n bytes
+        replacing c_1, d_2..d_n (test hook); budget: cap on the committed bytes; samp: sample
+        with the draws of sequence index b instead of taking argmaxes."""
+        m, t = self.m, self.t
+        # draft (Algorithm 1, drafting step)
+        mbl = mb_draft_logits(m, self.Kp, self.o, self.u, t, n, self.x, y_last=self.y_last)
+        if samp is None:
+            c1 = greedy(self.nb_last)
+            drafts = [greedy(r) for r in mbl]
+            probs = [max_prob(r, d) for r, d in zip(mbl, drafts)]
+        else:
+            p1 = self.carried if self.carried is not None else sampling_dist(
+                self.nb_last, samp.temperature, samp.top_p)
+            c1 = sample_index(p1, draw(samp.seed, t, b, NEXT, 0))
+            drafts, probs = sampled_drafts(mbl, samp, t, b)
+        cand = bytes([c1] + drafts) if forced_cand is None else bytes(forced_cand)
+        P = self.run_candidates(cand)
+        nbl = P.nbl
         # accept (Algorithm 1, acceptance step) and commit the accepted prefix
         if samp is None:
             a = accept_count(mode, list(cand[1:]), probs, nbl, tau, forced)
@@ -283,25 +317,8 @@ class IncrementalDecoder:
                                          forced)
         e = 1 + a if budget is None else min(1 + a, budget)
         self.carried = None if samp is None else carried_dist(rejected, a, e, mbl, nbl, samp)
-        self.x += cand[:e]
-        self.b += [bool(f) for f in cb[:e]]
-        self.h_e = h_all[:t + e]
-        self.Kp += Kc[:e]
-        K_new = self.Kp[-1]
-        for s, new in (("enc", enc_new), ("nb", nb_new)):
-            for l, (k, v) in enumerate(new):
-                self.kv[s][l][0] = np.concatenate([self.kv[s][l][0], k[:e]], axis=0)
-                self.kv[s][l][1] = np.concatenate([self.kv[s][l][1], v[:e]], axis=0)
-        keep = K_new - K
-        if keep > 0:
-            for l, (k, v) in enumerate(lm_new):
-                self.kv["lm"][l][0] = np.concatenate([self.kv["lm"][l][0], k[:keep]], axis=0)
-                self.kv["lm"][l][1] = np.concatenate([self.kv["lm"][l][1], v[:keep]], axis=0)
-        self.u = u_ext[:K_new + 1]
-        self.o = o_ext[:K_new + 1]
-        self.nb_last = nbl[e - 1]
-        self.y_last = y_c[e - 1]
-        return StepRecord(c1, drafts, probs, a, cand[:e], mbl, nbl, t=self.t, K=K_new)
+        self.commit(P, e)
+        return StepRecord(c1, drafts, probs, a, cand[:e], mbl, nbl, t=self.t, K=self.K)
 
 
 def generate_incremental(model: Model, prompt, n, tau, mode, G, force=None, force_cand=None,
