@@ -108,3 +108,26 @@ def test_prefill_flops_of_the_paper_model():
     lin = 2 * 16 * d * d * (5 * 4 + 2 * 16)
     att = 2 * d * 5 * 6 * 4 + 2 * d * 2 * 3 * 16
     assert bench.prefill_flops(m, [p]) == lin + att + 2 * 256 * d
+
+
+def test_reference_arm_times_the_oracle_steps():
+    """`bench.py --impl reference` runs the oracle alone (no GPU): K timed decode steps after W
+    untimed ones, one JSON line with the arm's metric, e2e without copies and its cpu_baseline."""
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--workload", "tiny_b1",
+                        "--steps", "4", "--warmup", "3"], cwd=root, capture_output=True, text=True,
+                       timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["unit"] == "bytes/s" and line["higher_is_better"]
+    assert line["steps"] == 4 and line["warmup"] == 3 and line["value"] > 0 and line["ms_per_step"] > 0
+    assert line["e2e"] == {"value": line["value"], "unit": "bytes/s", "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["cores"] >= 1
+    assert "4 timed decode steps" in cb["sample"] and "3 untimed steps" in cb["sample"]
+    assert line["config"]["workload"] == "tiny_b1"
