@@ -131,3 +131,15 @@ def test_reference_arm_times_the_oracle_steps():
     assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["cores"] >= 1
     assert "4 timed decode steps" in cb["sample"] and "3 untimed steps" in cb["sample"]
     assert line["config"]["workload"] == "tiny_b1"
+
+
+def test_reference_arm_runs_on_rank_zero_only():
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--workload", "tiny_b1",
+                        "--gpus", "2", "--steps", "2", "--warmup", "3"], cwd=root, env=env,
+                       capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0 and r.stdout.strip() == ""
