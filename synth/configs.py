@@ -80,6 +80,10 @@ PAPER = ModelConfig(d_model=1024, n_heads=16, head_dim=64, d_ff=4096,
 
 PAPER_MLP = PAPER.replace(mb_kind="mlp", n_mb=3, n_mlp_heads=6)
 
+# The external verifier of Section 6.3 (FxT): a learned boundary predictor (hidden width d), a
+# four-layer next-byte decoder and no multi-byte head.
+FXT = PAPER.replace(boundary="learned", d_bp=1024, n_nb=4, n_mb=0)
+
 WORKLOADS = {
     "tiny_b1": Workload("tiny_b1", TINY, batch=1, prompt_len=256, gen=128,
                         n_list=(3,), tau_list=(0.75,), text="words",
