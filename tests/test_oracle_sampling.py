@@ -212,3 +212,33 @@ def test_speculative_sampling_matches_plain_sampling():
     exp = [joint[k] * S for k in big] + [S * (1 - sum(joint[k] for k in big))]
     assert len(big) >= 4
     assert stats.chisquare(obs, exp).pvalue > 1e-3
+
+
+@pytest.mark.parametrize("pq", _pairs())
+def test_speculative_acceptance_rate_is_the_overlap(pq):
+    """The probability that a draft drawn from q is kept is sum_x min(p(x), q(x)) (the expected
+    acceptance rate of speculative sampling), by quadrature over the draft's and the test's
+    uniforms."""
+    p, q = pq
+    N = 2048
+    grid = (np.arange(N) + 0.5) / N
+    kept = 0.0
+    for ud in grid:
+        d = sample_index(q, ud)
+        kept += np.mean([spec_keep(p, q, d, ua) for ua in grid[::4]])
+    np.testing.assert_allclose(kept / N, np.minimum(p, q).sum(), atol=3.0 * len(p) / N)
+
+
+def test_n1_sampling_is_plain_sampling():
+    """With n = 1 there are no drafts: every step draws one byte from the next-byte sampling
+    distribution with the step's NEXT uniform (c_1 of the step that starts at length t)."""
+    M = micro_model(gain=8.0)
+    samp = Sampling(0.7, 0.9, 77)
+    x = bytearray(PROMPT)
+    for _ in range(10):
+        p = sampling_dist(om.forward_full(M, x).nb_logits[-1], samp.temperature, samp.top_p)
+        x.append(sample_index(p, draw(samp.seed, len(x), 0, NEXT, 0)))
+    want = bytes(x[len(PROMPT):])
+    for mode in (THRESH, SPEC):
+        assert generate_reference(M, PROMPT, 1, 0.75, mode, 10, samp=samp)[0] == want
+        assert generate_incremental(M, PROMPT, 1, 0.75, mode, 10, samp=samp)[0] == want
