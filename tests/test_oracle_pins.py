@@ -442,3 +442,21 @@ def test_learned_predictor_that_fires_on_spaces_is_the_space_rule():
         assert [(r.a, r.t, r.K) for r in rg] == [(r.a, r.t, r.K) for r in rw]
         ref, rr = generate_reference(ML, PROMPT, 4, 0.6, mode, 24, force_cand=fc)
         assert ref == want and [r.K for r in rr] == [r.K for r in rw]
+
+
+def test_incremental_equals_full_recompute_at_paper_size():
+    """The cached decoder against the full recompute on the paper-size model (2/16/2/2 blocks,
+    d = 1024, 16 heads of 64, the calibrated gains of the batch-1 workload) over a short prompt:
+    shapes that the micro models do not reach (16 heads, 16 LM blocks, bf16-rounded weights)."""
+    from synth import WORKLOADS, cached_weights, prompt, weight_gains
+    w = WORKLOADS["paper_b1"]
+    M = om.Model(w.model, cached_weights(w.model, **weight_gains(w, True)))
+    p = prompt(w, 0, 96)
+    out_r, rr = generate_reference(M, p, 3, 0.75, THRESH, 6, record_nb=True)
+    out_i, ri = generate_incremental(M, p, 3, 0.75, THRESH, 6)
+    assert out_r == out_i
+    for a, b in zip(rr, ri):
+        assert (a.c1, a.drafts, a.a, a.t, a.K) == (b.c1, b.drafts, b.a, b.t, b.K)
+        np.testing.assert_allclose(b.mb_logits, a.mb_logits, rtol=1e-8, atol=1e-8)
+        np.testing.assert_allclose(b.nb_logits, a.nb_logits, rtol=1e-8, atol=1e-8)
+    assert p.count(b" ") >= 5  # the prompt has closed segments for the LM module
